@@ -1,0 +1,258 @@
+"""fp64 CPU oracle for the Pair estimator hot path: TEST INFRASTRUCTURE ONLY.
+
+Only tests/, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` may import this package. The CUDA
+library shares no code with it, and it imports nothing from the library
+package except the seeded input generator's bf16 upcast helper (which holds
+none of the estimator's arithmetic).
+
+Contents, each following the paper's definitions literally:
+
+* ``coeffs``: per-rollout coefficients of Eq. (pair-advantage), observed and
+  contrast edge counts, active mask. Plain C in fp64 (``pair_oracle.c``),
+  computed twice (edge-sum form of Algorithm 1 and the direct row form) and
+  cross-checked.
+* ``estimate_dense``: Eq. (pair-ht) by explicit enumeration of every observed
+  edge with the pair kernel h_ij of Eq. (pair-kernel) formed per coordinate.
+* ``head_*`` / ``pair_grad_ref``: the policy objective sum_i A_i log pi(o_i|q)
+  of Sec. 4.5 realised on an LM output head: logits z = W h, log-softmax,
+  target gather, and the exact gradients of the objective w.r.t. the hidden
+  states and the head weight, in fp64 numpy (matmul as a library step).
+
+Parity status: the coefficient, dense and head functions are pinned by the
+paper's identities (Thm. 1, Thm. 2, Prop. bias/covariance, the edge-sum /
+coefficient-collapse identity) and by library/brute-force checks in
+tests/test_oracle_pins.py.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_BUILD = os.path.join(_HERE, "_build")
+_SO = os.path.join(_BUILD, "liboracle.so")
+_SRC = os.path.join(_HERE, "pair_oracle.c")
+
+ORACLE_OK = 0
+ORACLE_ERR_NONPOSITIVE_INCLUSION = 1
+ORACLE_ERR_FORMS_DISAGREE = 2
+
+
+class OracleError(RuntimeError):
+    pass
+
+
+def build_oracle(force: bool = False) -> str:
+    """Compile the C oracle with gcc (no fast-math, no FMA contraction)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_SO)
+            and os.path.getmtime(_SO) >= os.path.getmtime(_SRC)):
+        return _SO
+    tmp = _SO + ".tmp%d" % os.getpid()
+    cmd = ["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC",
+           "-shared", "-pthread", "-o", tmp, _SRC, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _SO)
+    return _SO
+
+
+_lib = None
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(build_oracle())
+        P = ctypes.c_void_p
+        lib.oracle_pair_coeffs.argtypes = [
+            ctypes.c_int, ctypes.c_int, P, P, P, ctypes.c_double, ctypes.c_int,
+            P, P, P, P, P, ctypes.c_int]
+        lib.oracle_pair_coeffs.restype = ctypes.c_int
+        lib.oracle_pair_estimate_dense.argtypes = [
+            ctypes.c_int, ctypes.c_int, ctypes.c_int, P, P, P, P, P,
+            ctypes.c_double, P, ctypes.c_int]
+        lib.oracle_pair_estimate_dense.restype = ctypes.c_int
+        _lib = lib
+    return _lib
+
+
+def n_threads() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:  # pragma: no cover
+        return os.cpu_count() or 1
+
+
+def _ptr(a):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def coeffs(r, J, rho, scale=1.0, center=False, threads=None, check=True):
+    """Eq. (pair-advantage) without the 1/(2M) -> scale * 1/2 factor.
+
+    r [B,G], J [B,G] (0/1), rho [B,G,G] (only i<j read). Returns dict with
+    a, a_mag (scale * 1/2 sum |terms|), active, edges, contrast, status.
+    """
+    r = np.ascontiguousarray(r, dtype=np.float64)
+    J = np.ascontiguousarray(J, dtype=np.uint8)
+    rho = np.ascontiguousarray(rho, dtype=np.float64)
+    B, G = r.shape
+    assert J.shape == (B, G) and rho.shape == (B, G, G)
+    a = np.zeros((B, G), np.float64)
+    a_mag = np.zeros((B, G), np.float64)
+    active = np.zeros((B, G), np.uint8)
+    edges = np.zeros(B, np.int32)
+    contrast = np.zeros(B, np.int32)
+    st = _load().oracle_pair_coeffs(
+        B, G, _ptr(r), _ptr(J), _ptr(rho), float(scale), int(bool(center)),
+        _ptr(a), _ptr(a_mag), _ptr(active), _ptr(edges), _ptr(contrast),
+        threads or n_threads())
+    if check and st == ORACLE_ERR_FORMS_DISAGREE:
+        raise OracleError("edge-sum and row forms disagree")
+    return dict(a=a, a_mag=a_mag, active=active, edges=edges,
+                contrast=contrast, status=st)
+
+
+def estimate_dense(r, J, rho, S, scale=1.0, threads=None):
+    """Eq. (pair-ht) times M*scale: scale * sum_{i<j} J_iJ_j h_ij/rho_ij with
+    h_ij = 1/2 (r_i - r_j)(s_i - s_j) formed explicitly. S [B,G,D]."""
+    r = np.ascontiguousarray(r, dtype=np.float64)
+    J = np.ascontiguousarray(J, dtype=np.uint8)
+    rho = np.ascontiguousarray(rho, dtype=np.float64)
+    B, G = r.shape
+    D = S.shape[2]
+    g = np.zeros((B, D), np.float64)
+    if S.dtype == np.float32:
+        S32 = np.ascontiguousarray(S)
+        p32, p64 = _ptr(S32), None
+    else:
+        S64 = np.ascontiguousarray(S, dtype=np.float64)
+        p32, p64 = None, _ptr(S64)
+    st = _load().oracle_pair_estimate_dense(
+        B, G, D, _ptr(r), _ptr(J), _ptr(rho), p32, p64, float(scale),
+        _ptr(g), threads or n_threads())
+    return g, st
+
+
+# ----------------------------------------------------------------------------
+# LM-head objective: sum_i A_i log pi(o_i | q)   (Sec. 4.5)
+# log pi(o_i | q) = sum over the response tokens t of rollout i of
+# log softmax(W h_t)[y_t]  (the sequence-level score of Sec. 3.1 is its
+# gradient). Ascent convention: the returned gradients are of the objective.
+# ----------------------------------------------------------------------------
+
+def segment_ids(cu_seqlens):
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    return np.repeat(np.arange(cu.size - 1), np.diff(cu))
+
+
+def compact_tokens(cu_seqlens, mask, a):
+    """Tokens that enter the objective: mask_t = 1 inside a rollout whose
+    coefficient is nonzero. Returns (token index, c_t = a_seg(t), seg(t))."""
+    seg = segment_ids(cu_seqlens)
+    a = np.asarray(a)
+    keep = (np.asarray(mask) == 1) & (a[seg] != 0)
+    idx = np.nonzero(keep)[0]
+    return idx, np.asarray(a, np.float64)[seg[idx]], seg[idx]
+
+
+def head_logits(Hrows, W):
+    """z_tv = <h_t, W_v> in fp64."""
+    return np.asarray(Hrows, np.float64) @ np.asarray(W, np.float64).T
+
+
+def head_lse(Hrows, W, y, chunk=256):
+    """Per token: log-sum-exp over the vocabulary (max-shifted) and the
+    target logit. Returns (lse, z_target), fp64."""
+    W64 = np.asarray(W, np.float64)
+    n = Hrows.shape[0]
+    lse = np.empty(n, np.float64)
+    zy = np.empty(n, np.float64)
+    for s in range(0, n, chunk):
+        e = min(n, s + chunk)
+        Z = np.asarray(Hrows[s:e], np.float64) @ W64.T
+        m = Z.max(axis=1)
+        lse[s:e] = m + np.log(np.exp(Z - m[:, None]).sum(axis=1))
+        zy[s:e] = Z[np.arange(e - s), y[s:e]]
+    return lse, zy
+
+
+def head_dh_rows(Hrows, W, y, c, lse):
+    """dJ/dh_t = c_t (W_{y_t} - sum_v softmax(z_t)_v W_v) for the given rows."""
+    W64 = np.asarray(W, np.float64)
+    Z = np.asarray(Hrows, np.float64) @ W64.T
+    P = np.exp(Z - lse[:, None])
+    return np.asarray(c, np.float64)[:, None] * (W64[y] - P @ W64)
+
+
+def head_dw_rows(Hact, W, yact, cact, lse_act, vrows, chunk=4096):
+    """dJ/dW_v = sum_t c_t (1[y_t = v] - softmax(z_t)_v) h_t for v in vrows,
+    summed over every active token t (rows Hact with targets yact)."""
+    H64 = np.asarray(Hact, np.float64)
+    W64 = np.asarray(W, np.float64)
+    vrows = np.asarray(vrows, np.int64)
+    out = np.empty((vrows.size, H64.shape[1]), np.float64)
+    for s in range(0, vrows.size, chunk):
+        vs = vrows[s:s + chunk]
+        Z = H64 @ W64[vs].T
+        P = np.exp(Z - lse_act[:, None])
+        onehot = (np.asarray(yact)[:, None] == vs[None, :]).astype(np.float64)
+        Gt = np.asarray(cact, np.float64)[:, None] * (onehot - P)
+        out[s:s + chunk] = Gt.T @ H64
+    return out
+
+
+def pair_grad_ref(inp, a, dh_rows=None, dw_rows=None, lse_tokens=None,
+                  full=False):
+    """Reference outputs of pair_grad for inputs from synth.make_head_workload.
+
+    a: per-rollout coefficients [R]. With full=True every output is computed
+    (J, logp_seq, dH over all T rows, dW over all V rows). Otherwise:
+    dh_rows / dw_rows select the rows to compute; lse_tokens selects the
+    tokens whose lse/logp are returned (indices into the packed batch).
+    """
+    from paper_2608_11368_gb300.synth import as_float  # exact upcast only
+    Hf = as_float(inp["H"], inp["dtype"])
+    Wf = as_float(inp["W"], inp["dtype"])
+    y = inp["y"]
+    idx, c, seg = compact_tokens(inp["cu_seqlens"], inp["mask"], a)
+    out = {"active_tokens": idx, "c": c}
+    R = inp["R"]
+    if full:
+        lse, zy = head_lse(Hf[idx], Wf, y[idx])
+        logp = zy - lse
+        out["lse"], out["logp"] = lse, logp
+        out["J"] = float(np.sum(c * logp))
+        out["J_abs"] = float(np.sum(np.abs(c * logp)))
+        lps = np.zeros(R, np.float64)
+        np.add.at(lps, seg, logp)
+        out["logp_seq"] = lps
+        dH = np.zeros((inp["T"], inp["d"]), np.float64)
+        if idx.size:
+            dH[idx] = head_dh_rows(Hf[idx], Wf, y[idx], c, lse)
+        out["dH"] = dH
+        out["dW"] = head_dw_rows(Hf[idx], Wf, y[idx], c, lse,
+                                 np.arange(inp["V"]))
+        return out
+    if lse_tokens is not None:
+        t = np.asarray(lse_tokens, np.int64)
+        lse_t, zy_t = head_lse(Hf[t], Wf, y[t])
+        out["lse_sel"], out["logp_sel"] = lse_t, zy_t - lse_t
+    if dh_rows is not None:
+        t = np.asarray(dh_rows, np.int64)
+        seg_all = segment_ids(inp["cu_seqlens"])
+        ct = np.asarray(a, np.float64)[seg_all[t]] * (inp["mask"][t] == 1)
+        lse_t, _ = head_lse(Hf[t], Wf, y[t])
+        rows = np.zeros((t.size, inp["d"]), np.float64)
+        nz = ct != 0
+        if nz.any():
+            rows[nz] = head_dh_rows(Hf[t[nz]], Wf, y[t[nz]], ct[nz], lse_t[nz])
+        out["dH_rows"] = rows
+    if dw_rows is not None:
+        lse_a, _ = head_lse(Hf[idx], Wf, y[idx])
+        out["dW_rows"] = head_dw_rows(Hf[idx], Wf, y[idx], c, lse_a, dw_rows)
+    return out
