@@ -1,0 +1,206 @@
+/*
+ * pair.h -- C ABI of the GB300 (sm_103a) hot path of the Pair estimator
+ * (Pairwise-Aware Inclusion Reweighting for adaptive rollout allocation).
+ *
+ * Problem statement (Sec. 3): a prompt has G candidate rollouts with
+ * verifiable rewards r_i and sequence scores s_i = d log pi(o_i|q) / d theta.
+ * An adaptive continuation design completes rollout i iff J_i = 1; the
+ * sampler logs the joint inclusion probabilities rho_ij = P(J_i = J_j = 1)
+ * > 0 (Sec. 3.3). With the pair kernel h_ij = 1/2 (r_i - r_j)(s_i - s_j)
+ * (Sec. 3.2, Eq. pair-kernel) the design-unbiased estimator is
+ *     g = (1/M) sum_{i<j} J_i J_j h_ij / rho_ij,      M = C(G, 2)
+ * (Sec. 4.5, Eq. pair-ht), which collapses to g = sum_i A_i s_i with
+ *     A_i = 1/(2M) sum_{j != i} J_i J_j (r_i - r_j) / rho_ij
+ * (Eq. pair-advantage); the policy is updated through the objective
+ * sum_i A_i log pi(o_i | q) (Sec. 4.5, Algorithm 1).
+ *
+ * Normalisation: every entry point takes `scale`. The coefficient computed
+ * is a_i = scale * 1/2 sum_{j != i} J_i J_j (r_i - r_j) / rho_ij, so
+ * scale = 1 gives the plain completed-edge sum and scale = 1/C(G,2) gives
+ * the paper's A_i (M counts all G candidates, not the completed ones).
+ *
+ * Conventions shared by all calls:
+ *  - All array pointers are caller-owned DEVICE memory unless stated.
+ *    Outputs are overwritten (never accumulated). The library never
+ *    allocates, frees or synchronises inside a compute call; every call is
+ *    asynchronous on `stream` (0 = legacy default stream).
+ *  - Row-major layouts; group b, candidate i is element b*G + i.
+ *  - rho [B][G][G] float32: only the strict upper triangle (i < j) is read;
+ *    the diagonal and lower triangle are ignored (rho is symmetric by
+ *    definition, Sec. 3.3).
+ *  - Host-detected argument errors return immediately, before any launch.
+ *  - Device-detected data errors (rho_ij <= 0 or NaN on a completed edge;
+ *    a target id outside [0, V) at a mask = 1 token) never trap: the kernel
+ *    finishes, the affected outputs are unspecified, and a bit is OR-ed into
+ *    the caller's device word `dev_err`, which `pair_status_sync` decodes.
+ *  - Requires a compute capability 10.3 device (GB300). Other devices get
+ *    PAIR_ERR_UNSUPPORTED.
+ */
+#ifndef PAIR_H_
+#define PAIR_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define PAIR_API __attribute__((visibility("default")))
+#else
+#define PAIR_API
+#endif
+
+/* Opaque CUDA stream handle (a cudaStream_t). */
+typedef struct CUstream_st *pair_stream_t;
+
+typedef enum {
+  PAIR_OK = 0,
+  PAIR_ERR_INVALID_ARG = 1,           /* null pointer, bad size or layout   */
+  PAIR_ERR_UNSUPPORTED = 2,           /* device or shape not supported      */
+  PAIR_ERR_WORKSPACE = 3,             /* workspace missing or too small     */
+  PAIR_ERR_NONPOSITIVE_INCLUSION = 4, /* rho_ij <= 0 or NaN, completed edge */
+  PAIR_ERR_TARGET_RANGE = 5,          /* y_t outside [0, V) at a mask=1 token */
+  PAIR_ERR_CUDA = 6,                  /* a CUDA runtime call failed         */
+  PAIR_ERR_DEVICE_TIMEOUT = 7         /* a bounded on-device wait gave up;
+                                         outputs of that call are invalid  */
+} pair_status;
+
+typedef enum { PAIR_F32 = 0, PAIR_BF16 = 1 } pair_dtype;
+
+/* Bits of the device error word written by the kernels. */
+#define PAIR_DEV_ERR_NONPOSITIVE_INCLUSION 1
+#define PAIR_DEV_ERR_TARGET_RANGE 2
+#define PAIR_DEV_ERR_TIMEOUT 4 /* a pipeline wait exceeded its limit (~2 s) */
+
+/* pair_coeffs flags. */
+#define PAIR_CENTER 1u /* subtract the mean of a over completed vertices
+                          (App. C, numerical stability). Off by default:
+                          in exact arithmetic the sum is already zero. */
+
+/* Largest group size G accepted by pair_coeffs / pair_estimate_dense. */
+#define PAIR_MAX_G 128
+
+/*
+ * pair_coeffs -- per-rollout coefficients of Eq. (pair-advantage) and the
+ * observed-edge bookkeeping of Algorithm 1 (enumerate induced edges,
+ * accumulate each edge term into both endpoints).
+ *
+ * In:  B >= 1 groups of G candidates, 2 <= G <= PAIR_MAX_G.
+ *      r      [B][G] float32  rewards (any real value; binary in RLVR).
+ *      J      [B][G] uint8    completion indicators (0 or nonzero).
+ *      rho    [B][G][G] float32 logged joint inclusion probabilities.
+ *      scale  multiplies every coefficient (see the header comment).
+ *      flags  0 or PAIR_CENTER.
+ * Out: a      [B][G] float32  a_i = scale * 1/2 sum_{j != i} J_iJ_j
+ *                             (r_i - r_j)/rho_ij; exactly 0 where J_i = 0
+ *                             or no completed partner has another reward.
+ *      active [B][G] uint8    1 iff J_i = 1 and some completed j != i has
+ *                             r_j != r_i (nullable).
+ *      edges  [B] int32       number of observed edges C(K_b, 2),
+ *                             K_b = sum_i J_i (nullable).
+ *      contrast_edges [B] int32 observed edges with r_i != r_j (nullable).
+ *      dev_err: device int32 error word (nullable; if null, device data
+ *               errors are not reported).
+ * Arithmetic: fp32, IEEE division, tree summation over the partners (a
+ * relative error of a few ulp of sum_j |term_j|); deterministic.
+ */
+PAIR_API pair_status pair_coeffs(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                        const float *rho, float scale, uint32_t flags,
+                        float *a, uint8_t *active, int32_t *edges,
+                        int32_t *contrast_edges, int32_t *dev_err,
+                        pair_stream_t stream);
+
+/*
+ * pair_estimate_dense -- Eq. (pair-ht) for explicit score vectors:
+ *     g_b = scale * sum_{i<j} J_iJ_j h_ij / rho_ij = sum_i a_i s_{b,i}
+ * (the coefficient collapse of Eq. pair-advantage; rows with a_i = 0 are
+ * never read).
+ *
+ * In:  r, J, rho, scale as for pair_coeffs (flags = 0);
+ *      S [B][G][D] float32 score vectors, D >= 1.
+ * Out: g [B][D] float32; exactly 0 for a group without an active vertex.
+ *      a [B][G] float32 coefficients (nullable).
+ *      dev_err as for pair_coeffs.
+ */
+PAIR_API pair_status pair_estimate_dense(int32_t B, int32_t G, int32_t D,
+                                const float *r, const uint8_t *J,
+                                const float *rho, const float *S, float scale,
+                                float *g, float *a, int32_t *dev_err,
+                                pair_stream_t stream);
+
+/*
+ * pair_grad_workspace_size -- bytes of device workspace pair_grad needs for
+ * T packed tokens, hidden size d, vocabulary V, R rollouts and dtype dt.
+ * Returns 0 for arguments pair_grad would reject.
+ */
+PAIR_API size_t pair_grad_workspace_size(int64_t T, int32_t d, int32_t V, int32_t R,
+                                pair_dtype dt);
+
+/*
+ * pair_grad -- the policy objective of Sec. 4.5, sum_i a_i log pi(o_i | q),
+ * realised on an LM output head over a packed variable-length batch, with
+ * its exact gradients (ascent convention: derivatives OF the objective; a
+ * trainer minimising a loss negates them):
+ *     z_t = W h_t,  logp_t = z_t[y_t] - logsumexp(z_t),
+ *     Jobj = sum_i a_i sum_{t in rollout i, mask_t = 1} logp_t,
+ *     dH = dJobj/dH  [T][d],   dW = dJobj/dW  [V][d].
+ * The sequence score of Sec. 3.1 is the per-rollout sum over tokens (no
+ * length normalisation). Rollouts with a_i == 0 (+0 or -0) are skipped
+ * entirely; their tokens' dH rows, like those of mask = 0 tokens, are
+ * written as exact zeros. Logits never leave the chip (vocabulary-tiled
+ * on-chip softmax).
+ *
+ * In:  T >= 1 packed tokens; d hidden size; V vocabulary size; dt dtype of
+ *      H and W (PAIR_BF16: fp32 accumulation on the tensor cores, requires
+ *      d % 64 == 0; PAIR_F32: fp32 CUDA-core path).
+ *      Shapes: T >= 1, R >= 1, V >= 1, d % 16 == 0 (PAIR_F32) or
+ *      d % 64 == 0 (PAIR_BF16); H, W 16-byte aligned.
+ *      H [T][d] (dt)     hidden state that predicts y_t (targets are NOT
+ *                        shifted by the library).
+ *      W [V][d] (dt)     head weight (nn.Linear layout).
+ *      y [T] int32       target ids; read only where mask_t = 1.
+ *      mask [T] uint8    1 = response token, 0 = padding (padding rows of H
+ *                        and y may hold anything, NaN included).
+ *      cu_seqlens [R+1] int32  rollout i owns tokens [cu[i], cu[i+1]);
+ *                        cu[0] = 0, non-decreasing, cu[R] = T (R >= 1).
+ *      a [R] float32     per-rollout coefficients (e.g. from pair_coeffs,
+ *                        group-major b*G + i).
+ * Out: dH [T][d] float32, dW [V][d] float32,
+ *      Jobj [1] double   (device pointer),
+ *      logp_seq [R] float32 (nullable): sum of logp_t over the rollout's
+ *                        mask = 1 tokens where a_i != 0, 0 elsewhere.
+ * Workspace: ws (device, >= pair_grad_workspace_size bytes, any contents,
+ *      256-byte aligned). dev_err as for pair_coeffs (target-range and
+ *      pipeline-timeout errors).
+ * Deterministic: repeated calls give bit-identical outputs.
+ */
+PAIR_API pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
+                      const void *H, const void *W, const int32_t *y,
+                      const uint8_t *mask, const int32_t *cu_seqlens,
+                      int32_t R, const float *a, float *dH, float *dW,
+                      double *Jobj, float *logp_seq, void *ws,
+                      size_t ws_bytes, int32_t *dev_err, pair_stream_t stream);
+
+/*
+ * pair_status_sync -- synchronise `stream`, read the device error word
+ * (if non-null), reset it to 0, and return the status it encodes
+ * (PAIR_ERR_DEVICE_TIMEOUT, then PAIR_ERR_NONPOSITIVE_INCLUSION, then
+ * PAIR_ERR_TARGET_RANGE), or
+ * PAIR_ERR_CUDA if the stream reports an error. Not for hot loops.
+ */
+PAIR_API pair_status pair_status_sync(pair_stream_t stream, int32_t *dev_err);
+
+/* Static description of a status code. */
+PAIR_API const char *pair_status_string(pair_status st);
+
+/* Kernel launches issued by the most recent compute call on this thread
+ * (used to report how many of this library's kernels ran). */
+PAIR_API int32_t pair_last_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PAIR_H_ */

@@ -181,12 +181,18 @@ def head_lse(Hrows, W, y, chunk=256):
     return lse, zy
 
 
-def head_dh_rows(Hrows, W, y, c, lse):
+def head_dh_rows(Hrows, W, y, c, lse, chunk=256):
     """dJ/dh_t = c_t (W_{y_t} - sum_v softmax(z_t)_v W_v) for the given rows."""
     W64 = np.asarray(W, np.float64)
-    Z = np.asarray(Hrows, np.float64) @ W64.T
-    P = np.exp(Z - lse[:, None])
-    return np.asarray(c, np.float64)[:, None] * (W64[y] - P @ W64)
+    n = Hrows.shape[0]
+    out = np.empty((n, W64.shape[1]), np.float64)
+    c = np.asarray(c, np.float64)
+    for s in range(0, n, chunk):
+        e = min(n, s + chunk)
+        Z = np.asarray(Hrows[s:e], np.float64) @ W64.T
+        P = np.exp(Z - lse[s:e, None])
+        out[s:e] = c[s:e, None] * (W64[y[s:e]] - P @ W64)
+    return out
 
 
 def head_dw_rows(Hact, W, yact, cact, lse_act, vrows, chunk=4096):
@@ -207,23 +213,30 @@ def head_dw_rows(Hact, W, yact, cact, lse_act, vrows, chunk=4096):
 
 
 def pair_grad_ref(inp, a, dh_rows=None, dw_rows=None, lse_tokens=None,
-                  full=False):
+                  full=False, logp_rollouts=None):
     """Reference outputs of pair_grad for inputs from synth.make_head_workload.
 
     a: per-rollout coefficients [R]. With full=True every output is computed
-    (J, logp_seq, dH over all T rows, dW over all V rows). Otherwise:
-    dh_rows / dw_rows select the rows to compute; lse_tokens selects the
-    tokens whose lse/logp are returned (indices into the packed batch).
+    (J, logp_seq, dH over all T rows, dW over all V rows). Otherwise only the
+    requested pieces: dh_rows / dw_rows select dH / dW rows, lse_tokens
+    selects tokens whose lse / logp are returned, logp_rollouts selects
+    rollouts whose summed logp is returned. Only the hidden rows that a
+    requested output depends on are read.
     """
     from paper_2608_11368_gb300.synth import as_float  # exact upcast only
-    Hf = as_float(inp["H"], inp["dtype"])
-    Wf = as_float(inp["W"], inp["dtype"])
+    dtype = inp["dtype"]
+
+    def hrows(t):
+        return as_float(inp["H"][np.asarray(t, np.int64)], dtype)
+
+    Wf = as_float(inp["W"], dtype).astype(np.float64)
     y = inp["y"]
     idx, c, seg = compact_tokens(inp["cu_seqlens"], inp["mask"], a)
     out = {"active_tokens": idx, "c": c}
     R = inp["R"]
     if full:
-        lse, zy = head_lse(Hf[idx], Wf, y[idx])
+        Ha = hrows(idx)
+        lse, zy = head_lse(Ha, Wf, y[idx])
         logp = zy - lse
         out["lse"], out["logp"] = lse, logp
         out["J"] = float(np.sum(c * logp))
@@ -233,26 +246,39 @@ def pair_grad_ref(inp, a, dh_rows=None, dw_rows=None, lse_tokens=None,
         out["logp_seq"] = lps
         dH = np.zeros((inp["T"], inp["d"]), np.float64)
         if idx.size:
-            dH[idx] = head_dh_rows(Hf[idx], Wf, y[idx], c, lse)
+            dH[idx] = head_dh_rows(Ha, Wf, y[idx], c, lse)
         out["dH"] = dH
-        out["dW"] = head_dw_rows(Hf[idx], Wf, y[idx], c, lse,
-                                 np.arange(inp["V"]))
+        out["dW"] = head_dw_rows(Ha, Wf, y[idx], c, lse, np.arange(inp["V"]))
         return out
     if lse_tokens is not None:
         t = np.asarray(lse_tokens, np.int64)
-        lse_t, zy_t = head_lse(Hf[t], Wf, y[t])
+        lse_t, zy_t = head_lse(hrows(t), Wf, y[t])
         out["lse_sel"], out["logp_sel"] = lse_t, zy_t - lse_t
+    if logp_rollouts is not None:
+        cu = inp["cu_seqlens"]
+        vals = []
+        for i in logp_rollouts:
+            t = np.arange(cu[i], cu[i + 1])
+            t = t[inp["mask"][t] == 1]
+            if a[i] == 0 or t.size == 0:
+                vals.append(0.0)
+                continue
+            lse_t, zy_t = head_lse(hrows(t), Wf, y[t])
+            vals.append(float(np.sum(zy_t - lse_t)))
+        out["logp_seq_sel"] = np.array(vals)
     if dh_rows is not None:
         t = np.asarray(dh_rows, np.int64)
         seg_all = segment_ids(inp["cu_seqlens"])
         ct = np.asarray(a, np.float64)[seg_all[t]] * (inp["mask"][t] == 1)
-        lse_t, _ = head_lse(Hf[t], Wf, y[t])
         rows = np.zeros((t.size, inp["d"]), np.float64)
         nz = ct != 0
         if nz.any():
-            rows[nz] = head_dh_rows(Hf[t[nz]], Wf, y[t[nz]], ct[nz], lse_t[nz])
+            Ht = hrows(t[nz])
+            lse_t, _ = head_lse(Ht, Wf, y[t[nz]])
+            rows[nz] = head_dh_rows(Ht, Wf, y[t[nz]], ct[nz], lse_t)
         out["dH_rows"] = rows
     if dw_rows is not None:
-        lse_a, _ = head_lse(Hf[idx], Wf, y[idx])
-        out["dW_rows"] = head_dw_rows(Hf[idx], Wf, y[idx], c, lse_a, dw_rows)
+        Ha = hrows(idx)
+        lse_a, _ = head_lse(Ha, Wf, y[idx])
+        out["dW_rows"] = head_dw_rows(Ha, Wf, y[idx], c, lse_a, dw_rows)
     return out

@@ -1,0 +1,193 @@
+"""ctypes binding of libpair.so for torch tensors: argument marshalling only.
+
+The functions carry the C-ABI names (include/pair.h). Every step of the
+estimator runs in the library's CUDA kernels; this module only checks
+tensor placement/dtypes, allocates outputs with torch when the caller does
+not pass them, and forwards raw device pointers plus the current CUDA stream.
+There is no CPU fallback: if libpair.so is missing, importing the binding's
+library raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libpair.so")
+HEADER = os.path.join(os.path.dirname(_PKG), "include", "pair.h")
+
+PAIR_OK = 0
+PAIR_F32, PAIR_BF16 = 0, 1
+PAIR_CENTER = 1
+STATUS_NAMES = {0: "PAIR_OK", 1: "PAIR_ERR_INVALID_ARG", 2: "PAIR_ERR_UNSUPPORTED",
+                3: "PAIR_ERR_WORKSPACE", 4: "PAIR_ERR_NONPOSITIVE_INCLUSION",
+                5: "PAIR_ERR_TARGET_RANGE", 6: "PAIR_ERR_CUDA",
+                7: "PAIR_ERR_DEVICE_TIMEOUT"}
+
+
+class PairError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__("%s: %s (%s)" % (where, STATUS_NAMES.get(status, status),
+                                          pair_status_string(status)))
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libpair.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError("libpair.so is not built (run __graft_entry__.build())")
+    L = ctypes.CDLL(LIB_PATH)
+    P, I32, I64, F32, U32, SZ = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64,
+                                 ctypes.c_float, ctypes.c_uint32, ctypes.c_size_t)
+    L.pair_coeffs.argtypes = [I32, I32, P, P, P, F32, U32, P, P, P, P, P, P]
+    L.pair_coeffs.restype = ctypes.c_int
+    L.pair_estimate_dense.argtypes = [I32, I32, I32, P, P, P, P, F32, P, P, P, P]
+    L.pair_estimate_dense.restype = ctypes.c_int
+    L.pair_grad_workspace_size.argtypes = [I64, I32, I32, I32, ctypes.c_int]
+    L.pair_grad_workspace_size.restype = SZ
+    L.pair_grad.argtypes = [I64, I32, I32, ctypes.c_int, P, P, P, P, P, I32, P,
+                            P, P, P, P, P, SZ, P, P]
+    L.pair_grad.restype = ctypes.c_int
+    L.pair_status_sync.argtypes = [P, P]
+    L.pair_status_sync.restype = ctypes.c_int
+    L.pair_status_string.argtypes = [ctypes.c_int]
+    L.pair_status_string.restype = ctypes.c_char_p
+    L.pair_last_launch_count.argtypes = []
+    L.pair_last_launch_count.restype = I32
+    _lib = L
+    return L
+
+
+def header_functions():
+    """Names of the functions declared in include/pair.h."""
+    txt = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:[\w\s\*]+?)\b(pair_\w+)\s*\(", txt,
+                                 flags=re.M)))
+
+
+def pair_status_string(status: int) -> str:
+    return lib().pair_status_string(int(status)).decode()
+
+
+def pair_last_launch_count() -> int:
+    return int(lib().pair_last_launch_count())
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t, name, dtype, shape=None):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError("%s must be a CUDA tensor" % name)
+    if t.dtype != dtype:
+        raise TypeError("%s must be %s, got %s" % (name, dtype, t.dtype))
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError("%s must have shape %s, got %s" % (name, tuple(shape),
+                                                            tuple(t.shape)))
+
+
+def _check(st, where):
+    if st != PAIR_OK:
+        raise PairError(st, where)
+
+
+def pair_coeffs(r, J, rho, scale=1.0, flags=0, a=None, active=None, edges=None,
+                contrast_edges=None, dev_err=None, stream=None):
+    """Coefficients of Eq. (pair-advantage) (times `scale`, see pair.h).
+    Returns (a, active, edges, contrast_edges)."""
+    B, G = r.shape
+    dev = r.device
+    _need(r, "r", torch.float32)
+    _need(J, "J", torch.uint8, (B, G))
+    _need(rho, "rho", torch.float32, (B, G, G))
+    a = torch.empty((B, G), dtype=torch.float32, device=dev) if a is None else a
+    active = torch.empty((B, G), dtype=torch.uint8, device=dev) if active is None else active
+    edges = torch.empty(B, dtype=torch.int32, device=dev) if edges is None else edges
+    contrast_edges = (torch.empty(B, dtype=torch.int32, device=dev)
+                      if contrast_edges is None else contrast_edges)
+    st = lib().pair_coeffs(B, G, _p(r), _p(J), _p(rho), float(scale), int(flags),
+                           _p(a), _p(active), _p(edges), _p(contrast_edges),
+                           _p(dev_err), _stream(stream))
+    _check(st, "pair_coeffs")
+    return a, active, edges, contrast_edges
+
+
+def pair_estimate_dense(r, J, rho, S, scale=1.0, g=None, a=None, dev_err=None,
+                        stream=None):
+    """Eq. (pair-ht) for explicit scores S [B,G,D]. Returns (g, a)."""
+    B, G, D = S.shape
+    _need(r, "r", torch.float32, (B, G))
+    _need(J, "J", torch.uint8, (B, G))
+    _need(rho, "rho", torch.float32, (B, G, G))
+    _need(S, "S", torch.float32)
+    g = torch.empty((B, D), dtype=torch.float32, device=S.device) if g is None else g
+    st = lib().pair_estimate_dense(B, G, D, _p(r), _p(J), _p(rho), _p(S),
+                                   float(scale), _p(g), _p(a), _p(dev_err),
+                                   _stream(stream))
+    _check(st, "pair_estimate_dense")
+    return g, a
+
+
+def pair_grad_workspace_size(T, d, V, R, dtype) -> int:
+    return int(lib().pair_grad_workspace_size(int(T), int(d), int(V), int(R),
+                                              int(dtype)))
+
+
+def _pair_dtype(t):
+    if t.dtype == torch.bfloat16:
+        return PAIR_BF16
+    if t.dtype == torch.float32:
+        return PAIR_F32
+    raise TypeError("H/W must be bfloat16 or float32")
+
+
+def pair_grad(H, W, y, mask, cu_seqlens, a, dH=None, dW=None, Jobj=None,
+              logp_seq=None, ws=None, dev_err=None, stream=None):
+    """LM-head realisation of sum_i a_i log pi(o_i|q) and its gradients.
+    Returns (Jobj [1] f64, dH [T,d] f32, dW [V,d] f32, logp_seq [R] f32)."""
+    T, d = H.shape
+    V = W.shape[0]
+    R = cu_seqlens.numel() - 1
+    dt = _pair_dtype(H)
+    _need(H, "H", H.dtype)
+    _need(W, "W", H.dtype, (V, d))
+    _need(y, "y", torch.int32, (T,))
+    _need(mask, "mask", torch.uint8, (T,))
+    _need(cu_seqlens, "cu_seqlens", torch.int32, (R + 1,))
+    _need(a, "a", torch.float32, (R,))
+    dev = H.device
+    dH = torch.empty((T, d), dtype=torch.float32, device=dev) if dH is None else dH
+    dW = torch.empty((V, d), dtype=torch.float32, device=dev) if dW is None else dW
+    Jobj = torch.empty(1, dtype=torch.float64, device=dev) if Jobj is None else Jobj
+    logp_seq = torch.empty(R, dtype=torch.float32, device=dev) if logp_seq is None else logp_seq
+    need = pair_grad_workspace_size(T, d, V, R, dt)
+    if ws is None:
+        ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    st = lib().pair_grad(T, d, V, dt, _p(H), _p(W), _p(y), _p(mask),
+                         _p(cu_seqlens), R, _p(a), _p(dH), _p(dW), _p(Jobj),
+                         _p(logp_seq), _p(ws), ws.numel(), _p(dev_err),
+                         _stream(stream))
+    _check(st, "pair_grad")
+    return Jobj, dH, dW, logp_seq
+
+
+def pair_status_sync(dev_err=None, stream=None) -> int:
+    """Synchronise the stream and decode/reset the device error word."""
+    return int(lib().pair_status_sync(_stream(stream), _p(dev_err)))

@@ -1,0 +1,155 @@
+// C-ABI entry points of libpair (see include/pair.h for the contract).
+//
+// Host side only: argument validation, device check, workspace carving and
+// the launch sequence. Every compute step runs in this library's kernels.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "pair_common.cuh"
+
+namespace pairk {
+
+static thread_local int32_t g_launches = 0;
+void note_launch() { ++g_launches; }
+void reset_launches() { g_launches = 0; }
+
+static pair_status check_device() {
+  static int cached_dev = -1;
+  static pair_status cached = PAIR_OK;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return PAIR_ERR_CUDA;
+  if (dev != cached_dev) {
+    int major = 0, minor = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) !=
+            cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) !=
+            cudaSuccess)
+      return PAIR_ERR_CUDA;
+    cached = (major == 10 && minor == 3) ? PAIR_OK : PAIR_ERR_UNSUPPORTED;
+    cached_dev = dev;
+  }
+  return cached;
+}
+
+static bool aligned16(const void *p) {
+  return (reinterpret_cast<uintptr_t>(p) & 15u) == 0;
+}
+
+}  // namespace pairk
+
+using namespace pairk;
+
+extern "C" {
+
+pair_status pair_coeffs(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                        const float *rho, float scale, uint32_t flags,
+                        float *a, uint8_t *active, int32_t *edges,
+                        int32_t *contrast_edges, int32_t *dev_err,
+                        pair_stream_t stream) {
+  reset_launches();
+  if (B < 1 || G < 2 || G > PAIR_MAX_G || !r || !J || !rho || !a ||
+      (flags & ~PAIR_CENTER) != 0)
+    return PAIR_ERR_INVALID_ARG;
+  const pair_status dv = check_device();
+  if (dv != PAIR_OK) return dv;
+  return launch_coeffs(B, G, r, J, rho, scale, flags, a, active, edges,
+                       contrast_edges, dev_err,
+                       reinterpret_cast<cudaStream_t>(stream));
+}
+
+pair_status pair_estimate_dense(int32_t B, int32_t G, int32_t D,
+                                const float *r, const uint8_t *J,
+                                const float *rho, const float *S, float scale,
+                                float *g, float *a, int32_t *dev_err,
+                                pair_stream_t stream) {
+  reset_launches();
+  if (B < 1 || G < 2 || G > PAIR_MAX_G || D < 1 || !r || !J || !rho || !S ||
+      !g)
+    return PAIR_ERR_INVALID_ARG;
+  const pair_status dv = check_device();
+  if (dv != PAIR_OK) return dv;
+  return launch_estimate_dense(B, G, D, r, J, rho, S, scale, g, a, dev_err,
+                               reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t pair_grad_workspace_size(int64_t T, int32_t d, int32_t V, int32_t R,
+                                pair_dtype dt) {
+  if (T < 1 || R < 1 || V < 1 || d < 16 || (d % 16) != 0) return 0;
+  if (dt != PAIR_F32 && dt != PAIR_BF16) return 0;
+  if (dt == PAIR_BF16 && (d % 64) != 0) return 0;
+  if (T > (int64_t)INT32_MAX - 1024) return 0;
+  return grad_workspace_bytes(T, d, V, R, dt, nullptr, nullptr);
+}
+
+pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
+                      const void *H, const void *W, const int32_t *y,
+                      const uint8_t *mask, const int32_t *cu_seqlens,
+                      int32_t R, const float *a, float *dH, float *dW,
+                      double *Jobj, float *logp_seq, void *ws,
+                      size_t ws_bytes, int32_t *dev_err,
+                      pair_stream_t stream) {
+  reset_launches();
+  if (!H || !W || !y || !mask || !cu_seqlens || !a || !dH || !dW || !Jobj)
+    return PAIR_ERR_INVALID_ARG;
+  if (!aligned16(H) || !aligned16(W) || !aligned16(dH) || !aligned16(dW))
+    return PAIR_ERR_INVALID_ARG;
+  const size_t need = pair_grad_workspace_size(T, d, V, R, dt);
+  if (need == 0) return (dt == PAIR_BF16 && d % 64 != 0 && d % 16 == 0)
+                            ? PAIR_ERR_UNSUPPORTED
+                            : PAIR_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return PAIR_ERR_WORKSPACE;
+  const pair_status dv = check_device();
+  if (dv != PAIR_OK) return dv;
+
+  GradWorkspace w;
+  grad_workspace_bytes(T, d, V, R, dt, &w, ws);
+  GradArgs g{T, d, V, R, dt, H, W, y, mask, cu_seqlens, a,
+             dH, dW, Jobj, logp_seq, dev_err};
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  pair_status st = grad_prepare(g, w, s);
+  if (st != PAIR_OK) return st;
+  if (dt == PAIR_BF16) {
+    st = grad_head_tc(g, w, s);
+    if (st != PAIR_OK) return st;
+    st = grad_onehot(g, w, s);
+  } else {
+    st = grad_head_simt(g, w, s);
+  }
+  if (st != PAIR_OK) return st;
+  return grad_finalize(g, w, s);
+}
+
+pair_status pair_status_sync(pair_stream_t stream, int32_t *dev_err) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return PAIR_ERR_CUDA;
+  if (!dev_err) return PAIR_OK;
+  int32_t h = 0;
+  if (cudaMemcpy(&h, dev_err, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return PAIR_ERR_CUDA;
+  if (h != 0 && cudaMemset(dev_err, 0, sizeof(h)) != cudaSuccess)
+    return PAIR_ERR_CUDA;
+  if (h & PAIR_DEV_ERR_TIMEOUT) return PAIR_ERR_DEVICE_TIMEOUT;
+  if (h & PAIR_DEV_ERR_NONPOSITIVE_INCLUSION) return PAIR_ERR_NONPOSITIVE_INCLUSION;
+  if (h & PAIR_DEV_ERR_TARGET_RANGE) return PAIR_ERR_TARGET_RANGE;
+  return PAIR_OK;
+}
+
+const char *pair_status_string(pair_status st) {
+  switch (st) {
+    case PAIR_OK: return "ok";
+    case PAIR_ERR_INVALID_ARG: return "invalid argument";
+    case PAIR_ERR_UNSUPPORTED: return "unsupported device or shape";
+    case PAIR_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case PAIR_ERR_NONPOSITIVE_INCLUSION:
+      return "joint inclusion probability <= 0 or NaN on a completed edge";
+    case PAIR_ERR_TARGET_RANGE: return "target id outside [0, V) at a mask=1 token";
+    case PAIR_ERR_CUDA: return "CUDA runtime error";
+    case PAIR_ERR_DEVICE_TIMEOUT: return "device pipeline wait timed out";
+  }
+  return "unknown status";
+}
+
+int32_t pair_last_launch_count(void) { return g_launches; }
+
+}  // extern "C"

@@ -1,0 +1,313 @@
+// Per-group coefficient collapse and the dense estimator.
+//
+// Sec. 4.5, Eq. (pair-advantage): a_i = scale * 1/2 sum_{j != i} J_iJ_j
+// (r_i - r_j) / rho_ij, and Eq. (pair-ht) collapsed to g = sum_i a_i s_i.
+// Algorithm 1 enumerates the observed induced edges; here every edge (i<j)
+// is read once from the upper triangle of rho and its antisymmetric term is
+// placed at (i, j) and (j, i) of a shared-memory matrix, after which each
+// vertex sums its row with a fixed binary tree (deterministic, error
+// O(log2 G) ulp of sum_j |term_j|).
+//
+// Memory: the upper triangle is read by "row pairs": rows k and GP-1-k
+// together hold exactly GP-1 upper entries, so a block of >= GP threads reads
+// them as two contiguous runs per step, fully unrolled to keep every load
+// of the group in flight at once.
+#include "pair_common.cuh"
+
+namespace pairk {
+namespace {
+
+template <int GP>
+struct GroupSmem {
+  float T[GP][GP + 1];  // antisymmetric edge terms; +1 pad: conflict-free rows
+  float r[GP];
+  float a[GP];
+  int8_t J[GP];
+  int red_i[32];
+  float red_f[32];
+};
+
+// Deterministic block sum of one int per thread (all threads call).
+__device__ int block_sum_int(int v, int *red) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[w] = v;
+  __syncthreads();
+  int s = 0;
+  for (int k = 0; k < nw; ++k) s += red[k];
+  return s;
+}
+
+// Deterministic block sum of one float per thread in a fixed tree order.
+__device__ float block_sum_float(float v, float *red) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[w] = v;
+  __syncthreads();
+  float s = 0.f;
+  for (int k = 0; k < nw; ++k) s += red[k];
+  return s;
+}
+
+// Computes the coefficients of group `b` into sm.a[0..G) (scale applied).
+// Requires blockDim.x >= GP. Returns (in thread 0) K and the contrast count.
+template <int GP>
+__device__ void group_coeffs(GroupSmem<GP> &sm, int b, int G, const float *r,
+                             const uint8_t *J, const float *rho, float scale,
+                             bool center, int32_t *dev_err, int &K_out,
+                             int &contrast_out, uint8_t &active_out) {
+  const int tid = threadIdx.x;
+  const size_t gbase = (size_t)b * G;
+  if (tid < GP) {
+    const bool in = tid < G;
+    sm.r[tid] = in ? r[gbase + tid] : 0.f;
+    sm.J[tid] = in ? (J[gbase + tid] != 0) : 0;
+    sm.T[tid][tid] = 0.f;
+  }
+  __syncthreads();
+
+  const float *rho_g = rho + (size_t)b * G * G;
+  int my_contrast = 0, bad = 0;
+  if (tid < GP - 1) {
+    // Load phase: every upper entry this thread owns, all loads in flight.
+    float v[GP / 2];
+#pragma unroll
+    for (int k = 0; k < GP / 2; ++k) {
+      const int n1 = GP - 1 - k;  // entries of row k
+      int i, j;
+      if (tid < n1) { i = k; j = k + 1 + tid; }
+      else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
+      const bool live = (j < G) && sm.J[i] && sm.J[j];
+      v[k] = live ? __ldg(rho_g + (size_t)i * G + j) : 1.f;
+    }
+#pragma unroll
+    for (int k = 0; k < GP / 2; ++k) {
+      const int n1 = GP - 1 - k;
+      int i, j;
+      if (tid < n1) { i = k; j = k + 1 + tid; }
+      else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
+      const bool live = (j < G) && sm.J[i] && sm.J[j];
+      float t = 0.f;
+      if (live) {
+        const float rij = v[k];
+        if (!(rij > 0.f)) {
+          bad = 1;
+        } else {
+          const float dr = sm.r[i] - sm.r[j];
+          t = __fdiv_rn(dr, rij);
+          my_contrast += (sm.r[i] != sm.r[j]);
+        }
+      }
+      sm.T[i][j] = t;
+      sm.T[j][i] = -t;
+    }
+  }
+  if (bad) flag_error(dev_err, PAIR_DEV_ERR_NONPOSITIVE_INCLUSION);
+  __syncthreads();
+
+  // Row sums by a fixed pairwise tree.
+  float a = 0.f;
+  uint8_t act = 0;
+  if (tid < GP) {
+    float x[GP];
+    bool nz = false;
+#pragma unroll
+    for (int k = 0; k < GP; ++k) {
+      x[k] = sm.T[tid][k];
+      nz |= (x[k] != 0.f);
+    }
+#pragma unroll
+    for (int s = GP / 2; s >= 1; s >>= 1) {
+#pragma unroll
+      for (int k = 0; k < s; ++k) x[k] += x[k + s];
+    }
+    a = (x[0] == 0.f) ? 0.f : 0.5f * x[0];
+    act = (tid < G && sm.J[tid] && nz) ? 1 : 0;
+  }
+  const int K = block_sum_int((tid < GP) ? (int)sm.J[tid] : 0, sm.red_i);
+  const int C = block_sum_int(my_contrast, sm.red_i);
+  if (center && K > 0) {
+    // App. C: centre across the observed endpoints.
+    const float s = block_sum_float((tid < GP && sm.J[tid]) ? a : 0.f, sm.red_f);
+    const float mean = s / (float)K;
+    if (tid < GP && sm.J[tid]) a -= mean;
+  }
+  if (tid < GP) sm.a[tid] = (tid < G) ? a * scale : 0.f;
+  __syncthreads();
+  K_out = K;
+  contrast_out = C;
+  active_out = act;
+}
+
+template <int GP>
+__global__ void __launch_bounds__(128) coeffs_kernel(
+    int B, int G, const float *__restrict__ r, const uint8_t *__restrict__ J,
+    const float *__restrict__ rho, float scale, int center,
+    float *__restrict__ a, uint8_t *__restrict__ active,
+    int32_t *__restrict__ edges, int32_t *__restrict__ contrast,
+    int32_t *dev_err) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  GroupSmem<GP> &sm = *reinterpret_cast<GroupSmem<GP> *>(smem_raw);
+  const int b = blockIdx.x;
+  int K, C;
+  uint8_t act;
+  group_coeffs<GP>(sm, b, G, r, J, rho, scale, center != 0, dev_err, K, C, act);
+  const int tid = threadIdx.x;
+  if (tid < G) {
+    a[(size_t)b * G + tid] = sm.a[tid];
+    if (active) active[(size_t)b * G + tid] = act;
+  }
+  if (tid == 0) {
+    if (edges) edges[b] = K * (K - 1) / 2;
+    if (contrast) contrast[b] = C;
+  }
+}
+
+// One block per group: coefficients, then g_b = sum_i a_i s_{b,i} streamed
+// over D with 16-byte loads; rows with a_i == 0 are never read.
+template <int GP>
+__global__ void __launch_bounds__(256) dense_kernel(
+    int B, int G, int D, const float *__restrict__ r,
+    const uint8_t *__restrict__ J, const float *__restrict__ rho,
+    const float *__restrict__ S, float scale, float *__restrict__ g,
+    float *__restrict__ a_out, int32_t *dev_err) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  GroupSmem<GP> &sm = *reinterpret_cast<GroupSmem<GP> *>(smem_raw);
+  __shared__ int rows[GP];
+  __shared__ float coef[GP];
+  __shared__ int n_rows;
+  const int b = blockIdx.x, tid = threadIdx.x;
+  int K, C;
+  uint8_t act;
+  group_coeffs<GP>(sm, b, G, r, J, rho, scale, false, dev_err, K, C, act);
+  if (a_out && tid < G) a_out[(size_t)b * G + tid] = sm.a[tid];
+  if (tid == 0) {
+    int n = 0;
+    for (int i = 0; i < G; ++i)
+      if (sm.a[i] != 0.f) { rows[n] = i; coef[n] = sm.a[i]; ++n; }
+    n_rows = n;
+  }
+  __syncthreads();
+  const int n = n_rows;
+  const float *Sb = S + (size_t)b * G * D;
+  float *gb = g + (size_t)b * D;
+  const bool vec = ((D & 3) == 0) && ((reinterpret_cast<uintptr_t>(S) & 15) == 0) &&
+                   ((reinterpret_cast<uintptr_t>(g) & 15) == 0);
+  if (vec) {
+    const int D4 = D >> 2;
+    for (int c0 = tid; c0 < D4; c0 += 4 * blockDim.x) {
+      float4 acc[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      int q = 0;
+      for (; q + 1 < n; q += 2) {
+        float4 x0[4], x1[4];
+        const float4 *p0 = reinterpret_cast<const float4 *>(Sb + (size_t)rows[q] * D);
+        const float4 *p1 = reinterpret_cast<const float4 *>(Sb + (size_t)rows[q + 1] * D);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int c = c0 + u * blockDim.x;
+          x0[u] = c < D4 ? __ldcs(p0 + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+          x1[u] = c < D4 ? __ldcs(p1 + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        const float w0 = coef[q], w1 = coef[q + 1];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          acc[u].x = fmaf(w0, x0[u].x, acc[u].x); acc[u].y = fmaf(w0, x0[u].y, acc[u].y);
+          acc[u].z = fmaf(w0, x0[u].z, acc[u].z); acc[u].w = fmaf(w0, x0[u].w, acc[u].w);
+          acc[u].x = fmaf(w1, x1[u].x, acc[u].x); acc[u].y = fmaf(w1, x1[u].y, acc[u].y);
+          acc[u].z = fmaf(w1, x1[u].z, acc[u].z); acc[u].w = fmaf(w1, x1[u].w, acc[u].w);
+        }
+      }
+      if (q < n) {
+        const float4 *p0 = reinterpret_cast<const float4 *>(Sb + (size_t)rows[q] * D);
+        const float w0 = coef[q];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int c = c0 + u * blockDim.x;
+          if (c < D4) {
+            const float4 x = __ldcs(p0 + c);
+            acc[u].x = fmaf(w0, x.x, acc[u].x); acc[u].y = fmaf(w0, x.y, acc[u].y);
+            acc[u].z = fmaf(w0, x.z, acc[u].z); acc[u].w = fmaf(w0, x.w, acc[u].w);
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = c0 + u * blockDim.x;
+        if (c < D4) __stcs(reinterpret_cast<float4 *>(gb) + c, acc[u]);
+      }
+    }
+  } else {
+    for (int c = tid; c < D; c += blockDim.x) {
+      float acc = 0.f;
+      for (int q = 0; q < n; ++q) acc = fmaf(coef[q], Sb[(size_t)rows[q] * D + c], acc);
+      gb[c] = acc;
+    }
+  }
+}
+
+template <int GP>
+pair_status launch_coeffs_gp(int32_t B, int32_t G, const float *r,
+                             const uint8_t *J, const float *rho, float scale,
+                             uint32_t flags, float *a, uint8_t *active,
+                             int32_t *edges, int32_t *contrast,
+                             int32_t *dev_err, cudaStream_t s) {
+  const size_t smem = sizeof(GroupSmem<GP>);
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(coeffs_kernel<GP>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)smem));
+  coeffs_kernel<GP><<<B, GP, smem, s>>>(B, G, r, J, rho, scale,
+                                        (flags & PAIR_CENTER) ? 1 : 0, a,
+                                        active, edges, contrast, dev_err);
+  PAIR_LAUNCH_CHECK();
+  return PAIR_OK;
+}
+
+template <int GP>
+pair_status launch_dense_gp(int32_t B, int32_t G, int32_t D, const float *r,
+                            const uint8_t *J, const float *rho, const float *S,
+                            float scale, float *g, float *a, int32_t *dev_err,
+                            cudaStream_t s) {
+  const size_t smem = sizeof(GroupSmem<GP>);
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(dense_kernel<GP>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)smem));
+  dense_kernel<GP><<<B, 256, smem, s>>>(B, G, D, r, J, rho, S, scale, g, a,
+                                        dev_err);
+  PAIR_LAUNCH_CHECK();
+  return PAIR_OK;
+}
+
+}  // namespace
+
+pair_status launch_coeffs(int32_t B, int32_t G, const float *r,
+                          const uint8_t *J, const float *rho, float scale,
+                          uint32_t flags, float *a, uint8_t *active,
+                          int32_t *edges, int32_t *contrast, int32_t *dev_err,
+                          cudaStream_t s) {
+  if (G <= 32)
+    return launch_coeffs_gp<32>(B, G, r, J, rho, scale, flags, a, active,
+                                edges, contrast, dev_err, s);
+  if (G <= 64)
+    return launch_coeffs_gp<64>(B, G, r, J, rho, scale, flags, a, active,
+                                edges, contrast, dev_err, s);
+  return launch_coeffs_gp<128>(B, G, r, J, rho, scale, flags, a, active,
+                               edges, contrast, dev_err, s);
+}
+
+pair_status launch_estimate_dense(int32_t B, int32_t G, int32_t D,
+                                  const float *r, const uint8_t *J,
+                                  const float *rho, const float *S,
+                                  float scale, float *g, float *a,
+                                  int32_t *dev_err, cudaStream_t s) {
+  if (G <= 32)
+    return launch_dense_gp<32>(B, G, D, r, J, rho, S, scale, g, a, dev_err, s);
+  if (G <= 64)
+    return launch_dense_gp<64>(B, G, D, r, J, rho, S, scale, g, a, dev_err, s);
+  return launch_dense_gp<128>(B, G, D, r, J, rho, S, scale, g, a, dev_err, s);
+}
+
+}  // namespace pairk

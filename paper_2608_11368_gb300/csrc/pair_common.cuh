@@ -1,0 +1,97 @@
+// Shared definitions for the Pair estimator CUDA library (sm_103a).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "pair.h"
+
+namespace pairk {
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+// Counts kernel launches of the current entry-point call (per host thread).
+void note_launch();
+void reset_launches();
+
+__device__ __forceinline__ void flag_error(int32_t *err, int bit) {
+  if (err) atomicOr(err, bit);
+}
+
+__host__ __device__ __forceinline__ int64_t ceil_div(int64_t a, int64_t b) {
+  return (a + b - 1) / b;
+}
+
+// Group coefficient kernels (pair_coeffs.cu).
+pair_status launch_coeffs(int32_t B, int32_t G, const float *r,
+                          const uint8_t *J, const float *rho, float scale,
+                          uint32_t flags, float *a, uint8_t *active,
+                          int32_t *edges, int32_t *contrast, int32_t *dev_err,
+                          cudaStream_t s);
+pair_status launch_estimate_dense(int32_t B, int32_t G, int32_t D,
+                                  const float *r, const uint8_t *J,
+                                  const float *rho, const float *S,
+                                  float scale, float *g, float *a,
+                                  int32_t *dev_err, cudaStream_t s);
+
+// pair_grad pieces (pair_grad_prep.cu, pair_grad_simt.cu, pair_grad_tc.cu).
+struct GradWorkspace {
+  int32_t *counters;   // [0] = number of active tokens T_eff
+  int32_t *seg_cnt;    // [R] active tokens per rollout
+  int32_t *seg_off;    // [R+1] exclusive prefix of seg_cnt
+  int32_t *tok_idx;    // [T] packed position of each active token
+  int32_t *tok_y;      // [T] its target id
+  float *tok_c;        // [T] its coefficient c_t = a_seg(t)
+  float *lse;          // [Tpad] log-sum-exp of the active token's logits
+  float *zy;           // [Tpad] target logit
+  float2 *part;        // [nsplit][Tpad] partial (max, sum-exp) per split
+  double *seg_logp;    // [R] per-rollout sum of logp (fp64)
+  void *Hc;            // [Tpad][d] compacted hidden rows (dt), zero tail
+  int64_t Tpad;
+  int nsplit;
+};
+
+size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
+                            pair_dtype dt, GradWorkspace *out, void *base);
+
+struct GradArgs {
+  int64_t T;
+  int32_t d, V, R;
+  pair_dtype dt;
+  const void *H, *W;
+  const int32_t *y;
+  const uint8_t *mask;
+  const int32_t *cu;
+  const float *a;
+  float *dH, *dW;
+  double *Jobj;
+  float *logp_seq;
+  int32_t *dev_err;
+};
+
+pair_status grad_prepare(const GradArgs &g, const GradWorkspace &w,
+                         cudaStream_t s);
+pair_status grad_finalize(const GradArgs &g, const GradWorkspace &w,
+                          cudaStream_t s);
+pair_status grad_head_simt(const GradArgs &g, const GradWorkspace &w,
+                           cudaStream_t s);
+pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
+                         cudaStream_t s);
+// Exact one-hot parts (added after the tensor-core softmax parts).
+pair_status grad_onehot(const GradArgs &g, const GradWorkspace &w,
+                        cudaStream_t s);
+
+}  // namespace pairk
+
+#define PAIR_CUDA_TRY(expr)                                   \
+  do {                                                        \
+    cudaError_t e_ = (expr);                                  \
+    if (e_ != cudaSuccess) return PAIR_ERR_CUDA;              \
+  } while (0)
+
+#define PAIR_LAUNCH_CHECK()                                   \
+  do {                                                        \
+    ::pairk::note_launch();                                   \
+    cudaError_t e_ = cudaGetLastError();                      \
+    if (e_ != cudaSuccess) return PAIR_ERR_CUDA;              \
+  } while (0)

@@ -1,0 +1,357 @@
+// pair_grad bookkeeping kernels: active-token compaction, per-rollout and
+// total objective, exact one-hot gradient parts, workspace layout.
+//
+// The objective of Sec. 4.5 is sum_i a_i log pi(o_i | q) with log pi a sum
+// over response tokens; rollouts with a_i == 0 contribute nothing and are
+// removed before any head arithmetic. The surviving tokens are packed in
+// their original order (rollout by rollout), so every per-rollout sum below
+// runs over a contiguous range in a fixed order (bit-reproducible).
+#include <cuda_bf16.h>
+
+#include "pair_common.cuh"
+
+namespace pairk {
+namespace {
+
+constexpr int kNSplit = 16;  // vocabulary splits of the log-sum-exp pass
+
+__device__ __forceinline__ bool coef_nonzero(float a) {
+  return (__float_as_uint(a) & 0x7fffffffu) != 0u;
+}
+
+__device__ __forceinline__ int clamp_i(int v, int lo, int hi) {
+  return v < lo ? lo : (v > hi ? hi : v);
+}
+
+// Counts the active tokens of each rollout; validates every mask=1 target.
+__global__ void seg_count_kernel(int R, int T, int V, const int32_t *cu,
+                                 const uint8_t *mask, const int32_t *y,
+                                 const float *a, int32_t *seg_cnt,
+                                 int32_t *dev_err) {
+  const int i = blockIdx.x;
+  const int beg = clamp_i(cu[i], 0, T), end = clamp_i(cu[i + 1], beg, T);
+  const bool on = coef_nonzero(a[i]);
+  int n = 0, bad = 0;
+  for (int t = beg + threadIdx.x; t < end; t += blockDim.x) {
+    if (mask[t]) {
+      ++n;
+      const int yt = y[t];
+      bad |= (yt < 0 || yt >= V);
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) n += __shfl_xor_sync(0xffffffffu, n, o);
+  __shared__ int red[32];
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = n;
+  if (bad) flag_error(dev_err, PAIR_DEV_ERR_TARGET_RANGE);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int s = 0;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) s += red[k];
+    seg_cnt[i] = on ? s : 0;
+  }
+}
+
+// Exclusive prefix over rollouts (one block, sequential chunks of 1024).
+__global__ void seg_scan_kernel(int R, const int32_t *seg_cnt, int32_t *seg_off,
+                                int32_t *counters) {
+  __shared__ int buf[1024];
+  __shared__ int carry;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int base = 0; base < R; base += 1024) {
+    const int i = base + threadIdx.x;
+    const int v = i < R ? seg_cnt[i] : 0;
+    buf[threadIdx.x] = v;
+    __syncthreads();
+    for (int o = 1; o < 1024; o <<= 1) {
+      const int add = threadIdx.x >= o ? buf[threadIdx.x - o] : 0;
+      __syncthreads();
+      buf[threadIdx.x] += add;
+      __syncthreads();
+    }
+    if (i < R) seg_off[i] = carry + buf[threadIdx.x] - v;
+    __syncthreads();
+    if (threadIdx.x == 1023) carry += buf[1023];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    seg_off[R] = carry;
+    counters[0] = carry;
+  }
+}
+
+// In-order compaction of each active rollout's mask=1 tokens.
+__global__ void gather_kernel(int R, int T, const int32_t *cu,
+                              const uint8_t *mask, const int32_t *y,
+                              const float *a, const int32_t *seg_off,
+                              int32_t *tok_idx, int32_t *tok_y, float *tok_c) {
+  const int i = blockIdx.x;
+  if (!coef_nonzero(a[i])) return;
+  const int beg = clamp_i(cu[i], 0, T), end = clamp_i(cu[i + 1], beg, T);
+  const float c = a[i];
+  __shared__ int wsum[32];
+  __shared__ int carry;
+  if (threadIdx.x == 0) carry = seg_off[i];
+  __syncthreads();
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int nw = blockDim.x >> 5;
+  for (int base = beg; base < end; base += blockDim.x) {
+    const int t = base + threadIdx.x;
+    const int f = (t < end && mask[t]) ? 1 : 0;
+    const unsigned bal = __ballot_sync(0xffffffffu, f);
+    const int rank_w = __popc(bal & ((1u << lane) - 1u));
+    if (lane == 0) wsum[w] = __popc(bal);
+    __syncthreads();
+    int before = 0, total = 0;
+    for (int k = 0; k < nw; ++k) {
+      before += (k < w) ? wsum[k] : 0;
+      total += wsum[k];
+    }
+    if (f) {
+      const int p = carry + before + rank_w;
+      tok_idx[p] = t;
+      tok_y[p] = y[t];
+      tok_c[p] = c;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) carry += total;
+    __syncthreads();
+  }
+}
+
+// Hc[p] = H[tok_idx[p]] for p < T_eff; zero rows up to the next multiple of
+// 128 (the token-tile height), so tail tiles carry finite zeros.
+template <typename Tin>
+__global__ void copy_rows_kernel(int64_t Tpad, int d, const int32_t *counters,
+                                 const int32_t *tok_idx, const Tin *H, Tin *Hc) {
+  const int Teff = counters[0];
+  const int64_t Tz = ((int64_t)Teff + 127) / 128 * 128;
+  const int vec = 16 / (int)sizeof(Tin);
+  const int dv = d / vec;
+  for (int64_t p = blockIdx.x; p < Tz && p < Tpad; p += gridDim.x) {
+    uint4 *dst = reinterpret_cast<uint4 *>(Hc + p * d);
+    if (p < Teff) {
+      const uint4 *src = reinterpret_cast<const uint4 *>(H + (int64_t)tok_idx[p] * d);
+      for (int k = threadIdx.x; k < dv; k += blockDim.x) dst[k] = src[k];
+    } else {
+      for (int k = threadIdx.x; k < dv; k += blockDim.x) dst[k] = make_uint4(0, 0, 0, 0);
+    }
+  }
+}
+
+// Zero the dH rows of tokens outside the objective (mask = 0 or a = 0).
+__global__ void zero_inactive_rows_kernel(int64_t T, int d, int R,
+                                          const int32_t *cu,
+                                          const uint8_t *mask, const float *a,
+                                          float *dH) {
+  for (int64_t t = blockIdx.x; t < T; t += gridDim.x) {
+    // rollout of t: last i with cu[i] <= t
+    int lo = 0, hi = R - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (cu[mid] <= t) lo = mid; else hi = mid - 1;
+    }
+    const bool live = mask[t] && coef_nonzero(a[lo]) && cu[lo] <= t && t < cu[lo + 1];
+    if (live) continue;
+    float4 *row = reinterpret_cast<float4 *>(dH + t * d);
+    if ((d & 3) == 0) {
+      for (int k = threadIdx.x; k < d / 4; k += blockDim.x)
+        row[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    } else {
+      for (int k = threadIdx.x; k < d; k += blockDim.x) dH[t * d + k] = 0.f;
+    }
+  }
+}
+
+// Per-rollout sum of logp_t = zy - lse over the rollout's compacted range
+// (fp64, fixed tree order).
+__global__ void seg_logp_kernel(int R, const int32_t *seg_off, const float *zy,
+                                const float *lse, double *seg_logp) {
+  const int i = blockIdx.x;
+  const int beg = seg_off[i], end = seg_off[i + 1];
+  double s = 0.0;
+  for (int p = beg + threadIdx.x; p < end; p += blockDim.x)
+    s += (double)zy[p] - (double)lse[p];
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  __shared__ double red[32];
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) t += red[k];
+    seg_logp[i] = t;
+  }
+}
+
+// Jobj = sum_i a_i * logp_seq_i (fp64, fixed order); logp_seq out.
+__global__ void objective_kernel(int R, const float *a, const double *seg_logp,
+                                 double *Jobj, float *logp_seq) {
+  __shared__ double red[32];
+  double s = 0.0;
+  for (int i = threadIdx.x; i < R; i += blockDim.x) {
+    const bool on = coef_nonzero(a[i]);
+    const double lp = on ? seg_logp[i] : 0.0;
+    if (logp_seq) logp_seq[i] = (float)lp;
+    s += on ? (double)a[i] * lp : 0.0;
+  }
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) t += red[k];
+    *Jobj = t;
+  }
+}
+
+// dH_t += c_t W[y_t]  (the one-hot part of dJ/dh_t, exact in fp32).
+template <typename Tin>
+__global__ void onehot_dh_kernel(int d, const int32_t *counters,
+                                 const int32_t *tok_idx, const int32_t *tok_y,
+                                 const float *tok_c, const Tin *W, float *dH) {
+  const int Teff = counters[0];
+  for (int p = blockIdx.x; p < Teff; p += gridDim.x) {
+    const float c = tok_c[p];
+    const Tin *w = W + (int64_t)tok_y[p] * d;
+    float *row = dH + (int64_t)tok_idx[p] * d;
+    for (int k = threadIdx.x; k < d; k += blockDim.x)
+      row[k] = fmaf(c, (float)w[k], row[k]);
+  }
+}
+
+// dW_v += sum_{t: y_t = v} c_t h_t (the one-hot part of dJ/dW_v), exact in
+// fp32, tokens added in their packed order. One warp owns a bucket of
+// vocabulary rows and scans the compacted targets for matches.
+template <typename Tin>
+__global__ void onehot_dw_kernel(int d, int V, int bucket,
+                                 const int32_t *counters, const int32_t *tok_y,
+                                 const float *tok_c, const Tin *Hc, float *dW) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  const int v0 = warp * bucket;
+  if (v0 >= V) return;
+  const int v1 = min(V, v0 + bucket);
+  const int Teff = counters[0];
+  for (int base = 0; base < Teff; base += 32) {
+    const int p = base + lane;
+    const int yt = p < Teff ? tok_y[p] : -1;
+    unsigned hit = __ballot_sync(0xffffffffu, yt >= v0 && yt < v1);
+    while (hit) {
+      const int src = __ffs(hit) - 1;
+      hit &= hit - 1;
+      const int q = base + src;
+      const int v = __shfl_sync(0xffffffffu, yt, src);
+      const float c = tok_c[q];
+      const Tin *h = Hc + (int64_t)q * d;
+      float *row = dW + (int64_t)v * d;
+      for (int k = lane; k < d; k += 32) row[k] = fmaf(c, (float)h[k], row[k]);
+    }
+  }
+}
+
+}  // namespace
+
+size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
+                            pair_dtype dt, GradWorkspace *out, void *base) {
+  const int64_t Tpad = (T + 127) / 128 * 128 + 128;
+  const size_t esz = dt == PAIR_BF16 ? 2 : 4;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += (bytes + 255) / 256 * 256;
+    return o;
+  };
+  const size_t o_cnt = take(64 * sizeof(int32_t));
+  const size_t o_segc = take((size_t)R * 4);
+  const size_t o_sego = take((size_t)(R + 1) * 4);
+  const size_t o_idx = take((size_t)Tpad * 4);
+  const size_t o_y = take((size_t)Tpad * 4);
+  const size_t o_c = take((size_t)Tpad * 4);
+  const size_t o_lse = take((size_t)Tpad * 4);
+  const size_t o_zy = take((size_t)Tpad * 4);
+  const size_t o_part = take((size_t)kNSplit * Tpad * sizeof(float2));
+  const size_t o_segl = take((size_t)R * 8);
+  const size_t o_hc = take((size_t)Tpad * d * esz);
+  if (out) {
+    char *b = static_cast<char *>(base);
+    out->counters = reinterpret_cast<int32_t *>(b + o_cnt);
+    out->seg_cnt = reinterpret_cast<int32_t *>(b + o_segc);
+    out->seg_off = reinterpret_cast<int32_t *>(b + o_sego);
+    out->tok_idx = reinterpret_cast<int32_t *>(b + o_idx);
+    out->tok_y = reinterpret_cast<int32_t *>(b + o_y);
+    out->tok_c = reinterpret_cast<float *>(b + o_c);
+    out->lse = reinterpret_cast<float *>(b + o_lse);
+    out->zy = reinterpret_cast<float *>(b + o_zy);
+    out->part = reinterpret_cast<float2 *>(b + o_part);
+    out->seg_logp = reinterpret_cast<double *>(b + o_segl);
+    out->Hc = b + o_hc;
+    out->Tpad = Tpad;
+    out->nsplit = kNSplit;
+  }
+  (void)V;
+  return off;
+}
+
+pair_status grad_prepare(const GradArgs &g, const GradWorkspace &w,
+                         cudaStream_t s) {
+  seg_count_kernel<<<g.R, 256, 0, s>>>(g.R, (int)g.T, g.V, g.cu, g.mask, g.y,
+                                       g.a, w.seg_cnt, g.dev_err);
+  PAIR_LAUNCH_CHECK();
+  seg_scan_kernel<<<1, 1024, 0, s>>>(g.R, w.seg_cnt, w.seg_off, w.counters);
+  PAIR_LAUNCH_CHECK();
+  gather_kernel<<<g.R, 256, 0, s>>>(g.R, (int)g.T, g.cu, g.mask, g.y, g.a,
+                                    w.seg_off, w.tok_idx, w.tok_y, w.tok_c);
+  PAIR_LAUNCH_CHECK();
+  const int rows_grid = 152 * 16;
+  if (g.dt == PAIR_BF16)
+    copy_rows_kernel<uint16_t><<<rows_grid, 128, 0, s>>>(
+        w.Tpad, g.d, w.counters, w.tok_idx,
+        static_cast<const uint16_t *>(g.H), static_cast<uint16_t *>(w.Hc));
+  else
+    copy_rows_kernel<float><<<rows_grid, 128, 0, s>>>(
+        w.Tpad, g.d, w.counters, w.tok_idx, static_cast<const float *>(g.H),
+        static_cast<float *>(w.Hc));
+  PAIR_LAUNCH_CHECK();
+  zero_inactive_rows_kernel<<<rows_grid, 128, 0, s>>>(g.T, g.d, g.R, g.cu,
+                                                      g.mask, g.a, g.dH);
+  PAIR_LAUNCH_CHECK();
+  return PAIR_OK;
+}
+
+pair_status grad_finalize(const GradArgs &g, const GradWorkspace &w,
+                          cudaStream_t s) {
+  seg_logp_kernel<<<g.R, 256, 0, s>>>(g.R, w.seg_off, w.zy, w.lse, w.seg_logp);
+  PAIR_LAUNCH_CHECK();
+  objective_kernel<<<1, 1024, 0, s>>>(g.R, g.a, w.seg_logp, g.Jobj,
+                                      g.logp_seq);
+  PAIR_LAUNCH_CHECK();
+  return PAIR_OK;
+}
+
+pair_status grad_onehot(const GradArgs &g, const GradWorkspace &w,
+                        cudaStream_t s) {
+  const int bucket = 128;
+  const int warps = (int)ceil_div(g.V, bucket);
+  if (g.dt == PAIR_BF16) {
+    const __nv_bfloat16 *W = static_cast<const __nv_bfloat16 *>(g.W);
+    onehot_dh_kernel<__nv_bfloat16><<<152 * 16, 256, 0, s>>>(
+        g.d, w.counters, w.tok_idx, w.tok_y, w.tok_c, W, g.dH);
+    PAIR_LAUNCH_CHECK();
+    onehot_dw_kernel<__nv_bfloat16><<<(int)ceil_div(warps, 8), 256, 0, s>>>(
+        g.d, g.V, bucket, w.counters, w.tok_y, w.tok_c,
+        static_cast<const __nv_bfloat16 *>(w.Hc), g.dW);
+    PAIR_LAUNCH_CHECK();
+  } else {
+    onehot_dh_kernel<float><<<152 * 16, 256, 0, s>>>(
+        g.d, w.counters, w.tok_idx, w.tok_y, w.tok_c,
+        static_cast<const float *>(g.W), g.dH);
+    PAIR_LAUNCH_CHECK();
+    onehot_dw_kernel<float><<<(int)ceil_div(warps, 8), 256, 0, s>>>(
+        g.d, g.V, bucket, w.counters, w.tok_y, w.tok_c,
+        static_cast<const float *>(w.Hc), g.dW);
+    PAIR_LAUNCH_CHECK();
+  }
+  return PAIR_OK;
+}
+
+}  // namespace pairk

@@ -1,0 +1,613 @@
+// bf16 LM-head path of pair_grad on the 5th-generation tensor cores
+// (tcgen05 + TMEM + TMA, sm_103a).
+//
+// Objective (Sec. 4.5): J = sum_t c_t logp_t over compacted active tokens,
+// logp_t = z_{t,y_t} - lse_t, z = W h. Its gradients split into an exact
+// one-hot part (added in fp32 by grad_onehot) and a softmax part that is a
+// pair of dense contractions through the logit-gradient tile
+//     Gs_tv = -c_t exp(z_tv - lse_t)      (bf16 on chip, never in HBM):
+//     dH_t += sum_v Gs_tv W_v,     dW_v += sum_t Gs_tv h_t.
+//
+// Kernels (all persistent, one 192-thread CTA per SM, warp-specialised:
+// warp 0 = TMA producer, warp 1 = TMEM owner + single-thread MMA issuer,
+// warps 2..5 = epilogue, one TMEM lane / tile row per thread):
+//   lse_kernel  : 128-token x 256-vocab tiles, K = d streamed in 64-wide
+//                 SWIZZLE_128B atoms; fp32 accumulators double-buffered in
+//                 TMEM (2 x 256 columns); the epilogue folds each tile into
+//                 an online (max, sum-exp) per token and picks the target
+//                 logit. Work unit = (token block, vocabulary split).
+//   bwd_kernel  : rows x 128-column S tiles recomputed from the operands,
+//                 Gs formed in registers and written to shared memory as a
+//                 K-major SWIZZLE_128B bf16 tile, then a second MMA
+//                 out[rows, slice] += Gs . C[cols, slice] with the column
+//                 operand's d-slice read MN-major. Token rows give dH,
+//                 vocabulary rows give dW. The output slice (<= 256 fp32
+//                 columns) stays in TMEM for the whole unit, beside the two
+//                 128-column S buffers.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+
+#include "pair_common.cuh"
+#include "tc_ptx.cuh"
+
+namespace pairk {
+namespace {
+
+using namespace tc;
+
+constexpr int kThreads = 192;
+constexpr int kAtom128 = 128 * 64 * 2;  // 128 rows x 64 bf16 (16 KB)
+
+// ------------------------------------------------------------------ LSE
+constexpr int kLseBN = 256;
+constexpr int kLseStages = 4;
+constexpr uint32_t kLseStageTx = (128 + kLseBN) * 64 * 2;
+constexpr uint32_t kIdescLse = idesc_bf16(128, kLseBN, 0, 0);
+
+struct LseSmem {
+  uint8_t a[kLseStages][kAtom128];
+  uint8_t b[kLseStages][2 * kAtom128];
+  uint64_t full[kLseStages], empty[kLseStages];
+  uint64_t acc_full[2], acc_empty[2];
+  uint64_t mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ uint8_t *align1k(uint8_t *p) {
+  return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) &
+                                     ~static_cast<uintptr_t>(1023));
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    lse_kernel(const __grid_constant__ CUtensorMap tmH,
+               const __grid_constant__ CUtensorMap tmW, int d, int V,
+               int nsplit, int64_t Tpad, const int32_t *counters,
+               const int32_t *tok_y, float2 *part, float *zy,
+               int32_t *dev_err) {
+  extern __shared__ uint8_t smem_raw[];
+  LseSmem &sm = *reinterpret_cast<LseSmem *>(align1k(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int Teff = counters[0];
+  const int n_tb = (Teff + 127) / 128;
+  const int n_vt = (V + kLseBN - 1) / kLseBN;
+  const int n_units = n_tb * nsplit;
+  const int nk = d / 64;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kLseStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.acc_full[s], 1);
+      mbar_init(&sm.acc_empty[s], 128);
+    }
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmH);
+    prefetch_tmap(&tmW);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  volatile int *abort = &sm.abort;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0;
+      int last_ph[kLseStages];
+      for (int s = 0; s < kLseStages; ++s) last_ph[s] = -1;
+      bool ok = true;
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+        const int tb = u / nsplit, sp = u % nsplit;
+        const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
+        const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
+        for (int vt = vt0; vt < vt1 && ok; ++vt) {
+          for (int k = 0; k < nk; ++k) {
+            if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+            mbar_expect_tx(&sm.full[stage], kLseStageTx);
+            tma_load_2d(sm.a[stage], &tmH, &sm.full[stage], k * 64, tb * 128);
+            tma_load_2d(sm.b[stage], &tmW, &sm.full[stage], k * 64, vt * kLseBN);
+            last_ph[stage] = (int)ph;
+            if (++stage == kLseStages) { stage = 0; ph ^= 1; }
+          }
+        }
+      }
+      // Never leave a copy in flight: wait (bounded) for the last one issued
+      // on every stage.
+      for (int s = 0; s < kLseStages; ++s)
+        if (last_ph[s] >= 0) {
+          volatile int never = 0;
+          wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+        }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0, acc = 0;
+      uint32_t ph = 0, acc_ph = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+        const int sp = u % nsplit;
+        const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
+        const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
+        for (int vt = vt0; vt < vt1 && ok; ++vt) {
+          if (!(ok = wait(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
+          tc_fence_after();
+          const uint32_t dt = tmem + acc * kLseBN;
+          for (int k = 0; k < nk; ++k) {
+            if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+            tc_fence_after();
+            const uint32_t sa = smem_u32(sm.a[stage]), sb = smem_u32(sm.b[stage]);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_bf16(dt, sdesc_sw128(sa + kk * 32, 16, 1024),
+                       sdesc_sw128(sb + kk * 32, 16, 1024), kIdescLse,
+                       (k | kk) != 0);
+            mma_commit(&sm.empty[stage]);
+            if (++stage == kLseStages) { stage = 0; ph ^= 1; }
+          }
+          if (!ok) break;
+          mma_commit(&sm.acc_full[acc]);
+          if (++acc == 2) { acc = 0; acc_ph ^= 1; }
+        }
+      }
+      mma_commit(&sm.mma_done);
+      volatile int never = 0;
+      wait(&sm.mma_done, 0, &never, dev_err);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    int acc = 0;
+    uint32_t acc_ph = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+      const int tb = u / nsplit, sp = u % nsplit;
+      const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
+      const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
+      const int p = tb * 128 + row;
+      const bool valid = p < Teff;
+      const int yt = valid ? tok_y[p] : -1;
+      float m2 = -INFINITY, l = 0.f, zt = 0.f;
+      bool found = false;
+      for (int vt = vt0; vt < vt1; ++vt) {
+        if (!(ok = wait(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < kLseBN / 32; ++c) {
+          float v[32];
+          tmem_ld32(lane_addr + acc * kLseBN + c * 32, v);
+          const int col0 = vt * kLseBN + c * 32;
+          const int off = yt - col0;
+          if (off >= 0 && off < 32) {
+            found = true;
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (j == off) zt = v[j];
+          }
+          const int nvalid = V - col0;  // columns >= V are padding
+          float mc = -INFINITY;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            v[j] = (j < nvalid) ? v[j] * kLog2e : -INFINITY;
+            mc = fmaxf(mc, v[j]);
+          }
+          if (mc == -INFINITY) continue;
+          if (mc > m2) {
+            l *= exp2f(m2 - mc);
+            m2 = mc;
+          }
+          float s = 0.f;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) s += exp2f(v[j] - m2);
+          l += s;
+        }
+        tc_fence_before();
+        mbar_arrive(&sm.acc_empty[acc]);
+        if (++acc == 2) { acc = 0; acc_ph ^= 1; }
+      }
+      if (!ok) break;
+      if (valid) {
+        part[(int64_t)sp * Tpad + p] = make_float2(m2, l);
+        if (found) zy[p] = zt;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// lse_t = ln 2 * (M + log2 sum_s l_s 2^(m_s - M)) over the vocabulary splits.
+__global__ void lse_combine_kernel(int nsplit, int64_t Tpad,
+                                   const int32_t *counters, const float2 *part,
+                                   float *lse) {
+  const int Teff = counters[0];
+  for (int p = blockIdx.x * blockDim.x + threadIdx.x; p < Teff;
+       p += gridDim.x * blockDim.x) {
+    float M = -INFINITY;
+    for (int s = 0; s < nsplit; ++s) M = fmaxf(M, part[(int64_t)s * Tpad + p].x);
+    float L = 0.f;
+    for (int s = 0; s < nsplit; ++s) {
+      const float2 q = part[(int64_t)s * Tpad + p];
+      if (q.y > 0.f) L += q.y * exp2f(q.x - M);
+    }
+    lse[p] = (M + log2f(L)) * 0.6931471805599453f;
+  }
+}
+
+// ------------------------------------------------------------- backward
+constexpr int kBwdBN = 128;     // S tile columns
+constexpr int kSlice = 256;     // output columns held in TMEM per unit
+constexpr int kBwdStages = 3;
+constexpr uint32_t kBwdStageTx = 2 * kAtom128;
+constexpr uint32_t kIdescS = idesc_bf16(128, kBwdBN, 0, 0);
+
+struct BwdSmem {
+  uint8_t a[kBwdStages][kAtom128];   // rows-operand atoms (128 x 64)
+  uint8_t b[kBwdStages][kAtom128];   // cols-operand atoms (128 x 64)
+  uint8_t cs[kSlice / 64][kAtom128]; // cols operand, d-slice (MN-major B)
+  uint8_t g[kBwdBN / 64][kAtom128];  // Gs tile, K-major A (2 atoms along K)
+  float col_c[kBwdBN], col_l[kBwdBN];
+  uint64_t full[kBwdStages], empty[kBwdStages];
+  uint64_t s_full[2], s_empty[2];
+  uint64_t g_full, g_empty, cs_full, cs_empty, o_full, o_empty, mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ void epi_sync() {
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+}
+
+// kTokenRows: rows = tokens (output dH), cols = vocabulary.
+// otherwise : rows = vocabulary (output dW), cols = tokens.
+template <bool kTokenRows>
+__global__ void __launch_bounds__(kThreads, 1)
+    bwd_kernel(const __grid_constant__ CUtensorMap tmR,
+               const __grid_constant__ CUtensorMap tmC, int d, int V,
+               const int32_t *counters, const int32_t *tok_idx,
+               const float *tok_c, const float *lse, float *out,
+               int32_t *dev_err) {
+  extern __shared__ uint8_t smem_raw[];
+  BwdSmem &sm = *reinterpret_cast<BwdSmem *>(align1k(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int Teff = counters[0];
+  const int nsl = (d + kSlice - 1) / kSlice;
+  const int n_rb = kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128;
+  const int n_ct = kTokenRows ? (V + kBwdBN - 1) / kBwdBN : (Teff + kBwdBN - 1) / kBwdBN;
+  const int n_units = n_rb * nsl;
+  const int nk = d / 64;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kBwdStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.s_full[s], 1);
+      mbar_init(&sm.s_empty[s], 128);
+    }
+    mbar_init(&sm.g_full, 128);
+    mbar_init(&sm.g_empty, 1);
+    mbar_init(&sm.cs_full, 1);
+    mbar_init(&sm.cs_empty, 1);
+    mbar_init(&sm.o_full, 1);
+    mbar_init(&sm.o_empty, 128);
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmR);
+    prefetch_tmap(&tmC);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  const uint32_t tmem_o = tmem + 2 * kBwdBN;  // columns [256, 512)
+  volatile int *abort = &sm.abort;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0, cs_ph = 0;
+      int last_ph[kBwdStages];
+      for (int s = 0; s < kBwdStages; ++s) last_ph[s] = -1;
+      int cs_last = -1;
+      bool ok = true;
+      auto load_s = [&](int rb, int ct) {
+        for (int k = 0; k < nk && ok; ++k) {
+          if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+          mbar_expect_tx(&sm.full[stage], kBwdStageTx);
+          tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], k * 64, rb * 128);
+          tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], k * 64, ct * kBwdBN);
+          last_ph[stage] = (int)ph;
+          if (++stage == kBwdStages) { stage = 0; ph ^= 1; }
+        }
+      };
+      auto load_cs = [&](int sl, int w, int ct) {
+        if (!ok) return;
+        if (!(ok = wait(&sm.cs_empty, cs_ph ^ 1, abort, dev_err))) return;
+        mbar_expect_tx(&sm.cs_full, (uint32_t)(w / 64) * kAtom128);
+        for (int j = 0; j < w / 64; ++j)
+          tma_load_2d(sm.cs[j], &tmC, &sm.cs_full, sl * kSlice + j * 64, ct * kBwdBN);
+        cs_last = (int)cs_ph;
+        cs_ph ^= 1;
+      };
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+        const int rb = u / nsl, sl = u % nsl;
+        const int w = min(kSlice, d - sl * kSlice);
+        if (n_ct == 0) continue;
+        load_s(rb, 0);
+        for (int ct = 1; ct < n_ct && ok; ++ct) {
+          load_s(rb, ct);
+          load_cs(sl, w, ct - 1);
+        }
+        load_cs(sl, w, n_ct - 1);
+      }
+      volatile int never = 0;
+      for (int s = 0; s < kBwdStages; ++s)
+        if (last_ph[s] >= 0) wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+      if (cs_last >= 0) wait(&sm.cs_full, (uint32_t)cs_last, &never, dev_err);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0, s_ph[2] = {0, 0}, g_ph = 0, cs_ph = 0, o_ph = 0;
+      bool ok = true;
+      auto issue_s = [&](int ct) {
+        const int buf = ct & 1;
+        if (!(ok = wait(&sm.s_empty[buf], s_ph[buf] ^ 1, abort, dev_err))) return;
+        tc_fence_after();
+        const uint32_t dt = tmem + buf * kBwdBN;
+        for (int k = 0; k < nk; ++k) {
+          if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) return;
+          tc_fence_after();
+          const uint32_t sa = smem_u32(sm.a[stage]), sb = smem_u32(sm.b[stage]);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            mma_bf16(dt, sdesc_sw128(sa + kk * 32, 16, 1024),
+                     sdesc_sw128(sb + kk * 32, 16, 1024), kIdescS,
+                     (k | kk) != 0);
+          mma_commit(&sm.empty[stage]);
+          if (++stage == kBwdStages) { stage = 0; ph ^= 1; }
+        }
+        mma_commit(&sm.s_full[buf]);
+        s_ph[buf] ^= 1;
+      };
+      auto issue_o = [&](int ct, int w) {
+        if (!ok) return;
+        if (!(ok = wait(&sm.g_full, g_ph, abort, dev_err))) return;
+        if (!(ok = wait(&sm.cs_full, cs_ph, abort, dev_err))) return;
+        if (ct == 0 && !(ok = wait(&sm.o_empty, o_ph ^ 1, abort, dev_err))) return;
+        tc_fence_after();
+        const uint32_t idesc = idesc_bf16(128, w, 0, 1);
+        const uint32_t sg = smem_u32(sm.g[0]), sc = smem_u32(sm.cs[0]);
+#pragma unroll
+        for (int kk = 0; kk < kBwdBN / 16; ++kk) {
+          const uint64_t ad = sdesc_sw128(sg + (kk >> 2) * kAtom128 + (kk & 3) * 32, 16, 1024);
+          const uint64_t bd = sdesc_sw128(sc + kk * 2048, kAtom128, 1024);
+          mma_bf16(tmem_o, ad, bd, idesc, (ct | kk) != 0);
+        }
+        mma_commit(&sm.g_empty);
+        mma_commit(&sm.cs_empty);
+        g_ph ^= 1;
+        cs_ph ^= 1;
+      };
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+        const int sl = u % nsl;
+        const int w = min(kSlice, d - sl * kSlice);
+        if (n_ct == 0) continue;
+        issue_s(0);
+        for (int ct = 0; ct < n_ct && ok; ++ct) {
+          if (ct + 1 < n_ct) issue_s(ct + 1);
+          issue_o(ct, w);
+        }
+        if (!ok) break;
+        mma_commit(&sm.o_full);
+        o_ph ^= 1;
+      }
+      mma_commit(&sm.mma_done);
+      volatile int never = 0;
+      wait(&sm.mma_done, 0, &never, dev_err);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    uint32_t s_ph[2] = {0, 0}, g_ph = 0, o_ph = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+      const int rb = u / nsl, sl = u % nsl;
+      const int w = min(kSlice, d - sl * kSlice);
+      const int rid = rb * 128 + row;  // token position or vocabulary id
+      float rc = 0.f, rl = 0.f;
+      if (kTokenRows && rid < Teff) {
+        rc = tok_c[rid];
+        rl = lse[rid] * kLog2e;
+      }
+      for (int ct = 0; ct < n_ct; ++ct) {
+        if (!kTokenRows) {
+          epi_sync();
+          const int p = ct * kBwdBN + row;
+          sm.col_c[row] = p < Teff ? tok_c[p] : 0.f;
+          sm.col_l[row] = p < Teff ? lse[p] * kLog2e : 0.f;
+          epi_sync();
+        }
+        const int buf = ct & 1;
+        if (!(ok = wait(&sm.s_full[buf], s_ph[buf], abort, dev_err))) break;
+        s_ph[buf] ^= 1;
+        if (!(ok = wait(&sm.g_empty, g_ph ^ 1, abort, dev_err))) break;
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < kBwdBN / 32; ++c) {
+          float v[32];
+          tmem_ld32(tmem + lane_off + buf * kBwdBN + c * 32, v);
+          uint32_t pk[16];
+#pragma unroll
+          for (int j = 0; j < 32; j += 2) {
+            float g2[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int col = c * 32 + j + e;
+              float cc, ll;
+              bool live;
+              if (kTokenRows) {
+                cc = rc; ll = rl;
+                live = (rc != 0.f) && (ct * kBwdBN + col < V);
+              } else {
+                cc = sm.col_c[col]; ll = sm.col_l[col];
+                live = cc != 0.f;
+              }
+              g2[e] = live ? -cc * exp2f(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
+            }
+            __nv_bfloat162 b2 = __floats2bfloat162_rn(g2[0], g2[1]);
+            pk[j >> 1] = *reinterpret_cast<uint32_t *>(&b2);
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int k = c * 32 + q * 8;  // first column of this 16-byte piece
+            uint8_t *dst = sm.g[k >> 6] + sw128_offset(row, k & 63);
+            *reinterpret_cast<uint4 *>(dst) =
+                make_uint4(pk[q * 4], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(&sm.s_empty[buf]);
+        fence_async_smem();
+        mbar_arrive(&sm.g_full);
+        g_ph ^= 1;
+      }
+      if (!ok) break;
+      const bool valid = kTokenRows ? (rid < Teff) : (rid < V);
+      float *dst = nullptr;
+      if (valid)
+        dst = out + (kTokenRows ? (int64_t)tok_idx[rid] : (int64_t)rid) * d + sl * kSlice;
+      if (n_ct == 0) {
+        if (valid)
+          for (int k = 0; k < w; ++k) dst[k] = 0.f;
+        continue;
+      }
+      if (!(ok = wait(&sm.o_full, o_ph, abort, dev_err))) break;
+      o_ph ^= 1;
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < w / 32; ++c) {
+        float v[32];
+        tmem_ld32(tmem_o + lane_off + c * 32, v);
+        if (valid) {
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            reinterpret_cast<float4 *>(dst + c * 32)[q] =
+                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&sm.o_empty);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// --------------------------------------------------------------- host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 row-major [rows][cols] map with 64 x box_rows SWIZZLE_128B boxes.
+bool make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t cols,
+              int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr),
+            dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int num_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+}  // namespace
+
+pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
+                         cudaStream_t s) {
+  CUtensorMap mH, mW128, mW256;
+  if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) ||
+      !make_map(&mW128, g.W, g.V, g.d, 128) ||
+      !make_map(&mW256, g.W, g.V, g.d, 256))
+    return PAIR_ERR_CUDA;
+  const int nsm = num_sms();
+  const size_t lse_smem = sizeof(LseSmem) + 1024;
+  const size_t bwd_smem = sizeof(BwdSmem) + 1024;
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(lse_kernel,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)lse_smem));
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_kernel<true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bwd_smem));
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_kernel<false>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bwd_smem));
+
+  lse_kernel<<<nsm, kThreads, lse_smem, s>>>(mH, mW256, g.d, g.V, w.nsplit,
+                                             w.Tpad, w.counters, w.tok_y,
+                                             w.part, w.zy, g.dev_err);
+  PAIR_LAUNCH_CHECK();
+  lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters,
+                                             w.part, w.lse);
+  PAIR_LAUNCH_CHECK();
+  bwd_kernel<true><<<nsm, kThreads, bwd_smem, s>>>(
+      mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
+      g.dev_err);
+  PAIR_LAUNCH_CHECK();
+  bwd_kernel<false><<<nsm, kThreads, bwd_smem, s>>>(
+      mW128, mH, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
+      g.dev_err);
+  PAIR_LAUNCH_CHECK();
+  return PAIR_OK;
+}
+
+}  // namespace pairk

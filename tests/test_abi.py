@@ -1,0 +1,74 @@
+"""The C-ABI library builds for sm_103a, loads, exports every function that
+include/pair.h declares, and validates arguments on the host (no GPU needed:
+invalid arguments are rejected before any device call)."""
+import ctypes
+
+import pytest
+
+from paper_2608_11368_gb300 import build
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    from paper_2608_11368_gb300 import binding
+    return binding
+
+
+def test_exports_every_header_function(L):
+    names = L.header_functions()
+    assert {"pair_coeffs", "pair_grad", "pair_estimate_dense",
+            "pair_grad_workspace_size", "pair_status_sync",
+            "pair_status_string", "pair_last_launch_count"} <= set(names)
+    lib = L.lib()
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_strings(L):
+    for st in range(8):
+        s = L.pair_status_string(st)
+        assert s and s != "unknown status"
+    assert L.pair_status_string(99) == "unknown status"
+
+
+def test_workspace_size_rules(L):
+    ws = L.pair_grad_workspace_size
+    assert ws(1000, 2048, 151936, 64, L.PAIR_BF16) > 1000 * 2048 * 2
+    assert ws(1000, 2048, 151936, 64, L.PAIR_F32) > ws(1000, 2048, 151936, 64, L.PAIR_BF16)
+    assert ws(1000, 96, 100, 4, L.PAIR_BF16) == 0      # bf16 needs d % 64 == 0
+    assert ws(1000, 96, 100, 4, L.PAIR_F32) > 0
+    assert ws(1000, 20, 100, 4, L.PAIR_F32) == 0       # d % 16 != 0
+    assert ws(0, 64, 100, 4, L.PAIR_F32) == 0
+    assert ws(10, 64, 100, 0, L.PAIR_F32) == 0
+    assert ws(10, 64, 0, 1, L.PAIR_F32) == 0
+
+
+def test_host_validation_without_device(L):
+    lib = L.lib()
+    P = ctypes.c_void_p
+    one = P(16)  # never dereferenced: validation fails first
+    # G < 2, G > PAIR_MAX_G, B < 1, null pointers, bad flags.
+    for B, G in [(1, 1), (1, 129), (0, 8)]:
+        assert lib.pair_coeffs(B, G, one, one, one, 1.0, 0, one, None, None,
+                               None, None, None) == 1
+    assert lib.pair_coeffs(1, 8, None, one, one, 1.0, 0, one, None, None, None,
+                           None, None) == 1
+    assert lib.pair_coeffs(1, 8, one, one, one, 1.0, 2, one, None, None, None,
+                           None, None) == 1
+    assert lib.pair_estimate_dense(1, 8, 0, one, one, one, one, 1.0, one, None,
+                                   None, None) == 1
+    # pair_grad: nulls, misalignment, bad shapes, workspace too small.
+    args = [100, 128, 256, L.PAIR_BF16, one, one, one, one, one, 2, one, one,
+            one, one, None, one, 1 << 30, None, None]
+    assert lib.pair_grad(*args) != 0
+    bad = list(args); bad[4] = None
+    assert lib.pair_grad(*bad) == 1
+    bad = list(args); bad[4] = P(8)
+    assert lib.pair_grad(*bad) == 1
+    bad = list(args); bad[1] = 96
+    assert lib.pair_grad(*bad) == 2          # bf16 with d % 64 != 0
+    bad = list(args); bad[16] = 1024
+    assert lib.pair_grad(*bad) == 3          # workspace too small
+    bad = list(args); bad[15] = P(16 + 128)
+    assert lib.pair_grad(*bad) == 3          # workspace not 256-aligned

@@ -1,0 +1,199 @@
+"""GPU parity of pair_grad (the LM-head realisation of sum_i a_i log pi of
+Sec. 4.5) against the fp64 oracle.
+
+Tolerances: J, dH, dW within a relative Frobenius error of 2e-3 (bf16 inputs,
+fp32 accumulation); for J the denominator is sum_t |c_t logp_t| because the
+coefficients sum to zero within a group. The softmax parts alone (dH minus
+its exact one-hot part, dW on non-target rows) are held to 1e-2: their only
+approximation is the bf16 rounding of the on-chip logit gradient
+(relative 2^-9 per element, about 1.1e-3 RMS).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_11368_gb300 import synth
+from tests.gpu_util import dev_err_word, head_inputs, rel_fro
+
+pytestmark = pytest.mark.gpu
+
+TOL = 2e-3
+TOL_SOFT = 1e-2
+
+
+def _binding():
+    from paper_2608_11368_gb300 import binding
+    return binding
+
+
+def _coeffs(inp, scale=1.0):
+    c = oracle.coeffs(inp["r"], inp["J"], inp["rho"], scale=scale)
+    return c["a"].reshape(-1).astype(np.float32)
+
+
+def _run(inp, a, **kw):
+    B = _binding()
+    t = head_inputs(inp, a)
+    err = dev_err_word()
+    Jo, dH, dW, lps = B.pair_grad(t["H"], t["W"], t["y"], t["mask"],
+                                  t["cu_seqlens"], t["a"], dev_err=err, **kw)
+    st = B.pair_status_sync(err)
+    return st, Jo.item(), dH, dW, lps, t
+
+
+def _full_check(inp, a):
+    st, J, dH, dW, lps, t = _run(inp, a)
+    assert st == 0
+    ref = oracle.pair_grad_ref(inp, a.astype(np.float64), full=True)
+    dHn, dWn = dH.cpu().numpy(), dW.cpu().numpy()
+    assert abs(J - ref["J"]) <= TOL * max(ref["J_abs"], 1e-30)
+    assert rel_fro(dHn, ref["dH"]) <= TOL
+    assert rel_fro(dWn, ref["dW"]) <= TOL
+    np.testing.assert_allclose(lps.cpu().numpy(), ref["logp_seq"], rtol=1e-4,
+                               atol=1e-3)
+    # Rows outside the objective are exact zeros.
+    seg = oracle.segment_ids(inp["cu_seqlens"])
+    off = (inp["mask"] == 0) | (a[seg] == 0)
+    assert (dHn[off] == 0).all()
+    # Softmax parts on their own.
+    Wf = synth.as_float(inp["W"], inp["dtype"]).astype(np.float64)
+    idx, c, _ = oracle.compact_tokens(inp["cu_seqlens"], inp["mask"], a)
+    if idx.size:
+        one = c[:, None] * Wf[inp["y"][idx]]
+        assert rel_fro(dHn[idx] - one, ref["dH"][idx] - one) <= TOL_SOFT
+        untargeted = np.setdiff1d(np.arange(inp["V"]), inp["y"][idx])
+        assert rel_fro(dWn[untargeted], ref["dW"][untargeted]) <= TOL_SOFT
+    return J, dH, dW
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_grad_fp32_reference_workload(seed):
+    inp = synth.make_head_workload(synth.WORKLOADS["pr1_ref_fp32"], seed)
+    _full_check(inp, _coeffs(inp))
+
+
+CASES = [
+    # name, d, V, B, G, len_scale, w_mult
+    ("qwen3_1p7b_head", 2048, 151936, 2, 4, 0.06, 1.0),  # full head, tail tile
+    ("qwen3_1p7b_head", 192, 1000, 3, 5, 0.05, 8.0),     # ragged V, N=192 slice
+    ("qwen3_4b_head", 320, 777, 2, 6, 0.03, 8.0),        # two slices (256 + 64)
+    ("longctx_skew", 64, 300, 4, 4, 0.02, 1.0),          # minimal d
+    ("qwen3_4b_head", 2560, 4099, 2, 3, 0.05, 3.0),      # ten slices
+]
+
+
+@pytest.mark.parametrize("case", CASES, ids=[f"d{c[1]}_V{c[2]}" for c in CASES])
+def test_grad_bf16_full_parity(case):
+    name, d, V, B, G, ls, wm = case
+    inp = synth.make_head_workload(synth.WORKLOADS[name], 5, B=B, G=G, d=d, V=V,
+                                   len_scale=ls, w_std_mult=wm)
+    a = _coeffs(inp)
+    if not (a != 0).any():
+        a[0] = 0.75
+    _full_check(inp, a)
+
+
+def test_grad_no_active_rollout():
+    inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 1, B=2,
+                                   G=2, d=128, V=520, len_scale=0.05)
+    a = np.zeros(inp["R"], np.float32)
+    a[1] = -0.0
+    st, J, dH, dW, lps, _ = _run(inp, a)
+    assert st == 0 and J == 0.0
+    assert (dH == 0).all() and (dW == 0).all() and (lps == 0).all()
+
+
+def test_grad_nan_padding_is_ignored_and_deterministic():
+    wl = synth.WORKLOADS["longctx_skew"]
+    kw = dict(B=3, G=4, d=256, V=2000, len_scale=0.05, w_std_mult=2.0)
+    inp = synth.make_head_workload(wl, 4, **kw)
+    inp_nan = synth.make_head_workload(wl, 4, pad_fill="nan", **kw)
+    a = _coeffs(inp)
+    r0 = _run(inp, a)
+    r1 = _run(inp_nan, a)
+    r2 = _run(inp, a)
+    for x, y in ((r0, r1), (r0, r2)):
+        assert x[1] == y[1]
+        assert torch.equal(x[2], y[2]) and torch.equal(x[3], y[3])
+
+
+def test_grad_target_out_of_range_flagged():
+    inp = synth.make_head_workload(synth.WORKLOADS["pr1_ref_fp32"], 0, V=64,
+                                   d=32)
+    a = _coeffs(inp)
+    t = np.nonzero(inp["mask"])[0][3]
+    inp["y"][t] = 64
+    st = _run(inp, a)[0]
+    assert st == 5
+    # -100 on padding tokens is fine (the generator's default).
+    inp["y"][t] = 5
+    assert _run(inp, a)[0] == 0
+
+
+FULL = ["qwen3_1p7b_head", "qwen3_4b_head", "longctx_skew"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_grad_full_size_sampled(name):
+    """Full-size workload in the benchmark's launch configuration: sampled
+    rows against the oracle, and size-independent identities for the rest."""
+    wl = synth.WORKLOADS[name]
+    inp = synth.make_head_workload(wl, 0)
+    a = _coeffs(inp)
+    st, J, dH, dW, lps, t = _run(inp, a)
+    assert st == 0
+    rng = np.random.default_rng(11)
+    idx, c, seg = oracle.compact_tokens(inp["cu_seqlens"], inp["mask"], a)
+    assert idx.size > 0
+    # dH: 1024 sampled active rows plus every row of the two shortest active
+    # rollouts (whose summed logp is checked too).
+    act_r = np.nonzero(a)[0]
+    L = np.diff(inp["cu_seqlens"])[act_r]
+    two = act_r[np.argsort(L)[:2]]
+    cu = inp["cu_seqlens"]
+    whole = np.concatenate([np.arange(cu[i], cu[i + 1]) for i in two])
+    rows = np.unique(np.concatenate([rng.choice(idx, 1024, replace=False), whole]))
+    ref = oracle.pair_grad_ref(inp, a.astype(np.float64), dh_rows=rows,
+                               logp_rollouts=two)
+    dHn = dH.cpu().numpy()
+    assert rel_fro(dHn[rows], ref["dH_rows"]) <= TOL
+    lps_n = lps.cpu().numpy()
+    np.testing.assert_allclose(lps_n[two], ref["logp_seq_sel"], rtol=1e-4)
+    # J is the coefficient-weighted sum of the per-rollout log-probabilities.
+    assert abs(J - float(np.dot(a.astype(np.float64), lps_n.astype(np.float64)))) \
+        <= 1e-4 * float(np.abs(a).dot(np.abs(lps_n)))
+    # Inactive rows exactly zero.
+    seg_all = oracle.segment_ids(cu)
+    off = (inp["mask"] == 0) | (a[seg_all] == 0)
+    assert not dH[torch.from_numpy(off).cuda()].any()
+    # Identities that hold at any size: sum_v dJ/dW_v = 0 (softmax rows sum
+    # to one), and <dW, W> = <dH, H> = sum_tv G_tv z_tv.
+    colsum = dW.double().sum(dim=0)
+    assert colsum.abs().max().item() <= 1e-3 * dW.double().abs().sum(dim=0).max().item()
+    ip_w = (dW.double() * t["W"].double()).sum().item()
+    ip_h = (dH.double() * t["H"].double()).sum().item()
+    assert abs(ip_w - ip_h) <= 1e-3 * max(abs(ip_h), 1e-30)
+    del dH, dW
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_grad_full_head_single_rollout_dw(name):
+    """dW rows at the full head size against the oracle, with one active
+    rollout (the oracle's dW costs one pass per active token)."""
+    wl = synth.WORKLOADS[name]
+    inp = synth.make_head_workload(wl, 1, B=2, G=wl.G, len_scale=0.25)
+    a = np.zeros(inp["R"], np.float32)
+    a[int(np.argmax(np.diff(inp["cu_seqlens"]) > 0))] = 0.625
+    st, J, dH, dW, lps, _ = _run(inp, a)
+    assert st == 0
+    rng = np.random.default_rng(3)
+    idx, _, _ = oracle.compact_tokens(inp["cu_seqlens"], inp["mask"], a)
+    targeted = np.unique(inp["y"][idx])
+    vrows = np.unique(np.concatenate([
+        rng.choice(inp["V"], 192, replace=False),
+        rng.choice(targeted, min(64, targeted.size), replace=False),
+        [inp["V"] - 1]]))
+    ref = oracle.pair_grad_ref(inp, a.astype(np.float64), dw_rows=vrows)
+    assert rel_fro(dW.cpu().numpy()[vrows], ref["dW_rows"]) <= TOL
