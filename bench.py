@@ -1,0 +1,463 @@
+#!/usr/bin/env python
+"""Benchmark of the Pair estimator hot path on GB300.
+
+One step = one pass of the whole hot path over one batch of the Qwen3-1.7B
+head workload (8 prompts x 8 rollouts, d = 2048, V = 151936, response
+lengths U[256, 2048], packed): pair_coeffs (per-rollout coefficients of
+Eq. pair-advantage from rewards, completion mask and the logged inclusion
+matrix) followed by pair_grad (LM-head GEMM, vocabulary log-softmax, target
+gather, scaling by a_i and the backward to dHidden and dW). The metric is
+pair_grad tokens/s (packed tokens per second, forward + backward); the JSON
+line also carries pair_coeffs / pair_estimate_dense GB/s on the
+4096 x 64 coefficient stress workload.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
+For N > 1 launch with torch.distributed.run; each rank runs its own batch
+(groups are independent: weak scaling, no data-path collective).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2608_11368_gb300 import synth  # noqa: E402
+
+WORKLOAD = "qwen3_1p7b_head"
+STRESS = "coeffs_dense_stress"
+METRIC = "pair_grad tokens/s (fwd+bwd) and % dense-BF16 peak; pair_coeffs GB/s vs HBM"
+FLUSH_BYTES = 256 << 20          # > 129 MB L2
+CPU_SAMPLE_TOKENS = 256          # oracle sample for the CPU baseline
+REF_SAMPLE_TOKENS = 48           # oracle sample per --impl reference step
+TC_KERNELS = ("lse_tc", "bwd_dh_tc", "bwd_dw_tc")
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
+    p.add_argument("--seed", type=int, default=0)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-stress", action="store_true")
+    return p.parse_args()
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        pk = json.load(open(path))
+        return dict(hbm=float(pk["hbm_gbs"]), bf16=float(pk["bf16_tflops"]),
+                    bf16_sus=float(pk["bf16_tflops_sustained"]), src="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+def load_traffic():
+    """Per-launch DRAM bytes from the committed ncu summary, keyed by kernel,
+    valid only while the kernel source is unchanged (hash recorded there)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    out = {}
+    if not os.path.exists(path):
+        return out
+    for line in open(path):
+        parts = line.split()
+        if len(parts) < 5 or line.startswith("#"):
+            continue
+        name, wl, bytes_, src, sha = parts[:5]
+        try:
+            cur = hashlib.sha256(open(os.path.join(ROOT, src), "rb").read()).hexdigest()[:16]
+        except OSError:
+            continue
+        if cur == sha:
+            out[(name, wl)] = float(bytes_)
+    return out
+
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,"
+         "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.rows = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append([x.strip() for x in line.split(",")])
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=5)
+        sm, mx, reasons, power = [], [], set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in self.rows:
+            if len(r) < 10:
+                continue
+            try:
+                sm.append(float(r[1])); mx.append(float(r[2])); power.append(float(r[3]))
+            except ValueError:
+                continue
+            for k, nm in enumerate(names):
+                if r[6 + k].lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_max": max(power) if power else None}
+
+
+def count_active_tokens(inp, a):
+    cu = inp["cu_seqlens"]
+    seg = np.repeat(np.arange(cu.size - 1), np.diff(cu))
+    return int(((inp["mask"] == 1) & (a[seg] != 0)).sum())
+
+
+def cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+# ------------------------------------------------------------- CPU oracle leg
+
+def oracle_sample_time(inp, n_tok):
+    """Time the fp64 oracle (as it stands) on the coefficients of every group
+    plus the complete head work (lse, logp, dH rows, dW contribution over all
+    V rows) of the first n_tok active tokens. Returns (seconds for the sample,
+    seconds for the coefficients, T_eff)."""
+    import oracle
+    t0 = time.perf_counter()
+    c = oracle.coeffs(inp["r"], inp["J"], inp["rho"])
+    t_coef = time.perf_counter() - t0
+    a = c["a"].reshape(-1)
+    idx, cc, _ = oracle.compact_tokens(inp["cu_seqlens"], inp["mask"], a)
+    sub = idx[:n_tok]
+    W64 = synth.as_float(inp["W"], inp["dtype"]).astype(np.float64)
+    Hs = synth.as_float(inp["H"][sub], inp["dtype"]).astype(np.float64)
+    ys = inp["y"][sub]
+    t0 = time.perf_counter()
+    lse, zy = oracle.head_lse(Hs, W64, ys)
+    oracle.head_dh_rows(Hs, W64, ys, cc[:sub.size], lse)
+    oracle.head_dw_rows(Hs, W64, ys, cc[:sub.size], lse, np.arange(inp["V"]))
+    t_head = time.perf_counter() - t0
+    return t_head, t_coef, int(idx.size), int(sub.size)
+
+
+def cpu_baseline(inp):
+    t_head, t_coef, T_eff, n = oracle_sample_time(inp, CPU_SAMPLE_TOKENS)
+    est = t_coef + t_head * T_eff / max(n, 1)
+    return {"value": inp["T"] / est, "unit": "tokens/s", "cores": cores(),
+            "kind": "oracle",
+            "sample": ("fp64 oracle: coefficients of all %d groups + full head "
+                       "work (lse, dH rows, dW over all V) of %d of %d active "
+                       "tokens, %.1f s; step time extrapolated by T_eff/%d"
+                       % (inp["B"], n, T_eff, t_head + t_coef, n))}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return 0
+    wl = synth.WORKLOADS[WORKLOAD]
+    inp = synth.make_head_workload(wl, args.seed)
+    times = []
+    T_eff = n = 0
+    t_coef = 0.0
+    for k in range(args.warmup + args.steps):
+        t_head, t_coef, T_eff, n = oracle_sample_time(inp, REF_SAMPLE_TOKENS)
+        if k >= args.warmup:
+            times.append(t_coef + t_head * T_eff / max(n, 1))
+    step_s = statistics.mean(times)
+    value = inp["T"] * world / step_s
+    line = {"impl": "reference", "metric": METRIC, "value": value,
+            "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "global_batch": wl.B * wl.G * world,
+                       "tokens_packed": inp["T"], "tokens_active": T_eff,
+                       "parallelism": "replicas"},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores(),
+                             "kind": "oracle",
+                             "sample": "per step: coefficients of all groups + "
+                                       "full head work of %d active tokens, "
+                                       "extrapolated to T_eff=%d" % (n, T_eff)},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------- GPU leg
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+
+    import torch
+    import torch.distributed as dist
+    from paper_2608_11368_gb300 import binding as B
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    peaks = load_peaks()
+    traffic = load_traffic()
+    wl = synth.WORKLOADS[WORKLOAD]
+    inp = synth.make_head_workload(wl, args.seed + rank)
+    T, d, V, R = inp["T"], inp["d"], inp["V"], inp["R"]
+
+    def pinned(x):
+        t = torch.from_numpy(np.ascontiguousarray(x))
+        return t.pin_memory()
+
+    host = {
+        "H": pinned(inp["H"].view(np.int16)), "W": pinned(inp["W"].view(np.int16)),
+        "y": pinned(inp["y"]), "mask": pinned(inp["mask"]),
+        "cu": pinned(inp["cu_seqlens"]), "r": pinned(inp["r"]),
+        "J": pinned(inp["J"]), "rho": pinned(inp["rho"]),
+    }
+    devb = {k: v.to("cuda", non_blocking=False) for k, v in host.items()}
+    H = devb["H"].view(torch.bfloat16)
+    W = devb["W"].view(torch.bfloat16)
+    a = torch.empty((wl.B, wl.G), dtype=torch.float32, device="cuda")
+    active = torch.empty((wl.B, wl.G), dtype=torch.uint8, device="cuda")
+    edges = torch.empty(wl.B, dtype=torch.int32, device="cuda")
+    contrast = torch.empty(wl.B, dtype=torch.int32, device="cuda")
+    dH = torch.empty((T, d), dtype=torch.float32, device="cuda")
+    dW = torch.empty((V, d), dtype=torch.float32, device="cuda")
+    Jobj = torch.empty(1, dtype=torch.float64, device="cuda")
+    lps = torch.empty(R, dtype=torch.float32, device="cuda")
+    ws = torch.empty(B.pair_grad_workspace_size(T, d, V, R, B.PAIR_BF16),
+                     dtype=torch.uint8, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    launches = [0]
+
+    def step():
+        B.pair_coeffs(devb["r"], devb["J"], devb["rho"], a=a, active=active,
+                      edges=edges, contrast_edges=contrast, dev_err=err)
+        n = B.pair_last_launch_count()
+        B.pair_grad(H, W, devb["y"], devb["mask"], devb["cu"], a.view(-1),
+                    dH=dH, dW=dW, Jobj=Jobj, logp_seq=lps, ws=ws, dev_err=err)
+        launches[0] += n + B.pair_last_launch_count()
+
+    for _ in range(args.warmup):
+        step()
+    st = B.pair_status_sync(err)
+    if st != 0:
+        raise SystemExit("warm-up step failed: %s" % B.pair_status_string(st))
+    T_eff = count_active_tokens(inp, a.view(-1).cpu().numpy())
+
+    # ---- timed region: inputs resident in HBM, L2 flushed between steps.
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    sampler = ClockSampler(local)
+    sampler.start()
+    barrier()
+    torch.cuda.synchronize()
+    launches[0] = 0
+    B.pair_timing_enable(True)
+    for k in range(args.steps):
+        flush.zero_()
+        ev[k][0].record()
+        step()
+        ev[k][1].record()
+    torch.cuda.synchronize()
+    barrier()
+    kern = B.pair_timing_read()
+    B.pair_timing_enable(False)
+    clocks = sampler.stop()
+    gpu_launches = launches[0]
+    step_ms = [s.elapsed_time(e) for s, e in ev]
+    total_ms = max_over_ranks(sum(step_ms))
+    if B.pair_status_sync(err) != 0:
+        raise SystemExit("timed steps reported a device error")
+    value = T * world * args.steps / (total_ms / 1e3)
+
+    # Per-kernel durations over the timed region (CUDA events on the library's
+    # launch stream).
+    agg = {}
+    for name, ms in kern:
+        n, tot = agg.get(name, (0, 0.0))
+        agg[name] = (n + 1, tot + ms)
+    flops_gemm = 2.0 * T_eff * V * d
+    dominant = max(agg.items(), key=lambda kv: kv[1][1])[0]
+    dn, dt_ms = agg[dominant]
+    dom_avg = dt_ms / dn
+    dom_flops = flops_gemm if dominant in TC_KERNELS else None
+    achieved = dom_flops / (dom_avg / 1e3) / 1e12 if dom_flops else None
+    roofline = {"kernel": dominant, "bound": "tensor",
+                "achieved": achieved, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
+                "frac": (achieved / peaks["bf16_sus"]) if achieved else None,
+                "traffic": traffic.get((dominant, WORKLOAD)),
+                "peak_source": peaks["src"] + " sustained bf16 (kernel timed inside a long step)",
+                "algorithmic_flops_per_launch": dom_flops,
+                "avg_launch_ms": dom_avg}
+    tc_ms = sum(agg[k][1] for k in TC_KERNELS if k in agg) / args.steps
+    grad_ms = sum(t for nm, (n, t) in agg.items() if nm not in ("coeffs",)) / args.steps
+    pair_grad_info = {
+        "algorithmic_tflops": 3 * flops_gemm / (grad_ms / 1e3) / 1e12,
+        "frac_of_sustained_bf16": 3 * flops_gemm / (grad_ms / 1e3) / 1e12 / peaks["bf16_sus"],
+        "ms_per_call": grad_ms, "tensor_kernels_ms": tc_ms,
+        "tokens_active_per_s": T_eff * world / (grad_ms / 1e3),
+        "kernels": {k: {"launches": n, "total_ms": t, "share": t / sum(x[1] for x in agg.values())}
+                    for k, (n, t) in sorted(agg.items(), key=lambda kv: -kv[1][1])}}
+
+    # ---- end-to-end through the C-ABI with host buffers.
+    out_h = torch.empty(1 + R, dtype=torch.float64).pin_memory()
+    names_in = ["H", "W", "y", "mask", "cu", "r", "J", "rho"]
+    h2d = sum(host[k].numel() * host[k].element_size() for k in names_in)
+    d2h = Jobj.numel() * 8 + lps.numel() * 4
+    lps_h = torch.empty(R, dtype=torch.float32).pin_memory()
+    e2e_ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    barrier()
+    torch.cuda.synchronize()
+    e2e_ev[0].record()
+    for _ in range(args.steps):
+        for k in names_in:
+            devb[k].copy_(host[k], non_blocking=True)
+        step()
+        out_h[:1].copy_(Jobj, non_blocking=True)
+        lps_h.copy_(lps, non_blocking=True)
+    e2e_ev[1].record()
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e2e_ev[0].elapsed_time(e2e_ev[1]))
+    e2e = {"value": T * world * args.steps / (e2e_ms / 1e3), "unit": "tokens/s",
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    # ---- pair_coeffs / pair_estimate_dense on the 4096 x 64 stress workload.
+    stress = None
+    if not args.no_stress:
+        stress = bench_stress(B, torch, peaks, flush, args.steps, rank, traffic)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(inp)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; Qwen3-1.7B head shapes, random-init weights)",
+        "config": {"workload": WORKLOAD, "d": d, "V": V,
+                   "global_batch": wl.B * wl.G * world, "prompts": wl.B * world,
+                   "rollouts_per_prompt": wl.G, "tokens_packed": T,
+                   "tokens_active": T_eff,
+                   "l2": "flushed between timed steps (256 MiB write); inputs exceed L2",
+                   "parallelism": "replicas" if world == 1 else "dp%d weak (independent groups)" % world},
+        "roofline": roofline, "pair_grad": pair_grad_info,
+        "stress": stress, "cpu_baseline": cpu, "e2e": e2e,
+        "clocks": clocks, "gpu_launches": gpu_launches,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
+    wl = synth.WORKLOADS[STRESS]
+    inp = synth.make_dense_workload(wl, 100 + rank)
+    dv = lambda x: torch.from_numpy(np.ascontiguousarray(x)).cuda()
+    r, J, rho, S = dv(inp["r"]), dv(inp["J"]), dv(inp["rho"]), dv(inp["S"])
+    Bn, G, D = wl.B, wl.G, wl.d
+    a = torch.empty((Bn, G), dtype=torch.float32, device="cuda")
+    g = torch.empty((Bn, D), dtype=torch.float32, device="cuda")
+    act = torch.empty((Bn, G), dtype=torch.uint8, device="cuda")
+    e1 = torch.empty(Bn, dtype=torch.int32, device="cuda")
+    e2 = torch.empty(Bn, dtype=torch.int32, device="cuda")
+
+    def timed(fn, n):
+        fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(n):
+            flush.zero_()
+            s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s.record(); fn(); e.record()
+            torch.cuda.synchronize()
+            ts.append(s.elapsed_time(e))
+        return statistics.median(ts)
+
+    reps = max(20, steps)
+    t_c = timed(lambda: B.pair_coeffs(r, J, rho, a=a, active=act, edges=e1,
+                                      contrast_edges=e2), reps)
+    t_d = timed(lambda: B.pair_estimate_dense(r, J, rho, S, g=g, a=a), reps)
+    n_act = int((a != 0).sum().item())
+    bytes_c = Bn * (4 * G * (G - 1) // 2 + 4 * G + G + 4 * G + G + 8)
+    bytes_d = 4 * D * n_act + Bn * (4 * G * (G - 1) // 2 + 4 * G + G) + 4 * Bn * D + 4 * Bn * G
+    gbs_c = bytes_c / (t_c / 1e3) / 1e9
+    gbs_d = bytes_d / (t_d / 1e3) / 1e9
+    return {
+        "workload": STRESS,
+        "pair_coeffs": {"bound": "hbm", "achieved": gbs_c, "peak": peaks["hbm"],
+                        "unit": "GB/s", "frac": gbs_c / peaks["hbm"],
+                        "traffic": traffic.get(("coeffs", STRESS)),
+                        "ms": t_c, "algorithmic_bytes": bytes_c},
+        "pair_estimate_dense": {"bound": "hbm", "achieved": gbs_d, "peak": peaks["hbm"],
+                                "unit": "GB/s", "frac": gbs_d / peaks["hbm"],
+                                "traffic": traffic.get(("dense", STRESS)),
+                                "ms": t_d, "algorithmic_bytes": bytes_d},
+        "timing": "median of %d single launches, CUDA events, L2 flushed before each" % reps,
+    }
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -199,6 +199,19 @@ PAIR_API const char *pair_status_string(pair_status st);
  * (used to report how many of this library's kernels ran). */
 PAIR_API int32_t pair_last_launch_count(void);
 
+/*
+ * Optional per-kernel timing (tracing). While enabled on a host thread,
+ * every kernel this library launches from that thread is bracketed by CUDA
+ * events recorded on the launch stream (at most 4096 launches are kept).
+ * pair_timing_enable(1) starts a fresh record; pair_timing_read waits for
+ * the recorded events, writes up to `max` durations in milliseconds and
+ * static kernel names (either array may be null), clears the record and
+ * returns the number written. Off by default; costs two event records per
+ * launch when on.
+ */
+PAIR_API void pair_timing_enable(int32_t on);
+PAIR_API int32_t pair_timing_read(int32_t max, float *ms, const char **names);
+
 #ifdef __cplusplus
 }
 #endif

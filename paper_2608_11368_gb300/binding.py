@@ -63,6 +63,10 @@ def lib() -> ctypes.CDLL:
     L.pair_status_string.restype = ctypes.c_char_p
     L.pair_last_launch_count.argtypes = []
     L.pair_last_launch_count.restype = I32
+    L.pair_timing_enable.argtypes = [I32]
+    L.pair_timing_enable.restype = None
+    L.pair_timing_read.argtypes = [I32, P, P]
+    L.pair_timing_read.restype = I32
     _lib = L
     return L
 
@@ -80,6 +84,20 @@ def pair_status_string(status: int) -> str:
 
 def pair_last_launch_count() -> int:
     return int(lib().pair_last_launch_count())
+
+
+def pair_timing_enable(on: bool) -> None:
+    """Start (or stop) recording per-kernel CUDA events for this thread."""
+    lib().pair_timing_enable(1 if on else 0)
+
+
+def pair_timing_read(max_launches: int = 4096):
+    """[(kernel name, milliseconds)] of the launches recorded since the last
+    enable/read (waits for their events)."""
+    ms = (ctypes.c_float * max_launches)()
+    names = (ctypes.c_char_p * max_launches)()
+    n = lib().pair_timing_read(max_launches, ms, names)
+    return [(names[i].decode(), float(ms[i])) for i in range(n)]
 
 
 def _p(t):

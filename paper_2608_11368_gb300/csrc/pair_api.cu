@@ -9,9 +9,46 @@
 
 namespace pairk {
 
-static thread_local int32_t g_launches = 0;
-void note_launch() { ++g_launches; }
-void reset_launches() { g_launches = 0; }
+// Per-host-thread launch bookkeeping and the optional per-kernel timer.
+namespace {
+constexpr int kMaxTimed = 4096;
+struct TimedLaunch {
+  const char *name;
+  cudaEvent_t start, stop;
+};
+struct LaunchLog {
+  int32_t launches = 0;
+  bool timing = false;
+  int n = 0;           // recorded launches since the last read
+  int n_events = 0;    // events created so far (reused across reads)
+  TimedLaunch rec[kMaxTimed];
+};
+thread_local LaunchLog g_log;
+}  // namespace
+
+void launch_begin(const char *name, cudaStream_t s) {
+  LaunchLog &L = g_log;
+  if (!L.timing || L.n >= kMaxTimed) return;
+  TimedLaunch &t = L.rec[L.n];
+  if (L.n >= L.n_events) {
+    if (cudaEventCreate(&t.start) != cudaSuccess ||
+        cudaEventCreate(&t.stop) != cudaSuccess)
+      return;
+    ++L.n_events;
+  }
+  t.name = name;
+  cudaEventRecord(t.start, s);
+}
+
+void launch_end(cudaStream_t s) {
+  LaunchLog &L = g_log;
+  ++L.launches;
+  if (!L.timing || L.n >= kMaxTimed || L.n >= L.n_events) return;
+  cudaEventRecord(L.rec[L.n].stop, s);
+  ++L.n;
+}
+
+void reset_launches() { g_log.launches = 0; }
 
 static pair_status check_device() {
   static int cached_dev = -1;
@@ -150,6 +187,25 @@ const char *pair_status_string(pair_status st) {
   return "unknown status";
 }
 
-int32_t pair_last_launch_count(void) { return g_launches; }
+int32_t pair_last_launch_count(void) { return g_log.launches; }
+
+void pair_timing_enable(int32_t on) {
+  g_log.timing = on != 0;
+  g_log.n = 0;
+}
+
+int32_t pair_timing_read(int32_t max, float *ms, const char **names) {
+  LaunchLog &L = g_log;
+  const int n = L.n < max ? L.n : max;
+  for (int i = 0; i < n; ++i) {
+    float t = -1.f;
+    if (cudaEventSynchronize(L.rec[i].stop) == cudaSuccess)
+      cudaEventElapsedTime(&t, L.rec[i].start, L.rec[i].stop);
+    if (ms) ms[i] = t;
+    if (names) names[i] = L.rec[i].name;
+  }
+  L.n = 0;
+  return n;
+}
 
 }  // extern "C"

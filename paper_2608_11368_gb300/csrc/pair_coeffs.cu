@@ -259,10 +259,11 @@ pair_status launch_coeffs_gp(int32_t B, int32_t G, const float *r,
   PAIR_CUDA_TRY(cudaFuncSetAttribute(coeffs_kernel<GP>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)smem));
+  PAIR_BEGIN("coeffs", s);
   coeffs_kernel<GP><<<B, GP, smem, s>>>(B, G, r, J, rho, scale,
                                         (flags & PAIR_CENTER) ? 1 : 0, a,
                                         active, edges, contrast, dev_err);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
 
@@ -275,9 +276,10 @@ pair_status launch_dense_gp(int32_t B, int32_t G, int32_t D, const float *r,
   PAIR_CUDA_TRY(cudaFuncSetAttribute(dense_kernel<GP>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)smem));
+  PAIR_BEGIN("dense", s);
   dense_kernel<GP><<<B, 256, smem, s>>>(B, G, D, r, J, rho, S, scale, g, a,
                                         dev_err);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
 

@@ -10,8 +10,11 @@ namespace pairk {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
-// Counts kernel launches of the current entry-point call (per host thread).
-void note_launch();
+// Launch bookkeeping (per host thread): counts the kernels of the current
+// entry-point call and, when timing is enabled, brackets each launch with
+// CUDA events on its stream.
+void launch_begin(const char *name, cudaStream_t s);
+void launch_end(cudaStream_t s);
 void reset_launches();
 
 __device__ __forceinline__ void flag_error(int32_t *err, int bit) {
@@ -89,9 +92,11 @@ pair_status grad_onehot(const GradArgs &g, const GradWorkspace &w,
     if (e_ != cudaSuccess) return PAIR_ERR_CUDA;              \
   } while (0)
 
-#define PAIR_LAUNCH_CHECK()                                   \
+#define PAIR_BEGIN(name, s) ::pairk::launch_begin(name, s)
+
+#define PAIR_LAUNCH_CHECK(s)                                  \
   do {                                                        \
-    ::pairk::note_launch();                                   \
+    ::pairk::launch_end(s);                                   \
     cudaError_t e_ = cudaGetLastError();                      \
     if (e_ != cudaSuccess) return PAIR_ERR_CUDA;              \
   } while (0)

@@ -294,15 +294,19 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
 
 pair_status grad_prepare(const GradArgs &g, const GradWorkspace &w,
                          cudaStream_t s) {
+  PAIR_BEGIN("seg_count", s);
   seg_count_kernel<<<g.R, 256, 0, s>>>(g.R, (int)g.T, g.V, g.cu, g.mask, g.y,
                                        g.a, w.seg_cnt, g.dev_err);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("seg_scan", s);
   seg_scan_kernel<<<1, 1024, 0, s>>>(g.R, w.seg_cnt, w.seg_off, w.counters);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("gather", s);
   gather_kernel<<<g.R, 256, 0, s>>>(g.R, (int)g.T, g.cu, g.mask, g.y, g.a,
                                     w.seg_off, w.tok_idx, w.tok_y, w.tok_c);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
   const int rows_grid = 152 * 16;
+  PAIR_BEGIN("copy_rows", s);
   if (g.dt == PAIR_BF16)
     copy_rows_kernel<uint16_t><<<rows_grid, 128, 0, s>>>(
         w.Tpad, g.d, w.counters, w.tok_idx,
@@ -311,20 +315,23 @@ pair_status grad_prepare(const GradArgs &g, const GradWorkspace &w,
     copy_rows_kernel<float><<<rows_grid, 128, 0, s>>>(
         w.Tpad, g.d, w.counters, w.tok_idx, static_cast<const float *>(g.H),
         static_cast<float *>(w.Hc));
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("zero_inactive", s);
   zero_inactive_rows_kernel<<<rows_grid, 128, 0, s>>>(g.T, g.d, g.R, g.cu,
                                                       g.mask, g.a, g.dH);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
 
 pair_status grad_finalize(const GradArgs &g, const GradWorkspace &w,
                           cudaStream_t s) {
+  PAIR_BEGIN("seg_logp", s);
   seg_logp_kernel<<<g.R, 256, 0, s>>>(g.R, w.seg_off, w.zy, w.lse, w.seg_logp);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("objective", s);
   objective_kernel<<<1, 1024, 0, s>>>(g.R, g.a, w.seg_logp, g.Jobj,
                                       g.logp_seq);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
 
@@ -334,22 +341,26 @@ pair_status grad_onehot(const GradArgs &g, const GradWorkspace &w,
   const int warps = (int)ceil_div(g.V, bucket);
   if (g.dt == PAIR_BF16) {
     const __nv_bfloat16 *W = static_cast<const __nv_bfloat16 *>(g.W);
+    PAIR_BEGIN("onehot_dh", s);
     onehot_dh_kernel<__nv_bfloat16><<<152 * 16, 256, 0, s>>>(
         g.d, w.counters, w.tok_idx, w.tok_y, w.tok_c, W, g.dH);
-    PAIR_LAUNCH_CHECK();
+    PAIR_LAUNCH_CHECK(s);
+    PAIR_BEGIN("onehot_dw", s);
     onehot_dw_kernel<__nv_bfloat16><<<(int)ceil_div(warps, 8), 256, 0, s>>>(
         g.d, g.V, bucket, w.counters, w.tok_y, w.tok_c,
         static_cast<const __nv_bfloat16 *>(w.Hc), g.dW);
-    PAIR_LAUNCH_CHECK();
+    PAIR_LAUNCH_CHECK(s);
   } else {
+    PAIR_BEGIN("onehot_dh", s);
     onehot_dh_kernel<float><<<152 * 16, 256, 0, s>>>(
         g.d, w.counters, w.tok_idx, w.tok_y, w.tok_c,
         static_cast<const float *>(g.W), g.dH);
-    PAIR_LAUNCH_CHECK();
+    PAIR_LAUNCH_CHECK(s);
+    PAIR_BEGIN("onehot_dw", s);
     onehot_dw_kernel<float><<<(int)ceil_div(warps, 8), 256, 0, s>>>(
         g.d, g.V, bucket, w.counters, w.tok_y, w.tok_c,
         static_cast<const float *>(w.Hc), g.dW);
-    PAIR_LAUNCH_CHECK();
+    PAIR_LAUNCH_CHECK(s);
   }
   return PAIR_OK;
 }

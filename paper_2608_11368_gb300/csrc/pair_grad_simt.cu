@@ -146,17 +146,20 @@ pair_status grad_head_simt(const GradArgs &g, const GradWorkspace &w,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2));
   PAIR_CUDA_TRY(cudaFuncSetAttribute(simt_dw_kernel,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2));
+  PAIR_BEGIN("simt_lse", s);
   simt_lse_kernel<<<grid, kWarps * 32, sm1, s>>>(g.d, g.V, w.counters, Hc, W,
                                                  w.tok_y, w.lse, w.zy);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("simt_dh", s);
   simt_dh_kernel<<<grid, kWarps * 32, sm2, s>>>(g.d, g.V, w.counters,
                                                 w.tok_idx, Hc, W, w.tok_y,
                                                 w.tok_c, w.lse, g.dH);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
   const int gridv = (int)(g.V < 152 * 16 ? g.V : 152 * 16);
+  PAIR_BEGIN("simt_dw", s);
   simt_dw_kernel<<<gridv, kWarps * 32, sm2, s>>>(g.d, g.V, w.counters, Hc, W,
                                                  w.tok_y, w.tok_c, w.lse, g.dW);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
 

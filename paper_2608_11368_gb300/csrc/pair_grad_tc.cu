@@ -592,21 +592,25 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
   PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_kernel<false>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bwd_smem));
 
+  PAIR_BEGIN("lse_tc", s);
   lse_kernel<<<nsm, kThreads, lse_smem, s>>>(mH, mW256, g.d, g.V, w.nsplit,
                                              w.Tpad, w.counters, w.tok_y,
                                              w.part, w.zy, g.dev_err);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("lse_combine", s);
   lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters,
                                              w.part, w.lse);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("bwd_dh_tc", s);
   bwd_kernel<true><<<nsm, kThreads, bwd_smem, s>>>(
       mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
       g.dev_err);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("bwd_dw_tc", s);
   bwd_kernel<false><<<nsm, kThreads, bwd_smem, s>>>(
       mW128, mH, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
       g.dev_err);
-  PAIR_LAUNCH_CHECK();
+  PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
 
