@@ -53,6 +53,10 @@ def parse_args():
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-stress", action="store_true")
+    # Smaller variants of the workload, for profiling captures only.
+    p.add_argument("--workload", default=WORKLOAD,
+                   choices=["qwen3_1p7b_head", "qwen3_4b_head", "longctx_skew"])
+    p.add_argument("--len-scale", type=float, default=1.0)
     return p.parse_args()
 
 
@@ -257,8 +261,8 @@ def main():
 
     peaks = load_peaks()
     traffic = load_traffic()
-    wl = synth.WORKLOADS[WORKLOAD]
-    inp = synth.make_head_workload(wl, args.seed + rank)
+    wl = synth.WORKLOADS[args.workload]
+    inp = synth.make_head_workload(wl, args.seed + rank, len_scale=args.len_scale)
     T, d, V, R = inp["T"], inp["d"], inp["V"], inp["R"]
 
     def pinned(x):
@@ -344,7 +348,7 @@ def main():
     roofline = {"kernel": dominant, "bound": "tensor",
                 "achieved": achieved, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
                 "frac": (achieved / peaks["bf16_sus"]) if achieved else None,
-                "traffic": traffic.get((dominant, WORKLOAD)),
+                "traffic": traffic.get((dominant, args.workload)),
                 "peak_source": peaks["src"] + " sustained bf16 (kernel timed inside a long step)",
                 "algorithmic_flops_per_launch": dom_flops,
                 "avg_launch_ms": dom_avg}
@@ -395,7 +399,8 @@ def main():
         "ms_per_step": total_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; Qwen3-1.7B head shapes, random-init weights)",
-        "config": {"workload": WORKLOAD, "d": d, "V": V,
+        "config": {"workload": args.workload, "len_scale": args.len_scale,
+                   "d": d, "V": V,
                    "global_batch": wl.B * wl.G * world, "prompts": wl.B * world,
                    "rollouts_per_prompt": wl.G, "tokens_packed": T,
                    "tokens_active": T_eff,
