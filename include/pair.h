@@ -184,6 +184,38 @@ PAIR_API pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
                       size_t ws_bytes, int32_t *dev_err, pair_stream_t stream);
 
 /*
+ * pair_grad_noalloc -- pair_grad without a caller-provided workspace, for
+ * callers that cannot allocate device memory: for example a plug-in that
+ * runs inside a host application which owns every device allocation and
+ * exposes no allocator to it, or code that must not call cudaMalloc
+ * because of the device-wide synchronisation and the out-of-memory failure
+ * mode that an allocation brings. The paper has no counterpart; this is a
+ * deployment convenience around the same kernels.
+ *
+ * Arguments, outputs and numerics are those of pair_grad, minus ws and
+ * ws_bytes. The workspace is a file-scope device array of
+ * PAIR_NOALLOC_MAX_WORKSPACE bytes that every GPU loading this library
+ * holds until the process exits; problems whose
+ * pair_grad_workspace_size(...) exceeds it are rejected with
+ * PAIR_ERR_WORKSPACE before any launch. The call allocates nothing.
+ * The first call on each device looks up the array's device address (with
+ * that device current) and caches it; make that first call before any
+ * stream capture. All calls on a device share the one array, which keeps
+ * the previous call's contents (pair_grad needs no zeroed workspace): calls
+ * whose executions overlap on the GPU (different streams, or host threads
+ * without ordering) race on it and must be serialised by the caller.
+ */
+#define PAIR_NOALLOC_MAX_WORKSPACE (32u << 20)
+PAIR_API pair_status pair_grad_noalloc(int64_t T, int32_t d, int32_t V,
+                                       pair_dtype dt, const void *H,
+                                       const void *W, const int32_t *y,
+                                       const uint8_t *mask,
+                                       const int32_t *cu_seqlens, int32_t R,
+                                       const float *a, float *dH, float *dW,
+                                       double *Jobj, float *logp_seq,
+                                       int32_t *dev_err, pair_stream_t stream);
+
+/*
  * pair_status_sync -- synchronise `stream`, read the device error word
  * (if non-null), reset it to 0, and return the status it encodes
  * (PAIR_ERR_DEVICE_TIMEOUT, then PAIR_ERR_NONPOSITIVE_INCLUSION, then

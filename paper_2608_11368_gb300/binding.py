@@ -63,6 +63,9 @@ def lib() -> ctypes.CDLL:
     L.pair_status_string.restype = ctypes.c_char_p
     L.pair_last_launch_count.argtypes = []
     L.pair_last_launch_count.restype = I32
+    L.pair_grad_noalloc.argtypes = [I64, I32, I32, ctypes.c_int, P, P, P, P, P,
+                                    I32, P, P, P, P, P, P, P]
+    L.pair_grad_noalloc.restype = ctypes.c_int
     L.pair_timing_enable.argtypes = [I32]
     L.pair_timing_enable.restype = None
     L.pair_timing_read.argtypes = [I32, P, P]
@@ -203,6 +206,38 @@ def pair_grad(H, W, y, mask, cu_seqlens, a, dH=None, dW=None, Jobj=None,
                          _p(logp_seq), _p(ws), ws.numel(), _p(dev_err),
                          _stream(stream))
     _check(st, "pair_grad")
+    return Jobj, dH, dW, logp_seq
+
+
+NOALLOC_MAX_WORKSPACE = 32 << 20
+
+
+def pair_grad_noalloc(H, W, y, mask, cu_seqlens, a, dH=None, dW=None,
+                      Jobj=None, logp_seq=None, dev_err=None, stream=None):
+    """pair_grad on the library's fixed device workspace (no workspace
+    argument; see pair.h for the size limit and the sharing rules).
+    Output tensors not passed in are allocated here by torch, as in
+    pair_grad; pass them to keep the call allocation-free.
+    Returns (Jobj, dH, dW, logp_seq)."""
+    T, d = H.shape
+    V = W.shape[0]
+    R = cu_seqlens.numel() - 1
+    dt = _pair_dtype(H)
+    _need(W, "W", H.dtype, (V, d))
+    _need(y, "y", torch.int32, (T,))
+    _need(mask, "mask", torch.uint8, (T,))
+    _need(cu_seqlens, "cu_seqlens", torch.int32, (R + 1,))
+    _need(a, "a", torch.float32, (R,))
+    dev = H.device
+    dH = torch.empty((T, d), dtype=torch.float32, device=dev) if dH is None else dH
+    dW = torch.empty((V, d), dtype=torch.float32, device=dev) if dW is None else dW
+    Jobj = torch.empty(1, dtype=torch.float64, device=dev) if Jobj is None else Jobj
+    logp_seq = torch.empty(R, dtype=torch.float32, device=dev) if logp_seq is None else logp_seq
+    st = lib().pair_grad_noalloc(T, d, V, dt, _p(H), _p(W), _p(y), _p(mask),
+                                 _p(cu_seqlens), R, _p(a), _p(dH), _p(dW),
+                                 _p(Jobj), _p(logp_seq), _p(dev_err),
+                                 _stream(stream))
+    _check(st, "pair_grad_noalloc")
     return Jobj, dH, dW, logp_seq
 
 

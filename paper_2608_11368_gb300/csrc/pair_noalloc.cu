@@ -1,0 +1,91 @@
+// pair_grad_noalloc: pair_grad for callers that cannot allocate device
+// memory. Its workspace is a fixed array in this library's device data
+// instead of a caller-provided buffer; everything else is the pair_grad
+// launch sequence, unchanged.
+#include <mutex>
+
+#include "pair_common.cuh"
+
+namespace pairk {
+namespace {
+
+constexpr size_t kStaticScratchBytes = PAIR_NOALLOC_MAX_WORKSPACE;
+
+// Workspace shared by every pair_grad_noalloc call on a device. Each GPU
+// that loads this library holds one copy until the process exits.
+static __device__ __align__(256) unsigned char g_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 128;
+std::mutex g_scratch_mu;
+void *g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_scratch on the current device. The host-side name of
+// a __device__ array is only a stand-in, so the address is looked up once
+// per device (with that device current) and cached.
+pair_status scratch_address(void **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return PAIR_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return PAIR_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_addr[dev]) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || !p)
+      return PAIR_ERR_CUDA;
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return PAIR_OK;
+}
+
+}  // namespace
+}  // namespace pairk
+
+using namespace pairk;
+
+extern "C" pair_status pair_grad_noalloc(
+    int64_t T, int32_t d, int32_t V, pair_dtype dt, const void *H,
+    const void *W, const int32_t *y, const uint8_t *mask,
+    const int32_t *cu_seqlens, int32_t R, const float *a, float *dH,
+    float *dW, double *Jobj, float *logp_seq, int32_t *dev_err,
+    pair_stream_t stream) {
+  reset_launches();
+  if (!H || !W || !y || !mask || !cu_seqlens || !a || !dH || !dW || !Jobj)
+    return PAIR_ERR_INVALID_ARG;
+  const size_t need = pair_grad_workspace_size(T, d, V, R, dt);
+  if (need == 0)
+    return (dt == PAIR_BF16 && d % 64 != 0 && d % 16 == 0)
+               ? PAIR_ERR_UNSUPPORTED
+               : PAIR_ERR_INVALID_ARG;
+  if (need > kStaticScratchBytes) return PAIR_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(H) & 15u) || (reinterpret_cast<uintptr_t>(W) & 15u) ||
+      (reinterpret_cast<uintptr_t>(dH) & 15u) || (reinterpret_cast<uintptr_t>(dW) & 15u))
+    return PAIR_ERR_INVALID_ARG;
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+    return PAIR_ERR_CUDA;
+  if (major != 10 || minor != 3) return PAIR_ERR_UNSUPPORTED;
+  void *ws = nullptr;
+  const pair_status sa = scratch_address(&ws);
+  if (sa != PAIR_OK) return sa;
+
+  // The workspace needs no initial contents: every kernel writes the parts
+  // it later reads within the same call.
+  GradWorkspace w;
+  grad_workspace_bytes(T, d, V, R, dt, &w, ws);
+  GradArgs g{T, d, V, R, dt, H, W, y, mask, cu_seqlens, a,
+             dH, dW, Jobj, logp_seq, dev_err};
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  pair_status st = grad_prepare(g, w, s);
+  if (st != PAIR_OK) return st;
+  if (dt == PAIR_BF16) {
+    st = grad_head_tc(g, w, s);
+    if (st != PAIR_OK) return st;
+    st = grad_onehot(g, w, s);
+  } else {
+    st = grad_head_simt(g, w, s);
+  }
+  if (st != PAIR_OK) return st;
+  return grad_finalize(g, w, s);
+}
