@@ -8,6 +8,11 @@
 
 namespace pairk {
 
+// Clusters the cluster backward may run at once (ring buffers are sized for
+// this many); each ring holds 8 owners x 2 tiles x 32 KB.
+constexpr int kMaxClusters = 24;
+constexpr size_t kRingBytesPerCluster = 8 * 2 * 32768;
+
 constexpr float kLog2e = 1.4426950408889634f;
 
 // Launch bookkeeping (per host thread): counts the kernels of the current
@@ -50,6 +55,7 @@ struct GradWorkspace {
   float2 *part;        // [nsplit][Tpad] partial (max, sum-exp) per split
   double *seg_logp;    // [R] per-rollout sum of logp (fp64)
   void *Hc;            // [Tpad][d] compacted hidden rows (dt), zero tail
+  void *gring;         // per-cluster ring of published Gs tiles
   int64_t Tpad;
   int nsplit;
 };

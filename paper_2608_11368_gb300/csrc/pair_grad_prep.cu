@@ -272,6 +272,7 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   const size_t o_part = take((size_t)kNSplit * Tpad * sizeof(float2));
   const size_t o_segl = take((size_t)R * 8);
   const size_t o_hc = take((size_t)Tpad * d * esz);
+  const size_t o_ring = dt == PAIR_BF16 ? take((size_t)kMaxClusters * kRingBytesPerCluster) : off;
   if (out) {
     char *b = static_cast<char *>(base);
     out->counters = reinterpret_cast<int32_t *>(b + o_cnt);
@@ -285,6 +286,7 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->part = reinterpret_cast<float2 *>(b + o_part);
     out->seg_logp = reinterpret_cast<double *>(b + o_segl);
     out->Hc = b + o_hc;
+    out->gring = b + o_ring;
     out->Tpad = Tpad;
     out->nsplit = kNSplit;
   }

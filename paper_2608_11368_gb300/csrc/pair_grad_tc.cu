@@ -533,6 +533,376 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ------------------------------------------------- backward, cluster form
+//
+// One 8-CTA cluster owns a row block (128 tokens for dH, 128 vocabulary rows
+// for dW); CTA k of the cluster keeps out[rows, k*w : (k+1)*w] (w = d/8) in
+// TMEM for the whole unit, so each logit-gradient tile Gs is formed once per
+// cluster instead of once per d-slice.
+//
+// Tile ownership rotates: the owner of column tile g (g mod 8) accumulates
+// the full-depth S tile in TMEM, spread evenly over the 8 slots that end
+// kClLag slots before the tile is used (d/512 K-atoms per slot), converts it
+// to bf16 Gs and publishes the 32 KB tile (already in the swizzled K-major
+// layout of the MMA operand) once, to a per-cluster ring in global memory,
+// then signals every CTA of the cluster through its pub[owner] mbarrier.
+// Every CTA pulls Gs(s) into one of its two shared-memory slots with a bulk
+// copy and updates out += Gs(s) . C[s, slice]. The exchange goes through L2
+// because distributed shared memory sustains far less per-SM egress than a
+// broadcast of a 32 KB tile to 7 peers per slot needs. In every slot every
+// CTA issues the same tensor work: a share of one S accumulation plus one
+// output update. The slot counter runs across units, so the staggered S
+// schedule never drains at unit boundaries.
+constexpr int kCl = 8;          // cluster size
+constexpr int kClBN = 128;      // column tile
+constexpr int kClStages = 3;
+constexpr int kClLag = 2;       // slots between an S tile's completion and its use
+constexpr int kClJ = kCl + kClLag;
+constexpr uint32_t kGsBytes = 2 * kAtom128;   // one Gs tile (128 x 128 bf16)
+constexpr uint32_t kIdescClS = idesc_bf16(128, kClBN, 0, 0);
+
+struct ClSmem {
+  uint8_t a[kClStages][kAtom128];
+  uint8_t b[kClStages][kAtom128];
+  uint8_t cs[4][kAtom128];           // C[s, slice] (MN-major B, <= 4 atoms)
+  uint8_t g[2][2][kAtom128];         // Gs slots: 128 x 128 bf16 (2 K-atoms)
+  float col_c[kClBN], col_l[kClBN];
+  uint64_t full[kClStages], empty[kClStages];
+  uint64_t s_full[2], s_empty[2];
+  uint64_t g_full[2], gs_empty[2];   // local Gs slots
+  uint64_t pub[kCl];                 // owner o published its next tile
+  uint64_t gfree[2];                 // (owner) all CTAs done with its tile m (by m & 1)
+  uint64_t cs_full, cs_empty, o_full, o_empty, mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ int pmod(int a, int m) {
+  const int r = a % m;
+  return r < 0 ? r + m : r;
+}
+
+// Bulk copy global -> this CTA's shared memory, completing on `bar`.
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes,
+                                          uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes "
+      "[%0], [%1], %2, [%3];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+template <bool kTokenRows>
+__global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
+    bwd_cluster_kernel(const __grid_constant__ CUtensorMap tmR,
+                       const __grid_constant__ CUtensorMap tmC, int d, int V,
+                       const int32_t *counters, const int32_t *tok_idx,
+                       const float *tok_c, const float *lse, float *out,
+                       uint8_t *gring, int32_t *dev_err) {
+  extern __shared__ uint8_t smem_raw[];
+  ClSmem &sm = *reinterpret_cast<ClSmem *>(align1k(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int k = (int)cluster_rank();
+  const int cid = (int)cluster_id_x(), ncl = (int)num_clusters_x();
+  const int Teff = counters[0];
+  const int A = d / (64 * kCl);            // K-atoms per slot (d / 512)
+  const int w = 64 * A;                    // this CTA's d-slice width
+  const int nk = d / 64;
+  const int n_rb = kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128;
+  const int n_ct = kTokenRows ? (V + kClBN - 1) / kClBN : (Teff + kClBN - 1) / kClBN;
+  const int n_my = cid < n_rb ? (n_rb - cid + ncl - 1) / ncl : 0;
+  const long long N = (long long)n_my * n_ct;   // global tiles of this cluster
+  // Ring of published Gs tiles: [owner][job parity] for this cluster.
+  uint8_t *ring = gring + (size_t)cid * kCl * 2 * kGsBytes;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kClStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.s_full[s], 1);
+      mbar_init(&sm.s_empty[s], 128);
+      mbar_init(&sm.g_full[s], 1);
+      mbar_init(&sm.gs_empty[s], 1);
+      mbar_init(&sm.gfree[s], kCl);
+    }
+    for (int o = 0; o < kCl; ++o) mbar_init(&sm.pub[o], 1);
+    mbar_init(&sm.cs_full, 1);
+    mbar_init(&sm.cs_empty, 1);
+    mbar_init(&sm.o_full, 1);
+    mbar_init(&sm.o_empty, 128);
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmR);
+    prefetch_tmap(&tmC);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // every CTA's barriers exist before anyone signals them
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  const uint32_t tmem_o = tmem + 2 * kClBN;
+  volatile int *abort = &sm.abort;
+
+  auto rb_of = [&](long long g) { return cid + (int)(g / n_ct) * ncl; };
+  auto ct_of = [&](long long g) { return (int)(g % n_ct); };
+  // The tile whose S this CTA accumulates during slot s (may be < 0 or >= N).
+  auto job_of = [&](long long s) {
+    return s + kClLag + 1 + pmod(k - (int)((s + kClLag + 1) % kCl), kCl);
+  };
+  auto ring_tile = [&](long long g) {
+    return ring + ((size_t)(g % kCl) * 2 + (size_t)((g / kCl) & 1)) * kGsBytes;
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0, cs_ph = 0, ge_ph[2] = {0, 0};
+      int last_ph[kClStages], g_last[2] = {-1, -1};
+      for (int s = 0; s < kClStages; ++s) last_ph[s] = -1;
+      int cs_last = -1;
+      bool ok = true;
+      for (long long s = -kClJ; s < N && ok; ++s) {
+        const long long gj = job_of(s);
+        if (gj >= 0 && gj < N) {
+          const int rb = rb_of(gj), ct = ct_of(gj);
+          const int a0 = (int)(s - (gj - kClJ)) * A;
+          for (int a = a0; a < a0 + A; ++a) {
+            if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+            mbar_expect_tx(&sm.full[stage], 2 * kAtom128);
+            tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, rb * 128);
+            tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], a * 64, ct * kClBN);
+            last_ph[stage] = (int)ph;
+            if (++stage == kClStages) { stage = 0; ph ^= 1; }
+          }
+        }
+        if (!ok || s < 0) continue;
+        // Output operand C[s, slice].
+        if (!(ok = wait(&sm.cs_empty, cs_ph ^ 1, abort, dev_err))) break;
+        mbar_expect_tx(&sm.cs_full, (uint32_t)A * kAtom128);
+        const int ct = ct_of(s);
+        for (int j = 0; j < A; ++j)
+          tma_load_2d(sm.cs[j], &tmC, &sm.cs_full, k * w + j * 64, ct * kClBN);
+        cs_last = (int)cs_ph;
+        cs_ph ^= 1;
+        // Gs(s): published by its owner, pulled into local slot s & 1.
+        const int slot = (int)(s & 1);
+        if (!(ok = wait_cluster(&sm.pub[s % kCl], (uint32_t)((s / kCl) & 1), abort, dev_err)))
+          break;
+        fence_proxy_async_global();
+        if (!(ok = wait(&sm.gs_empty[slot], ge_ph[slot] ^ 1, abort, dev_err))) break;
+        ge_ph[slot] ^= 1;
+        mbar_expect_tx(&sm.g_full[slot], kGsBytes);
+        bulk_load(sm.g[slot][0], ring_tile(s), kGsBytes, &sm.g_full[slot]);
+        g_last[slot] = (int)((s >> 1) & 1);
+      }
+      // Never leave a copy in flight: wait (bounded) for the last one issued
+      // on every buffer.
+      volatile int never = 0;
+      for (int s = 0; s < kClStages; ++s)
+        if (last_ph[s] >= 0) wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+      if (cs_last >= 0) wait(&sm.cs_full, (uint32_t)cs_last, &never, dev_err);
+      for (int sl = 0; sl < 2; ++sl)
+        if (g_last[sl] >= 0) wait(&sm.g_full[sl], (uint32_t)g_last[sl], &never, dev_err);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0, cs_ph = 0, o_ph = 0, s_ph[2] = {0, 0}, g_ph[2] = {0, 0};
+      const uint32_t idesc_o = idesc_bf16(128, w, 0, 1);
+      bool ok = true;
+      for (long long s = -kClJ; s < N && ok; ++s) {
+        const long long gj = job_of(s);
+        if (gj >= 0 && gj < N) {
+          const int buf = (int)((gj / kCl) & 1);
+          const int a0 = (int)(s - (gj - kClJ)) * A;
+          if (a0 == 0) {
+            if (!(ok = wait(&sm.s_empty[buf], s_ph[buf] ^ 1, abort, dev_err))) break;
+            tc_fence_after();
+          }
+          const uint32_t dt = tmem + buf * kClBN;
+          for (int a = a0; a < a0 + A; ++a) {
+            if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+            tc_fence_after();
+            const uint32_t sa = smem_u32(sm.a[stage]), sb = smem_u32(sm.b[stage]);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_bf16(dt, sdesc_sw128(sa + kk * 32, 16, 1024),
+                       sdesc_sw128(sb + kk * 32, 16, 1024), kIdescClS,
+                       (a | kk) != 0);
+            mma_commit(&sm.empty[stage]);
+            if (++stage == kClStages) { stage = 0; ph ^= 1; }
+          }
+          if (!ok) break;
+          if (a0 + A == nk) {
+            mma_commit(&sm.s_full[buf]);
+            s_ph[buf] ^= 1;
+          }
+        }
+        if (s < 0) continue;
+        const int ct = ct_of(s), slot = (int)(s & 1);
+        if (ct == 0 && !(ok = wait(&sm.o_empty, o_ph ^ 1, abort, dev_err))) break;
+        if (!(ok = wait(&sm.g_full[slot], g_ph[slot], abort, dev_err))) break;
+        g_ph[slot] ^= 1;
+        if (!(ok = wait(&sm.cs_full, cs_ph, abort, dev_err))) break;
+        cs_ph ^= 1;
+        tc_fence_after();
+        const uint32_t sg = smem_u32(sm.g[slot][0]), sc = smem_u32(sm.cs[0]);
+#pragma unroll
+        for (int kk = 0; kk < kClBN / 16; ++kk)
+          mma_bf16(tmem_o,
+                   sdesc_sw128(sg + (kk >> 2) * kAtom128 + (kk & 3) * 32, 16, 1024),
+                   sdesc_sw128(sc + kk * 2048, kAtom128, 1024), idesc_o,
+                   (ct | kk) != 0);
+        mma_commit(&sm.cs_empty);
+        mma_commit(&sm.gs_empty[slot]);
+        // Tell the owner of s that this CTA is done with tile s. The owner
+        // publishes its next tile (s + 8) only after all 8 CTAs are, so no
+        // pub[] phase can run ahead of a consumer still waiting on the
+        // previous one, and ring slot reuse (tile s + 16) is safe.
+        if (s + kCl < N)
+          mma_commit_multicast(&sm.gfree[(s / kCl) & 1], (uint16_t)(1u << (int)(s % kCl)));
+        if (ct == n_ct - 1) {
+          mma_commit(&sm.o_full);
+          o_ph ^= 1;
+        }
+      }
+      mma_commit(&sm.mma_done);
+      volatile int never = 0;
+      wait(&sm.mma_done, 0, &never, dev_err);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    uint32_t sf_ph[2] = {0, 0}, free_ph[2] = {0, 0}, o_ph = 0;
+    bool ok = true;
+    for (long long s = -kClJ; s < N && ok; ++s) {
+      const long long g = s + kClLag + 1;  // tile whose S completes in slot s
+      if (g >= 0 && g < N && (int)(g % kCl) == k) {
+        const long long m = g / kCl;
+        const int buf = (int)(m & 1);
+        const int rb = rb_of(g), ct = ct_of(g);
+        float rc = 0.f, rl = 0.f;
+        if (kTokenRows) {
+          const int p = rb * 128 + row;
+          if (p < Teff) { rc = tok_c[p]; rl = lse[p] * kLog2e; }
+        } else {
+          epi_sync();
+          const int p = ct * kClBN + row;
+          sm.col_c[row] = p < Teff ? tok_c[p] : 0.f;
+          sm.col_l[row] = p < Teff ? lse[p] * kLog2e : 0.f;
+          epi_sync();
+        }
+        if (!(ok = wait(&sm.s_full[buf], sf_ph[buf], abort, dev_err))) break;
+        sf_ph[buf] ^= 1;
+        if (m >= 1) {
+          // Every CTA has finished with this owner's previous tile g - 8.
+          const int pb = (int)((m - 1) & 1);
+          if (!(ok = wait_cluster(&sm.gfree[pb], free_ph[pb], abort, dev_err))) break;
+          free_ph[pb] ^= 1;
+        }
+        tc_fence_after();
+        uint8_t *dst_tile = ring_tile(g);
+#pragma unroll 1
+        for (int c = 0; c < kClBN / 32; ++c) {
+          float v[32];
+          tmem_ld32(tmem + lane_off + buf * kClBN + c * 32, v);
+          uint32_t pk[16];
+#pragma unroll
+          for (int j = 0; j < 32; j += 2) {
+            float g2[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int col = c * 32 + j + e;
+              float cc, ll;
+              bool live;
+              if (kTokenRows) {
+                cc = rc; ll = rl;
+                live = (rc != 0.f) && (ct * kClBN + col < V);
+              } else {
+                cc = sm.col_c[col]; ll = sm.col_l[col];
+                live = cc != 0.f;
+              }
+              g2[e] = live ? -cc * exp2f(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
+            }
+            __nv_bfloat162 b2 = __floats2bfloat162_rn(g2[0], g2[1]);
+            pk[j >> 1] = *reinterpret_cast<uint32_t *>(&b2);
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int kc = c * 32 + q * 8;
+            uint8_t *dst = dst_tile + (kc >> 6) * kAtom128 + sw128_offset(row, kc & 63);
+            *reinterpret_cast<uint4 *>(dst) =
+                make_uint4(pk[q * 4], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
+          }
+        }
+        fence_proxy_async_global();
+        fence_acq_rel_cluster();
+        tc_fence_before();
+        mbar_arrive(&sm.s_empty[buf]);
+        epi_sync();
+        if (warp == 2 && lane == 0) {
+          fence_acq_rel_cluster();
+          const uint32_t pb = smem_u32(&sm.pub[k]);
+          for (int r = 0; r < kCl; ++r) mbar_arrive_cluster(mapa(pb, (uint32_t)r));
+        }
+      }
+      if (s >= 0 && ct_of(s) == n_ct - 1) {
+        // Drain the finished unit: out[rows, k*w : (k+1)*w].
+        if (!(ok = wait(&sm.o_full, o_ph, abort, dev_err))) break;
+        o_ph ^= 1;
+        tc_fence_after();
+        const int rb = rb_of(s);
+        const int rid = rb * 128 + row;
+        const bool valid = kTokenRows ? (rid < Teff) : (rid < V);
+        float *dst = nullptr;
+        if (valid)
+          dst = out + (kTokenRows ? (int64_t)tok_idx[rid] : (int64_t)rid) * d + k * w;
+#pragma unroll 1
+        for (int c = 0; c < w / 32; ++c) {
+          float v[32];
+          tmem_ld32(tmem_o + lane_off + c * 32, v);
+          if (valid) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              reinterpret_cast<float4 *>(dst + c * 32)[q] =
+                  make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(&sm.o_empty);
+      }
+    }
+    // No column tiles at all (no active token): the slice is zero.
+    if (ok && n_ct == 0) {
+      for (int j = 0; j < n_my; ++j) {
+        const int rid = (cid + j * ncl) * 128 + row;
+        if (!kTokenRows && rid < V)
+          for (int c = 0; c < w; ++c) out[(int64_t)rid * d + k * w + c] = 0.f;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while a peer may still signal its barriers
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
 // --------------------------------------------------------------- host side
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -573,6 +943,28 @@ int num_sms() {
   return n;
 }
 
+// The cluster backward needs d = 8 * 64 * A with 1 <= A <= 4 (each CTA's
+// output slice of 64 * A columns stays in TMEM beside the S buffers).
+bool use_cluster_path(int d) { return d % 512 == 0 && d >= 512 && d <= 2048; }
+
+// Clusters that fit at once (persistent grid), from the occupancy API.
+int cluster_grid(const void *kernel, size_t smem) {
+  static int cached = 0;
+  if (cached) return cached;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kCl * 64, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    n = num_sms() / kCl;
+  }
+  if (n > kMaxClusters) n = kMaxClusters;
+  cached = n > 0 ? n : 1;
+  return cached;
+}
+
 }  // namespace
 
 pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
@@ -602,6 +994,24 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
                                              w.part, w.lse);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("bwd_dh_tc", s);
+  if (use_cluster_path(g.d)) {
+    const size_t cl_smem = sizeof(ClSmem) + 1024;
+    PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<true>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
+    PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
+    const int ncl = cluster_grid((const void *)bwd_cluster_kernel<true>, cl_smem);
+    bwd_cluster_kernel<true><<<ncl * kCl, kThreads, cl_smem, s>>>(
+        mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
+        static_cast<uint8_t *>(w.gring), g.dev_err);
+    PAIR_LAUNCH_CHECK(s);
+    PAIR_BEGIN("bwd_dw_tc", s);
+    bwd_cluster_kernel<false><<<ncl * kCl, kThreads, cl_smem, s>>>(
+        mW128, mH, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
+        static_cast<uint8_t *>(w.gring), g.dev_err);
+    PAIR_LAUNCH_CHECK(s);
+    return PAIR_OK;
+  }
   bwd_kernel<true><<<nsm, kThreads, bwd_smem, s>>>(
       mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
       g.dev_err);

@@ -80,6 +80,11 @@ CASES = [
     ("qwen3_4b_head", 320, 777, 2, 6, 0.03, 8.0),        # two slices (256 + 64)
     ("longctx_skew", 64, 300, 4, 4, 0.02, 1.0),          # minimal d
     ("qwen3_4b_head", 2560, 4099, 2, 3, 0.05, 3.0),      # ten slices
+    # Cluster backward (d = 512 * A): slice widths 64, 128, 192, with
+    # ragged vocabulary tails and several row blocks per cluster.
+    ("qwen3_1p7b_head", 512, 1000, 3, 8, 0.3, 4.0),
+    ("longctx_skew", 1024, 5003, 2, 8, 0.15, 2.0),
+    ("qwen3_4b_head", 1536, 777, 2, 6, 0.08, 8.0),
 ]
 
 
