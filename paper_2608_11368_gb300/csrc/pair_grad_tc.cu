@@ -553,34 +553,32 @@ __global__ void __launch_bounds__(kThreads, 1)
 // CTA issues the same tensor work: a share of one S accumulation plus one
 // output update. The slot counter runs across units, so the staggered S
 // schedule never drains at unit boundaries.
-constexpr int kCl = 8;          // cluster size
-constexpr int kClBN = 128;      // column tile
-constexpr int kClStages = 3;
-constexpr int kClLag = 2;       // slots between an S tile's completion and its use
+constexpr int kCl = 8;          // cluster size (power of two)
+constexpr int kClBN = 128;      // column tile (S is 128 x 128)
+constexpr int kClStages = 3;    // S operand stages
+constexpr int kClLag = 3;       // slots between an S tile's completion and its use
 constexpr int kClJ = kCl + kClLag;
-constexpr uint32_t kGsBytes = 2 * kAtom128;   // one Gs tile (128 x 128 bf16)
+constexpr int kGSlots = 2;      // Gs tiles staged in shared memory
+constexpr int kClThreads = 224; // + warp 6: loads of C[s, slice] and Gs
+constexpr uint32_t kGsBytes = 128 * kClBN * 2; // one Gs tile (32 KB)
 constexpr uint32_t kIdescClS = idesc_bf16(128, kClBN, 0, 0);
 
 struct ClSmem {
-  uint8_t a[kClStages][kAtom128];
-  uint8_t b[kClStages][kAtom128];
-  uint8_t cs[4][kAtom128];           // C[s, slice] (MN-major B, <= 4 atoms)
-  uint8_t g[2][2][kAtom128];         // Gs slots: 128 x 128 bf16 (2 K-atoms)
+  uint8_t a[kClStages][kAtom128];    // rows operand atoms (128 x 64)
+  uint8_t b[kClStages][kAtom128];    // column operand atoms (128 x 64)
+  uint8_t cs[4][kAtom128];           // C[s, slice]: MN-major B, <= 4 atoms
+  uint8_t g[kGSlots][2][kAtom128];   // Gs tiles: 128 x 128 bf16, K-major A
   float col_c[kClBN], col_l[kClBN];
   uint64_t full[kClStages], empty[kClStages];
   uint64_t s_full[2], s_empty[2];
-  uint64_t g_full[2], gs_empty[2];   // local Gs slots
+  uint64_t g_full[kGSlots], gs_empty[kGSlots];
+  uint64_t cs_full, cs_empty;
   uint64_t pub[kCl];                 // owner o published its next tile
   uint64_t gfree[2];                 // (owner) all CTAs done with its tile m (by m & 1)
-  uint64_t cs_full, cs_empty, o_full, o_empty, mma_done;
+  uint64_t o_full, o_empty, mma_done;
   uint32_t tmem_base;
   int abort;
 };
-
-__device__ __forceinline__ int pmod(int a, int m) {
-  const int r = a % m;
-  return r < 0 ? r + m : r;
-}
 
 // Bulk copy global -> this CTA's shared memory, completing on `bar`.
 __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes,
@@ -596,8 +594,24 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
+// Walks global tile indices 0, 1, 2, ... of a cluster as (row block,
+// column tile) pairs without divisions in the loop.
+struct TileCursor {
+  int ct, rb;
+  int n_ct, ncl;
+  __device__ void init(int g, int cid, int n_ct_, int ncl_) {
+    n_ct = n_ct_;
+    ncl = ncl_;
+    ct = n_ct ? g % n_ct : 0;
+    rb = cid + (n_ct ? g / n_ct : 0) * ncl;
+  }
+  __device__ void next() {
+    if (++ct == n_ct) { ct = 0; rb += ncl; }
+  }
+};
+
 template <bool kTokenRows>
-__global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
     bwd_cluster_kernel(const __grid_constant__ CUtensorMap tmR,
                        const __grid_constant__ CUtensorMap tmC, int d, int V,
                        const int32_t *counters, const int32_t *tok_idx,
@@ -615,9 +629,17 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
   const int n_rb = kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128;
   const int n_ct = kTokenRows ? (V + kClBN - 1) / kClBN : (Teff + kClBN - 1) / kClBN;
   const int n_my = cid < n_rb ? (n_rb - cid + ncl - 1) / ncl : 0;
-  const long long N = (long long)n_my * n_ct;   // global tiles of this cluster
+  const int N = n_my * n_ct;               // global tiles of this cluster
   // Ring of published Gs tiles: [owner][job parity] for this cluster.
   uint8_t *ring = gring + (size_t)cid * kCl * 2 * kGsBytes;
+  auto ring_tile = [&](int g) {
+    return ring + ((size_t)(g & (kCl - 1)) * 2 + (size_t)((g >> 3) & 1)) * kGsBytes;
+  };
+  // The tile whose S this CTA accumulates during slot s (may be < 0 or >= N).
+  auto job_of = [&](int s) {
+    const int g0 = s + kClLag + 1;
+    return g0 + ((k - g0) & (kCl - 1));
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kClStages; ++s) {
@@ -627,13 +649,15 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
     for (int s = 0; s < 2; ++s) {
       mbar_init(&sm.s_full[s], 1);
       mbar_init(&sm.s_empty[s], 128);
-      mbar_init(&sm.g_full[s], 1);
-      mbar_init(&sm.gs_empty[s], 1);
       mbar_init(&sm.gfree[s], kCl);
     }
-    for (int o = 0; o < kCl; ++o) mbar_init(&sm.pub[o], 1);
+    for (int s = 0; s < kGSlots; ++s) {
+      mbar_init(&sm.g_full[s], 1);
+      mbar_init(&sm.gs_empty[s], 1);
+    }
     mbar_init(&sm.cs_full, 1);
     mbar_init(&sm.cs_empty, 1);
+    for (int o = 0; o < kCl; ++o) mbar_init(&sm.pub[o], 1);
     mbar_init(&sm.o_full, 1);
     mbar_init(&sm.o_empty, 128);
     mbar_init(&sm.mma_done, 1);
@@ -654,78 +678,92 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
   const uint32_t tmem_o = tmem + 2 * kClBN;
   volatile int *abort = &sm.abort;
 
-  auto rb_of = [&](long long g) { return cid + (int)(g / n_ct) * ncl; };
-  auto ct_of = [&](long long g) { return (int)(g % n_ct); };
-  // The tile whose S this CTA accumulates during slot s (may be < 0 or >= N).
-  auto job_of = [&](long long s) {
-    return s + kClLag + 1 + pmod(k - (int)((s + kClLag + 1) % kCl), kCl);
-  };
-  auto ring_tile = [&](long long g) {
-    return ring + ((size_t)(g % kCl) * 2 + (size_t)((g / kCl) & 1)) * kGsBytes;
-  };
-
   if (warp == 0) {
+    // Producer of the S operands (this CTA's share of its owned tiles).
     if (lane == 0) {
       int stage = 0;
-      uint32_t ph = 0, cs_ph = 0, ge_ph[2] = {0, 0};
-      int last_ph[kClStages], g_last[2] = {-1, -1};
+      uint32_t ph = 0;
+      int last_ph[kClStages];
       for (int s = 0; s < kClStages; ++s) last_ph[s] = -1;
-      int cs_last = -1;
       bool ok = true;
-      for (long long s = -kClJ; s < N && ok; ++s) {
-        const long long gj = job_of(s);
-        if (gj >= 0 && gj < N) {
-          const int rb = rb_of(gj), ct = ct_of(gj);
-          const int a0 = (int)(s - (gj - kClJ)) * A;
-          for (int a = a0; a < a0 + A; ++a) {
-            if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
-            mbar_expect_tx(&sm.full[stage], 2 * kAtom128);
-            tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, rb * 128);
-            tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], a * 64, ct * kClBN);
-            last_ph[stage] = (int)ph;
-            if (++stage == kClStages) { stage = 0; ph ^= 1; }
-          }
+      int job_rb = 0, job_ct = 0, job_g = -1;
+      for (int s = -kClJ; s < N && ok; ++s) {
+        const int gj = job_of(s);
+        if (gj < 0 || gj >= N) continue;
+        if (gj != job_g) {
+          TileCursor c;
+          c.init(gj, cid, n_ct, ncl);
+          job_rb = c.rb; job_ct = c.ct; job_g = gj;
         }
-        if (!ok || s < 0) continue;
-        // Output operand C[s, slice].
-        if (!(ok = wait(&sm.cs_empty, cs_ph ^ 1, abort, dev_err))) break;
-        mbar_expect_tx(&sm.cs_full, (uint32_t)A * kAtom128);
-        const int ct = ct_of(s);
-        for (int j = 0; j < A; ++j)
-          tma_load_2d(sm.cs[j], &tmC, &sm.cs_full, k * w + j * 64, ct * kClBN);
-        cs_last = (int)cs_ph;
-        cs_ph ^= 1;
-        // Gs(s): published by its owner, pulled into local slot s & 1.
-        const int slot = (int)(s & 1);
-        if (!(ok = wait_cluster(&sm.pub[s % kCl], (uint32_t)((s / kCl) & 1), abort, dev_err)))
-          break;
-        fence_proxy_async_global();
-        if (!(ok = wait(&sm.gs_empty[slot], ge_ph[slot] ^ 1, abort, dev_err))) break;
-        ge_ph[slot] ^= 1;
-        mbar_expect_tx(&sm.g_full[slot], kGsBytes);
-        bulk_load(sm.g[slot][0], ring_tile(s), kGsBytes, &sm.g_full[slot]);
-        g_last[slot] = (int)((s >> 1) & 1);
+        const int a0 = (s - (gj - kClJ)) * A;
+        for (int a = a0; a < a0 + A; ++a) {
+          if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+          mbar_expect_tx(&sm.full[stage], 2 * kAtom128);
+          tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, job_rb * 128);
+          tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], a * 64, job_ct * kClBN);
+          last_ph[stage] = (int)ph;
+          if (++stage == kClStages) { stage = 0; ph ^= 1; }
+        }
       }
-      // Never leave a copy in flight: wait (bounded) for the last one issued
-      // on every buffer.
       volatile int never = 0;
       for (int s = 0; s < kClStages; ++s)
         if (last_ph[s] >= 0) wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+    }
+  } else if (warp == 6) {
+    // Producer of the output-update operands: C[s, slice] and Gs(s).
+    if (lane == 0) {
+      uint32_t cs_ph = 0, ge_ph[kGSlots] = {};
+      int cs_last = -1, g_last[kGSlots];
+      for (int i = 0; i < kGSlots; ++i) g_last[i] = -1;
+      bool ok = true;
+      TileCursor cur;
+      cur.init(0, cid, n_ct, ncl);
+      for (int s = 0; s < N && ok; ++s, cur.next()) {
+        // Gs(s) from its owner's ring slot.
+        const int gb = s & (kGSlots - 1);
+        if (!(ok = wait_cluster(&sm.pub[s & (kCl - 1)], (uint32_t)((s >> 3) & 1), abort,
+                                dev_err)))
+          break;
+        fence_proxy_async_global();
+        if (!(ok = wait(&sm.gs_empty[gb], ge_ph[gb] ^ 1, abort, dev_err))) break;
+        mbar_expect_tx(&sm.g_full[gb], kGsBytes);
+        bulk_load(sm.g[gb][0], ring_tile(s), kGsBytes, &sm.g_full[gb]);
+        g_last[gb] = (int)ge_ph[gb];
+        ge_ph[gb] ^= 1;
+        // Output operand C[s, slice].
+        if (!(ok = wait(&sm.cs_empty, cs_ph ^ 1, abort, dev_err))) break;
+        mbar_expect_tx(&sm.cs_full, (uint32_t)A * kAtom128);
+        for (int j = 0; j < A; ++j)
+          tma_load_2d(sm.cs[j], &tmC, &sm.cs_full, k * w + j * 64, cur.ct * kClBN);
+        cs_last = (int)cs_ph;
+        cs_ph ^= 1;
+      }
+      volatile int never = 0;
       if (cs_last >= 0) wait(&sm.cs_full, (uint32_t)cs_last, &never, dev_err);
-      for (int sl = 0; sl < 2; ++sl)
-        if (g_last[sl] >= 0) wait(&sm.g_full[sl], (uint32_t)g_last[sl], &never, dev_err);
+      for (int i = 0; i < kGSlots; ++i)
+        if (g_last[i] >= 0) wait(&sm.g_full[i], (uint32_t)g_last[i], &never, dev_err);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       int stage = 0;
-      uint32_t ph = 0, cs_ph = 0, o_ph = 0, s_ph[2] = {0, 0}, g_ph[2] = {0, 0};
+      uint32_t ph = 0, o_ph = 0, cs_ph = 0, s_ph[2] = {0, 0}, g_ph[kGSlots] = {};
       const uint32_t idesc_o = idesc_bf16(128, w, 0, 1);
+      // Descriptors of every buffer, built once; K steps add to the start
+      // address field (16-byte units).
+      // Buffers of one kind are contiguous, so buffer i adds i times its
+      // size (in 16-byte units) to the base descriptor.
+      const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
+      const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 16, 1024);
+      const uint64_t dg0 = sdesc_sw128(smem_u32(sm.g[0][0]), 16, 1024);
+      const uint64_t dc = sdesc_sw128(smem_u32(sm.cs[0]), kAtom128, 1024);
+      constexpr uint32_t kAtomU = kAtom128 >> 4, kGsU = kGsBytes >> 4;
       bool ok = true;
-      for (long long s = -kClJ; s < N && ok; ++s) {
-        const long long gj = job_of(s);
+      int ct = 0;  // column tile of slot s (s >= 0)
+      for (int s = -kClJ; s < N && ok; ++s) {
+        const int gj = job_of(s);
         if (gj >= 0 && gj < N) {
-          const int buf = (int)((gj / kCl) & 1);
-          const int a0 = (int)(s - (gj - kClJ)) * A;
+          const int buf = (gj >> 3) & 1;
+          const int a0 = (s - (gj - kClJ)) * A;
           if (a0 == 0) {
             if (!(ok = wait(&sm.s_empty[buf], s_ph[buf] ^ 1, abort, dev_err))) break;
             tc_fence_after();
@@ -734,12 +772,10 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
           for (int a = a0; a < a0 + A; ++a) {
             if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
             tc_fence_after();
-            const uint32_t sa = smem_u32(sm.a[stage]), sb = smem_u32(sm.b[stage]);
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              mma_bf16(dt, sdesc_sw128(sa + kk * 32, 16, 1024),
-                       sdesc_sw128(sb + kk * 32, 16, 1024), kIdescClS,
-                       (a | kk) != 0);
+              mma_bf16(dt, da0 + stage * kAtomU + 2 * kk, db0 + stage * kAtomU + 2 * kk,
+                       kIdescClS, (a | kk) != 0);
             mma_commit(&sm.empty[stage]);
             if (++stage == kClStages) { stage = 0; ph ^= 1; }
           }
@@ -750,29 +786,27 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
           }
         }
         if (s < 0) continue;
-        const int ct = ct_of(s), slot = (int)(s & 1);
+        const int gb = s & (kGSlots - 1);
         if (ct == 0 && !(ok = wait(&sm.o_empty, o_ph ^ 1, abort, dev_err))) break;
-        if (!(ok = wait(&sm.g_full[slot], g_ph[slot], abort, dev_err))) break;
-        g_ph[slot] ^= 1;
+        if (!(ok = wait(&sm.g_full[gb], g_ph[gb], abort, dev_err))) break;
+        g_ph[gb] ^= 1;
         if (!(ok = wait(&sm.cs_full, cs_ph, abort, dev_err))) break;
         cs_ph ^= 1;
         tc_fence_after();
-        const uint32_t sg = smem_u32(sm.g[slot][0]), sc = smem_u32(sm.cs[0]);
 #pragma unroll
         for (int kk = 0; kk < kClBN / 16; ++kk)
-          mma_bf16(tmem_o,
-                   sdesc_sw128(sg + (kk >> 2) * kAtom128 + (kk & 3) * 32, 16, 1024),
-                   sdesc_sw128(sc + kk * 2048, kAtom128, 1024), idesc_o,
-                   (ct | kk) != 0);
+          mma_bf16(tmem_o, dg0 + gb * kGsU + (kk >> 2) * kAtomU + (kk & 3) * 2,
+                   dc + kk * (2048 >> 4), idesc_o, (ct | kk) != 0);
         mma_commit(&sm.cs_empty);
-        mma_commit(&sm.gs_empty[slot]);
+        mma_commit(&sm.gs_empty[gb]);
         // Tell the owner of s that this CTA is done with tile s. The owner
         // publishes its next tile (s + 8) only after all 8 CTAs are, so no
         // pub[] phase can run ahead of a consumer still waiting on the
         // previous one, and ring slot reuse (tile s + 16) is safe.
         if (s + kCl < N)
-          mma_commit_multicast(&sm.gfree[(s / kCl) & 1], (uint16_t)(1u << (int)(s % kCl)));
-        if (ct == n_ct - 1) {
+          mma_commit_multicast(&sm.gfree[(s >> 3) & 1], (uint16_t)(1u << (s & (kCl - 1))));
+        if (++ct == n_ct) {
+          ct = 0;
           mma_commit(&sm.o_full);
           o_ph ^= 1;
         }
@@ -787,12 +821,16 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     uint32_t sf_ph[2] = {0, 0}, free_ph[2] = {0, 0}, o_ph = 0;
     bool ok = true;
-    for (long long s = -kClJ; s < N && ok; ++s) {
-      const long long g = s + kClLag + 1;  // tile whose S completes in slot s
-      if (g >= 0 && g < N && (int)(g % kCl) == k) {
-        const long long m = g / kCl;
-        const int buf = (int)(m & 1);
-        const int rb = rb_of(g), ct = ct_of(g);
+    TileCursor cur;  // tile of slot s (s >= 0), for unit drains
+    cur.init(0, cid, n_ct, ncl);
+    for (int s = -kClJ; s < N && ok; ++s) {
+      const int g = s + kClLag + 1;  // tile whose S completes in slot s
+      if (g >= 0 && g < N && (g & (kCl - 1)) == k) {
+        const int m = g >> 3;
+        const int buf = m & 1;
+        TileCursor gt;
+        gt.init(g, cid, n_ct, ncl);
+        const int rb = gt.rb, ct = gt.ct;
         float rc = 0.f, rl = 0.f;
         if (kTokenRows) {
           const int p = rb * 128 + row;
@@ -808,7 +846,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
         sf_ph[buf] ^= 1;
         if (m >= 1) {
           // Every CTA has finished with this owner's previous tile g - 8.
-          const int pb = (int)((m - 1) & 1);
+          const int pb = (m - 1) & 1;
           if (!(ok = wait_cluster(&sm.gfree[pb], free_ph[pb], abort, dev_err))) break;
           free_ph[pb] ^= 1;
         }
@@ -842,8 +880,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const int kc = c * 32 + q * 8;
-            uint8_t *dst = dst_tile + (kc >> 6) * kAtom128 + sw128_offset(row, kc & 63);
-            *reinterpret_cast<uint4 *>(dst) =
+            *reinterpret_cast<uint4 *>(dst_tile + (kc >> 6) * kAtom128 +
+                                       sw128_offset(row, kc & 63)) =
                 make_uint4(pk[q * 4], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
           }
         }
@@ -858,12 +896,15 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kThreads, 1)
           for (int r = 0; r < kCl; ++r) mbar_arrive_cluster(mapa(pb, (uint32_t)r));
         }
       }
-      if (s >= 0 && ct_of(s) == n_ct - 1) {
+      if (s < 0) continue;
+      const bool unit_end = cur.ct == n_ct - 1;
+      const int rb = cur.rb;
+      cur.next();
+      if (unit_end) {
         // Drain the finished unit: out[rows, k*w : (k+1)*w].
         if (!(ok = wait(&sm.o_full, o_ph, abort, dev_err))) break;
         o_ph ^= 1;
         tc_fence_after();
-        const int rb = rb_of(s);
         const int rid = rb * 128 + row;
         const bool valid = kTokenRows ? (rid < Teff) : (rid < V);
         float *dst = nullptr;
@@ -953,7 +994,7 @@ int cluster_grid(const void *kernel, size_t smem) {
   if (cached) return cached;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(kCl * 64, 1, 1);
-  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.blockDim = dim3(kClThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   int n = 0;
   if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess || n <= 0) {
@@ -1001,12 +1042,12 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
     PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<false>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
     const int ncl = cluster_grid((const void *)bwd_cluster_kernel<true>, cl_smem);
-    bwd_cluster_kernel<true><<<ncl * kCl, kThreads, cl_smem, s>>>(
+    bwd_cluster_kernel<true><<<ncl * kCl, kClThreads, cl_smem, s>>>(
         mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
         static_cast<uint8_t *>(w.gring), g.dev_err);
     PAIR_LAUNCH_CHECK(s);
     PAIR_BEGIN("bwd_dw_tc", s);
-    bwd_cluster_kernel<false><<<ncl * kCl, kThreads, cl_smem, s>>>(
+    bwd_cluster_kernel<false><<<ncl * kCl, kClThreads, cl_smem, s>>>(
         mW128, mH, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
         static_cast<uint8_t *>(w.gring), g.dev_err);
     PAIR_LAUNCH_CHECK(s);
