@@ -771,7 +771,6 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           const uint32_t dt = tmem + buf * kClBN;
           for (int a = a0; a < a0 + A; ++a) {
             if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
-            tc_fence_after();
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
               mma_bf16(dt, da0 + stage * kAtomU + 2 * kk, db0 + stage * kAtomU + 2 * kk,
@@ -842,7 +841,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           sm.col_l[row] = p < Teff ? lse[p] * kLog2e : 0.f;
           epi_sync();
         }
-        if (!(ok = wait(&sm.s_full[buf], sf_ph[buf], abort, dev_err))) break;
+        if (!(ok = wait_sleepy(&sm.s_full[buf], sf_ph[buf], abort, dev_err))) break;
         sf_ph[buf] ^= 1;
         if (m >= 1) {
           // Every CTA has finished with this owner's previous tile g - 8.
@@ -902,7 +901,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
       cur.next();
       if (unit_end) {
         // Drain the finished unit: out[rows, k*w : (k+1)*w].
-        if (!(ok = wait(&sm.o_full, o_ph, abort, dev_err))) break;
+        if (!(ok = wait_sleepy(&sm.o_full, o_ph, abort, dev_err))) break;
         o_ph ^= 1;
         tc_fence_after();
         const int rid = rb * 128 + row;

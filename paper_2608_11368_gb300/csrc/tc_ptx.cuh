@@ -72,6 +72,25 @@ __device__ __forceinline__ bool wait(uint64_t *bar, uint32_t parity,
   }
 }
 
+// Bounded wait for threads off the critical issue path (epilogue warps):
+// sleeps between polls so that the warps sharing a scheduler with the MMA
+// issuer do not steal its issue slots.
+__device__ __forceinline__ bool wait_sleepy(uint64_t *bar, uint32_t parity,
+                                            volatile int *abort, int32_t *dev_err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    __nanosleep(128);
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *abort = 1;
+      flag_error(dev_err, PAIR_DEV_ERR_TIMEOUT);
+      return false;
+    }
+  }
+}
+
 // -------------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map,
                                             uint64_t *bar, int x, int y) {
