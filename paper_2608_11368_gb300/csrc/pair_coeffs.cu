@@ -19,13 +19,19 @@ namespace {
 
 template <int GP>
 struct GroupSmem {
-  float T[GP][GP + 1];  // antisymmetric edge terms; +1 pad: conflict-free rows
+  float U[GP * (GP - 1) / 2];  // strict upper triangle t_ij (i < j), row-major
   float r[GP];
   float a[GP];
   int8_t J[GP];
   int red_i[32];
   float red_f[32];
 };
+
+// Row-major offset of (i, j), i < j, in the packed strict upper triangle.
+template <int GP>
+__device__ __forceinline__ int upper_off(int i, int j) {
+  return i * (2 * GP - i - 1) / 2 + (j - i - 1);
+}
 
 // Deterministic block sum of one int per thread (all threads call).
 __device__ int block_sum_int(int v, int *red) {
@@ -52,7 +58,7 @@ __device__ float block_sum_float(float v, float *red) {
 }
 
 // Computes the coefficients of group `b` into sm.a[0..G) (scale applied).
-// Requires blockDim.x >= GP. Returns (in thread 0) K and the contrast count.
+// Requires blockDim.x >= GP. Returns K and the contrast count (all threads).
 template <int GP>
 __device__ void group_coeffs(GroupSmem<GP> &sm, int b, int G, const float *r,
                              const uint8_t *J, const float *rho, float scale,
@@ -64,7 +70,6 @@ __device__ void group_coeffs(GroupSmem<GP> &sm, int b, int G, const float *r,
     const bool in = tid < G;
     sm.r[tid] = in ? r[gbase + tid] : 0.f;
     sm.J[tid] = in ? (J[gbase + tid] != 0) : 0;
-    sm.T[tid][tid] = 0.f;
   }
   __syncthreads();
 
@@ -72,10 +77,11 @@ __device__ void group_coeffs(GroupSmem<GP> &sm, int b, int G, const float *r,
   int my_contrast = 0, bad = 0;
   if (tid < GP - 1) {
     // Load phase: every upper entry this thread owns, all loads in flight.
+    // Step k covers rows k (first GP-1-k threads) and GP-1-k (the rest).
     float v[GP / 2];
 #pragma unroll
     for (int k = 0; k < GP / 2; ++k) {
-      const int n1 = GP - 1 - k;  // entries of row k
+      const int n1 = GP - 1 - k;
       int i, j;
       if (tid < n1) { i = k; j = k + 1 + tid; }
       else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
@@ -95,39 +101,46 @@ __device__ void group_coeffs(GroupSmem<GP> &sm, int b, int G, const float *r,
         if (!(rij > 0.f)) {
           bad = 1;
         } else {
-          const float dr = sm.r[i] - sm.r[j];
-          t = __fdiv_rn(dr, rij);
+          t = __fdiv_rn(sm.r[i] - sm.r[j], rij);
           my_contrast += (sm.r[i] != sm.r[j]);
         }
       }
-      sm.T[i][j] = t;
-      sm.T[j][i] = -t;
+      sm.U[upper_off<GP>(i, j)] = t;
     }
   }
   if (bad) flag_error(dev_err, PAIR_DEV_ERR_NONPOSITIVE_INCLUSION);
   __syncthreads();
 
-  // Row sums by a fixed pairwise tree.
+  // Row sum of the antisymmetric terms by a fixed pairwise tree, streamed:
+  // partial p[l] holds the sum of the last complete block of 2^l terms.
   float a = 0.f;
   uint8_t act = 0;
   if (tid < GP) {
-    float x[GP];
+    float p[8];
     bool nz = false;
 #pragma unroll
     for (int k = 0; k < GP; ++k) {
-      x[k] = sm.T[tid][k];
-      nz |= (x[k] != 0.f);
-    }
+      float x = 0.f;
+      if (k < tid) x = -sm.U[upper_off<GP>(k, tid)];
+      else if (k > tid) x = sm.U[upper_off<GP>(tid, k)];
+      nz |= (x != 0.f);
+      float c = x;
+      int m = k;
 #pragma unroll
-    for (int s = GP / 2; s >= 1; s >>= 1) {
-#pragma unroll
-      for (int k = 0; k < s; ++k) x[k] += x[k + s];
+      for (int l = 0; l < 8; ++l) {
+        if (m & 1) { c = p[l] + c; m >>= 1; }
+        else { p[l] = c; break; }
+      }
     }
-    a = (x[0] == 0.f) ? 0.f : 0.5f * x[0];
+    // GP is a power of two: the final carry landed in p[log2 GP].
+    const float sum = p[(GP == 32) ? 5 : (GP == 64) ? 6 : 7];
+    a = (sum == 0.f) ? 0.f : 0.5f * sum;
     act = (tid < G && sm.J[tid] && nz) ? 1 : 0;
   }
-  const int K = block_sum_int((tid < GP) ? (int)sm.J[tid] : 0, sm.red_i);
-  const int C = block_sum_int(my_contrast, sm.red_i);
+  // K (low 16 bits) and contrast edges (high bits) in one reduction.
+  const int packed = block_sum_int(((tid < GP) ? (int)sm.J[tid] : 0) | (my_contrast << 16),
+                                   sm.red_i);
+  const int K = packed & 0xffff, C = packed >> 16;
   if (center && K > 0) {
     // App. C: centre across the observed endpoints.
     const float s = block_sum_float((tid < GP && sm.J[tid]) ? a : 0.f, sm.red_f);
@@ -142,7 +155,7 @@ __device__ void group_coeffs(GroupSmem<GP> &sm, int b, int G, const float *r,
 }
 
 template <int GP>
-__global__ void __launch_bounds__(128) coeffs_kernel(
+__global__ void __launch_bounds__(GP, 1024 / GP) coeffs_kernel(
     int B, int G, const float *__restrict__ r, const uint8_t *__restrict__ J,
     const float *__restrict__ rho, float scale, int center,
     float *__restrict__ a, uint8_t *__restrict__ active,
@@ -168,7 +181,7 @@ __global__ void __launch_bounds__(128) coeffs_kernel(
 // One block per group: coefficients, then g_b = sum_i a_i s_{b,i} streamed
 // over D with 16-byte loads; rows with a_i == 0 are never read.
 template <int GP>
-__global__ void __launch_bounds__(256) dense_kernel(
+__global__ void __launch_bounds__(256, 4) dense_kernel(
     int B, int G, int D, const float *__restrict__ r,
     const uint8_t *__restrict__ J, const float *__restrict__ rho,
     const float *__restrict__ S, float scale, float *__restrict__ g,
