@@ -101,7 +101,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int *abort = &sm.abort;
 
   if (warp == 0) {
-    if (lane == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
       int stage = 0;
       uint32_t ph = 0;
       int last_ph[kLseStages];
@@ -114,9 +114,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int vt = vt0; vt < vt1 && ok; ++vt) {
           for (int k = 0; k < nk; ++k) {
             if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
-            mbar_expect_tx(&sm.full[stage], kLseStageTx);
-            tma_load_2d(sm.a[stage], &tmH, &sm.full[stage], k * 64, tb * 128);
-            tma_load_2d(sm.b[stage], &tmW, &sm.full[stage], k * 64, vt * kLseBN);
+            if (elect_one()) {
+              mbar_expect_tx(&sm.full[stage], kLseStageTx);
+              tma_load_2d(sm.a[stage], &tmH, &sm.full[stage], k * 64, tb * 128);
+              tma_load_2d(sm.b[stage], &tmW, &sm.full[stage], k * 64, vt * kLseBN);
+            }
+            __syncwarp();
             last_ph[stage] = (int)ph;
             if (++stage == kLseStages) { stage = 0; ph ^= 1; }
           }
@@ -131,9 +134,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
       int stage = 0, acc = 0;
       uint32_t ph = 0, acc_ph = 0;
+      const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
+      const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 16, 1024);
       bool ok = true;
       for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
         const int sp = u % nsplit;
@@ -145,22 +150,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t dt = tmem + acc * kLseBN;
           for (int k = 0; k < nk; ++k) {
             if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
-            tc_fence_after();
-            const uint32_t sa = smem_u32(sm.a[stage]), sb = smem_u32(sm.b[stage]);
+            const uint64_t da = da0 + (uint64_t)stage * (kAtom128 >> 4);
+            const uint64_t db = db0 + (uint64_t)stage * ((2 * kAtom128) >> 4);
+            if (elect_one()) {
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              mma_bf16(dt, sdesc_sw128(sa + kk * 32, 16, 1024),
-                       sdesc_sw128(sb + kk * 32, 16, 1024), kIdescLse,
-                       (k | kk) != 0);
-            mma_commit(&sm.empty[stage]);
+              for (int kk = 0; kk < 4; ++kk)
+                mma_bf16(dt, da + 2 * kk, db + 2 * kk, kIdescLse, (k | kk) != 0);
+              mma_commit(&sm.empty[stage]);
+            }
+            __syncwarp();
             if (++stage == kLseStages) { stage = 0; ph ^= 1; }
           }
           if (!ok) break;
-          mma_commit(&sm.acc_full[acc]);
+          if (elect_one()) mma_commit(&sm.acc_full[acc]);
+          __syncwarp();
           if (++acc == 2) { acc = 0; acc_ph ^= 1; }
         }
       }
-      mma_commit(&sm.mma_done);
+      if (elect_one()) mma_commit(&sm.mma_done);
+      __syncwarp();
       volatile int never = 0;
       wait(&sm.mma_done, 0, &never, dev_err);
     }
@@ -326,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int *abort = &sm.abort;
 
   if (warp == 0) {
-    if (lane == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
       int stage = 0;
       uint32_t ph = 0, cs_ph = 0;
       int last_ph[kBwdStages];
@@ -336,9 +344,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto load_s = [&](int rb, int ct) {
         for (int k = 0; k < nk && ok; ++k) {
           if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
-          mbar_expect_tx(&sm.full[stage], kBwdStageTx);
-          tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], k * 64, rb * 128);
-          tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], k * 64, ct * kBwdBN);
+          if (elect_one()) {
+            mbar_expect_tx(&sm.full[stage], kBwdStageTx);
+            tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], k * 64, rb * 128);
+            tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], k * 64, ct * kBwdBN);
+          }
+          __syncwarp();
           last_ph[stage] = (int)ph;
           if (++stage == kBwdStages) { stage = 0; ph ^= 1; }
         }
@@ -346,9 +357,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto load_cs = [&](int sl, int w, int ct) {
         if (!ok) return;
         if (!(ok = wait(&sm.cs_empty, cs_ph ^ 1, abort, dev_err))) return;
-        mbar_expect_tx(&sm.cs_full, (uint32_t)(w / 64) * kAtom128);
-        for (int j = 0; j < w / 64; ++j)
-          tma_load_2d(sm.cs[j], &tmC, &sm.cs_full, sl * kSlice + j * 64, ct * kBwdBN);
+        if (elect_one()) {
+          mbar_expect_tx(&sm.cs_full, (uint32_t)(w / 64) * kAtom128);
+          for (int j = 0; j < w / 64; ++j)
+            tma_load_2d(sm.cs[j], &tmC, &sm.cs_full, sl * kSlice + j * 64, ct * kBwdBN);
+        }
+        __syncwarp();
         cs_last = (int)cs_ph;
         cs_ph ^= 1;
       };
@@ -369,7 +383,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (cs_last >= 0) wait(&sm.cs_full, (uint32_t)cs_last, &never, dev_err);
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
       int stage = 0;
       uint32_t ph = 0, s_ph[2] = {0, 0}, g_ph = 0, cs_ph = 0, o_ph = 0;
       bool ok = true;
@@ -380,17 +394,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t dt = tmem + buf * kBwdBN;
         for (int k = 0; k < nk; ++k) {
           if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) return;
-          tc_fence_after();
           const uint32_t sa = smem_u32(sm.a[stage]), sb = smem_u32(sm.b[stage]);
+          if (elect_one()) {
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            mma_bf16(dt, sdesc_sw128(sa + kk * 32, 16, 1024),
-                     sdesc_sw128(sb + kk * 32, 16, 1024), kIdescS,
-                     (k | kk) != 0);
-          mma_commit(&sm.empty[stage]);
+            for (int kk = 0; kk < 4; ++kk)
+              mma_bf16(dt, sdesc_sw128(sa + kk * 32, 16, 1024),
+                       sdesc_sw128(sb + kk * 32, 16, 1024), kIdescS,
+                       (k | kk) != 0);
+            mma_commit(&sm.empty[stage]);
+          }
+          __syncwarp();
           if (++stage == kBwdStages) { stage = 0; ph ^= 1; }
         }
-        mma_commit(&sm.s_full[buf]);
+        if (elect_one()) mma_commit(&sm.s_full[buf]);
+        __syncwarp();
         s_ph[buf] ^= 1;
       };
       auto issue_o = [&](int ct, int w) {
@@ -401,14 +418,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const uint32_t idesc = idesc_bf16(128, w, 0, 1);
         const uint32_t sg = smem_u32(sm.g[0]), sc = smem_u32(sm.cs[0]);
+        if (elect_one()) {
 #pragma unroll
-        for (int kk = 0; kk < kBwdBN / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(sg + (kk >> 2) * kAtom128 + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd = sdesc_sw128(sc + kk * 2048, kAtom128, 1024);
-          mma_bf16(tmem_o, ad, bd, idesc, (ct | kk) != 0);
+          for (int kk = 0; kk < kBwdBN / 16; ++kk) {
+            const uint64_t ad = sdesc_sw128(sg + (kk >> 2) * kAtom128 + (kk & 3) * 32, 16, 1024);
+            const uint64_t bd = sdesc_sw128(sc + kk * 2048, kAtom128, 1024);
+            mma_bf16(tmem_o, ad, bd, idesc, (ct | kk) != 0);
+          }
+          mma_commit(&sm.g_empty);
+          mma_commit(&sm.cs_empty);
         }
-        mma_commit(&sm.g_empty);
-        mma_commit(&sm.cs_empty);
+        __syncwarp();
         g_ph ^= 1;
         cs_ph ^= 1;
       };
@@ -422,10 +442,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue_o(ct, w);
         }
         if (!ok) break;
-        mma_commit(&sm.o_full);
+        if (elect_one()) mma_commit(&sm.o_full);
+        __syncwarp();
         o_ph ^= 1;
       }
-      mma_commit(&sm.mma_done);
+      if (elect_one()) mma_commit(&sm.mma_done);
+      __syncwarp();
       volatile int never = 0;
       wait(&sm.mma_done, 0, &never, dev_err);
     }
@@ -680,7 +702,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
 
   if (warp == 0) {
     // Producer of the S operands (this CTA's share of its owned tiles).
-    if (lane == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
       int stage = 0;
       uint32_t ph = 0;
       int last_ph[kClStages];
@@ -698,9 +720,12 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         const int a0 = (s - (gj - kClJ)) * A;
         for (int a = a0; a < a0 + A; ++a) {
           if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
-          mbar_expect_tx(&sm.full[stage], 2 * kAtom128);
-          tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, job_rb * 128);
-          tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], a * 64, job_ct * kClBN);
+          if (elect_one()) {
+            mbar_expect_tx(&sm.full[stage], 2 * kAtom128);
+            tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, job_rb * 128);
+            tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], a * 64, job_ct * kClBN);
+          }
+          __syncwarp();
           last_ph[stage] = (int)ph;
           if (++stage == kClStages) { stage = 0; ph ^= 1; }
         }
@@ -711,7 +736,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
     }
   } else if (warp == 6) {
     // Producer of the output-update operands: C[s, slice] and Gs(s).
-    if (lane == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
       uint32_t cs_ph = 0, ge_ph[kGSlots] = {};
       int cs_last = -1, g_last[kGSlots];
       for (int i = 0; i < kGSlots; ++i) g_last[i] = -1;
@@ -726,15 +751,21 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           break;
         fence_proxy_async_global();
         if (!(ok = wait(&sm.gs_empty[gb], ge_ph[gb] ^ 1, abort, dev_err))) break;
-        mbar_expect_tx(&sm.g_full[gb], kGsBytes);
-        bulk_load(sm.g[gb][0], ring_tile(s), kGsBytes, &sm.g_full[gb]);
+        if (elect_one()) {
+          mbar_expect_tx(&sm.g_full[gb], kGsBytes);
+          bulk_load(sm.g[gb][0], ring_tile(s), kGsBytes, &sm.g_full[gb]);
+        }
+        __syncwarp();
         g_last[gb] = (int)ge_ph[gb];
         ge_ph[gb] ^= 1;
         // Output operand C[s, slice].
         if (!(ok = wait(&sm.cs_empty, cs_ph ^ 1, abort, dev_err))) break;
-        mbar_expect_tx(&sm.cs_full, (uint32_t)A * kAtom128);
-        for (int j = 0; j < A; ++j)
-          tma_load_2d(sm.cs[j], &tmC, &sm.cs_full, k * w + j * 64, cur.ct * kClBN);
+        if (elect_one()) {
+          mbar_expect_tx(&sm.cs_full, (uint32_t)A * kAtom128);
+          for (int j = 0; j < A; ++j)
+            tma_load_2d(sm.cs[j], &tmC, &sm.cs_full, k * w + j * 64, cur.ct * kClBN);
+        }
+        __syncwarp();
         cs_last = (int)cs_ph;
         cs_ph ^= 1;
       }
@@ -744,7 +775,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         if (g_last[i] >= 0) wait(&sm.g_full[i], (uint32_t)g_last[i], &never, dev_err);
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
       int stage = 0;
       uint32_t ph = 0, o_ph = 0, cs_ph = 0, s_ph[2] = {0, 0}, g_ph[kGSlots] = {};
       const uint32_t idesc_o = idesc_bf16(128, w, 0, 1);
@@ -771,16 +802,20 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           const uint32_t dt = tmem + buf * kClBN;
           for (int a = a0; a < a0 + A; ++a) {
             if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+            const uint64_t da = da0 + stage * kAtomU, db = db0 + stage * kAtomU;
+            if (elect_one()) {
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              mma_bf16(dt, da0 + stage * kAtomU + 2 * kk, db0 + stage * kAtomU + 2 * kk,
-                       kIdescClS, (a | kk) != 0);
-            mma_commit(&sm.empty[stage]);
+              for (int kk = 0; kk < 4; ++kk)
+                mma_bf16(dt, da + 2 * kk, db + 2 * kk, kIdescClS, (a | kk) != 0);
+              mma_commit(&sm.empty[stage]);
+            }
+            __syncwarp();
             if (++stage == kClStages) { stage = 0; ph ^= 1; }
           }
           if (!ok) break;
           if (a0 + A == nk) {
-            mma_commit(&sm.s_full[buf]);
+            if (elect_one()) mma_commit(&sm.s_full[buf]);
+            __syncwarp();
             s_ph[buf] ^= 1;
           }
         }
@@ -792,25 +827,34 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         if (!(ok = wait(&sm.cs_full, cs_ph, abort, dev_err))) break;
         cs_ph ^= 1;
         tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < kClBN / 16; ++kk)
-          mma_bf16(tmem_o, dg0 + gb * kGsU + (kk >> 2) * kAtomU + (kk & 3) * 2,
-                   dc + kk * (2048 >> 4), idesc_o, (ct | kk) != 0);
-        mma_commit(&sm.cs_empty);
-        mma_commit(&sm.gs_empty[gb]);
+        const uint64_t dg = dg0 + gb * kGsU;
         // Tell the owner of s that this CTA is done with tile s. The owner
         // publishes its next tile (s + 8) only after all 8 CTAs are, so no
         // pub[] phase can run ahead of a consumer still waiting on the
         // previous one, and ring slot reuse (tile s + 16) is safe.
-        if (s + kCl < N)
-          mma_commit_multicast(&sm.gfree[(s >> 3) & 1], (uint16_t)(1u << (s & (kCl - 1))));
-        if (++ct == n_ct) {
+        const bool notify = s + kCl < N;
+        const bool unit_end = ct + 1 == n_ct;
+        if (elect_one()) {
+#pragma unroll
+          for (int kk = 0; kk < kClBN / 16; ++kk)
+            mma_bf16(tmem_o, dg + (kk >> 2) * kAtomU + (kk & 3) * 2, dc + kk * (2048 >> 4),
+                     idesc_o, (ct | kk) != 0);
+          mma_commit(&sm.cs_empty);
+          mma_commit(&sm.gs_empty[gb]);
+          if (notify)
+            mma_commit_multicast(&sm.gfree[(s >> 3) & 1], (uint16_t)(1u << (s & (kCl - 1))));
+          if (unit_end) mma_commit(&sm.o_full);
+        }
+        __syncwarp();
+        if (unit_end) {
           ct = 0;
-          mma_commit(&sm.o_full);
           o_ph ^= 1;
+        } else {
+          ++ct;
         }
       }
-      mma_commit(&sm.mma_done);
+      if (elect_one()) mma_commit(&sm.mma_done);
+      __syncwarp();
       volatile int never = 0;
       wait(&sm.mma_done, 0, &never, dev_err);
     }
