@@ -212,12 +212,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (mc == -INFINITY) continue;
           if (mc > m2) {
-            l *= exp2f(m2 - mc);
+            l *= ex2_approx(m2 - mc);
             m2 = mc;
           }
           float s = 0.f;
 #pragma unroll
-          for (int j = 0; j < 32; ++j) s += exp2f(v[j] - m2);
+          for (int j = 0; j < 32; ++j) s += ex2_approx(v[j] - m2);
           l += s;
         }
         tc_fence_before();
@@ -499,7 +499,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 cc = sm.col_c[col]; ll = sm.col_l[col];
                 live = cc != 0.f;
               }
-              g2[e] = live ? -cc * exp2f(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
+              g2[e] = live ? -cc * ex2_approx(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
             }
             __nv_bfloat162 b2 = __floats2bfloat162_rn(g2[0], g2[1]);
             pk[j >> 1] = *reinterpret_cast<uint32_t *>(&b2);
@@ -915,7 +915,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
                 cc = sm.col_c[col]; ll = sm.col_l[col];
                 live = cc != 0.f;
               }
-              g2[e] = live ? -cc * exp2f(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
+              g2[e] = live ? -cc * ex2_approx(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
             }
             __nv_bfloat162 b2 = __floats2bfloat162_rn(g2[0], g2[1]);
             pk[j >> 1] = *reinterpret_cast<uint32_t *>(&b2);
@@ -928,10 +928,11 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
                 make_uint4(pk[q * 4], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
           }
         }
-        fence_proxy_async_global();
-        fence_acq_rel_cluster();
         tc_fence_before();
         mbar_arrive(&sm.s_empty[buf]);
+        // The CTA barrier orders every epilogue thread's stores before the
+        // elected thread's cluster-scope release (cumulativity); readers
+        // fence the async proxy after acquiring pub[].
         epi_sync();
         if (warp == 2 && lane == 0) {
           fence_acq_rel_cluster();

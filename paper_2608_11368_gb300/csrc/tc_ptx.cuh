@@ -33,6 +33,15 @@ __device__ __forceinline__ bool elect_one() {
   return pred != 0;
 }
 
+// 2^x with the hardware approximation (ex2.approx.ftz.f32, relative error
+// about 2^-22); used where the result feeds bf16 operands or fp32 sums whose
+// tolerance is far looser.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)),
