@@ -934,10 +934,11 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         // elected thread's cluster-scope release (cumulativity); readers
         // fence the async proxy after acquiring pub[].
         epi_sync();
-        if (warp == 2 && lane == 0) {
+        if (warp == 2 && lane < kCl) {
+          // One lane per destination CTA, in parallel: fence, then a relaxed
+          // arrive (a release pattern per lane).
           fence_acq_rel_cluster();
-          const uint32_t pb = smem_u32(&sm.pub[k]);
-          for (int r = 0; r < kCl; ++r) mbar_arrive_cluster(mapa(pb, (uint32_t)r));
+          mbar_arrive_cluster_relaxed(mapa(smem_u32(&sm.pub[k]), (uint32_t)lane));
         }
       }
       if (s < 0) continue;
