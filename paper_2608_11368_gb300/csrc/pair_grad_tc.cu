@@ -577,10 +577,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 // schedule never drains at unit boundaries.
 constexpr int kCl = 8;          // cluster size (power of two)
 constexpr int kClBN = 128;      // column tile (S is 128 x 128)
-constexpr int kClStages = 3;    // S operand stages
+constexpr int kClStages = 4;    // S operand stages
 constexpr int kClLag = 3;       // slots between an S tile's completion and its use
 constexpr int kClJ = kCl + kClLag;
-constexpr int kGSlots = 2;      // Gs tiles staged in shared memory
+constexpr int kGSlots = 1;      // Gs tiles staged in shared memory
 constexpr int kClThreads = 224; // + warp 6: loads of C[s, slice] and Gs
 constexpr uint32_t kGsBytes = 128 * kClBN * 2; // one Gs tile (32 KB)
 constexpr uint32_t kIdescClS = idesc_bf16(128, kClBN, 0, 0);
