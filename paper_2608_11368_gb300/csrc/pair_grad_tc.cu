@@ -567,9 +567,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 // kClLag slots before the tile is used (d/512 K-atoms per slot), converts it
 // to bf16 Gs and publishes the 32 KB tile (already in the swizzled K-major
 // layout of the MMA operand) once, to a per-cluster ring in global memory,
-// then signals every CTA of the cluster through its pub[owner] mbarrier.
-// Every CTA pulls Gs(s) into one of its two shared-memory slots with a bulk
-// copy and updates out += Gs(s) . C[s, slice]. The exchange goes through L2
+// then signals every CTA of the cluster through its pub[owner][m & 1]
+// mbarrier (m = g / 8, the owner's tile count). Every CTA pulls Gs(s) into
+// shared memory with a bulk copy and updates out += Gs(s) . C[s, slice].
+// The ring holds two tiles per owner, and an owner overwrites its slot of
+// tile g - 16 only after every CTA is done with that tile; with two pub
+// barriers per owner this also keeps any consumer's parity wait unambiguous,
+// and it leaves 16 slots (not 8) for the round trip consume -> convert ->
+// publish -> load. The exchange goes through L2
 // because distributed shared memory sustains far less per-SM egress than a
 // broadcast of a 32 KB tile to 7 peers per slot needs. In every slot every
 // CTA issues the same tensor work: a share of one S accumulation plus one
@@ -581,7 +586,7 @@ constexpr int kClStages = 4;    // S operand stages
 constexpr int kClLag = 3;       // slots between an S tile's completion and its use
 constexpr int kClJ = kCl + kClLag;
 constexpr int kGSlots = 1;      // Gs tiles staged in shared memory
-constexpr int kClThreads = 224; // + warp 6: loads of C[s, slice] and Gs
+constexpr int kClThreads = 256; // + warp 6: loads of C[s, slice] and Gs; warp 7: output MMAs
 constexpr uint32_t kGsBytes = 128 * kClBN * 2; // one Gs tile (32 KB)
 constexpr uint32_t kIdescClS = idesc_bf16(128, kClBN, 0, 0);
 
@@ -594,8 +599,8 @@ struct ClSmem {
   uint64_t full[kClStages], empty[kClStages];
   uint64_t s_full[2], s_empty[2];
   uint64_t g_full[kGSlots], gs_empty[kGSlots];
-  uint64_t cs_full, cs_empty;
-  uint64_t pub[kCl];                 // owner o published its next tile
+  uint64_t cs_full[2], cs_empty[2];  // C[s, slice] in two column parts
+  uint64_t pub[kCl][2];              // owner o published its tile m (by m & 1)
   uint64_t gfree[2];                 // (owner) all CTAs done with its tile m (by m & 1)
   uint64_t o_full, o_empty, mma_done;
   uint32_t tmem_base;
@@ -648,6 +653,10 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   const int A = d / (64 * kCl);            // K-atoms per slot (d / 512)
   const int w = 64 * A;                    // this CTA's d-slice width
   const int nk = d / 64;
+  // The output update runs as two column parts of A0 and A - A0 atoms, each
+  // with its own C[s, slice] buffer barrier: part 0's operand of the next
+  // slot loads while part 1 still computes.
+  const int A0 = (A + 1) >> 1, A1 = A - A0;
   const int n_rb = kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128;
   const int n_ct = kTokenRows ? (V + kClBN - 1) / kClBN : (Teff + kClBN - 1) / kClBN;
   const int n_my = cid < n_rb ? (n_rb - cid + ncl - 1) / ncl : 0;
@@ -677,12 +686,17 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
       mbar_init(&sm.g_full[s], 1);
       mbar_init(&sm.gs_empty[s], 1);
     }
-    mbar_init(&sm.cs_full, 1);
-    mbar_init(&sm.cs_empty, 1);
-    for (int o = 0; o < kCl; ++o) mbar_init(&sm.pub[o], 1);
+    for (int p = 0; p < 2; ++p) {
+      mbar_init(&sm.cs_full[p], 1);
+      mbar_init(&sm.cs_empty[p], 1);
+    }
+    for (int o = 0; o < kCl; ++o) {
+      mbar_init(&sm.pub[o][0], 1);
+      mbar_init(&sm.pub[o][1], 1);
+    }
     mbar_init(&sm.o_full, 1);
     mbar_init(&sm.o_empty, 128);
-    mbar_init(&sm.mma_done, 1);
+    mbar_init(&sm.mma_done, 2);  // one final commit per MMA-issuing warp
     sm.abort = 0;
     fence_mbar_init();
     prefetch_tmap(&tmR);
@@ -737,16 +751,31 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   } else if (warp == 6) {
     // Producer of the output-update operands: C[s, slice] and Gs(s).
     {  // whole warp: uniform loop state; elected lane issues
-      uint32_t cs_ph = 0, ge_ph[kGSlots] = {};
-      int cs_last = -1, g_last[kGSlots];
+      uint32_t cs_ph[2] = {0, 0}, ge_ph[kGSlots] = {};
+      int cs_last[2] = {-1, -1}, g_last[kGSlots];
       for (int i = 0; i < kGSlots; ++i) g_last[i] = -1;
       bool ok = true;
       TileCursor cur;
       cur.init(0, cid, n_ct, ncl);
+      // Output operand C[s, slice], column part p (atoms [j0, j0 + na)).
+      auto load_cs = [&](int p, int j0, int na, int ct) {
+        if (!(ok = wait(&sm.cs_empty[p], cs_ph[p] ^ 1, abort, dev_err))) return;
+        if (elect_one()) {
+          mbar_expect_tx(&sm.cs_full[p], (uint32_t)na * kAtom128);
+          for (int j = j0; j < j0 + na; ++j)
+            tma_load_2d(sm.cs[j], &tmC, &sm.cs_full[p], k * w + j * 64, ct * kClBN);
+        }
+        __syncwarp();
+        cs_last[p] = (int)cs_ph[p];
+        cs_ph[p] ^= 1;
+      };
       for (int s = 0; s < N && ok; ++s, cur.next()) {
+        load_cs(0, 0, A0, cur.ct);
+        if (!ok) break;
         // Gs(s) from its owner's ring slot.
         const int gb = s & (kGSlots - 1);
-        if (!(ok = wait_cluster(&sm.pub[s & (kCl - 1)], (uint32_t)((s >> 3) & 1), abort,
+        // pub[o][b] completes once per two tiles of owner o: parity (m >> 1) & 1.
+        if (!(ok = wait_cluster(&sm.pub[s & (kCl - 1)][(s >> 3) & 1], (uint32_t)((s >> 4) & 1), abort,
                                 dev_err)))
           break;
         fence_proxy_async_global();
@@ -758,41 +787,38 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         __syncwarp();
         g_last[gb] = (int)ge_ph[gb];
         ge_ph[gb] ^= 1;
-        // Output operand C[s, slice].
-        if (!(ok = wait(&sm.cs_empty, cs_ph ^ 1, abort, dev_err))) break;
-        if (elect_one()) {
-          mbar_expect_tx(&sm.cs_full, (uint32_t)A * kAtom128);
-          for (int j = 0; j < A; ++j)
-            tma_load_2d(sm.cs[j], &tmC, &sm.cs_full, k * w + j * 64, cur.ct * kClBN);
-        }
-        __syncwarp();
-        cs_last = (int)cs_ph;
-        cs_ph ^= 1;
+        if (A1 > 0) load_cs(1, A0, A1, cur.ct);
       }
       volatile int never = 0;
-      if (cs_last >= 0) wait(&sm.cs_full, (uint32_t)cs_last, &never, dev_err);
+      for (int p = 0; p < 2; ++p)
+        if (cs_last[p] >= 0) wait(&sm.cs_full[p], (uint32_t)cs_last[p], &never, dev_err);
       for (int i = 0; i < kGSlots; ++i)
         if (g_last[i] >= 0) wait(&sm.g_full[i], (uint32_t)g_last[i], &never, dev_err);
     }
-  } else if (warp == 1) {
+  } else if (warp == 1 || warp == 7) {
+    // Two MMA issuers with independent instruction streams: warp 1 the S
+    // accumulations (TMEM columns [0, 256)), warp 7 the output update
+    // (columns [256, 512)). tcgen05.mma issue runs only about one instruction
+    // ahead of execution, so the bookkeeping between one warp's MMAs (barrier
+    // polls, loop state) would otherwise leave the tensor pipe idle; with two
+    // streams the other warp's MMAs fill those gaps. Each warp's commits
+    // track its own MMAs only.
     {  // whole warp: uniform loop state; elected lane issues
-      int stage = 0;
-      uint32_t ph = 0, o_ph = 0, cs_ph = 0, s_ph[2] = {0, 0}, g_ph[kGSlots] = {};
-      const uint32_t idesc_o = idesc_bf16(128, w, 0, 1);
       // Descriptors of every buffer, built once; K steps add to the start
-      // address field (16-byte units).
-      // Buffers of one kind are contiguous, so buffer i adds i times its
-      // size (in 16-byte units) to the base descriptor.
+      // address field (16-byte units). Buffers of one kind are contiguous,
+      // so buffer i adds i times its size (in 16-byte units) to the base.
       const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
       const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 16, 1024);
       const uint64_t dg0 = sdesc_sw128(smem_u32(sm.g[0][0]), 16, 1024);
       const uint64_t dc = sdesc_sw128(smem_u32(sm.cs[0]), kAtom128, 1024);
       constexpr uint32_t kAtomU = kAtom128 >> 4, kGsU = kGsBytes >> 4;
       bool ok = true;
-      int ct = 0;  // column tile of slot s (s >= 0)
-      for (int s = -kClJ; s < N && ok; ++s) {
-        const int gj = job_of(s);
-        if (gj >= 0 && gj < N) {
+      if (warp == 1) {
+        int stage = 0;
+        uint32_t ph = 0, s_ph[2] = {0, 0};
+        for (int s = -kClJ; s < N && ok; ++s) {
+          const int gj = job_of(s);
+          if (gj < 0 || gj >= N) continue;
           const int buf = (gj >> 3) & 1;
           const int a0 = (s - (gj - kClJ)) * A;
           if (a0 == 0) {
@@ -808,49 +834,67 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
               for (int kk = 0; kk < 4; ++kk)
                 mma_bf16(dt, da + 2 * kk, db + 2 * kk, kIdescClS, (a | kk) != 0);
               mma_commit(&sm.empty[stage]);
+              if (a + 1 == nk) mma_commit(&sm.s_full[buf]);
             }
             __syncwarp();
             if (++stage == kClStages) { stage = 0; ph ^= 1; }
           }
-          if (!ok) break;
-          if (a0 + A == nk) {
-            if (elect_one()) mma_commit(&sm.s_full[buf]);
-            __syncwarp();
-            s_ph[buf] ^= 1;
-          }
+          if (a0 + A == nk) s_ph[buf] ^= 1;
         }
-        if (s < 0) continue;
-        const int gb = s & (kGSlots - 1);
-        if (ct == 0 && !(ok = wait(&sm.o_empty, o_ph ^ 1, abort, dev_err))) break;
-        if (!(ok = wait(&sm.g_full[gb], g_ph[gb], abort, dev_err))) break;
-        g_ph[gb] ^= 1;
-        if (!(ok = wait(&sm.cs_full, cs_ph, abort, dev_err))) break;
-        cs_ph ^= 1;
-        tc_fence_after();
-        const uint64_t dg = dg0 + gb * kGsU;
-        // Tell the owner of s that this CTA is done with tile s. The owner
-        // publishes its next tile (s + 8) only after all 8 CTAs are, so no
-        // pub[] phase can run ahead of a consumer still waiting on the
-        // previous one, and ring slot reuse (tile s + 16) is safe.
-        const bool notify = s + kCl < N;
-        const bool unit_end = ct + 1 == n_ct;
-        if (elect_one()) {
+      } else {
+        uint32_t o_ph = 0, cs_ph[2] = {0, 0}, g_ph[kGSlots] = {};
+        const uint32_t idesc_o0 = idesc_bf16(128, 64 * A0, 0, 1);
+        const uint32_t idesc_o1 = idesc_bf16(128, 64 * (A1 > 0 ? A1 : 1), 0, 1);
+        const uint64_t dc1 = dc + (uint64_t)A0 * kAtomU;
+        int ct = 0;  // column tile of slot s
+        for (int s = 0; s < N && ok; ++s) {
+          const int gb = s & (kGSlots - 1);
+          if (ct == 0 && !(ok = wait(&sm.o_empty, o_ph ^ 1, abort, dev_err))) break;
+          if (!(ok = wait(&sm.g_full[gb], g_ph[gb], abort, dev_err))) break;
+          g_ph[gb] ^= 1;
+          if (!(ok = wait(&sm.cs_full[0], cs_ph[0], abort, dev_err))) break;
+          cs_ph[0] ^= 1;
+          tc_fence_after();
+          const uint64_t dg = dg0 + gb * kGsU;
+          if (elect_one()) {
 #pragma unroll
-          for (int kk = 0; kk < kClBN / 16; ++kk)
-            mma_bf16(tmem_o, dg + (kk >> 2) * kAtomU + (kk & 3) * 2, dc + kk * (2048 >> 4),
-                     idesc_o, (ct | kk) != 0);
-          mma_commit(&sm.cs_empty);
-          mma_commit(&sm.gs_empty[gb]);
-          if (notify)
-            mma_commit_multicast(&sm.gfree[(s >> 3) & 1], (uint16_t)(1u << (s & (kCl - 1))));
-          if (unit_end) mma_commit(&sm.o_full);
-        }
-        __syncwarp();
-        if (unit_end) {
-          ct = 0;
-          o_ph ^= 1;
-        } else {
-          ++ct;
+            for (int kk = 0; kk < kClBN / 16; ++kk)
+              mma_bf16(tmem_o, dg + (kk >> 2) * kAtomU + (kk & 3) * 2, dc + kk * (2048 >> 4),
+                       idesc_o0, (ct | kk) != 0);
+            mma_commit(&sm.cs_empty[0]);
+          }
+          __syncwarp();
+          if (A1 > 0) {
+            if (!(ok = wait(&sm.cs_full[1], cs_ph[1], abort, dev_err))) break;
+            cs_ph[1] ^= 1;
+            tc_fence_after();
+          }
+          // Tell the owner of s that this CTA is done with tile s. The owner
+          // publishes tile s + 16 (same ring slot, same pub barrier) only after
+          // all 8 CTAs are, so no pub phase can run ahead of a consumer still
+          // waiting on an earlier one.
+          const bool notify = s + 2 * kCl < N;
+          const bool unit_end = ct + 1 == n_ct;
+          if (elect_one()) {
+            if (A1 > 0) {
+#pragma unroll
+              for (int kk = 0; kk < kClBN / 16; ++kk)
+                mma_bf16(tmem_o + 64 * A0, dg + (kk >> 2) * kAtomU + (kk & 3) * 2,
+                         dc1 + kk * (2048 >> 4), idesc_o1, (ct | kk) != 0);
+              mma_commit(&sm.cs_empty[1]);
+            }
+            mma_commit(&sm.gs_empty[gb]);
+            if (notify)
+              mma_commit_multicast(&sm.gfree[(s >> 3) & 1], (uint16_t)(1u << (s & (kCl - 1))));
+            if (unit_end) mma_commit(&sm.o_full);
+          }
+          __syncwarp();
+          if (unit_end) {
+            ct = 0;
+            o_ph ^= 1;
+          } else {
+            ++ct;
+          }
         }
       }
       if (elect_one()) mma_commit(&sm.mma_done);
@@ -887,9 +931,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         }
         if (!(ok = wait_sleepy(&sm.s_full[buf], sf_ph[buf], abort, dev_err))) break;
         sf_ph[buf] ^= 1;
-        if (m >= 1) {
-          // Every CTA has finished with this owner's previous tile g - 8.
-          const int pb = (m - 1) & 1;
+        if (m >= 2) {
+          // Every CTA has finished with this owner's tile g - 16.
+          const int pb = m & 1;
           if (!(ok = wait_cluster(&sm.gfree[pb], free_ph[pb], abort, dev_err))) break;
           free_ph[pb] ^= 1;
         }
@@ -938,7 +982,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           // One lane per destination CTA, in parallel: fence, then a relaxed
           // arrive (a release pattern per lane).
           fence_acq_rel_cluster();
-          mbar_arrive_cluster_relaxed(mapa(smem_u32(&sm.pub[k]), (uint32_t)lane));
+          mbar_arrive_cluster_relaxed(mapa(smem_u32(&sm.pub[k][m & 1]), (uint32_t)lane));
         }
       }
       if (s < 0) continue;
