@@ -621,21 +621,79 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
-// Walks global tile indices 0, 1, 2, ... of a cluster as (row block,
-// column tile) pairs without divisions in the loop.
-struct TileCursor {
-  int ct, rb;
-  int n_ct, ncl;
-  __device__ void init(int g, int cid, int n_ct_, int ncl_) {
+// The tiles of one cluster, in processing order: first its F = n_rb / ncl
+// full row blocks (cid, cid + ncl, ...), each with all n_ct column tiles;
+// then an even share [t0, t1) of the row-major tiles of the remaining
+// n_rb mod ncl row blocks, so that all clusters finish within a tile of each
+// other. A unit (run of tiles with one row block) in that tail may cover only
+// part of its row block; its rows are zeroed beforehand and its result is
+// added atomically.
+struct TileMap {
+  int n_ct, ncl, cid, gT, t0, rbT, N;
+  __device__ void setup(int n_rb, int n_ct_, int cid_, int ncl_) {
     n_ct = n_ct_;
     ncl = ncl_;
-    ct = n_ct ? g % n_ct : 0;
-    rb = cid + (n_ct ? g / n_ct : 0) * ncl;
+    cid = cid_;
+    const int F = n_ct ? n_rb / ncl : 0;
+    const int R = n_ct ? n_rb - F * ncl : 0;
+    const int64_t T = (int64_t)R * n_ct;
+    gT = F * n_ct;
+    rbT = F * ncl;
+    t0 = (int)(T * cid / ncl);
+    N = gT + (int)(T * (cid + 1) / ncl) - t0;
   }
-  __device__ void next() {
-    if (++ct == n_ct) { ct = 0; rb += ncl; }
-  }
+  __device__ bool tail(int g) const { return g >= gT; }
 };
+
+// Walks tile indices g = 0, 1, 2, ... of a TileMap as (row block, column
+// tile) pairs without divisions in the loop.
+struct TileCursor {
+  int ct, rb, g;
+  __device__ void init(const TileMap &mp, int g_) {
+    g = g_;
+    if (mp.n_ct == 0) {
+      ct = 0;
+      rb = mp.cid;
+    } else if (g < mp.gT) {
+      ct = g % mp.n_ct;
+      rb = mp.cid + (g / mp.n_ct) * mp.ncl;
+    } else {
+      const int t = mp.t0 + (g - mp.gT);
+      ct = t % mp.n_ct;
+      rb = mp.rbT + t / mp.n_ct;
+    }
+  }
+  __device__ void next(const TileMap &mp) {
+    ++g;
+    if (g == mp.gT) {
+      ct = mp.t0 % mp.n_ct;
+      rb = mp.rbT + mp.t0 / mp.n_ct;
+    } else if (++ct == mp.n_ct) {
+      ct = 0;
+      rb += g < mp.gT ? mp.ncl : 1;
+    }
+  }
+  __device__ bool unit_start(const TileMap &mp) const { return ct == 0 || g == mp.gT; }
+  __device__ bool unit_end(const TileMap &mp) const { return ct == mp.n_ct - 1 || g == mp.N - 1; }
+};
+
+// Zeroes the output rows of the tail row blocks (see TileMap) before the
+// cluster backward adds partial units into them.
+template <bool kTokenRows>
+__global__ void zero_tail_rows_kernel(int d, int V, int ncl, const int32_t *counters,
+                                      const int32_t *tok_idx, float *out) {
+  const int Teff = counters[0];
+  const int n_rows = kTokenRows ? Teff : V;
+  const int n_rb = (n_rows + 127) / 128;
+  const int r0 = (n_rb / ncl) * ncl * 128;
+  const int vec = d / 4;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+       i < (int64_t)(n_rows - r0) * vec; i += (int64_t)gridDim.x * blockDim.x) {
+    const int rid = r0 + (int)(i / vec);
+    const int64_t row = kTokenRows ? (int64_t)tok_idx[rid] : (int64_t)rid;
+    reinterpret_cast<float4 *>(out + row * d)[i % vec] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+}
 
 template <bool kTokenRows>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
@@ -660,7 +718,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   const int n_rb = kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128;
   const int n_ct = kTokenRows ? (V + kClBN - 1) / kClBN : (Teff + kClBN - 1) / kClBN;
   const int n_my = cid < n_rb ? (n_rb - cid + ncl - 1) / ncl : 0;
-  const int N = n_my * n_ct;               // global tiles of this cluster
+  TileMap mp;
+  mp.setup(n_rb, n_ct, cid, ncl);
+  const int N = mp.N;                      // tiles of this cluster
   // Ring of published Gs tiles: [owner][job parity] for this cluster.
   uint8_t *ring = gring + (size_t)cid * kCl * 2 * kGsBytes;
   auto ring_tile = [&](int g) {
@@ -728,7 +788,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         if (gj < 0 || gj >= N) continue;
         if (gj != job_g) {
           TileCursor c;
-          c.init(gj, cid, n_ct, ncl);
+          c.init(mp, gj);
           job_rb = c.rb; job_ct = c.ct; job_g = gj;
         }
         const int a0 = (s - (gj - kClJ)) * A;
@@ -756,7 +816,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
       for (int i = 0; i < kGSlots; ++i) g_last[i] = -1;
       bool ok = true;
       TileCursor cur;
-      cur.init(0, cid, n_ct, ncl);
+      cur.init(mp, 0);
       // Output operand C[s, slice], column part p (atoms [j0, j0 + na)).
       auto load_cs = [&](int p, int j0, int na, int ct) {
         if (!(ok = wait(&sm.cs_empty[p], cs_ph[p] ^ 1, abort, dev_err))) return;
@@ -769,7 +829,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         cs_last[p] = (int)cs_ph[p];
         cs_ph[p] ^= 1;
       };
-      for (int s = 0; s < N && ok; ++s, cur.next()) {
+      for (int s = 0; s < N && ok; ++s, cur.next(mp)) {
         load_cs(0, 0, A0, cur.ct);
         if (!ok) break;
         // Gs(s) from its owner's ring slot.
@@ -846,10 +906,13 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         const uint32_t idesc_o0 = idesc_bf16(128, 64 * A0, 0, 1);
         const uint32_t idesc_o1 = idesc_bf16(128, 64 * (A1 > 0 ? A1 : 1), 0, 1);
         const uint64_t dc1 = dc + (uint64_t)A0 * kAtomU;
-        int ct = 0;  // column tile of slot s
-        for (int s = 0; s < N && ok; ++s) {
+        TileCursor cur;  // tile of slot s
+        cur.init(mp, 0);
+        for (int s = 0; s < N && ok; ++s, cur.next(mp)) {
           const int gb = s & (kGSlots - 1);
-          if (ct == 0 && !(ok = wait(&sm.o_empty, o_ph ^ 1, abort, dev_err))) break;
+          const bool unit_start = cur.unit_start(mp);
+          const bool unit_end = cur.unit_end(mp);
+          if (unit_start && !(ok = wait(&sm.o_empty, o_ph ^ 1, abort, dev_err))) break;
           if (!(ok = wait(&sm.g_full[gb], g_ph[gb], abort, dev_err))) break;
           g_ph[gb] ^= 1;
           if (!(ok = wait(&sm.cs_full[0], cs_ph[0], abort, dev_err))) break;
@@ -860,7 +923,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
 #pragma unroll
             for (int kk = 0; kk < kClBN / 16; ++kk)
               mma_bf16(tmem_o, dg + (kk >> 2) * kAtomU + (kk & 3) * 2, dc + kk * (2048 >> 4),
-                       idesc_o0, (ct | kk) != 0);
+                       idesc_o0, !(unit_start && kk == 0));
             mma_commit(&sm.cs_empty[0]);
           }
           __syncwarp();
@@ -874,13 +937,12 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           // all 8 CTAs are, so no pub phase can run ahead of a consumer still
           // waiting on an earlier one.
           const bool notify = s + 2 * kCl < N;
-          const bool unit_end = ct + 1 == n_ct;
           if (elect_one()) {
             if (A1 > 0) {
 #pragma unroll
               for (int kk = 0; kk < kClBN / 16; ++kk)
                 mma_bf16(tmem_o + 64 * A0, dg + (kk >> 2) * kAtomU + (kk & 3) * 2,
-                         dc1 + kk * (2048 >> 4), idesc_o1, (ct | kk) != 0);
+                         dc1 + kk * (2048 >> 4), idesc_o1, !(unit_start && kk == 0));
               mma_commit(&sm.cs_empty[1]);
             }
             mma_commit(&sm.gs_empty[gb]);
@@ -889,12 +951,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
             if (unit_end) mma_commit(&sm.o_full);
           }
           __syncwarp();
-          if (unit_end) {
-            ct = 0;
-            o_ph ^= 1;
-          } else {
-            ++ct;
-          }
+          if (unit_end) o_ph ^= 1;
         }
       }
       if (elect_one()) mma_commit(&sm.mma_done);
@@ -909,14 +966,14 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
     uint32_t sf_ph[2] = {0, 0}, free_ph[2] = {0, 0}, o_ph = 0;
     bool ok = true;
     TileCursor cur;  // tile of slot s (s >= 0), for unit drains
-    cur.init(0, cid, n_ct, ncl);
+    cur.init(mp, 0);
     for (int s = -kClJ; s < N && ok; ++s) {
       const int g = s + kClLag + 1;  // tile whose S completes in slot s
       if (g >= 0 && g < N && (g & (kCl - 1)) == k) {
         const int m = g >> 3;
         const int buf = m & 1;
         TileCursor gt;
-        gt.init(g, cid, n_ct, ncl);
+        gt.init(mp, g);
         const int rb = gt.rb, ct = gt.ct;
         float rc = 0.f, rl = 0.f;
         if (kTokenRows) {
@@ -986,9 +1043,10 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         }
       }
       if (s < 0) continue;
-      const bool unit_end = cur.ct == n_ct - 1;
+      const bool unit_end = cur.unit_end(mp);
+      const bool add = mp.tail(cur.g);
       const int rb = cur.rb;
-      cur.next();
+      cur.next(mp);
       if (unit_end) {
         // Drain the finished unit: out[rows, k*w : (k+1)*w].
         if (!(ok = wait_sleepy(&sm.o_full, o_ph, abort, dev_err))) break;
@@ -1003,7 +1061,12 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         for (int c = 0; c < w / 32; ++c) {
           float v[32];
           tmem_ld32(tmem_o + lane_off + c * 32, v);
-          if (valid) {
+          if (valid && add) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              atomicAdd(reinterpret_cast<float4 *>(dst + c * 32) + q,
+                        make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+          } else if (valid) {
 #pragma unroll
             for (int q = 0; q < 8; ++q)
               reinterpret_cast<float4 *>(dst + c * 32)[q] =
@@ -1123,7 +1186,6 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
   lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters,
                                              w.part, w.lse);
   PAIR_LAUNCH_CHECK(s);
-  PAIR_BEGIN("bwd_dh_tc", s);
   if (use_cluster_path(g.d)) {
     const size_t cl_smem = sizeof(ClSmem) + 1024;
     PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<true>,
@@ -1131,9 +1193,16 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
     PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<false>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
     const int ncl = cluster_grid((const void *)bwd_cluster_kernel<true>, cl_smem);
+    PAIR_BEGIN("zero_tail_dh", s);
+    zero_tail_rows_kernel<true><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, w.counters, w.tok_idx, g.dH);
+    PAIR_LAUNCH_CHECK(s);
+    PAIR_BEGIN("bwd_dh_tc", s);
     bwd_cluster_kernel<true><<<ncl * kCl, kClThreads, cl_smem, s>>>(
         mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
         static_cast<uint8_t *>(w.gring), g.dev_err);
+    PAIR_LAUNCH_CHECK(s);
+    PAIR_BEGIN("zero_tail_dw", s);
+    zero_tail_rows_kernel<false><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, w.counters, w.tok_idx, g.dW);
     PAIR_LAUNCH_CHECK(s);
     PAIR_BEGIN("bwd_dw_tc", s);
     bwd_cluster_kernel<false><<<ncl * kCl, kClThreads, cl_smem, s>>>(
@@ -1142,6 +1211,7 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
     PAIR_LAUNCH_CHECK(s);
     return PAIR_OK;
   }
+  PAIR_BEGIN("bwd_dh_tc", s);
   bwd_kernel<true><<<nsm, kThreads, bwd_smem, s>>>(
       mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
       g.dev_err);
