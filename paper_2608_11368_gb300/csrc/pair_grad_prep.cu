@@ -221,7 +221,64 @@ __global__ void onehot_dh_kernel(int d, const int32_t *counters,
 
 // dW_v += sum_{t: y_t = v} c_t h_t (the one-hot part of dJ/dW_v), exact in
 // fp32, tokens added in their packed order. One warp owns a bucket of
-// vocabulary rows and scans the compacted targets for matches.
+// vocabulary rows and scans the compacted targets for matches (four 32-token
+// chunks per round, so the target loads overlap); a matching row is updated
+// with 16-byte vector accesses when d allows it.
+__device__ __forceinline__ void load8(const __nv_bfloat16 *h, float (&x)[8]) {
+  const uint4 u = *reinterpret_cast<const uint4 *>(h);
+  const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __bfloat1622float2(b[i]);
+    x[2 * i] = f.x;
+    x[2 * i + 1] = f.y;
+  }
+}
+__device__ __forceinline__ void load8(const float *h, float (&x)[8]) {
+  const float4 a = reinterpret_cast<const float4 *>(h)[0];
+  const float4 b = reinterpret_cast<const float4 *>(h)[1];
+  x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+  x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+}
+
+template <typename Tin>
+__device__ __forceinline__ void axpy_row(int d, float c, const Tin *__restrict__ h,
+                                         float *__restrict__ row, int lane) {
+  if ((d & 7) == 0) {
+    for (int k0 = lane * 8; k0 < d; k0 += 32 * 8 * 2) {
+      // Two independent 8-element groups per iteration.
+      const int k1 = k0 + 32 * 8;
+      float x0[8], x1[8];
+      load8(h + k0, x0);
+      float4 r0a = reinterpret_cast<float4 *>(row + k0)[0];
+      float4 r0b = reinterpret_cast<float4 *>(row + k0)[1];
+      float4 r1a = make_float4(0.f, 0.f, 0.f, 0.f), r1b = r1a;
+      const bool has1 = k1 < d;
+      if (has1) {
+        load8(h + k1, x1);
+        r1a = reinterpret_cast<float4 *>(row + k1)[0];
+        r1b = reinterpret_cast<float4 *>(row + k1)[1];
+      }
+      r0a = make_float4(fmaf(c, x0[0], r0a.x), fmaf(c, x0[1], r0a.y), fmaf(c, x0[2], r0a.z),
+                        fmaf(c, x0[3], r0a.w));
+      r0b = make_float4(fmaf(c, x0[4], r0b.x), fmaf(c, x0[5], r0b.y), fmaf(c, x0[6], r0b.z),
+                        fmaf(c, x0[7], r0b.w));
+      reinterpret_cast<float4 *>(row + k0)[0] = r0a;
+      reinterpret_cast<float4 *>(row + k0)[1] = r0b;
+      if (has1) {
+        r1a = make_float4(fmaf(c, x1[0], r1a.x), fmaf(c, x1[1], r1a.y), fmaf(c, x1[2], r1a.z),
+                          fmaf(c, x1[3], r1a.w));
+        r1b = make_float4(fmaf(c, x1[4], r1b.x), fmaf(c, x1[5], r1b.y), fmaf(c, x1[6], r1b.z),
+                          fmaf(c, x1[7], r1b.w));
+        reinterpret_cast<float4 *>(row + k1)[0] = r1a;
+        reinterpret_cast<float4 *>(row + k1)[1] = r1b;
+      }
+    }
+  } else {
+    for (int k = lane; k < d; k += 32) row[k] = fmaf(c, (float)h[k], row[k]);
+  }
+}
+
 template <typename Tin>
 __global__ void onehot_dw_kernel(int d, int V, int bucket,
                                  const int32_t *counters, const int32_t *tok_y,
@@ -232,19 +289,23 @@ __global__ void onehot_dw_kernel(int d, int V, int bucket,
   if (v0 >= V) return;
   const int v1 = min(V, v0 + bucket);
   const int Teff = counters[0];
-  for (int base = 0; base < Teff; base += 32) {
-    const int p = base + lane;
-    const int yt = p < Teff ? tok_y[p] : -1;
-    unsigned hit = __ballot_sync(0xffffffffu, yt >= v0 && yt < v1);
-    while (hit) {
-      const int src = __ffs(hit) - 1;
-      hit &= hit - 1;
-      const int q = base + src;
-      const int v = __shfl_sync(0xffffffffu, yt, src);
-      const float c = tok_c[q];
-      const Tin *h = Hc + (int64_t)q * d;
-      float *row = dW + (int64_t)v * d;
-      for (int k = lane; k < d; k += 32) row[k] = fmaf(c, (float)h[k], row[k]);
+  for (int base = 0; base < Teff; base += 128) {
+    int yt[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int p = base + 32 * i + lane;
+      yt[i] = p < Teff ? tok_y[p] : -1;
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      unsigned hit = __ballot_sync(0xffffffffu, yt[i] >= v0 && yt[i] < v1);
+      while (hit) {
+        const int src = __ffs(hit) - 1;
+        hit &= hit - 1;
+        const int q = base + 32 * i + src;
+        const int v = __shfl_sync(0xffffffffu, yt[i], src);
+        axpy_row(d, tok_c[q], Hc + (int64_t)q * d, dW + (int64_t)v * d, lane);
+      }
     }
   }
 }
