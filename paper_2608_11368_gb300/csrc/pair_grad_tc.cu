@@ -580,22 +580,34 @@ __global__ void __launch_bounds__(kThreads, 1)
 // CTA issues the same tensor work: a share of one S accumulation plus one
 // output update. The slot counter runs across units, so the staggered S
 // schedule never drains at unit boundaries.
+//
+// The column tile is BN wide (BN = 128 for d <= 2048, 96 for d = 2560, 64
+// for d = 3072): TMEM holds two BN-column S buffers plus the d/8-column
+// output slice, 2 BN + d/8 <= 512.
 constexpr int kCl = 8;          // cluster size (power of two)
-constexpr int kClBN = 128;      // column tile (S is 128 x 128)
 constexpr int kClStages = 4;    // S operand stages
 constexpr int kClLag = 3;       // slots between an S tile's completion and its use
 constexpr int kClJ = kCl + kClLag;
 constexpr int kGSlots = 1;      // Gs tiles staged in shared memory
 constexpr int kClThreads = 256; // + warp 6: loads of C[s, slice] and Gs; warp 7: output MMAs
-constexpr uint32_t kGsBytes = 128 * kClBN * 2; // one Gs tile (32 KB)
-constexpr uint32_t kIdescClS = idesc_bf16(128, kClBN, 0, 0);
 
+template <int BN>
+struct ClTile {
+  static constexpr uint32_t kColAtom = BN * 64 * 2;         // BN rows x 64 bf16
+  static constexpr int kGsAtoms = (BN + 63) / 64;           // Gs K-major atoms
+  static constexpr uint32_t kGsBytes = kGsAtoms * kAtom128; // one Gs tile
+  static constexpr int kCsAtoms = (512 - 2 * BN) / 64;      // max output-slice atoms
+  static constexpr uint32_t kIdescS = idesc_bf16(128, BN, 0, 0);
+};
+
+template <int BN>
 struct ClSmem {
-  uint8_t a[kClStages][kAtom128];    // rows operand atoms (128 x 64)
-  uint8_t b[kClStages][kAtom128];    // column operand atoms (128 x 64)
-  uint8_t cs[4][kAtom128];           // C[s, slice]: MN-major B, <= 4 atoms
-  uint8_t g[kGSlots][2][kAtom128];   // Gs tiles: 128 x 128 bf16, K-major A
-  float col_c[kClBN], col_l[kClBN];
+  using T = ClTile<BN>;
+  uint8_t a[kClStages][kAtom128];                 // rows operand atoms (128 x 64)
+  uint8_t b[kClStages][T::kColAtom];              // column operand atoms (BN x 64)
+  uint8_t cs[T::kCsAtoms][T::kColAtom];           // C[s, slice]: MN-major B
+  uint8_t g[kGSlots][T::kGsAtoms][kAtom128];      // Gs tiles: 128 x BN bf16, K-major A
+  float col_c[BN], col_l[BN];
   uint64_t full[kClStages], empty[kClStages];
   uint64_t s_full[2], s_empty[2];
   uint64_t g_full[kGSlots], gs_empty[kGSlots];
@@ -695,7 +707,7 @@ __global__ void zero_tail_rows_kernel(int d, int V, int ncl, const int32_t *coun
   }
 }
 
-template <bool kTokenRows>
+template <bool kTokenRows, int BN>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
     bwd_cluster_kernel(const __grid_constant__ CUtensorMap tmR,
                        const __grid_constant__ CUtensorMap tmC, int d, int V,
@@ -703,7 +715,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
                        const float *tok_c, const float *lse, float *out,
                        uint8_t *gring, int32_t *dev_err) {
   extern __shared__ uint8_t smem_raw[];
-  ClSmem &sm = *reinterpret_cast<ClSmem *>(align1k(smem_raw));
+  ClSmem<BN> &sm = *reinterpret_cast<ClSmem<BN> *>(align1k(smem_raw));
+  using Tl = ClTile<BN>;
+  constexpr uint32_t kGsBytes = Tl::kGsBytes, kColAtom = Tl::kColAtom;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int k = (int)cluster_rank();
   const int cid = (int)cluster_id_x(), ncl = (int)num_clusters_x();
@@ -716,7 +730,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   // slot loads while part 1 still computes.
   const int A0 = (A + 1) >> 1, A1 = A - A0;
   const int n_rb = kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128;
-  const int n_ct = kTokenRows ? (V + kClBN - 1) / kClBN : (Teff + kClBN - 1) / kClBN;
+  const int n_ct = kTokenRows ? (V + BN - 1) / BN : (Teff + BN - 1) / BN;
   const int n_my = cid < n_rb ? (n_rb - cid + ncl - 1) / ncl : 0;
   TileMap mp;
   mp.setup(n_rb, n_ct, cid, ncl);
@@ -771,7 +785,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   cluster_sync();  // every CTA's barriers exist before anyone signals them
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  const uint32_t tmem_o = tmem + 2 * kClBN;
+  const uint32_t tmem_o = tmem + 2 * BN;
   volatile int *abort = &sm.abort;
 
   if (warp == 0) {
@@ -795,9 +809,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         for (int a = a0; a < a0 + A; ++a) {
           if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
           if (elect_one()) {
-            mbar_expect_tx(&sm.full[stage], 2 * kAtom128);
+            mbar_expect_tx(&sm.full[stage], kAtom128 + kColAtom);
             tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, job_rb * 128);
-            tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], a * 64, job_ct * kClBN);
+            tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], a * 64, job_ct * BN);
           }
           __syncwarp();
           last_ph[stage] = (int)ph;
@@ -821,9 +835,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
       auto load_cs = [&](int p, int j0, int na, int ct) {
         if (!(ok = wait(&sm.cs_empty[p], cs_ph[p] ^ 1, abort, dev_err))) return;
         if (elect_one()) {
-          mbar_expect_tx(&sm.cs_full[p], (uint32_t)na * kAtom128);
+          mbar_expect_tx(&sm.cs_full[p], (uint32_t)na * kColAtom);
           for (int j = j0; j < j0 + na; ++j)
-            tma_load_2d(sm.cs[j], &tmC, &sm.cs_full[p], k * w + j * 64, ct * kClBN);
+            tma_load_2d(sm.cs[j], &tmC, &sm.cs_full[p], k * w + j * 64, ct * BN);
         }
         __syncwarp();
         cs_last[p] = (int)cs_ph[p];
@@ -870,8 +884,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
       const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
       const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 16, 1024);
       const uint64_t dg0 = sdesc_sw128(smem_u32(sm.g[0][0]), 16, 1024);
-      const uint64_t dc = sdesc_sw128(smem_u32(sm.cs[0]), kAtom128, 1024);
-      constexpr uint32_t kAtomU = kAtom128 >> 4, kGsU = kGsBytes >> 4;
+      const uint64_t dc = sdesc_sw128(smem_u32(sm.cs[0]), kColAtom, 1024);
+      constexpr uint32_t kAtomU = kAtom128 >> 4, kColU = kColAtom >> 4, kGsU = kGsBytes >> 4;
       bool ok = true;
       if (warp == 1) {
         int stage = 0;
@@ -885,14 +899,14 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
             if (!(ok = wait(&sm.s_empty[buf], s_ph[buf] ^ 1, abort, dev_err))) break;
             tc_fence_after();
           }
-          const uint32_t dt = tmem + buf * kClBN;
+          const uint32_t dt = tmem + buf * BN;
           for (int a = a0; a < a0 + A; ++a) {
             if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
-            const uint64_t da = da0 + stage * kAtomU, db = db0 + stage * kAtomU;
+            const uint64_t da = da0 + stage * kAtomU, db = db0 + stage * kColU;
             if (elect_one()) {
 #pragma unroll
               for (int kk = 0; kk < 4; ++kk)
-                mma_bf16(dt, da + 2 * kk, db + 2 * kk, kIdescClS, (a | kk) != 0);
+                mma_bf16(dt, da + 2 * kk, db + 2 * kk, Tl::kIdescS, (a | kk) != 0);
               mma_commit(&sm.empty[stage]);
               if (a + 1 == nk) mma_commit(&sm.s_full[buf]);
             }
@@ -905,7 +919,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         uint32_t o_ph = 0, cs_ph[2] = {0, 0}, g_ph[kGSlots] = {};
         const uint32_t idesc_o0 = idesc_bf16(128, 64 * A0, 0, 1);
         const uint32_t idesc_o1 = idesc_bf16(128, 64 * (A1 > 0 ? A1 : 1), 0, 1);
-        const uint64_t dc1 = dc + (uint64_t)A0 * kAtomU;
+        const uint64_t dc1 = dc + (uint64_t)A0 * kColU;
         TileCursor cur;  // tile of slot s
         cur.init(mp, 0);
         for (int s = 0; s < N && ok; ++s, cur.next(mp)) {
@@ -921,7 +935,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           const uint64_t dg = dg0 + gb * kGsU;
           if (elect_one()) {
 #pragma unroll
-            for (int kk = 0; kk < kClBN / 16; ++kk)
+            for (int kk = 0; kk < BN / 16; ++kk)
               mma_bf16(tmem_o, dg + (kk >> 2) * kAtomU + (kk & 3) * 2, dc + kk * (2048 >> 4),
                        idesc_o0, !(unit_start && kk == 0));
             mma_commit(&sm.cs_empty[0]);
@@ -940,7 +954,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           if (elect_one()) {
             if (A1 > 0) {
 #pragma unroll
-              for (int kk = 0; kk < kClBN / 16; ++kk)
+              for (int kk = 0; kk < BN / 16; ++kk)
                 mma_bf16(tmem_o + 64 * A0, dg + (kk >> 2) * kAtomU + (kk & 3) * 2,
                          dc1 + kk * (2048 >> 4), idesc_o1, !(unit_start && kk == 0));
               mma_commit(&sm.cs_empty[1]);
@@ -981,9 +995,11 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           if (p < Teff) { rc = tok_c[p]; rl = lse[p] * kLog2e; }
         } else {
           epi_sync();
-          const int p = ct * kClBN + row;
-          sm.col_c[row] = p < Teff ? tok_c[p] : 0.f;
-          sm.col_l[row] = p < Teff ? lse[p] * kLog2e : 0.f;
+          const int p = ct * BN + row;
+          if (row < BN) {
+            sm.col_c[row] = p < Teff ? tok_c[p] : 0.f;
+            sm.col_l[row] = p < Teff ? lse[p] * kLog2e : 0.f;
+          }
           epi_sync();
         }
         if (!(ok = wait_sleepy(&sm.s_full[buf], sf_ph[buf], abort, dev_err))) break;
@@ -997,9 +1013,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         tc_fence_after();
         uint8_t *dst_tile = ring_tile(g);
 #pragma unroll 1
-        for (int c = 0; c < kClBN / 32; ++c) {
+        for (int c = 0; c < BN / 32; ++c) {
           float v[32];
-          tmem_ld32(tmem + lane_off + buf * kClBN + c * 32, v);
+          tmem_ld32(tmem + lane_off + buf * BN + c * 32, v);
           uint32_t pk[16];
 #pragma unroll
           for (int j = 0; j < 32; j += 2) {
@@ -1011,7 +1027,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
               bool live;
               if (kTokenRows) {
                 cc = rc; ll = rl;
-                live = (rc != 0.f) && (ct * kClBN + col < V);
+                live = (rc != 0.f) && (ct * BN + col < V);
               } else {
                 cc = sm.col_c[col]; ll = sm.col_l[col];
                 live = cc != 0.f;
@@ -1136,11 +1152,14 @@ int num_sms() {
   return n;
 }
 
-// The cluster backward needs d = 8 * 64 * A with 1 <= A <= 4 (each CTA's
-// output slice of 64 * A columns stays in TMEM beside the S buffers).
-bool use_cluster_path(int d) { return d % 512 == 0 && d >= 512 && d <= 2048; }
+// The cluster backward needs d = 8 * 64 * A with 1 <= A <= 6: each CTA's
+// output slice of 64 * A columns stays in TMEM beside two S buffers of the
+// column-tile width BN (2 BN + 64 A <= 512).
+bool use_cluster_path(int d) { return d % 512 == 0 && d >= 512 && d <= 3072; }
+int cluster_tile_width(int d) { return d <= 2048 ? 128 : d <= 2560 ? 96 : 64; }
 
 // Clusters that fit at once (persistent grid), from the occupancy API.
+template <int BN>
 int cluster_grid(const void *kernel, size_t smem) {
   static int cached = 0;
   if (cached) return cached;
@@ -1156,6 +1175,40 @@ int cluster_grid(const void *kernel, size_t smem) {
   if (n > kMaxClusters) n = kMaxClusters;
   cached = n > 0 ? n : 1;
   return cached;
+}
+
+// dH and dW by the cluster kernels with BN-wide column tiles. Row operands
+// use 128-row boxes (mH for dH, mW128 for dW); column operands BN-row boxes.
+template <int BN>
+pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStream_t s,
+                             const CUtensorMap &mH, const CUtensorMap &mW128) {
+  CUtensorMap mHc, mWc;
+  if (!make_map(&mHc, w.Hc, w.Tpad, g.d, BN) || !make_map(&mWc, g.W, g.V, g.d, BN))
+    return PAIR_ERR_CUDA;
+  const int nsm = num_sms();
+  const size_t cl_smem = sizeof(ClSmem<BN>) + 1024;
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<true, BN>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<false, BN>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
+  const int ncl = cluster_grid<BN>((const void *)bwd_cluster_kernel<true, BN>, cl_smem);
+  PAIR_BEGIN("zero_tail_dh", s);
+  zero_tail_rows_kernel<true><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, w.counters, w.tok_idx, g.dH);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("bwd_dh_tc", s);
+  bwd_cluster_kernel<true, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
+      mH, mWc, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
+      static_cast<uint8_t *>(w.gring), g.dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("zero_tail_dw", s);
+  zero_tail_rows_kernel<false><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, w.counters, w.tok_idx, g.dW);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("bwd_dw_tc", s);
+  bwd_cluster_kernel<false, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
+      mW128, mHc, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
+      static_cast<uint8_t *>(w.gring), g.dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
 }
 
 }  // namespace
@@ -1187,29 +1240,11 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
                                              w.part, w.lse);
   PAIR_LAUNCH_CHECK(s);
   if (use_cluster_path(g.d)) {
-    const size_t cl_smem = sizeof(ClSmem) + 1024;
-    PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<true>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
-    PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<false>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
-    const int ncl = cluster_grid((const void *)bwd_cluster_kernel<true>, cl_smem);
-    PAIR_BEGIN("zero_tail_dh", s);
-    zero_tail_rows_kernel<true><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, w.counters, w.tok_idx, g.dH);
-    PAIR_LAUNCH_CHECK(s);
-    PAIR_BEGIN("bwd_dh_tc", s);
-    bwd_cluster_kernel<true><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-        mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
-        static_cast<uint8_t *>(w.gring), g.dev_err);
-    PAIR_LAUNCH_CHECK(s);
-    PAIR_BEGIN("zero_tail_dw", s);
-    zero_tail_rows_kernel<false><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, w.counters, w.tok_idx, g.dW);
-    PAIR_LAUNCH_CHECK(s);
-    PAIR_BEGIN("bwd_dw_tc", s);
-    bwd_cluster_kernel<false><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-        mW128, mH, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
-        static_cast<uint8_t *>(w.gring), g.dev_err);
-    PAIR_LAUNCH_CHECK(s);
-    return PAIR_OK;
+    switch (cluster_tile_width(g.d)) {
+      case 128: return grad_bwd_cluster<128>(g, w, s, mH, mW128);
+      case 96: return grad_bwd_cluster<96>(g, w, s, mH, mW128);
+      default: return grad_bwd_cluster<64>(g, w, s, mH, mW128);
+    }
   }
   PAIR_BEGIN("bwd_dh_tc", s);
   bwd_kernel<true><<<nsm, kThreads, bwd_smem, s>>>(

@@ -79,12 +79,15 @@ CASES = [
     ("qwen3_1p7b_head", 192, 1000, 3, 5, 0.05, 8.0),     # ragged V, N=192 slice
     ("qwen3_4b_head", 320, 777, 2, 6, 0.03, 8.0),        # two slices (256 + 64)
     ("longctx_skew", 64, 300, 4, 4, 0.02, 1.0),          # minimal d
-    ("qwen3_4b_head", 2560, 4099, 2, 3, 0.05, 3.0),      # ten slices
     # Cluster backward (d = 512 * A): slice widths 64, 128, 192, with
     # ragged vocabulary tails and several row blocks per cluster.
     ("qwen3_1p7b_head", 512, 1000, 3, 8, 0.3, 4.0),
     ("longctx_skew", 1024, 5003, 2, 8, 0.15, 2.0),
     ("qwen3_4b_head", 1536, 777, 2, 6, 0.08, 8.0),
+    # Wider hidden sizes: 96-wide (d = 2560, slice 320) and 64-wide
+    # (d = 3072, slice 384) column tiles, ragged in both directions.
+    ("qwen3_4b_head", 2560, 4099, 2, 3, 0.05, 3.0),
+    ("longctx_skew", 3072, 2011, 2, 4, 0.04, 3.0),
 ]
 
 
