@@ -43,6 +43,7 @@ constexpr int kAtom128 = 128 * 64 * 2;  // 128 rows x 64 bf16 (16 KB)
 constexpr int kLseBN = 256;
 constexpr int kLseStages = 4;
 constexpr uint32_t kLseStageTx = (128 + kLseBN) * 64 * 2;
+constexpr int kLsePair = 2;  // CTAs per cluster sharing each vocabulary tile
 constexpr uint32_t kIdescLse = idesc_bf16(128, kLseBN, 0, 0);
 
 struct LseSmem {
@@ -60,7 +61,14 @@ __device__ __forceinline__ uint8_t *align1k(uint8_t *p) {
                                      ~static_cast<uintptr_t>(1023));
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+// CTA pairs (2-CTA clusters) work on two token blocks of the same vocabulary
+// split in lockstep: each CTA fetches its own token atom and one half (128
+// rows) of the shared 256-row vocabulary atom, multicast into both CTAs'
+// stage. A stage is refilled only after both CTAs' MMAs released it (each
+// MMA warp commits to the empty barrier of both CTAs). This halves the
+// vocabulary bytes each SM's copy engine requests, which is what limits the
+// loads here (the engine's outstanding requests wait on DRAM-latency tiles).
+__global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
     lse_kernel(const __grid_constant__ CUtensorMap tmH,
                const __grid_constant__ CUtensorMap tmW, int d, int V,
                int nsplit, int64_t Tpad, const int32_t *counters,
@@ -72,13 +80,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int Teff = counters[0];
   const int n_tb = (Teff + 127) / 128;
   const int n_vt = (V + kLseBN - 1) / kLseBN;
-  const int n_units = n_tb * nsplit;
+  // Work unit = (pair of token blocks, vocabulary split); CTA r of the pair
+  // takes token block 2 * pair + r (past the last block for an odd count:
+  // in-bounds padding rows whose results are never written).
+  const int n_units = (n_tb + 1) / 2 * nsplit;
   const int nk = d / 64;
+  const int r = (int)cluster_rank();
+  const int pid = (int)cluster_id_x(), npairs = (int)num_clusters_x();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kLseStages; ++s) {
       mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], 1);
+      mbar_init(&sm.empty[s], kLsePair);  // both CTAs' MMAs done with the stage
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&sm.acc_full[s], 1);
@@ -96,6 +109,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // the peer's barriers exist before any multicast lands
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   volatile int *abort = &sm.abort;
@@ -107,17 +121,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       int last_ph[kLseStages];
       for (int s = 0; s < kLseStages; ++s) last_ph[s] = -1;
       bool ok = true;
-      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
-        const int tb = u / nsplit, sp = u % nsplit;
+      for (int u = pid; u < n_units && ok; u += npairs) {
+        const int tb = 2 * (u / nsplit) + r, sp = u % nsplit;
         const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
         const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
         for (int vt = vt0; vt < vt1 && ok; ++vt) {
           for (int k = 0; k < nk; ++k) {
-            if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+            if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
             if (elect_one()) {
               mbar_expect_tx(&sm.full[stage], kLseStageTx);
               tma_load_2d(sm.a[stage], &tmH, &sm.full[stage], k * 64, tb * 128);
-              tma_load_2d(sm.b[stage], &tmW, &sm.full[stage], k * 64, vt * kLseBN);
+              tma_load_2d_mc(sm.b[stage] + r * (kLseBN / 2) * 128, &tmW, &sm.full[stage],
+                             k * 64, vt * kLseBN + r * (kLseBN / 2), (uint16_t)3);
             }
             __syncwarp();
             last_ph[stage] = (int)ph;
@@ -140,7 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
       const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 16, 1024);
       bool ok = true;
-      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+      for (int u = pid; u < n_units && ok; u += npairs) {
         const int sp = u % nsplit;
         const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
         const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
@@ -156,7 +171,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
               for (int kk = 0; kk < 4; ++kk)
                 mma_bf16(dt, da + 2 * kk, db + 2 * kk, kIdescLse, (k | kk) != 0);
-              mma_commit(&sm.empty[stage]);
+              mma_commit_multicast(&sm.empty[stage], (uint16_t)3);
             }
             __syncwarp();
             if (++stage == kLseStages) { stage = 0; ph ^= 1; }
@@ -179,8 +194,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     int acc = 0;
     uint32_t acc_ph = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
-      const int tb = u / nsplit, sp = u % nsplit;
+    for (int u = pid; u < n_units && ok; u += npairs) {
+      const int tb = 2 * (u / nsplit) + r, sp = u % nsplit;
       const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
       const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
       const int p = tb * 128 + row;
@@ -234,6 +249,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still signal or fill it
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
@@ -1141,6 +1157,25 @@ bool make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t cols,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+int num_sms();
+
+// CTAs of the LSE grid: every 2-CTA cluster that fits at once (persistent).
+int lse_grid(size_t smem) {
+  static int cached = 0;
+  if (cached) return cached;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kLsePair * 64, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, (const void *)lse_kernel, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    n = num_sms() / kLsePair;
+  }
+  cached = kLsePair * (n > 0 ? n : 1);
+  return cached;
+}
+
 int num_sms() {
   static int n = 0;
   if (!n) {
@@ -1231,7 +1266,7 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bwd_smem));
 
   PAIR_BEGIN("lse_tc", s);
-  lse_kernel<<<nsm, kThreads, lse_smem, s>>>(mH, mW256, g.d, g.V, w.nsplit,
+  lse_kernel<<<lse_grid(lse_smem), kThreads, lse_smem, s>>>(mH, mW128, g.d, g.V, w.nsplit,
                                              w.Tpad, w.counters, w.tok_y,
                                              w.part, w.zy, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
