@@ -244,6 +244,24 @@ PAIR_API int32_t pair_last_launch_count(void);
 PAIR_API void pair_timing_enable(int32_t on);
 PAIR_API int32_t pair_timing_read(int32_t max, float *ms, const char **names);
 
+/*
+ * pair_selftest_wait_timeout -- exercises the failure path of the pipeline
+ * waits (a diagnostic for tests; no counterpart in the paper).
+ * Launches one block that waits on an mbarrier nothing ever arrives on,
+ * through the same bounded-wait code every tensor-core kernel uses, with a
+ * limit of limit_cycles SM clocks (1 .. 4e9). The wait gives up, raises the
+ * block's abort flag (a second role then stops waiting at once) and ORs
+ * PAIR_DEV_ERR_TIMEOUT into *dev_err; the kernel then returns normally, so
+ * the context stays usable. seen (2 int32, device) receives bit 0 = the wait
+ * gave up, bit 1 = the abort flag was raised, and seen[1] = 1 when the second
+ * role saw the flag. Asynchronous on `stream`; follow with pair_status_sync,
+ * which then returns PAIR_ERR_DEVICE_TIMEOUT.
+ * Errors: PAIR_ERR_INVALID_ARG (null pointer, limit out of range),
+ * PAIR_ERR_UNSUPPORTED, PAIR_ERR_CUDA.
+ */
+PAIR_API pair_status pair_selftest_wait_timeout(int64_t limit_cycles, int32_t *dev_err,
+                                                int32_t *seen, pair_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

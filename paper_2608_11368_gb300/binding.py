@@ -70,6 +70,8 @@ def lib() -> ctypes.CDLL:
     L.pair_timing_enable.restype = None
     L.pair_timing_read.argtypes = [I32, P, P]
     L.pair_timing_read.restype = I32
+    L.pair_selftest_wait_timeout.argtypes = [I64, P, P, P]
+    L.pair_selftest_wait_timeout.restype = ctypes.c_int
     _lib = L
     return L
 
@@ -239,6 +241,15 @@ def pair_grad_noalloc(H, W, y, mask, cu_seqlens, a, dH=None, dW=None,
                                  _stream(stream))
     _check(st, "pair_grad_noalloc")
     return Jobj, dH, dW, logp_seq
+
+
+def pair_selftest_wait_timeout(limit_cycles, dev_err, seen, stream=None):
+    """Launch the bounded-wait failure-path check (see pair.h)."""
+    _need(dev_err, "dev_err", torch.int32)
+    _need(seen, "seen", torch.int32, (2,))
+    st = lib().pair_selftest_wait_timeout(int(limit_cycles), _p(dev_err), _p(seen),
+                                          _stream(stream))
+    _check(st, "pair_selftest_wait_timeout")
 
 
 def pair_status_sync(dev_err=None, stream=None) -> int:

@@ -50,7 +50,8 @@ void launch_end(cudaStream_t s) {
 
 void reset_launches() { g_log.launches = 0; }
 
-static pair_status check_device() {
+// Compute capability 10.3 (GB300) on the current device; cached per device.
+pair_status check_device() {
   static int cached_dev = -1;
   static pair_status cached = PAIR_OK;
   int dev = 0;

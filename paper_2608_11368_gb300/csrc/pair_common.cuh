@@ -21,6 +21,8 @@ constexpr float kLog2e = 1.4426950408889634f;
 void launch_begin(const char *name, cudaStream_t s);
 void launch_end(cudaStream_t s);
 void reset_launches();
+// PAIR_OK on a compute-capability 10.3 device, else PAIR_ERR_UNSUPPORTED.
+pair_status check_device();
 
 __device__ __forceinline__ void flag_error(int32_t *err, int bit) {
   if (err) atomicOr(err, bit);

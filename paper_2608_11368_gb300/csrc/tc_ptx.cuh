@@ -78,20 +78,26 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase of parity `parity` to complete. Returns false
-// (and raises *abort) on timeout, or if another role already aborted.
-__device__ __forceinline__ bool wait(uint64_t *bar, uint32_t parity,
-                                     volatile int *abort, int32_t *dev_err) {
+// (and raises *abort) after `limit` SM clocks, or if another role already
+// aborted.
+__device__ __forceinline__ bool wait_limit(uint64_t *bar, uint32_t parity, volatile int *abort,
+                                           int32_t *dev_err, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > limit) {
       *abort = 1;
       flag_error(dev_err, PAIR_DEV_ERR_TIMEOUT);
       return false;
     }
   }
+}
+
+__device__ __forceinline__ bool wait(uint64_t *bar, uint32_t parity,
+                                     volatile int *abort, int32_t *dev_err) {
+  return wait_limit(bar, parity, abort, dev_err, kWaitCycles);
 }
 
 // Bounded wait for threads off the critical issue path (epilogue warps):
