@@ -726,7 +726,8 @@ __global__ void zero_tail_rows_kernel(int d, int V, int ncl, const int32_t *coun
 template <bool kTokenRows, int BN>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
     bwd_cluster_kernel(const __grid_constant__ CUtensorMap tmR,
-                       const __grid_constant__ CUtensorMap tmC, int d, int V,
+                       const __grid_constant__ CUtensorMap tmC,
+                       const __grid_constant__ CUtensorMap tmC64, int d, int V,
                        const int32_t *counters, const int32_t *tok_idx,
                        const float *tok_c, const float *lse, float *out,
                        uint8_t *gring, int32_t *dev_err) {
@@ -741,10 +742,14 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   const int A = d / (64 * kCl);            // K-atoms per slot (d / 512)
   const int w = 64 * A;                    // this CTA's d-slice width
   const int nk = d / 64;
-  // The output update runs as two column parts of A0 and A - A0 atoms, each
-  // with its own C[s, slice] buffer barrier: part 0's operand of the next
-  // slot loads while part 1 still computes.
-  const int A0 = (A + 1) >> 1, A1 = A - A0;
+  // The output update runs in two parts with their own operand barriers, so
+  // part 0's operands of the next slot load while part 1 still computes.
+  // With a 128-wide tile and a slice of at most 256 columns (d <= 2048) the
+  // parts are the two 64-row K halves of the tile (Gs atom p with rows
+  // [64p, 64p + 64) of C[s, slice]; 256-wide MMAs); otherwise they are two
+  // column parts of A0 and A - A0 atoms of the slice.
+  const bool ksplit = BN == 128 && A <= 4;
+  const int A0 = ksplit ? A : (A + 1) >> 1, A1 = ksplit ? A : A - A0;
   const int n_rb = kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128;
   const int n_ct = kTokenRows ? (V + BN - 1) / BN : (Teff + BN - 1) / BN;
   const int n_my = cid < n_rb ? (n_rb - cid + ncl - 1) / ncl : 0;
@@ -791,6 +796,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
     fence_mbar_init();
     prefetch_tmap(&tmR);
     prefetch_tmap(&tmC);
+    prefetch_tmap(&tmC64);
   }
   if (warp == 1) {
     tmem_alloc(&sm.tmem_base, 512);
@@ -859,7 +865,34 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         cs_last[p] = (int)cs_ph[p];
         cs_ph[p] ^= 1;
       };
-      for (int s = 0; s < N && ok; ++s, cur.next(mp)) {
+      // K-split: part p = Gs atom p and rows [64p, 64p + 64) of every slice
+      // atom, on one barrier.
+      auto load_khalf = [&](int p, int s, int ct) {
+        if (!(ok = wait(&sm.cs_empty[p], cs_ph[p] ^ 1, abort, dev_err))) return;
+        if (p == 0) {
+          // pub[o][b] completes once per two tiles of owner o: parity (m >> 1) & 1.
+          if (!(ok = wait_cluster(&sm.pub[s & (kCl - 1)][(s >> 3) & 1], (uint32_t)((s >> 4) & 1),
+                                  abort, dev_err)))
+            return;
+          fence_proxy_async_global();
+        }
+        if (elect_one()) {
+          mbar_expect_tx(&sm.cs_full[p], kAtom128 + (uint32_t)A * (kColAtom / 2));
+          bulk_load(sm.g[0][p], ring_tile(s) + p * kAtom128, kAtom128, &sm.cs_full[p]);
+          for (int j = 0; j < A; ++j)
+            tma_load_2d(sm.cs[j] + p * (kColAtom / 2), &tmC64, &sm.cs_full[p], k * w + j * 64,
+                        ct * BN + 64 * p);
+        }
+        __syncwarp();
+        cs_last[p] = (int)cs_ph[p];
+        cs_ph[p] ^= 1;
+      };
+      for (int s = 0; s < N && ok && ksplit; ++s, cur.next(mp)) {
+        load_khalf(0, s, cur.ct);
+        if (!ok) break;
+        load_khalf(1, s, cur.ct);
+      }
+      for (int s = 0; s < N && ok && !ksplit; ++s, cur.next(mp)) {
         load_cs(0, 0, A0, cur.ct);
         if (!ok) break;
         // Gs(s) from its owner's ring slot.
@@ -938,7 +971,34 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         const uint64_t dc1 = dc + (uint64_t)A0 * kColU;
         TileCursor cur;  // tile of slot s
         cur.init(mp, 0);
-        for (int s = 0; s < N && ok; ++s, cur.next(mp)) {
+        const uint32_t idesc_w = idesc_bf16(128, 64 * A, 0, 1);
+        for (int s = 0; s < N && ok && ksplit; ++s, cur.next(mp)) {
+          const bool unit_start = cur.unit_start(mp);
+          const bool unit_end = cur.unit_end(mp);
+          if (unit_start && !(ok = wait(&sm.o_empty, o_ph ^ 1, abort, dev_err))) break;
+          for (int p = 0; p < 2 && ok; ++p) {
+            if (!(ok = wait(&sm.cs_full[p], cs_ph[p], abort, dev_err))) break;
+            cs_ph[p] ^= 1;
+            tc_fence_after();
+            if (elect_one()) {
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+                mma_bf16(tmem_o, dg0 + p * kAtomU + q * 2,
+                         dc + p * (kColU / 2) + q * (2048 >> 4), idesc_w,
+                         !(unit_start && p == 0 && q == 0));
+              mma_commit(&sm.cs_empty[p]);
+              if (p == 1) {
+                // Tell the owner of s that this CTA is done with tile s (see below).
+                if (s + 2 * kCl < N)
+                  mma_commit_multicast(&sm.gfree[(s >> 3) & 1], (uint16_t)(1u << (s & (kCl - 1))));
+                if (unit_end) mma_commit(&sm.o_full);
+              }
+            }
+            __syncwarp();
+          }
+          if (ok && unit_end) o_ph ^= 1;
+        }
+        for (int s = 0; s < N && ok && !ksplit; ++s, cur.next(mp)) {
           const int gb = s & (kGSlots - 1);
           const bool unit_start = cur.unit_start(mp);
           const bool unit_end = cur.unit_end(mp);
@@ -1217,8 +1277,9 @@ int cluster_grid(const void *kernel, size_t smem) {
 template <int BN>
 pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStream_t s,
                              const CUtensorMap &mH, const CUtensorMap &mW128) {
-  CUtensorMap mHc, mWc;
-  if (!make_map(&mHc, w.Hc, w.Tpad, g.d, BN) || !make_map(&mWc, g.W, g.V, g.d, BN))
+  CUtensorMap mHc, mWc, mHc64, mWc64;
+  if (!make_map(&mHc, w.Hc, w.Tpad, g.d, BN) || !make_map(&mWc, g.W, g.V, g.d, BN) ||
+      !make_map(&mHc64, w.Hc, w.Tpad, g.d, 64) || !make_map(&mWc64, g.W, g.V, g.d, 64))
     return PAIR_ERR_CUDA;
   const int nsm = num_sms();
   const size_t cl_smem = sizeof(ClSmem<BN>) + 1024;
@@ -1232,7 +1293,7 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("bwd_dh_tc", s);
   bwd_cluster_kernel<true, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-      mH, mWc, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
+      mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
       static_cast<uint8_t *>(w.gring), g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("zero_tail_dw", s);
@@ -1240,7 +1301,7 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("bwd_dw_tc", s);
   bwd_cluster_kernel<false, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-      mW128, mHc, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
+      mW128, mHc, mHc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
       static_cast<uint8_t *>(w.gring), g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
