@@ -76,6 +76,14 @@ def _load():
             ctypes.c_int, ctypes.c_int, ctypes.c_int, P, P, P, P, P,
             ctypes.c_double, P, ctypes.c_int]
         lib.oracle_pair_estimate_dense.restype = ctypes.c_int
+        lib.oracle_pair_coeffs_w.argtypes = [
+            ctypes.c_int, ctypes.c_int, P, P, P, ctypes.c_double, ctypes.c_int,
+            ctypes.c_int, ctypes.c_double, P, P, P, P, P, P, P, ctypes.c_int]
+        lib.oracle_pair_coeffs_w.restype = ctypes.c_int
+        lib.oracle_pair_coeffs_product.argtypes = [
+            ctypes.c_int, ctypes.c_int, P, P, P, ctypes.c_double, ctypes.c_int,
+            P, P, P, P, P, P, P, ctypes.c_int]
+        lib.oracle_pair_coeffs_product.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -115,6 +123,53 @@ def coeffs(r, J, rho, scale=1.0, center=False, threads=None, check=True):
         raise OracleError("edge-sum and row forms disagree")
     return dict(a=a, a_mag=a_mag, active=active, edges=edges,
                 contrast=contrast, status=st)
+
+
+# Weighting variants (App. "Estimated and stabilized propensities"; ablation
+# table): edge weight 1/rho, 1, 1/(pi_i pi_j) with pi = diag(rho),
+# min(1/rho, w_max), and 1/rho self-normalised by the group's weight sum.
+W_HT, W_UNWEIGHTED, W_MARGINAL, W_CLIPPED, W_HAJEK = 0, 1, 2, 3, 4
+
+
+def _coeffs_out(B, G):
+    return dict(a=np.zeros((B, G), np.float64), a_mag=np.zeros((B, G), np.float64),
+                active=np.zeros((B, G), np.uint8), edges=np.zeros(B, np.int32),
+                contrast=np.zeros(B, np.int32), ess=np.zeros(B, np.float64),
+                max_w=np.zeros(B, np.float64))
+
+
+def coeffs_w(r, J, rho, scale=1.0, center=False, wmode=W_HT, w_max=0.0, threads=None):
+    """Coefficients under weighting variant `wmode`, with the per-group ESS
+    (sum w)^2 / sum w^2 and largest weight over the completed edges.
+    rho [B,G,G]: strict upper triangle read for the joint probabilities, its
+    diagonal for the marginals (W_MARGINAL)."""
+    r = np.ascontiguousarray(r, dtype=np.float64)
+    J = np.ascontiguousarray(J, dtype=np.uint8)
+    rho = np.ascontiguousarray(rho, dtype=np.float64)
+    B, G = r.shape
+    o = _coeffs_out(B, G)
+    st = _load().oracle_pair_coeffs_w(
+        B, G, _ptr(r), _ptr(J), _ptr(rho), float(scale), int(bool(center)), int(wmode),
+        float(w_max), _ptr(o["a"]), _ptr(o["a_mag"]), _ptr(o["active"]), _ptr(o["edges"]),
+        _ptr(o["contrast"]), _ptr(o["ess"]), _ptr(o["max_w"]), threads or n_threads())
+    o["status"] = st
+    return o
+
+
+def coeffs_product(r, J, p, scale=1.0, center=False, threads=None):
+    """Inverse-probability coefficients of the independent design, rho_ij =
+    p_i p_j, from the marginals p [B,G]; plus ESS and largest weight."""
+    r = np.ascontiguousarray(r, dtype=np.float64)
+    J = np.ascontiguousarray(J, dtype=np.uint8)
+    p = np.ascontiguousarray(p, dtype=np.float64)
+    B, G = r.shape
+    o = _coeffs_out(B, G)
+    st = _load().oracle_pair_coeffs_product(
+        B, G, _ptr(r), _ptr(J), _ptr(p), float(scale), int(bool(center)),
+        _ptr(o["a"]), _ptr(o["a_mag"]), _ptr(o["active"]), _ptr(o["edges"]),
+        _ptr(o["contrast"]), _ptr(o["ess"]), _ptr(o["max_w"]), threads or n_threads())
+    o["status"] = st
+    return o
 
 
 def estimate_dense(r, J, rho, S, scale=1.0, threads=None):

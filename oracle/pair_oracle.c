@@ -105,6 +105,94 @@ static int coeffs_group(int G, const double *r, const uint8_t *J,
     return err;
 }
 
+/*
+ * Edge weights of the estimator variants (App. "Estimated and stabilized
+ * propensities" and the ablation table of Sec. 5): for a completed edge e =
+ * (i, j) the coefficient term is 1/2 (r_i - r_j) w_e with
+ *   ORACLE_W_HT          w_e = 1 / rho_ij                (Eq. pair-ht)
+ *   ORACLE_W_UNWEIGHTED  w_e = 1                         (no pair correction)
+ *   ORACLE_W_MARGINAL    w_e = 1 / (pi_i pi_j), pi_i = rho_ii (marginal-only)
+ *   ORACLE_W_CLIPPED     w_e = min(1 / rho_ij, w_max)
+ *   ORACLE_W_HAJEK       w_e = 1 / rho_ij, and the group's coefficients are
+ *                        divided by sum_e w_e (self-normalised ratio form)
+ * Diagnostics per group over its completed edges: ESS = (sum w)^2 / sum w^2
+ * (Sec. 5 metrics) and the largest weight; both 0 without completed edges.
+ */
+#define ORACLE_W_HT 0
+#define ORACLE_W_UNWEIGHTED 1
+#define ORACLE_W_MARGINAL 2
+#define ORACLE_W_CLIPPED 3
+#define ORACLE_W_HAJEK 4
+
+/* One group, weighting variant `wmode`. Returns an ORACLE_* code. */
+static int coeffs_group_w(int G, const double *r, const uint8_t *J,
+                          const double *rho_g, double scale, int center,
+                          int wmode, double w_max, double *a, double *a_mag,
+                          uint8_t *active, int32_t *edges, int32_t *contrast,
+                          double *ess, double *max_w)
+{
+    int n_edges = 0, n_contrast = 0, err = ORACLE_OK;
+    double sum_w = 0.0, sum_w2 = 0.0, mw = 0.0;
+    for (int i = 0; i < G; ++i) { a[i] = 0.0; a_mag[i] = 0.0; active[i] = 0; }
+    /* Every completed edge i < j once; its term goes to both endpoints. */
+    for (int i = 0; i < G; ++i) {
+        for (int j = i + 1; j < G; ++j) {
+            if (!(J[i] && J[j])) continue;
+            double w;
+            if (wmode == ORACLE_W_UNWEIGHTED) {
+                w = 1.0;
+            } else if (wmode == ORACLE_W_MARGINAL) {
+                double pi = rho_g[(size_t)i * G + i], pj = rho_g[(size_t)j * G + j];
+                if (!(pi > 0.0) || !(pj > 0.0)) { err = ORACLE_ERR_NONPOSITIVE_INCLUSION; continue; }
+                w = 1.0 / (pi * pj);
+            } else {
+                double rij = rho_g[(size_t)i * G + j];
+                if (!(rij > 0.0)) { err = ORACLE_ERR_NONPOSITIVE_INCLUSION; continue; }
+                w = 1.0 / rij;
+                if (wmode == ORACLE_W_CLIPPED && w > w_max) w = w_max;
+            }
+            ++n_edges;
+            if (r[i] != r[j]) {
+                ++n_contrast;
+                active[i] = 1;
+                active[j] = 1;
+            }
+            double t = 0.5 * (r[i] - r[j]) * w;
+            a[i] += t;
+            a[j] -= t;
+            a_mag[i] += fabs(t);
+            a_mag[j] += fabs(t);
+            sum_w += w;
+            sum_w2 += w * w;
+            if (w > mw) mw = w;
+        }
+    }
+    if (wmode == ORACLE_W_HAJEK) {
+        for (int i = 0; i < G; ++i) {
+            a[i] = sum_w > 0.0 ? a[i] / sum_w : 0.0;
+            a_mag[i] = sum_w > 0.0 ? a_mag[i] / sum_w : 0.0;
+        }
+    }
+    if (center) {
+        int K = 0;
+        double sum = 0.0;
+        for (int i = 0; i < G; ++i) if (J[i]) { ++K; sum += a[i]; }
+        if (K > 0) {
+            double mean = sum / K;
+            for (int i = 0; i < G; ++i) if (J[i]) a[i] -= mean;
+        }
+    }
+    for (int i = 0; i < G; ++i) {
+        a[i] *= scale;
+        a_mag[i] *= fabs(scale);
+    }
+    *edges = n_edges;
+    *contrast = n_contrast;
+    *ess = sum_w2 > 0.0 ? sum_w * sum_w / sum_w2 : 0.0;
+    *max_w = mw;
+    return err;
+}
+
 typedef struct {
     int B, G, D, center, nthreads, tid;
     const double *r, *rho;
@@ -115,6 +203,10 @@ typedef struct {
     double *a, *a_mag, *g;
     uint8_t *active;
     int32_t *edges, *contrast;
+    int wmode;
+    double w_max;
+    const double *p;       /* product design: marginals [B][G] */
+    double *ess, *max_w;
     int err;
 } job_t;
 
@@ -129,6 +221,38 @@ static void *coeffs_worker(void *p)
                              jb->active + o, jb->edges + b, jb->contrast + b);
         if (e && !jb->err) jb->err = e;
     }
+    return NULL;
+}
+
+static void *coeffs_w_worker(void *p)
+{
+    job_t *jb = (job_t *)p;
+    int G = jb->G;
+    double *rho_tmp = NULL;
+    if (jb->p) {
+        rho_tmp = (double *)malloc(sizeof(double) * (size_t)G * G);
+        if (!rho_tmp) { jb->err = ORACLE_ERR_ALLOC; return NULL; }
+    }
+    for (int b = jb->tid; b < jb->B; b += jb->nthreads) {
+        size_t o = (size_t)b * G;
+        const double *rho_g;
+        if (jb->p) {
+            /* Independent Bernoulli design: rho_ij = p_i p_j (Sec. 4, the
+             * product design), rho_ii = p_i. */
+            for (int i = 0; i < G; ++i)
+                for (int j = 0; j < G; ++j)
+                    rho_tmp[(size_t)i * G + j] = i == j ? jb->p[o + i] : jb->p[o + i] * jb->p[o + j];
+            rho_g = rho_tmp;
+        } else {
+            rho_g = jb->rho + o * G;
+        }
+        int e = coeffs_group_w(G, jb->r + o, jb->J + o, rho_g, jb->scale, jb->center,
+                               jb->wmode, jb->w_max, jb->a + o, jb->a_mag + o,
+                               jb->active + o, jb->edges + b, jb->contrast + b,
+                               jb->ess + b, jb->max_w + b);
+        if (e && !jb->err) jb->err = e;
+    }
+    free(rho_tmp);
     return NULL;
 }
 
@@ -221,4 +345,41 @@ int oracle_pair_estimate_dense(int B, int G, int D, const double *r,
     jb.B = B; jb.G = G; jb.D = D; jb.r = r; jb.J = J; jb.rho = rho;
     jb.S32 = S32; jb.S64 = S64; jb.scale = scale; jb.g = g;
     return run_jobs(&jb, nthreads, dense_worker);
+}
+
+/*
+ * Coefficients under a weighting variant (ORACLE_W_*, see coeffs_group_w),
+ * with the per-group ESS and largest weight of the completed edges.
+ */
+int oracle_pair_coeffs_w(int B, int G, const double *r, const uint8_t *J,
+                         const double *rho, double scale, int center, int wmode,
+                         double w_max, double *a, double *a_mag, uint8_t *active,
+                         int32_t *edges, int32_t *contrast, double *ess,
+                         double *max_w, int nthreads)
+{
+    job_t jb = {0};
+    jb.B = B; jb.G = G; jb.center = center; jb.r = r; jb.J = J; jb.rho = rho;
+    jb.scale = scale; jb.a = a; jb.a_mag = a_mag; jb.active = active;
+    jb.edges = edges; jb.contrast = contrast; jb.wmode = wmode; jb.w_max = w_max;
+    jb.ess = ess; jb.max_w = max_w;
+    return run_jobs(&jb, nthreads, coeffs_w_worker);
+}
+
+/*
+ * Inverse-probability coefficients of the independent (product) design:
+ * rho_ij = p_i p_j, i.e. ORACLE_W_HT on the joint probabilities formed from
+ * the marginals p[B][G].
+ */
+int oracle_pair_coeffs_product(int B, int G, const double *r, const uint8_t *J,
+                               const double *p, double scale, int center,
+                               double *a, double *a_mag, uint8_t *active,
+                               int32_t *edges, int32_t *contrast, double *ess,
+                               double *max_w, int nthreads)
+{
+    job_t jb = {0};
+    jb.B = B; jb.G = G; jb.center = center; jb.r = r; jb.J = J; jb.p = p;
+    jb.scale = scale; jb.a = a; jb.a_mag = a_mag; jb.active = active;
+    jb.edges = edges; jb.contrast = contrast; jb.wmode = ORACLE_W_HT;
+    jb.ess = ess; jb.max_w = max_w;
+    return run_jobs(&jb, nthreads, coeffs_w_worker);
 }
