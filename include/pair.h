@@ -113,6 +113,75 @@ PAIR_API pair_status pair_coeffs(int32_t B, int32_t G, const float *r, const uin
                         pair_stream_t stream);
 
 /*
+ * Edge weightings of pair_coeffs_weighted (App. "Estimated and stabilized
+ * propensities"; the ablation variants of Sec. 5). For a completed edge
+ * (i, j) the coefficient term is 1/2 (r_i - r_j) w_ij with
+ *   PAIR_W_HT          w = 1/rho_ij                  (Eq. pair-ht; exact)
+ *   PAIR_W_UNWEIGHTED  w = 1                         (no pair correction)
+ *   PAIR_W_MARGINAL    w = 1/(pi_i pi_j), pi_i = rho_ii (marginal-only)
+ *   PAIR_W_CLIPPED     w = min(1/rho_ij, w_max)
+ *   PAIR_W_HAJEK       w = 1/rho_ij, and the group's coefficients divided by
+ *                      the sum of w over its completed edges (self-normalised
+ *                      ratio form; 0 when there is no completed edge).
+ * Only PAIR_W_HT is unbiased for the complete-pair target (Thm. 2); the
+ * others are the paper's biased comparison variants.
+ */
+typedef enum {
+  PAIR_W_HT = 0,
+  PAIR_W_UNWEIGHTED = 1,
+  PAIR_W_MARGINAL = 2,
+  PAIR_W_CLIPPED = 3,
+  PAIR_W_HAJEK = 4
+} pair_weighting;
+
+/*
+ * pair_coeffs_weighted -- pair_coeffs under a weighting variant, with the
+ * per-group diagnostics of App. D: ESS = (sum_e w_e)^2 / sum_e w_e^2 and the
+ * largest weight over the completed edges (both 0 without one).
+ *
+ * In:  as pair_coeffs, plus wmode (pair_weighting) and w_max (> 0 and finite
+ *      for PAIR_W_CLIPPED, ignored otherwise). rho's strict upper triangle
+ *      is read for the joint probabilities (not at all for
+ *      PAIR_W_UNWEIGHTED); its diagonal only for PAIR_W_MARGINAL.
+ *      PAIR_CENTER centres after the weighting (and the Hajek division).
+ * Out: a, active, edges, contrast_edges as pair_coeffs (active and the edge
+ *      counts do not depend on the weighting);
+ *      ess [B], max_w [B] float32 (nullable).
+ * Errors: PAIR_ERR_INVALID_ARG for the pair_coeffs conditions, an unknown
+ *      wmode, or a non-positive / non-finite w_max with PAIR_W_CLIPPED;
+ *      device: rho_ij <= 0 or NaN on a completed edge (pi_i, pi_j for
+ *      PAIR_W_MARGINAL) -> PAIR_DEV_ERR_NONPOSITIVE_INCLUSION.
+ * Arithmetic: fp32, IEEE division and reciprocal, fixed tree sums.
+ */
+PAIR_API pair_status pair_coeffs_weighted(int32_t B, int32_t G, const float *r,
+                                          const uint8_t *J, const float *rho, float scale,
+                                          uint32_t flags, pair_weighting wmode, float w_max,
+                                          float *a, uint8_t *active, int32_t *edges,
+                                          int32_t *contrast_edges, float *ess, float *max_w,
+                                          int32_t *dev_err, pair_stream_t stream);
+
+/*
+ * pair_coeffs_product -- the coefficients of pair_coeffs for the independent
+ * (product) design, rho_ij = p_i p_j (Sec. 4: independent Bernoulli
+ * continuation), from the marginals alone:
+ *     a_i = scale * 1/2 (J_i / p_i) sum_{j != i} J_j (r_i - r_j) / p_j,
+ * reading 9 bytes per candidate instead of a G x G matrix per group.
+ *
+ * In:  r, J as pair_coeffs; p [B][G] float32 marginal inclusion probabilities
+ *      (read where J_i = 1); scale, flags as pair_coeffs.
+ * Out: a, active, edges, contrast_edges as pair_coeffs; ess, max_w as
+ *      pair_coeffs_weighted for the weights 1/(p_i p_j) (nullable).
+ * Errors: as pair_coeffs; device: p_i <= 0 or NaN where J_i = 1 ->
+ *      PAIR_DEV_ERR_NONPOSITIVE_INCLUSION.
+ */
+PAIR_API pair_status pair_coeffs_product(int32_t B, int32_t G, const float *r,
+                                         const uint8_t *J, const float *p, float scale,
+                                         uint32_t flags, float *a, uint8_t *active,
+                                         int32_t *edges, int32_t *contrast_edges, float *ess,
+                                         float *max_w, int32_t *dev_err,
+                                         pair_stream_t stream);
+
+/*
  * pair_estimate_dense -- Eq. (pair-ht) for explicit score vectors:
  *     g_b = scale * sum_{i<j} J_iJ_j h_ij / rho_ij = sum_i a_i s_{b,i}
  * (the coefficient collapse of Eq. pair-advantage; rows with a_i = 0 are

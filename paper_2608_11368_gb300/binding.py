@@ -70,6 +70,11 @@ def lib() -> ctypes.CDLL:
     L.pair_timing_enable.restype = None
     L.pair_timing_read.argtypes = [I32, P, P]
     L.pair_timing_read.restype = I32
+    L.pair_coeffs_weighted.argtypes = [I32, I32, P, P, P, F32, U32, ctypes.c_int, F32,
+                                       P, P, P, P, P, P, P, P]
+    L.pair_coeffs_weighted.restype = ctypes.c_int
+    L.pair_coeffs_product.argtypes = [I32, I32, P, P, P, F32, U32, P, P, P, P, P, P, P, P]
+    L.pair_coeffs_product.restype = ctypes.c_int
     L.pair_selftest_wait_timeout.argtypes = [I64, P, P, P]
     L.pair_selftest_wait_timeout.restype = ctypes.c_int
     _lib = L
@@ -150,6 +155,49 @@ def pair_coeffs(r, J, rho, scale=1.0, flags=0, a=None, active=None, edges=None,
                            _p(dev_err), _stream(stream))
     _check(st, "pair_coeffs")
     return a, active, edges, contrast_edges
+
+
+PAIR_W_HT, PAIR_W_UNWEIGHTED, PAIR_W_MARGINAL, PAIR_W_CLIPPED, PAIR_W_HAJEK = 0, 1, 2, 3, 4
+
+
+def _coeffs_outputs(B, G, dev, a, active, edges, contrast_edges, ess, max_w):
+    f = lambda t, shape, dt: torch.empty(shape, dtype=dt, device=dev) if t is None else t
+    return (f(a, (B, G), torch.float32), f(active, (B, G), torch.uint8),
+            f(edges, (B,), torch.int32), f(contrast_edges, (B,), torch.int32),
+            f(ess, (B,), torch.float32), f(max_w, (B,), torch.float32))
+
+
+def pair_coeffs_weighted(r, J, rho, wmode=PAIR_W_HT, w_max=0.0, scale=1.0, flags=0, a=None,
+                         active=None, edges=None, contrast_edges=None, ess=None, max_w=None,
+                         dev_err=None, stream=None):
+    """pair_coeffs under a weighting variant (see pair.h), with per-group ESS
+    and largest weight. Returns (a, active, edges, contrast_edges, ess, max_w)."""
+    B, G = r.shape
+    _need(r, "r", torch.float32)
+    _need(J, "J", torch.uint8, (B, G))
+    if rho is not None:
+        _need(rho, "rho", torch.float32, (B, G, G))
+    outs = _coeffs_outputs(B, G, r.device, a, active, edges, contrast_edges, ess, max_w)
+    st = lib().pair_coeffs_weighted(B, G, _p(r), _p(J), _p(rho), float(scale), int(flags),
+                                    int(wmode), float(w_max), *[_p(t) for t in outs],
+                                    _p(dev_err), _stream(stream))
+    _check(st, "pair_coeffs_weighted")
+    return outs
+
+
+def pair_coeffs_product(r, J, p, scale=1.0, flags=0, a=None, active=None, edges=None,
+                        contrast_edges=None, ess=None, max_w=None, dev_err=None, stream=None):
+    """Coefficients of the independent design rho_ij = p_i p_j from the
+    marginals p [B, G]. Returns (a, active, edges, contrast_edges, ess, max_w)."""
+    B, G = r.shape
+    _need(r, "r", torch.float32)
+    _need(J, "J", torch.uint8, (B, G))
+    _need(p, "p", torch.float32, (B, G))
+    outs = _coeffs_outputs(B, G, r.device, a, active, edges, contrast_edges, ess, max_w)
+    st = lib().pair_coeffs_product(B, G, _p(r), _p(J), _p(p), float(scale), int(flags),
+                                   *[_p(t) for t in outs], _p(dev_err), _stream(stream))
+    _check(st, "pair_coeffs_product")
+    return outs
 
 
 def pair_estimate_dense(r, J, rho, S, scale=1.0, g=None, a=None, dev_err=None,

@@ -95,6 +95,39 @@ pair_status pair_coeffs(int32_t B, int32_t G, const float *r, const uint8_t *J,
                        reinterpret_cast<cudaStream_t>(stream));
 }
 
+pair_status pair_coeffs_weighted(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                                 const float *rho, float scale, uint32_t flags,
+                                 pair_weighting wmode, float w_max, float *a, uint8_t *active,
+                                 int32_t *edges, int32_t *contrast_edges, float *ess,
+                                 float *max_w, int32_t *dev_err, pair_stream_t stream) {
+  reset_launches();
+  if (B < 1 || G < 2 || G > PAIR_MAX_G || !r || !J || !a || (flags & ~PAIR_CENTER) != 0)
+    return PAIR_ERR_INVALID_ARG;
+  const int wm = (int)wmode;
+  if (wm < PAIR_W_HT || wm > PAIR_W_HAJEK) return PAIR_ERR_INVALID_ARG;
+  if (wm != PAIR_W_UNWEIGHTED && !rho) return PAIR_ERR_INVALID_ARG;
+  if (wm == PAIR_W_CLIPPED && !(w_max > 0.f && w_max <= 3.0e38f)) return PAIR_ERR_INVALID_ARG;
+  const pair_status dv = check_device();
+  if (dv != PAIR_OK) return dv;
+  return launch_coeffs_weighted(B, G, r, J, rho, scale, flags, wm, w_max, a, active, edges,
+                                contrast_edges, ess, max_w, dev_err,
+                                reinterpret_cast<cudaStream_t>(stream));
+}
+
+pair_status pair_coeffs_product(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                                const float *p, float scale, uint32_t flags, float *a,
+                                uint8_t *active, int32_t *edges, int32_t *contrast_edges,
+                                float *ess, float *max_w, int32_t *dev_err,
+                                pair_stream_t stream) {
+  reset_launches();
+  if (B < 1 || G < 2 || G > PAIR_MAX_G || !r || !J || !p || !a || (flags & ~PAIR_CENTER) != 0)
+    return PAIR_ERR_INVALID_ARG;
+  const pair_status dv = check_device();
+  if (dv != PAIR_OK) return dv;
+  return launch_coeffs_product(B, G, r, J, p, scale, flags, a, active, edges, contrast_edges,
+                               ess, max_w, dev_err, reinterpret_cast<cudaStream_t>(stream));
+}
+
 pair_status pair_estimate_dense(int32_t B, int32_t G, int32_t D,
                                 const float *r, const uint8_t *J,
                                 const float *rho, const float *S, float scale,

@@ -262,6 +262,265 @@ __global__ void __launch_bounds__(256, 4) dense_kernel(
   }
 }
 
+// Deterministic block maximum of one float per thread (all threads call).
+__device__ float block_max_float(float v, float *red) {
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  const int w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[w] = v;
+  __syncthreads();
+  float m = 0.f;
+  for (int k = 0; k < nw; ++k) m = fmaxf(m, red[k]);
+  return m;
+}
+
+// Sum of the 2^l-blocked pairwise tree over x_0 .. x_{GP-1} (the same fixed
+// order the HT kernel uses for its row sums).
+template <int GP>
+struct PairwiseSum {
+  float p[8];
+  __device__ __forceinline__ void add(int k, float x) {
+    float c = x;
+    int m = k;
+#pragma unroll
+    for (int l = 0; l < 8; ++l) {
+      if (m & 1) { c = p[l] + c; m >>= 1; }
+      else { p[l] = c; break; }
+    }
+  }
+  __device__ __forceinline__ float total() const { return p[(GP == 32) ? 5 : (GP == 64) ? 6 : 7]; }
+};
+
+template <int GP>
+struct GroupSmemW {
+  float U[GP * (GP - 1) / 2];  // strict upper triangle of terms (r_i - r_j) w_ij
+  float r[GP];
+  float pi[GP];                // marginals (rho diagonal) or 1/p (product path)
+  int8_t J[GP];
+  int red_i[32];
+  float red_f[32];
+};
+
+// Coefficients under a weighting variant (see pair_coeffs_weighted), plus
+// the ESS and largest weight of the group's completed edges. One block of GP
+// threads per group; the upper triangle is read by row pairs as in
+// coeffs_kernel, every term placed once, every vertex summed by the fixed
+// pairwise tree.
+template <int GP>
+__global__ void __launch_bounds__(GP, 4) coeffs_w_kernel(
+    int B, int G, const float *__restrict__ r, const uint8_t *__restrict__ J,
+    const float *__restrict__ rho, float scale, int center, int wmode, float w_max,
+    float *__restrict__ a, uint8_t *__restrict__ active, int32_t *__restrict__ edges,
+    int32_t *__restrict__ contrast, float *__restrict__ ess, float *__restrict__ max_w,
+    int32_t *dev_err) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  GroupSmemW<GP> &sm = *reinterpret_cast<GroupSmemW<GP> *>(smem_raw);
+  const int b = blockIdx.x, tid = threadIdx.x;
+  const size_t gbase = (size_t)b * G;
+  const float *rho_g = rho + (size_t)b * G * G;
+  {
+    const bool in = tid < G;
+    sm.r[tid] = in ? r[gbase + tid] : 0.f;
+    sm.J[tid] = in ? (J[gbase + tid] != 0) : 0;
+    sm.pi[tid] = (in && wmode == PAIR_W_MARGINAL) ? rho_g[(size_t)tid * G + tid] : 1.f;
+  }
+  __syncthreads();
+  const bool needs_rho = wmode == PAIR_W_HT || wmode == PAIR_W_CLIPPED || wmode == PAIR_W_HAJEK;
+  int my_contrast = 0, bad = 0;
+  float sw = 0.f, sw2 = 0.f, mw = 0.f;
+  if (tid < GP - 1) {
+    float v[GP / 2];
+#pragma unroll
+    for (int k = 0; k < GP / 2; ++k) {
+      const int n1 = GP - 1 - k;
+      int i, j;
+      if (tid < n1) { i = k; j = k + 1 + tid; }
+      else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
+      const bool live = (j < G) && sm.J[i] && sm.J[j];
+      v[k] = (live && needs_rho) ? __ldg(rho_g + (size_t)i * G + j) : 1.f;
+    }
+#pragma unroll
+    for (int k = 0; k < GP / 2; ++k) {
+      const int n1 = GP - 1 - k;
+      int i, j;
+      if (tid < n1) { i = k; j = k + 1 + tid; }
+      else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
+      const bool live = (j < G) && sm.J[i] && sm.J[j];
+      float t = 0.f;
+      if (live) {
+        const float dr = sm.r[i] - sm.r[j];
+        float w = 1.f;
+        bool okw = true;
+        if (wmode == PAIR_W_UNWEIGHTED) {
+          t = dr;
+        } else if (wmode == PAIR_W_MARGINAL) {
+          const float pi = sm.pi[i], pj = sm.pi[j];
+          okw = (pi > 0.f) && (pj > 0.f);
+          const float den = pi * pj;
+          t = okw ? __fdiv_rn(dr, den) : 0.f;
+          w = okw ? __frcp_rn(den) : 0.f;
+        } else {
+          const float rij = v[k];
+          okw = rij > 0.f;
+          w = okw ? __frcp_rn(rij) : 0.f;
+          if (wmode == PAIR_W_CLIPPED && w > w_max) {
+            w = w_max;
+            t = dr * w_max;
+          } else {
+            t = okw ? __fdiv_rn(dr, rij) : 0.f;
+          }
+        }
+        if (!okw) {
+          bad = 1;
+        } else {
+          my_contrast += (sm.r[i] != sm.r[j]);
+          sw += w;
+          sw2 = fmaf(w, w, sw2);
+          mw = fmaxf(mw, w);
+        }
+      }
+      sm.U[upper_off<GP>(i, j)] = t;
+    }
+  }
+  if (bad) flag_error(dev_err, PAIR_DEV_ERR_NONPOSITIVE_INCLUSION);
+  const float W = block_sum_float(sw, sm.red_f);
+  const float W2 = block_sum_float(sw2, sm.red_f);
+  const float Wmax = block_max_float(mw, sm.red_f);
+  __syncthreads();
+
+  PairwiseSum<GP> ps;
+  bool nz = false;
+#pragma unroll
+  for (int k = 0; k < GP; ++k) {
+    float x = 0.f;
+    if (k < tid) x = -sm.U[upper_off<GP>(k, tid)];
+    else if (k > tid) x = sm.U[upper_off<GP>(tid, k)];
+    nz |= (x != 0.f);
+    ps.add(k, x);
+  }
+  const float sum = ps.total();
+  float av = (sum == 0.f) ? 0.f : 0.5f * sum;
+  if (wmode == PAIR_W_HAJEK) av = W > 0.f ? __fdiv_rn(av, W) : 0.f;
+  const uint8_t act = (tid < G && sm.J[tid] && nz) ? 1 : 0;
+  const int packed = block_sum_int((int)sm.J[tid] | (my_contrast << 16), sm.red_i);
+  const int K = packed & 0xffff, C = packed >> 16;
+  if (center && K > 0) {
+    const float s2 = block_sum_float(sm.J[tid] ? av : 0.f, sm.red_f);
+    const float mean = s2 / (float)K;
+    if (sm.J[tid]) av -= mean;
+  }
+  if (tid < G) {
+    a[gbase + tid] = av * scale;
+    if (active) active[gbase + tid] = act;
+  }
+  if (tid == 0) {
+    if (edges) edges[b] = K * (K - 1) / 2;
+    if (contrast) contrast[b] = C;
+    if (ess) ess[b] = W2 > 0.f ? __fdiv_rn(W * W, W2) : 0.f;
+    if (max_w) max_w[b] = Wmax;
+  }
+}
+
+// Independent (product) design: rho_ij = p_i p_j, so the coefficients need
+// only the marginals p [B][G]: a_i = 1/2 (J_i / p_i) sum_{j != i} J_j
+// (r_i - r_j) / p_j, summed per vertex by the fixed pairwise tree (the same
+// terms as the joint form, without reading a G x G matrix).
+template <int GP>
+__global__ void __launch_bounds__(GP, 4) coeffs_product_kernel(
+    int B, int G, const float *__restrict__ r, const uint8_t *__restrict__ J,
+    const float *__restrict__ p, float scale, int center, float *__restrict__ a,
+    uint8_t *__restrict__ active, int32_t *__restrict__ edges, int32_t *__restrict__ contrast,
+    float *__restrict__ ess, float *__restrict__ max_w, int32_t *dev_err) {
+  __shared__ float sr[GP], sq[GP];
+  __shared__ int8_t sJ[GP];
+  __shared__ int red_i[32];
+  __shared__ float red_f[32];
+  const int b = blockIdx.x, tid = threadIdx.x;
+  const size_t gbase = (size_t)b * G;
+  int bad = 0;
+  {
+    const bool in = tid < G;
+    const bool j = in && J[gbase + tid] != 0;
+    const float pv = in ? p[gbase + tid] : 1.f;
+    if (j && !(pv > 0.f)) bad = 1;
+    sr[tid] = in ? r[gbase + tid] : 0.f;
+    sJ[tid] = (j && pv > 0.f) ? 1 : 0;
+    sq[tid] = (j && pv > 0.f) ? __frcp_rn(pv) : 0.f;
+  }
+  if (bad) flag_error(dev_err, PAIR_DEV_ERR_NONPOSITIVE_INCLUSION);
+  __syncthreads();
+  PairwiseSum<GP> ps;
+  bool nz = false;
+  int my_contrast = 0;
+  float sw = 0.f, sw2 = 0.f, mw = 0.f;
+  const float ri = sr[tid], qi = sq[tid];
+  const bool Ji = sJ[tid] != 0;
+#pragma unroll
+  for (int k = 0; k < GP; ++k) {
+    const float x = (k != tid && Ji && sJ[k]) ? (ri - sr[k]) * sq[k] : 0.f;
+    nz |= (x != 0.f);
+    ps.add(k, x);
+    if (k > tid && Ji && sJ[k]) {
+      const float w = qi * sq[k];
+      sw += w;
+      sw2 = fmaf(w, w, sw2);
+      mw = fmaxf(mw, w);
+      my_contrast += (ri != sr[k]);
+    }
+  }
+  const float sum = ps.total();
+  float av = (sum == 0.f) ? 0.f : 0.5f * qi * sum;
+  const float W = block_sum_float(sw, red_f);
+  const float W2 = block_sum_float(sw2, red_f);
+  const float Wmax = block_max_float(mw, red_f);
+  const int packed = block_sum_int((int)sJ[tid] | (my_contrast << 16), red_i);
+  const int K = packed & 0xffff, C = packed >> 16;
+  if (center && K > 0) {
+    const float s2 = block_sum_float(Ji ? av : 0.f, red_f);
+    const float mean = s2 / (float)K;
+    if (Ji) av -= mean;
+  }
+  if (tid < G) {
+    a[gbase + tid] = av * scale;
+    if (active) active[gbase + tid] = (Ji && nz) ? 1 : 0;
+  }
+  if (tid == 0) {
+    if (edges) edges[b] = K * (K - 1) / 2;
+    if (contrast) contrast[b] = C;
+    if (ess) ess[b] = W2 > 0.f ? __fdiv_rn(W * W, W2) : 0.f;
+    if (max_w) max_w[b] = Wmax;
+  }
+}
+
+template <int GP>
+pair_status launch_coeffs_w_gp(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                               const float *rho, float scale, uint32_t flags, int wmode,
+                               float w_max, float *a, uint8_t *active, int32_t *edges,
+                               int32_t *contrast, float *ess, float *max_w, int32_t *dev_err,
+                               cudaStream_t s) {
+  const size_t smem = sizeof(GroupSmemW<GP>);
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(coeffs_w_kernel<GP>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  PAIR_BEGIN("coeffs_w", s);
+  coeffs_w_kernel<GP><<<B, GP, smem, s>>>(B, G, r, J, rho, scale, (flags & PAIR_CENTER) ? 1 : 0,
+                                          wmode, w_max, a, active, edges, contrast, ess, max_w,
+                                          dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+template <int GP>
+pair_status launch_coeffs_product_gp(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                                     const float *p, float scale, uint32_t flags, float *a,
+                                     uint8_t *active, int32_t *edges, int32_t *contrast,
+                                     float *ess, float *max_w, int32_t *dev_err, cudaStream_t s) {
+  PAIR_BEGIN("coeffs_product", s);
+  coeffs_product_kernel<GP><<<B, GP, 0, s>>>(B, G, r, J, p, scale, (flags & PAIR_CENTER) ? 1 : 0,
+                                             a, active, edges, contrast, ess, max_w, dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
 template <int GP>
 pair_status launch_coeffs_gp(int32_t B, int32_t G, const float *r,
                              const uint8_t *J, const float *rho, float scale,
@@ -311,6 +570,35 @@ pair_status launch_coeffs(int32_t B, int32_t G, const float *r,
                                 edges, contrast, dev_err, s);
   return launch_coeffs_gp<128>(B, G, r, J, rho, scale, flags, a, active,
                                edges, contrast, dev_err, s);
+}
+
+pair_status launch_coeffs_weighted(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                                   const float *rho, float scale, uint32_t flags, int wmode,
+                                   float w_max, float *a, uint8_t *active, int32_t *edges,
+                                   int32_t *contrast, float *ess, float *max_w,
+                                   int32_t *dev_err, cudaStream_t s) {
+  if (G <= 32)
+    return launch_coeffs_w_gp<32>(B, G, r, J, rho, scale, flags, wmode, w_max, a, active, edges,
+                                  contrast, ess, max_w, dev_err, s);
+  if (G <= 64)
+    return launch_coeffs_w_gp<64>(B, G, r, J, rho, scale, flags, wmode, w_max, a, active, edges,
+                                  contrast, ess, max_w, dev_err, s);
+  return launch_coeffs_w_gp<128>(B, G, r, J, rho, scale, flags, wmode, w_max, a, active, edges,
+                                 contrast, ess, max_w, dev_err, s);
+}
+
+pair_status launch_coeffs_product(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                                  const float *p, float scale, uint32_t flags, float *a,
+                                  uint8_t *active, int32_t *edges, int32_t *contrast, float *ess,
+                                  float *max_w, int32_t *dev_err, cudaStream_t s) {
+  if (G <= 32)
+    return launch_coeffs_product_gp<32>(B, G, r, J, p, scale, flags, a, active, edges, contrast,
+                                        ess, max_w, dev_err, s);
+  if (G <= 64)
+    return launch_coeffs_product_gp<64>(B, G, r, J, p, scale, flags, a, active, edges, contrast,
+                                        ess, max_w, dev_err, s);
+  return launch_coeffs_product_gp<128>(B, G, r, J, p, scale, flags, a, active, edges, contrast,
+                                       ess, max_w, dev_err, s);
 }
 
 pair_status launch_estimate_dense(int32_t B, int32_t G, int32_t D,

@@ -43,6 +43,15 @@ pair_status launch_estimate_dense(int32_t B, int32_t G, int32_t D,
                                   const float *rho, const float *S,
                                   float scale, float *g, float *a,
                                   int32_t *dev_err, cudaStream_t s);
+pair_status launch_coeffs_weighted(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                                   const float *rho, float scale, uint32_t flags, int wmode,
+                                   float w_max, float *a, uint8_t *active, int32_t *edges,
+                                   int32_t *contrast, float *ess, float *max_w,
+                                   int32_t *dev_err, cudaStream_t s);
+pair_status launch_coeffs_product(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                                  const float *p, float scale, uint32_t flags, float *a,
+                                  uint8_t *active, int32_t *edges, int32_t *contrast, float *ess,
+                                  float *max_w, int32_t *dev_err, cudaStream_t s);
 
 // pair_grad pieces (pair_grad_prep.cu, pair_grad_simt.cu, pair_grad_tc.cu).
 struct GradWorkspace {
