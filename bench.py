@@ -450,6 +450,25 @@ def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
     t_d = timed(lambda: B.pair_estimate_dense(r, J, rho, S, g=g, a=a), reps)
     n_act = int((a != 0).sum().item())
     bytes_c = Bn * (4 * G * (G - 1) // 2 + 4 * G + G + 4 * G + G + 8)
+    # Weighting variants (same rho traffic plus the two diagnostics words)
+    # and the product-design path (marginals only: r, J, p in; a, active,
+    # counts and diagnostics out).
+    ess = torch.empty(Bn, dtype=torch.float32, device="cuda")
+    mw = torch.empty(Bn, dtype=torch.float32, device="cuda")
+    p = dv(inp["p"])
+    variants = {}
+    for name, mode in (("clipped", B.PAIR_W_CLIPPED), ("self_normalised", B.PAIR_W_HAJEK)):
+        t_w = timed(lambda: B.pair_coeffs_weighted(r, J, rho, wmode=mode, w_max=20.0, a=a,
+                                                   active=act, edges=e1, contrast_edges=e2,
+                                                   ess=ess, max_w=mw), reps)
+        bw = bytes_c + 8 * Bn
+        variants[name] = {"bound": "hbm", "achieved": bw / (t_w / 1e3) / 1e9,
+                          "peak": peaks["hbm"], "unit": "GB/s",
+                          "frac": bw / (t_w / 1e3) / 1e9 / peaks["hbm"], "traffic": None,
+                          "ms": t_w, "algorithmic_bytes": bw}
+    t_p = timed(lambda: B.pair_coeffs_product(r, J, p, a=a, active=act, edges=e1,
+                                              contrast_edges=e2, ess=ess, max_w=mw), reps)
+    bytes_p = Bn * (4 * G + G + 4 * G + 4 * G + G + 16)
     bytes_d = 4 * D * n_act + Bn * (4 * G * (G - 1) // 2 + 4 * G + G) + 4 * Bn * D + 4 * Bn * G
     gbs_c = bytes_c / (t_c / 1e3) / 1e9
     gbs_d = bytes_d / (t_d / 1e3) / 1e9
@@ -463,6 +482,12 @@ def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
                                 "unit": "GB/s", "frac": gbs_d / peaks["hbm"],
                                 "traffic": traffic.get(("dense", STRESS)),
                                 "ms": t_d, "algorithmic_bytes": bytes_d},
+        "pair_coeffs_weighted": variants,
+        "pair_coeffs_product": {"bound": "hbm", "achieved": bytes_p / (t_p / 1e3) / 1e9,
+                                "peak": peaks["hbm"], "unit": "GB/s",
+                                "frac": bytes_p / (t_p / 1e3) / 1e9 / peaks["hbm"],
+                                "traffic": None, "ms": t_p, "algorithmic_bytes": bytes_p,
+                                "speedup_vs_joint_rho": t_c / t_p},
         "timing": ("median of %d single launches; CUDA events recorded by the library "
                    "around its own launch; L2 flushed before each" % reps),
     }

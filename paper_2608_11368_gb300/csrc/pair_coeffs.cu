@@ -307,7 +307,7 @@ struct GroupSmemW {
 // coeffs_kernel, every term placed once, every vertex summed by the fixed
 // pairwise tree.
 template <int GP>
-__global__ void __launch_bounds__(GP, 4) coeffs_w_kernel(
+__global__ void __launch_bounds__(GP, 1024 / GP) coeffs_w_kernel(
     int B, int G, const float *__restrict__ r, const uint8_t *__restrict__ J,
     const float *__restrict__ rho, float scale, int center, int wmode, float w_max,
     float *__restrict__ a, uint8_t *__restrict__ active, int32_t *__restrict__ edges,
