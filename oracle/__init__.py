@@ -172,6 +172,39 @@ def coeffs_product(r, J, p, scale=1.0, center=False, threads=None):
     return o
 
 
+def audit(r, rho, S, Jdraws, draw_weight=None, scale=1.0, center=False, wmode=W_HT,
+          w_max=0.0):
+    """Frozen-population audit (Sec. 5; App. D metrics) of one group over
+    design draws, formed explicitly in fp64: every draw's estimate
+    ghat_b = sum_i a_bi s_i from the oracle's coefficients (coefficient form of
+    Eq. pair-ht), the target g = scale * sum_{i<j} h_ij from explicit pair
+    kernels (Eq. pair-kernel). Returns dict of weighted means (see pair.h)."""
+    r = np.asarray(r, np.float64)
+    S = np.asarray(S, np.float64)
+    Jdraws = np.asarray(Jdraws, np.uint8)
+    N, G = Jdraws.shape
+    w = np.full(N, 1.0 / N) if draw_weight is None else np.asarray(draw_weight, np.float64)
+    rho = np.ones((G, G)) if rho is None else np.asarray(rho, np.float64)
+    g = np.zeros(S.shape[1])
+    for i in range(G):
+        for j in range(i + 1, G):
+            g += 0.5 * (r[i] - r[j]) * (S[i] - S[j])
+    g *= scale
+    o = coeffs_w(np.repeat(r[None], N, 0), Jdraws, np.repeat(rho[None], N, 0), scale=scale,
+                 center=center, wmode=wmode, w_max=w_max)
+    ghat = o["a"] @ S
+    W = w.sum()
+    err2 = ((ghat - g) ** 2).sum(axis=1)
+    nrm = np.sqrt((ghat ** 2).sum(axis=1)) * np.sqrt((g ** 2).sum())
+    cos = np.where(nrm > 0, (ghat @ g) / np.where(nrm > 0, nrm, 1.0), 0.0)
+    K = Jdraws.astype(np.int64).sum(axis=1)
+    bias = (w @ ghat) / W - g
+    return dict(bias_norm=float(np.sqrt((bias ** 2).sum())), mse=float(w @ err2 / W),
+                cos=float(w @ cos / W), vertices=float(w @ K / W),
+                edges=float(w @ (K * (K - 1) // 2) / W), ess=float(w @ o["ess"] / W),
+                target_sq=float((g ** 2).sum()), weight=float(W), bias=bias, status=o["status"])
+
+
 def estimate_dense(r, J, rho, S, scale=1.0, threads=None):
     """Eq. (pair-ht) times M*scale: scale * sum_{i<j} J_iJ_j h_ij/rho_ij with
     h_ij = 1/2 (r_i - r_j)(s_i - s_j) formed explicitly. S [B,G,D]."""

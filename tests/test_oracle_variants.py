@@ -254,3 +254,75 @@ def test_marginal_rejects_nonpositive_marginal():
     rho[0, 2, 2] = 0.0
     assert oracle.coeffs_w(r, J, rho, wmode=oracle.W_MARGINAL)["status"] == 1
     assert oracle.coeffs_w(r, J, rho, wmode=oracle.W_HT)["status"] == 0
+
+
+# ------------------------------------------------ frozen-population audit
+
+def _exhaustive_draws(p):
+    draws, probs = [], []
+    for J, prob in _independent_design(p):
+        draws.append(J); probs.append(prob)
+    return np.array(draws, np.uint8), np.array(probs)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_audit_exact_design_moments(seed):
+    """Over all 2^G inclusion sets weighted by their probability: HT has zero
+    bias (Thm. 2) and MSE equal to the trace of Prop. bias's covariance; the
+    vertex and edge counts have means sum p_i and sum_{i<j} p_i p_j."""
+    rng = _rng(700 + seed)
+    G = int(rng.integers(3, 8)); D = 4
+    r = rng.random(G)
+    S = rng.standard_normal((G, D))
+    p = rng.uniform(0.2, 0.95, G)
+    rho = np.outer(p, p)
+    M = math.comb(G, 2)
+    Jd, w = _exhaustive_draws(p)
+    o = oracle.audit(r, rho, S, Jd, w, scale=1.0 / M)
+    assert o["status"] == 0
+    assert o["bias_norm"] <= 1e-12 * math.sqrt(o["target_sq"])
+    tr = 0.0
+    for i in range(G):
+        for j in range(i + 1, G):
+            tr += (1.0 / (p[i] * p[j]) - 1.0) * float(_h(r, S, i, j) @ _h(r, S, i, j))
+    for i in range(G):
+        others = [j for j in range(G) if j != i]
+        for j, k in itertools.combinations(others, 2):
+            tr += 2.0 * (1.0 / p[i] - 1.0) * float(_h(r, S, i, j) @ _h(r, S, i, k))
+    tr /= M * M
+    assert o["mse"] == pytest.approx(tr, rel=1e-10)
+    assert o["vertices"] == pytest.approx(p.sum(), rel=1e-13)
+    pp = sum(p[i] * p[j] for i in range(G) for j in range(i + 1, G))
+    assert o["edges"] == pytest.approx(pp, rel=1e-13)
+    assert o["weight"] == pytest.approx(1.0, rel=1e-13)
+
+
+def test_audit_unweighted_bias_vector():
+    """Unweighted selection: bias (1/M) sum_e (rho_e - 1) h_e (Prop. bias)."""
+    rng = _rng(710)
+    G, D = 6, 3
+    r = _binary_rewards(rng, G)
+    S = rng.standard_normal((G, D))
+    p = rng.uniform(0.2, 0.9, G)
+    rho = np.outer(p, p)
+    M = math.comb(G, 2)
+    Jd, w = _exhaustive_draws(p)
+    o = oracle.audit(r, rho, S, Jd, w, scale=1.0 / M, wmode=oracle.W_UNWEIGHTED)
+    want = sum((rho[i, j] - 1.0) * _h(r, S, i, j) for i in range(G) for j in range(i + 1, G)) / M
+    np.testing.assert_allclose(o["bias"], want, rtol=1e-11, atol=1e-13)
+    assert o["bias_norm"] == pytest.approx(float(np.sqrt(want @ want)), rel=1e-11)
+
+
+def test_audit_full_inclusion_is_exact():
+    """Every draw completes the whole group with rho = 1: each estimate is the
+    target itself (zero bias, zero MSE, cosine 1)."""
+    rng = _rng(720)
+    G, D = 7, 5
+    r = rng.random(G)
+    S = rng.standard_normal((G, D))
+    Jd = np.ones((4, G), np.uint8)
+    o = oracle.audit(r, np.ones((G, G)), S, Jd)
+    assert o["bias_norm"] <= 1e-13 * math.sqrt(o["target_sq"])
+    assert o["mse"] <= 1e-26 * o["target_sq"]
+    assert o["cos"] == pytest.approx(1.0, abs=1e-14)
+    assert o["edges"] == G * (G - 1) / 2
