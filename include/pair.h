@@ -182,6 +182,47 @@ PAIR_API pair_status pair_coeffs_product(int32_t B, int32_t G, const float *r,
                                          pair_stream_t stream);
 
 /*
+ * pair_audit -- the frozen-population estimator audit (Sec. 5; metrics of
+ * App. D) of one candidate group: r [G], rho [G][G] (as pair_coeffs_weighted),
+ * explicit scores S [G][D], and N design draws Jdraws [N][G] (uint8). Each
+ * draw's estimate is ghat_b = sum_i a_bi s_i with a_b the
+ * pair_coeffs_weighted coefficients of that draw (wmode, w_max, scale,
+ * flags); the target is the complete-pair gradient g = scale * sum_{i<j}
+ * h_ij over all G candidates (Eq. pair-kernel). With draw weights w_b
+ * (draw_weight [N] double, nullable = 1/N each; e.g. exact design
+ * probabilities of an enumeration) and W = sum_b w_b, stats [8] (double) gets
+ *   [PAIR_AUDIT_BIAS_NORM]  || sum_b w_b ghat_b / W - g ||
+ *   [PAIR_AUDIT_MSE]        sum_b w_b || ghat_b - g ||^2 / W
+ *   [PAIR_AUDIT_COS]        sum_b w_b cos(ghat_b, g) / W (0 where ghat_b = 0)
+ *   [PAIR_AUDIT_VERTICES]   mean completed vertices, [PAIR_AUDIT_EDGES] mean
+ *                           completed edges, [PAIR_AUDIT_ESS] mean ESS
+ *   [PAIR_AUDIT_TARGET_SQ]  || g ||^2,  [PAIR_AUDIT_WEIGHT] W
+ * and bias [D] (double, nullable) the vector sum_b w_b ghat_b / W - g.
+ * Everything is formed through the Gram matrix S S^T in fp64 (the
+ * coefficients themselves are fp32); deterministic. ws: device workspace of
+ * pair_audit_workspace_size(N, G, D) bytes, 16-byte aligned, no initial
+ * contents needed.
+ * Errors: as pair_coeffs_weighted; PAIR_ERR_WORKSPACE.
+ */
+#define PAIR_AUDIT_BIAS_NORM 0
+#define PAIR_AUDIT_MSE 1
+#define PAIR_AUDIT_COS 2
+#define PAIR_AUDIT_VERTICES 3
+#define PAIR_AUDIT_EDGES 4
+#define PAIR_AUDIT_ESS 5
+#define PAIR_AUDIT_TARGET_SQ 6
+#define PAIR_AUDIT_WEIGHT 7
+#define PAIR_AUDIT_NSTATS 8
+
+PAIR_API size_t pair_audit_workspace_size(int32_t N, int32_t G, int32_t D);
+PAIR_API pair_status pair_audit(int32_t N, int32_t G, int32_t D, const float *r,
+                                const float *rho, const float *S, const uint8_t *Jdraws,
+                                const double *draw_weight, float scale, uint32_t flags,
+                                pair_weighting wmode, float w_max, double *stats, double *bias,
+                                void *ws, size_t ws_bytes, int32_t *dev_err,
+                                pair_stream_t stream);
+
+/*
  * pair_estimate_dense -- Eq. (pair-ht) for explicit score vectors:
  *     g_b = scale * sum_{i<j} J_iJ_j h_ij / rho_ij = sum_i a_i s_{b,i}
  * (the coefficient collapse of Eq. pair-advantage; rows with a_i = 0 are

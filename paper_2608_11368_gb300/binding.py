@@ -75,6 +75,11 @@ def lib() -> ctypes.CDLL:
     L.pair_coeffs_weighted.restype = ctypes.c_int
     L.pair_coeffs_product.argtypes = [I32, I32, P, P, P, F32, U32, P, P, P, P, P, P, P, P]
     L.pair_coeffs_product.restype = ctypes.c_int
+    L.pair_audit_workspace_size.argtypes = [I32, I32, I32]
+    L.pair_audit_workspace_size.restype = SZ
+    L.pair_audit.argtypes = [I32, I32, I32, P, P, P, P, P, F32, U32, ctypes.c_int, F32, P, P,
+                             P, SZ, P, P]
+    L.pair_audit.restype = ctypes.c_int
     L.pair_selftest_wait_timeout.argtypes = [I64, P, P, P]
     L.pair_selftest_wait_timeout.restype = ctypes.c_int
     _lib = L
@@ -198,6 +203,36 @@ def pair_coeffs_product(r, J, p, scale=1.0, flags=0, a=None, active=None, edges=
                                    *[_p(t) for t in outs], _p(dev_err), _stream(stream))
     _check(st, "pair_coeffs_product")
     return outs
+
+
+AUDIT_STATS = ("bias_norm", "mse", "cos", "vertices", "edges", "ess", "target_sq", "weight")
+
+
+def pair_audit(r, rho, S, Jdraws, draw_weight=None, wmode=PAIR_W_HT, w_max=0.0, scale=1.0,
+               flags=0, stats=None, bias=None, ws=None, dev_err=None, stream=None):
+    """Frozen-population audit of one group over design draws (see pair.h).
+    r [G], rho [G, G] (None for PAIR_W_UNWEIGHTED), S [G, D], Jdraws [N, G]
+    uint8, draw_weight [N] float64 or None. Returns (stats [8] f64, bias [D] f64)."""
+    N, G = Jdraws.shape
+    D = S.shape[1]
+    _need(r, "r", torch.float32, (G,))
+    if rho is not None:
+        _need(rho, "rho", torch.float32, (G, G))
+    _need(S, "S", torch.float32, (G, D))
+    _need(Jdraws, "Jdraws", torch.uint8, (N, G))
+    if draw_weight is not None:
+        _need(draw_weight, "draw_weight", torch.float64, (N,))
+    dev = r.device
+    stats = torch.empty(8, dtype=torch.float64, device=dev) if stats is None else stats
+    bias = torch.empty(D, dtype=torch.float64, device=dev) if bias is None else bias
+    need = int(lib().pair_audit_workspace_size(N, G, D))
+    if ws is None:
+        ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    st = lib().pair_audit(N, G, D, _p(r), _p(rho), _p(S), _p(Jdraws), _p(draw_weight),
+                          float(scale), int(flags), int(wmode), float(w_max), _p(stats),
+                          _p(bias), _p(ws), ws.numel(), _p(dev_err), _stream(stream))
+    _check(st, "pair_audit")
+    return stats, bias
 
 
 def pair_estimate_dense(r, J, rho, S, scale=1.0, g=None, a=None, dev_err=None,

@@ -12,7 +12,7 @@
 // together hold exactly GP-1 upper entries, so a block of >= GP threads reads
 // them as two contiguous runs per step, fully unrolled to keep every load
 // of the group in flight at once.
-#include "pair_common.cuh"
+#include "pair_coeffs_dev.cuh"
 
 namespace pairk {
 namespace {
@@ -26,36 +26,6 @@ struct GroupSmem {
   int red_i[32];
   float red_f[32];
 };
-
-// Row-major offset of (i, j), i < j, in the packed strict upper triangle.
-template <int GP>
-__device__ __forceinline__ int upper_off(int i, int j) {
-  return i * (2 * GP - i - 1) / 2 + (j - i - 1);
-}
-
-// Deterministic block sum of one int per thread (all threads call).
-__device__ int block_sum_int(int v, int *red) {
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  const int w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) red[w] = v;
-  __syncthreads();
-  int s = 0;
-  for (int k = 0; k < nw; ++k) s += red[k];
-  return s;
-}
-
-// Deterministic block sum of one float per thread in a fixed tree order.
-__device__ float block_sum_float(float v, float *red) {
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  const int w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) red[w] = v;
-  __syncthreads();
-  float s = 0.f;
-  for (int k = 0; k < nw; ++k) s += red[k];
-  return s;
-}
 
 // Computes the coefficients of group `b` into sm.a[0..G) (scale applied).
 // Requires blockDim.x >= GP. Returns K and the contrast count (all threads).
@@ -262,50 +232,9 @@ __global__ void __launch_bounds__(256, 4) dense_kernel(
   }
 }
 
-// Deterministic block maximum of one float per thread (all threads call).
-__device__ float block_max_float(float v, float *red) {
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  const int w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) red[w] = v;
-  __syncthreads();
-  float m = 0.f;
-  for (int k = 0; k < nw; ++k) m = fmaxf(m, red[k]);
-  return m;
-}
-
-// Sum of the 2^l-blocked pairwise tree over x_0 .. x_{GP-1} (the same fixed
-// order the HT kernel uses for its row sums).
-template <int GP>
-struct PairwiseSum {
-  float p[8];
-  __device__ __forceinline__ void add(int k, float x) {
-    float c = x;
-    int m = k;
-#pragma unroll
-    for (int l = 0; l < 8; ++l) {
-      if (m & 1) { c = p[l] + c; m >>= 1; }
-      else { p[l] = c; break; }
-    }
-  }
-  __device__ __forceinline__ float total() const { return p[(GP == 32) ? 5 : (GP == 64) ? 6 : 7]; }
-};
-
-template <int GP>
-struct GroupSmemW {
-  float U[GP * (GP - 1) / 2];  // strict upper triangle of terms (r_i - r_j) w_ij
-  float r[GP];
-  float pi[GP];                // marginals (rho diagonal) or 1/p (product path)
-  int8_t J[GP];
-  int red_i[32];
-  float red_f[32];
-};
-
 // Coefficients under a weighting variant (see pair_coeffs_weighted), plus
 // the ESS and largest weight of the group's completed edges. One block of GP
-// threads per group; the upper triangle is read by row pairs as in
-// coeffs_kernel, every term placed once, every vertex summed by the fixed
-// pairwise tree.
+// threads per group.
 template <int GP>
 __global__ void __launch_bounds__(GP, 1024 / GP) coeffs_w_kernel(
     int B, int G, const float *__restrict__ r, const uint8_t *__restrict__ J,
@@ -325,99 +254,16 @@ __global__ void __launch_bounds__(GP, 1024 / GP) coeffs_w_kernel(
     sm.pi[tid] = (in && wmode == PAIR_W_MARGINAL) ? rho_g[(size_t)tid * G + tid] : 1.f;
   }
   __syncthreads();
-  const bool needs_rho = wmode == PAIR_W_HT || wmode == PAIR_W_CLIPPED || wmode == PAIR_W_HAJEK;
-  int my_contrast = 0, bad = 0;
-  float sw = 0.f, sw2 = 0.f, mw = 0.f;
-  if (tid < GP - 1) {
-    float v[GP / 2];
-#pragma unroll
-    for (int k = 0; k < GP / 2; ++k) {
-      const int n1 = GP - 1 - k;
-      int i, j;
-      if (tid < n1) { i = k; j = k + 1 + tid; }
-      else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
-      const bool live = (j < G) && sm.J[i] && sm.J[j];
-      v[k] = (live && needs_rho) ? __ldg(rho_g + (size_t)i * G + j) : 1.f;
-    }
-#pragma unroll
-    for (int k = 0; k < GP / 2; ++k) {
-      const int n1 = GP - 1 - k;
-      int i, j;
-      if (tid < n1) { i = k; j = k + 1 + tid; }
-      else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
-      const bool live = (j < G) && sm.J[i] && sm.J[j];
-      float t = 0.f;
-      if (live) {
-        const float dr = sm.r[i] - sm.r[j];
-        float w = 1.f;
-        bool okw = true;
-        if (wmode == PAIR_W_UNWEIGHTED) {
-          t = dr;
-        } else if (wmode == PAIR_W_MARGINAL) {
-          const float pi = sm.pi[i], pj = sm.pi[j];
-          okw = (pi > 0.f) && (pj > 0.f);
-          const float den = pi * pj;
-          t = okw ? __fdiv_rn(dr, den) : 0.f;
-          w = okw ? __frcp_rn(den) : 0.f;
-        } else {
-          const float rij = v[k];
-          okw = rij > 0.f;
-          w = okw ? __frcp_rn(rij) : 0.f;
-          if (wmode == PAIR_W_CLIPPED && w > w_max) {
-            w = w_max;
-            t = dr * w_max;
-          } else {
-            t = okw ? __fdiv_rn(dr, rij) : 0.f;
-          }
-        }
-        if (!okw) {
-          bad = 1;
-        } else {
-          my_contrast += (sm.r[i] != sm.r[j]);
-          sw += w;
-          sw2 = fmaf(w, w, sw2);
-          mw = fmaxf(mw, w);
-        }
-      }
-      sm.U[upper_off<GP>(i, j)] = t;
-    }
-  }
-  if (bad) flag_error(dev_err, PAIR_DEV_ERR_NONPOSITIVE_INCLUSION);
-  const float W = block_sum_float(sw, sm.red_f);
-  const float W2 = block_sum_float(sw2, sm.red_f);
-  const float Wmax = block_max_float(mw, sm.red_f);
-  __syncthreads();
-
-  PairwiseSum<GP> ps;
-  bool nz = false;
-#pragma unroll
-  for (int k = 0; k < GP; ++k) {
-    float x = 0.f;
-    if (k < tid) x = -sm.U[upper_off<GP>(k, tid)];
-    else if (k > tid) x = sm.U[upper_off<GP>(tid, k)];
-    nz |= (x != 0.f);
-    ps.add(k, x);
-  }
-  const float sum = ps.total();
-  float av = (sum == 0.f) ? 0.f : 0.5f * sum;
-  if (wmode == PAIR_W_HAJEK) av = W > 0.f ? __fdiv_rn(av, W) : 0.f;
-  const uint8_t act = (tid < G && sm.J[tid] && nz) ? 1 : 0;
-  const int packed = block_sum_int((int)sm.J[tid] | (my_contrast << 16), sm.red_i);
-  const int K = packed & 0xffff, C = packed >> 16;
-  if (center && K > 0) {
-    const float s2 = block_sum_float(sm.J[tid] ? av : 0.f, sm.red_f);
-    const float mean = s2 / (float)K;
-    if (sm.J[tid]) av -= mean;
-  }
+  const WeightedOut o = group_coeffs_w<GP>(sm, rho_g, G, scale, center != 0, wmode, w_max, dev_err);
   if (tid < G) {
-    a[gbase + tid] = av * scale;
-    if (active) active[gbase + tid] = act;
+    a[gbase + tid] = o.a;
+    if (active) active[gbase + tid] = o.active;
   }
   if (tid == 0) {
-    if (edges) edges[b] = K * (K - 1) / 2;
-    if (contrast) contrast[b] = C;
-    if (ess) ess[b] = W2 > 0.f ? __fdiv_rn(W * W, W2) : 0.f;
-    if (max_w) max_w[b] = Wmax;
+    if (edges) edges[b] = o.K * (o.K - 1) / 2;
+    if (contrast) contrast[b] = o.C;
+    if (ess) ess[b] = o.W2 > 0.f ? __fdiv_rn(o.W * o.W, o.W2) : 0.f;
+    if (max_w) max_w[b] = o.Wmax;
   }
 }
 
