@@ -468,6 +468,24 @@ def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
                           "ms": t_w, "algorithmic_bytes": bw}
     t_p = timed(lambda: B.pair_coeffs_product(r, J, p, a=a, active=act, edges=e1,
                                               contrast_edges=e2, ess=ess, max_w=mw), reps)
+    # Frozen-population audit at the paper's audit scale: one 16-candidate
+    # group, 50,000 independent-design draws, scores of dimension 4096.
+    rng = np.random.default_rng(1234 + rank)
+    Ga, Da, Na = 16, 4096, 50000
+    pa = rng.uniform(0.1, 0.95, Ga)
+    ra = dv((rng.random(Ga) < 0.5).astype(np.float32))
+    rhoa_np = np.outer(pa, pa).astype(np.float32)
+    np.fill_diagonal(rhoa_np, pa.astype(np.float32))
+    rhoa = dv(rhoa_np)
+    Sa = dv(rng.standard_normal((Ga, Da)).astype(np.float32))
+    Jda = dv((rng.random((Na, Ga)) < pa[None]).astype(np.uint8))
+    st_a = torch.empty(8, dtype=torch.float64, device="cuda")
+    bias_a = torch.empty(Da, dtype=torch.float64, device="cuda")
+    ws_a = torch.empty(int(B.lib().pair_audit_workspace_size(Na, Ga, Da)), dtype=torch.uint8,
+                       device="cuda")
+    Ma = Ga * (Ga - 1) // 2
+    t_a = timed(lambda: B.pair_audit(ra, rhoa, Sa, Jda, scale=1.0 / Ma, stats=st_a, bias=bias_a,
+                                     ws=ws_a), max(5, min(reps, 10)))
     bytes_p = Bn * (4 * G + G + 4 * G + 4 * G + G + 16)
     bytes_d = 4 * D * n_act + Bn * (4 * G * (G - 1) // 2 + 4 * G + G) + 4 * Bn * D + 4 * Bn * G
     gbs_c = bytes_c / (t_c / 1e3) / 1e9
@@ -483,6 +501,10 @@ def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
                                 "traffic": traffic.get(("dense", STRESS)),
                                 "ms": t_d, "algorithmic_bytes": bytes_d},
         "pair_coeffs_weighted": variants,
+        "pair_audit": {"draws": Na, "G": Ga, "D": Da, "ms": t_a,
+                       "draws_per_s": Na / (t_a / 1e3),
+                       "stats": dict(zip(B.AUDIT_STATS, st_a.cpu().tolist())),
+                       "bound": "latency (per-draw coefficient collapse and quadratic forms)"},
         "pair_coeffs_product": {"bound": "hbm", "achieved": bytes_p / (t_p / 1e3) / 1e9,
                                 "peak": peaks["hbm"], "unit": "GB/s",
                                 "frac": bytes_p / (t_p / 1e3) / 1e9 / peaks["hbm"],
