@@ -138,7 +138,8 @@ def _coeffs_out(B, G):
                 max_w=np.zeros(B, np.float64))
 
 
-def coeffs_w(r, J, rho, scale=1.0, center=False, wmode=W_HT, w_max=0.0, threads=None):
+def coeffs_w(r, J, rho, scale=1.0, center=False, wmode=W_HT, w_max=0.0, threads=None,
+             standardize=False):
     """Coefficients under weighting variant `wmode`, with the per-group ESS
     (sum w)^2 / sum w^2 and largest weight over the completed edges.
     rho [B,G,G]: strict upper triangle read for the joint probabilities, its
@@ -149,14 +150,15 @@ def coeffs_w(r, J, rho, scale=1.0, center=False, wmode=W_HT, w_max=0.0, threads=
     B, G = r.shape
     o = _coeffs_out(B, G)
     st = _load().oracle_pair_coeffs_w(
-        B, G, _ptr(r), _ptr(J), _ptr(rho), float(scale), int(bool(center)), int(wmode),
+        B, G, _ptr(r), _ptr(J), _ptr(rho), float(scale),
+        int(bool(center)) | (2 if standardize else 0), int(wmode),
         float(w_max), _ptr(o["a"]), _ptr(o["a_mag"]), _ptr(o["active"]), _ptr(o["edges"]),
         _ptr(o["contrast"]), _ptr(o["ess"]), _ptr(o["max_w"]), threads or n_threads())
     o["status"] = st
     return o
 
 
-def coeffs_product(r, J, p, scale=1.0, center=False, threads=None):
+def coeffs_product(r, J, p, scale=1.0, center=False, threads=None, standardize=False):
     """Inverse-probability coefficients of the independent design, rho_ij =
     p_i p_j, from the marginals p [B,G]; plus ESS and largest weight."""
     r = np.ascontiguousarray(r, dtype=np.float64)
@@ -165,7 +167,8 @@ def coeffs_product(r, J, p, scale=1.0, center=False, threads=None):
     B, G = r.shape
     o = _coeffs_out(B, G)
     st = _load().oracle_pair_coeffs_product(
-        B, G, _ptr(r), _ptr(J), _ptr(p), float(scale), int(bool(center)),
+        B, G, _ptr(r), _ptr(J), _ptr(p), float(scale),
+        int(bool(center)) | (2 if standardize else 0),
         _ptr(o["a"]), _ptr(o["a_mag"]), _ptr(o["active"]), _ptr(o["edges"]),
         _ptr(o["contrast"]), _ptr(o["ess"]), _ptr(o["max_w"]), threads or n_threads())
     o["status"] = st

@@ -117,6 +117,8 @@ static int coeffs_group(int G, const double *r, const uint8_t *J,
  *                        divided by sum_e w_e (self-normalised ratio form)
  * Diagnostics per group over its completed edges: ESS = (sum w)^2 / sum w^2
  * (Sec. 5 metrics) and the largest weight; both 0 without completed edges.
+ * `center` holds flags: bit 0 centres over the completed vertices (App. C),
+ * bit 1 divides by the completed rewards' sample standard deviation.
  */
 #define ORACLE_W_HT 0
 #define ORACLE_W_UNWEIGHTED 1
@@ -173,7 +175,26 @@ static int coeffs_group_w(int G, const double *r, const uint8_t *J,
             a_mag[i] = sum_w > 0.0 ? a_mag[i] / sum_w : 0.0;
         }
     }
-    if (center) {
+    if (center & 2) {
+        /* Reward standardisation (App. "Practical departures"): divide by the
+         * sample standard deviation (n - 1) of the completed rewards; a group
+         * with fewer than two completed vertices or equal rewards has no
+         * contrast edge, so its coefficients are already 0 and stay 0. */
+        int K = 0;
+        double mean = 0.0;
+        for (int i = 0; i < G; ++i) if (J[i]) { ++K; mean += r[i]; }
+        if (K >= 2) {
+            mean /= K;
+            double ss = 0.0;
+            for (int i = 0; i < G; ++i) if (J[i]) ss += (r[i] - mean) * (r[i] - mean);
+            double sd = sqrt(ss / (K - 1));
+            for (int i = 0; i < G; ++i) {
+                a[i] = sd > 0.0 ? a[i] / sd : 0.0;
+                a_mag[i] = sd > 0.0 ? a_mag[i] / sd : 0.0;
+            }
+        }
+    }
+    if (center & 1) {
         int K = 0;
         double sum = 0.0;
         for (int i = 0; i < G; ++i) if (J[i]) { ++K; sum += a[i]; }

@@ -326,3 +326,37 @@ def test_audit_full_inclusion_is_exact():
     assert o["mse"] <= 1e-26 * o["target_sq"]
     assert o["cos"] == pytest.approx(1.0, abs=1e-14)
     assert o["edges"] == G * (G - 1) / 2
+
+
+# --------------------------------------------------- reward standardisation
+
+@pytest.mark.parametrize("seed", range(3))
+def test_standardised_coefficients_are_grpo_scaled(seed):
+    """rho = 1, every vertex completed: a_i = (G/2)(r_i - rbar) (Thm. 1), so the
+    standardised coefficients are G/2 times GRPO's (r_i - rbar) / std(r, ddof=1)."""
+    rng = _rng(730 + seed)
+    G = 9
+    r = rng.random(G)
+    J = np.ones(G, np.uint8)
+    o = oracle.coeffs_w(r[None], J[None], np.ones((1, G, G)), standardize=True)
+    want = 0.5 * G * (r - r.mean()) / np.std(r, ddof=1)
+    np.testing.assert_allclose(o["a"][0], want, rtol=1e-13, atol=1e-14)
+    p = rng.uniform(0.2, 1.0, G)
+    o2 = oracle.coeffs_product(r[None], J[None], p[None], standardize=True)
+    o3 = oracle.coeffs_product(r[None], J[None], p[None])
+    np.testing.assert_allclose(o2["a"][0], o3["a"][0] / np.std(r, ddof=1), rtol=1e-13)
+
+
+def test_standardisation_uses_completed_rewards_only():
+    r = np.array([[1.0, 0.0, 5.0, 1.0, 0.0]])
+    J = np.array([[1, 1, 0, 1, 1]], np.uint8)
+    rho = np.full((1, 5, 5), 0.5)
+    o = oracle.coeffs_w(r, J, rho, standardize=True)
+    o0 = oracle.coeffs_w(r, J, rho)
+    sd = np.std(r[0][J[0] == 1], ddof=1)
+    np.testing.assert_allclose(o["a"], o0["a"] / sd, rtol=1e-14)
+    # Saturated group (equal completed rewards): coefficients stay 0.
+    r2 = np.array([[1.0, 1.0, 0.0, 1.0]])
+    J2 = np.array([[1, 1, 0, 1]], np.uint8)
+    o2 = oracle.coeffs_w(r2, J2, np.full((1, 4, 4), 0.5), standardize=True)
+    assert np.all(o2["a"] == 0.0) and o2["status"] == 0
