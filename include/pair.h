@@ -78,6 +78,11 @@ typedef enum { PAIR_F32 = 0, PAIR_BF16 = 1 } pair_dtype;
 #define PAIR_CENTER 1u /* subtract the mean of a over completed vertices
                           (App. C, numerical stability). Off by default:
                           in exact arithmetic the sum is already zero. */
+#define PAIR_STANDARDIZE 2u /* divide the coefficients of each group by the
+                          sample standard deviation (n - 1) of its completed
+                          rewards (the practical reward standardisation of
+                          App. "Practical departures"; biased, see there).
+                          Groups with equal completed rewards stay 0. */
 
 /* Largest group size G accepted by pair_coeffs / pair_estimate_dense. */
 #define PAIR_MAX_G 128
@@ -92,7 +97,7 @@ typedef enum { PAIR_F32 = 0, PAIR_BF16 = 1 } pair_dtype;
  *      J      [B][G] uint8    completion indicators (0 or nonzero).
  *      rho    [B][G][G] float32 logged joint inclusion probabilities.
  *      scale  multiplies every coefficient (see the header comment).
- *      flags  0 or PAIR_CENTER.
+ *      flags  0 or PAIR_CENTER | PAIR_STANDARDIZE.
  * Out: a      [B][G] float32  a_i = scale * 1/2 sum_{j != i} J_iJ_j
  *                             (r_i - r_j)/rho_ij; exactly 0 where J_i = 0
  *                             or no completed partner has another reward.

@@ -22,6 +22,7 @@ HEADER = os.path.join(os.path.dirname(_PKG), "include", "pair.h")
 PAIR_OK = 0
 PAIR_F32, PAIR_BF16 = 0, 1
 PAIR_CENTER = 1
+PAIR_STANDARDIZE = 2
 STATUS_NAMES = {0: "PAIR_OK", 1: "PAIR_ERR_INVALID_ARG", 2: "PAIR_ERR_UNSUPPORTED",
                 3: "PAIR_ERR_WORKSPACE", 4: "PAIR_ERR_NONPOSITIVE_INCLUSION",
                 5: "PAIR_ERR_TARGET_RANGE", 6: "PAIR_ERR_CUDA",

@@ -86,7 +86,7 @@ pair_status pair_coeffs(int32_t B, int32_t G, const float *r, const uint8_t *J,
                         pair_stream_t stream) {
   reset_launches();
   if (B < 1 || G < 2 || G > PAIR_MAX_G || !r || !J || !rho || !a ||
-      (flags & ~PAIR_CENTER) != 0)
+      (flags & ~(PAIR_CENTER | PAIR_STANDARDIZE)) != 0)
     return PAIR_ERR_INVALID_ARG;
   const pair_status dv = check_device();
   if (dv != PAIR_OK) return dv;
@@ -101,7 +101,7 @@ pair_status pair_coeffs_weighted(int32_t B, int32_t G, const float *r, const uin
                                  int32_t *edges, int32_t *contrast_edges, float *ess,
                                  float *max_w, int32_t *dev_err, pair_stream_t stream) {
   reset_launches();
-  if (B < 1 || G < 2 || G > PAIR_MAX_G || !r || !J || !a || (flags & ~PAIR_CENTER) != 0)
+  if (B < 1 || G < 2 || G > PAIR_MAX_G || !r || !J || !a || (flags & ~(PAIR_CENTER | PAIR_STANDARDIZE)) != 0)
     return PAIR_ERR_INVALID_ARG;
   const int wm = (int)wmode;
   if (wm < PAIR_W_HT || wm > PAIR_W_HAJEK) return PAIR_ERR_INVALID_ARG;
@@ -120,7 +120,7 @@ pair_status pair_coeffs_product(int32_t B, int32_t G, const float *r, const uint
                                 float *ess, float *max_w, int32_t *dev_err,
                                 pair_stream_t stream) {
   reset_launches();
-  if (B < 1 || G < 2 || G > PAIR_MAX_G || !r || !J || !p || !a || (flags & ~PAIR_CENTER) != 0)
+  if (B < 1 || G < 2 || G > PAIR_MAX_G || !r || !J || !p || !a || (flags & ~(PAIR_CENTER | PAIR_STANDARDIZE)) != 0)
     return PAIR_ERR_INVALID_ARG;
   const pair_status dv = check_device();
   if (dv != PAIR_OK) return dv;

@@ -109,7 +109,7 @@ __global__ void __launch_bounds__(GP, 1) audit_draws_kernel(
     sm.grp.J[tid] = (tid < G) ? (Jd[(size_t)b * G + tid] != 0) : 0;
     __syncthreads();
     const WeightedOut o =
-        group_coeffs_w<GP>(sm.grp, rho, G, scale, center != 0, wmode, w_max, dev_err);
+        group_coeffs_w<GP>(sm.grp, rho, G, scale, (uint32_t)center, wmode, w_max, dev_err);
     const double ai = (double)o.a;
     const double ei = ai - sm.abar[tid];
     sm.e[tid] = ei;
@@ -201,7 +201,7 @@ pair_status launch_audit_gp(int N, int G, int D, const float *r, const float *rh
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   PAIR_BEGIN("audit_draws", s);
   audit_draws_kernel<GP><<<nblk, GP, smem, s>>>(N, G, r, rho, Jd, wd, scale,
-                                                (flags & PAIR_CENTER) ? 1 : 0, wmode, w_max, K,
+                                                (int)flags, wmode, w_max, K,
                                                 abar, u, gg, part, dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("audit_finish", s);
@@ -230,7 +230,8 @@ extern "C" pair_status pair_audit(int32_t N, int32_t G, int32_t D, const float *
                                   pair_stream_t stream) {
   reset_launches();
   const size_t need = pair_audit_workspace_size(N, G, D);
-  if (need == 0 || !r || !S || !Jdraws || !stats || (flags & ~PAIR_CENTER) != 0)
+  if (need == 0 || !r || !S || !Jdraws || !stats ||
+      (flags & ~(PAIR_CENTER | PAIR_STANDARDIZE)) != 0)
     return PAIR_ERR_INVALID_ARG;
   const int wm = (int)wmode;
   if (wm < PAIR_W_HT || wm > PAIR_W_HAJEK) return PAIR_ERR_INVALID_ARG;

@@ -254,7 +254,8 @@ __global__ void __launch_bounds__(GP, 1024 / GP) coeffs_w_kernel(
     sm.pi[tid] = (in && wmode == PAIR_W_MARGINAL) ? rho_g[(size_t)tid * G + tid] : 1.f;
   }
   __syncthreads();
-  const WeightedOut o = group_coeffs_w<GP>(sm, rho_g, G, scale, center != 0, wmode, w_max, dev_err);
+  const WeightedOut o = group_coeffs_w<GP>(sm, rho_g, G, scale, (uint32_t)center, wmode, w_max,
+                                           dev_err);
   if (tid < G) {
     a[gbase + tid] = o.a;
     if (active) active[gbase + tid] = o.active;
@@ -321,7 +322,8 @@ __global__ void __launch_bounds__(GP, 4) coeffs_product_kernel(
   const float Wmax = block_max_float(mw, red_f);
   const int packed = block_sum_int((int)sJ[tid] | (my_contrast << 16), red_i);
   const int K = packed & 0xffff, C = packed >> 16;
-  if (center && K > 0) {
+  if (center & PAIR_STANDARDIZE) av = standardize_by_rewards(av, ri, Ji, K, red_f);
+  if ((center & PAIR_CENTER) && K > 0) {
     const float s2 = block_sum_float(Ji ? av : 0.f, red_f);
     const float mean = s2 / (float)K;
     if (Ji) av -= mean;
@@ -348,9 +350,8 @@ pair_status launch_coeffs_w_gp(int32_t B, int32_t G, const float *r, const uint8
   PAIR_CUDA_TRY(cudaFuncSetAttribute(coeffs_w_kernel<GP>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   PAIR_BEGIN("coeffs_w", s);
-  coeffs_w_kernel<GP><<<B, GP, smem, s>>>(B, G, r, J, rho, scale, (flags & PAIR_CENTER) ? 1 : 0,
-                                          wmode, w_max, a, active, edges, contrast, ess, max_w,
-                                          dev_err);
+  coeffs_w_kernel<GP><<<B, GP, smem, s>>>(B, G, r, J, rho, scale, (int)flags, wmode, w_max, a,
+                                          active, edges, contrast, ess, max_w, dev_err);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
@@ -361,8 +362,8 @@ pair_status launch_coeffs_product_gp(int32_t B, int32_t G, const float *r, const
                                      uint8_t *active, int32_t *edges, int32_t *contrast,
                                      float *ess, float *max_w, int32_t *dev_err, cudaStream_t s) {
   PAIR_BEGIN("coeffs_product", s);
-  coeffs_product_kernel<GP><<<B, GP, 0, s>>>(B, G, r, J, p, scale, (flags & PAIR_CENTER) ? 1 : 0,
-                                             a, active, edges, contrast, ess, max_w, dev_err);
+  coeffs_product_kernel<GP><<<B, GP, 0, s>>>(B, G, r, J, p, scale, (int)flags, a, active, edges,
+                                             contrast, ess, max_w, dev_err);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
@@ -408,6 +409,9 @@ pair_status launch_coeffs(int32_t B, int32_t G, const float *r,
                           uint32_t flags, float *a, uint8_t *active,
                           int32_t *edges, int32_t *contrast, int32_t *dev_err,
                           cudaStream_t s) {
+  if (flags & PAIR_STANDARDIZE)  // HT through the weighted kernel (bit-identical HT terms)
+    return launch_coeffs_weighted(B, G, r, J, rho, scale, flags, PAIR_W_HT, 0.f, a, active, edges,
+                                  contrast, nullptr, nullptr, dev_err, s);
   if (G <= 32)
     return launch_coeffs_gp<32>(B, G, r, J, rho, scale, flags, a, active,
                                 edges, contrast, dev_err, s);

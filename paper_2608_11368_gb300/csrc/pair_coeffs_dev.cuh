@@ -77,6 +77,20 @@ struct GroupSmemW {
   float red_f[32];
 };
 
+// Reward standardisation (App. "Practical departures"): v divided by the
+// sample standard deviation (n - 1) of the completed rewards, two-pass. With
+// fewer than two completed vertices or equal rewards there is no contrast
+// edge and v is already 0. All threads call.
+__device__ __forceinline__ float standardize_by_rewards(float v, float r, bool completed, int K,
+                                                       float *red) {
+  if (K < 2) return v;
+  const float mean = block_sum_float(completed ? r : 0.f, red) / (float)K;
+  const float dv = completed ? r - mean : 0.f;
+  const float ss = block_sum_float(dv * dv, red);
+  const float sd = sqrtf(ss / (float)(K - 1));
+  return sd > 0.f ? __fdiv_rn(v, sd) : 0.f;
+}
+
 // Result of one group's weighted coefficients (per thread: its vertex).
 struct WeightedOut {
   float a;          // this vertex's coefficient (scale applied)
@@ -93,7 +107,7 @@ struct WeightedOut {
 // threads call.
 template <int GP>
 __device__ WeightedOut group_coeffs_w(GroupSmemW<GP> &sm, const float *rho_g, int G, float scale,
-                                      bool center, int wmode, float w_max, int32_t *dev_err) {
+                                      uint32_t flags, int wmode, float w_max, int32_t *dev_err) {
   const int tid = threadIdx.x;
   const bool needs_rho = wmode == PAIR_W_HT || wmode == PAIR_W_CLIPPED || wmode == PAIR_W_HAJEK;
   int my_contrast = 0, bad = 0;
@@ -176,7 +190,9 @@ __device__ WeightedOut group_coeffs_w(GroupSmemW<GP> &sm, const float *rho_g, in
   const int packed = block_sum_int((int)sm.J[tid] | (my_contrast << 16), sm.red_i);
   o.K = packed & 0xffff;
   o.C = packed >> 16;
-  if (center && o.K > 0) {
+  if (flags & PAIR_STANDARDIZE) av = standardize_by_rewards(av, sm.r[tid], sm.J[tid] != 0, o.K,
+                                                           sm.red_f);
+  if ((flags & PAIR_CENTER) && o.K > 0) {
     const float s2 = block_sum_float(sm.J[tid] ? av : 0.f, sm.red_f);
     const float mean = s2 / (float)o.K;
     if (sm.J[tid]) av -= mean;

@@ -2,10 +2,15 @@
 include/pair.h declares, and validates arguments on the host (no GPU needed:
 invalid arguments are rejected before any device call)."""
 import ctypes
+import os
+import subprocess
+import sys
 
 import pytest
 
 from paper_2608_11368_gb300 import build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 @pytest.fixture(scope="module")
@@ -47,7 +52,20 @@ def test_workspace_size_rules(L):
     assert ws(10, 64, 0, 1, L.PAIR_F32) == 0
 
 
-def test_host_validation_without_device(L):
+def test_host_validation_without_device():
+    """Host-side argument checks, run in a child process with no visible
+    device: the placeholder pointers below must never reach a kernel, even if
+    a check were to let a call through."""
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    code = ("import sys; sys.path.insert(0, %r); import tests.test_abi as t; "
+            "from paper_2608_11368_gb300 import binding; t._host_validation_checks(binding)"
+            % ROOT)
+    res = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True,
+                         text=True, timeout=300)
+    assert res.returncode == 0, res.stdout[-2000:] + res.stderr[-2000:]
+
+
+def _host_validation_checks(L):
     lib = L.lib()
     P = ctypes.c_void_p
     one = P(16)  # never dereferenced: validation fails first
@@ -57,7 +75,7 @@ def test_host_validation_without_device(L):
                                None, None, None) == 1
     assert lib.pair_coeffs(1, 8, None, one, one, 1.0, 0, one, None, None, None,
                            None, None) == 1
-    assert lib.pair_coeffs(1, 8, one, one, one, 1.0, 2, one, None, None, None,
+    assert lib.pair_coeffs(1, 8, one, one, one, 1.0, 4, one, None, None, None,
                            None, None) == 1
     assert lib.pair_estimate_dense(1, 8, 0, one, one, one, one, 1.0, one, None,
                                    None, None) == 1

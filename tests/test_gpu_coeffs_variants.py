@@ -135,3 +135,23 @@ def test_variant_host_validation():
     out = B.pair_coeffs_weighted(dev(r), dev(J), None, wmode=B.PAIR_W_UNWEIGHTED)
     ref = oracle.coeffs_w(r, J, rho, wmode=oracle.W_UNWEIGHTED)
     _check(ref, out)
+
+
+@pytest.mark.parametrize("G", [2, 9, 33, 64, 128])
+def test_standardised_parity(G):
+    B = _binding()
+    r, J, p, rho = _inputs(970 + G, 23, G)
+    J[3] = 0; J[3, 0] = 1; J[3, 1] = 1; r[3, 0] = r[3, 1] = 1.0   # saturated pair
+    flags = B.PAIR_STANDARDIZE | B.PAIR_CENTER
+    for wmode in (oracle.W_HT, oracle.W_CLIPPED, oracle.W_HAJEK):
+        out = B.pair_coeffs_weighted(dev(r), dev(J), dev(rho), wmode=wmode, w_max=6.0,
+                                     flags=flags)
+        ref = oracle.coeffs_w(r, J, rho, center=True, wmode=wmode, w_max=6.0, standardize=True)
+        _check(ref, out, tol=3e-6, center=True)
+    a, act, edges, contrast = B.pair_coeffs(dev(r), dev(J), dev(rho), flags=B.PAIR_STANDARDIZE)
+    ref = oracle.coeffs_w(r, J, rho, standardize=True)
+    err = np.abs(a.cpu().numpy().astype(np.float64) - ref["a"])
+    assert (err <= 3e-6 * ref["a_mag"] + 1e-30).all()
+    out = B.pair_coeffs_product(dev(r), dev(J), dev(p), flags=B.PAIR_STANDARDIZE)
+    ref = oracle.coeffs_product(r, J, p, standardize=True)
+    _check(ref, out, tol=4e-6)
