@@ -208,6 +208,37 @@ def audit(r, rho, S, Jdraws, draw_weight=None, scale=1.0, center=False, wmode=W_
                 target_sq=float((g ** 2).sum()), weight=float(W), bias=bias, status=o["status"])
 
 
+def ppo_surrogate(a, logp_seq, logp_old, eps):
+    """Clipped trajectory-ratio surrogate of the practical PPO epochs (Sec. 4.5
+    and App. "Practical departures"): with detached coefficients A_i and
+    trajectory ratios rho_i = exp(logp_seq_i - logp_old_i), rollout i
+    contributes L_i = min(rho_i A_i, clip(rho_i, 1 - eps, 1 + eps) A_i). Its
+    gradient is c_i * d logp_seq_i with c_i = A_i rho_i where the unclipped term
+    is the minimum (A_i > 0: rho_i <= 1 + eps; A_i < 0: rho_i >= 1 - eps) and 0
+    where the clip binds. Returns (c, L) in fp64; rollouts with A_i = 0 give 0."""
+    a = np.asarray(a, np.float64)
+    ratio = np.exp(np.asarray(logp_seq, np.float64) - np.asarray(logp_old, np.float64))
+    clipped = np.clip(ratio, 1.0 - eps, 1.0 + eps)
+    L = np.where(a != 0, np.minimum(ratio * a, clipped * a), 0.0)
+    unclipped = np.where(a > 0, ratio <= 1.0 + eps, ratio >= 1.0 - eps)
+    c = np.where((a != 0) & unclipped, a * ratio, 0.0)
+    return c, L
+
+
+def pair_grad_clipped_ref(inp, a, logp_old, eps):
+    """Reference outputs of pair_grad_clipped: the forward of pair_grad gives
+    every rollout's summed log-probability, the surrogate gives (c, L), and the
+    gradients are those of sum_i c_i logp_seq_i with c detached."""
+    base = pair_grad_ref(inp, a, full=True)
+    c, L = ppo_surrogate(a, base["logp_seq"], logp_old, eps)
+    out = pair_grad_ref(inp, c, full=True)
+    out["J"] = float(L.sum())
+    out["J_abs"] = float(np.abs(L).sum())
+    out["logp_seq"] = base["logp_seq"]
+    out["coef"] = c
+    return out
+
+
 def estimate_dense(r, J, rho, S, scale=1.0, threads=None):
     """Eq. (pair-ht) times M*scale: scale * sum_{i<j} J_iJ_j h_ij/rho_ij with
     h_ij = 1/2 (r_i - r_j)(s_i - s_j) formed explicitly. S [B,G,D]."""
