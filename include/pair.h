@@ -299,6 +299,33 @@ PAIR_API pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
                       size_t ws_bytes, int32_t *dev_err, pair_stream_t stream);
 
 /*
+ * pair_grad_clipped -- the clipped trajectory-ratio surrogate of the practical
+ * PPO epochs (Sec. 4.5; App. "Practical departures"), on the same LM-head
+ * realisation as pair_grad. With the detached coefficients A_i = a[i] and the
+ * trajectory ratio rho_i = exp(logp_seq_i - logp_old[i]) of every rollout
+ * (logp_seq_i this call's summed log-probability, formed in fp64),
+ *     J = sum_i min(rho_i A_i, clip(rho_i, 1 - clip_eps, 1 + clip_eps) A_i),
+ * and dH, dW are its gradients: those of sum_i c_i logp_seq_i with
+ * c_i = A_i rho_i where the unclipped term is the minimum (A_i > 0:
+ * rho_i <= 1 + eps; A_i < 0: rho_i >= 1 - eps) and c_i = 0 where the clip
+ * binds. At logp_old = logp_seq every ratio is 1 and the result is
+ * pair_grad's gradient (J = sum_i A_i). The paper marks this as a
+ * trust-region surrogate, not the design-unbiased gradient.
+ * In:  as pair_grad, plus logp_old [R] float32 (device; read where a_i != 0)
+ *      and clip_eps >= 0 (finite).
+ * Out: as pair_grad (Jobj = the surrogate J); coef [R] float32 (nullable):
+ *      the c_i used.
+ * Workspace: pair_grad_workspace_size. Errors: as pair_grad.
+ */
+PAIR_API pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dtype dt,
+                                       const void *H, const void *W, const int32_t *y,
+                                       const uint8_t *mask, const int32_t *cu_seqlens, int32_t R,
+                                       const float *a, const float *logp_old, float clip_eps,
+                                       float *dH, float *dW, double *Jobj, float *logp_seq,
+                                       float *coef, void *ws, size_t ws_bytes, int32_t *dev_err,
+                                       pair_stream_t stream);
+
+/*
  * pair_grad_noalloc -- pair_grad without a caller-provided workspace, for
  * callers that cannot allocate device memory: for example a plug-in that
  * runs inside a host application which owns every device allocation and

@@ -64,6 +64,9 @@ def lib() -> ctypes.CDLL:
     L.pair_status_string.restype = ctypes.c_char_p
     L.pair_last_launch_count.argtypes = []
     L.pair_last_launch_count.restype = I32
+    L.pair_grad_clipped.argtypes = [I64, I32, I32, ctypes.c_int, P, P, P, P, P, I32, P, P, F32,
+                                    P, P, P, P, P, P, SZ, P, P]
+    L.pair_grad_clipped.restype = ctypes.c_int
     L.pair_grad_noalloc.argtypes = [I64, I32, I32, ctypes.c_int, P, P, P, P, P,
                                     I32, P, P, P, P, P, P, P]
     L.pair_grad_noalloc.restype = ctypes.c_int
@@ -293,6 +296,38 @@ def pair_grad(H, W, y, mask, cu_seqlens, a, dH=None, dW=None, Jobj=None,
                          _stream(stream))
     _check(st, "pair_grad")
     return Jobj, dH, dW, logp_seq
+
+
+def pair_grad_clipped(H, W, y, mask, cu_seqlens, a, logp_old, clip_eps=0.2, dH=None, dW=None,
+                      Jobj=None, logp_seq=None, coef=None, ws=None, dev_err=None, stream=None):
+    """Clipped trajectory-ratio surrogate (see pair.h). Returns
+    (Jobj [1] f64, dH [T,d] f32, dW [V,d] f32, logp_seq [R] f32, coef [R] f32)."""
+    T, d = H.shape
+    V = W.shape[0]
+    R = cu_seqlens.numel() - 1
+    dt = _pair_dtype(H)
+    _need(H, "H", H.dtype)
+    _need(W, "W", H.dtype, (V, d))
+    _need(y, "y", torch.int32, (T,))
+    _need(mask, "mask", torch.uint8, (T,))
+    _need(cu_seqlens, "cu_seqlens", torch.int32, (R + 1,))
+    _need(a, "a", torch.float32, (R,))
+    _need(logp_old, "logp_old", torch.float32, (R,))
+    dev = H.device
+    dH = torch.empty((T, d), dtype=torch.float32, device=dev) if dH is None else dH
+    dW = torch.empty((V, d), dtype=torch.float32, device=dev) if dW is None else dW
+    Jobj = torch.empty(1, dtype=torch.float64, device=dev) if Jobj is None else Jobj
+    logp_seq = torch.empty(R, dtype=torch.float32, device=dev) if logp_seq is None else logp_seq
+    coef = torch.empty(R, dtype=torch.float32, device=dev) if coef is None else coef
+    need = pair_grad_workspace_size(T, d, V, R, dt)
+    if ws is None:
+        ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    st = lib().pair_grad_clipped(T, d, V, dt, _p(H), _p(W), _p(y), _p(mask), _p(cu_seqlens), R,
+                                 _p(a), _p(logp_old), float(clip_eps), _p(dH), _p(dW), _p(Jobj),
+                                 _p(logp_seq), _p(coef), _p(ws), ws.numel(), _p(dev_err),
+                                 _stream(stream))
+    _check(st, "pair_grad_clipped")
+    return Jobj, dH, dW, logp_seq, coef
 
 
 NOALLOC_MAX_WORKSPACE = 32 << 20

@@ -143,6 +143,43 @@ pair_status pair_estimate_dense(int32_t B, int32_t G, int32_t D,
                                reinterpret_cast<cudaStream_t>(stream));
 }
 
+pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dtype dt, const void *H,
+                              const void *W, const int32_t *y, const uint8_t *mask,
+                              const int32_t *cu_seqlens, int32_t R, const float *a,
+                              const float *logp_old, float clip_eps, float *dH, float *dW,
+                              double *Jobj, float *logp_seq, float *coef, void *ws,
+                              size_t ws_bytes, int32_t *dev_err, pair_stream_t stream) {
+  reset_launches();
+  if (!H || !W || !y || !mask || !cu_seqlens || !a || !logp_old || !dH || !dW || !Jobj)
+    return PAIR_ERR_INVALID_ARG;
+  if (!(clip_eps >= 0.f && clip_eps <= 1.0e30f)) return PAIR_ERR_INVALID_ARG;
+  if (!aligned16(H) || !aligned16(W) || !aligned16(dH) || !aligned16(dW))
+    return PAIR_ERR_INVALID_ARG;
+  const size_t need = pair_grad_workspace_size(T, d, V, R, dt);
+  if (need == 0) return (dt == PAIR_BF16 && d % 64 != 0 && d % 16 == 0)
+                            ? PAIR_ERR_UNSUPPORTED
+                            : PAIR_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return PAIR_ERR_WORKSPACE;
+  const pair_status dv = check_device();
+  if (dv != PAIR_OK) return dv;
+
+  GradWorkspace w;
+  grad_workspace_bytes(T, d, V, R, dt, &w, ws);
+  GradArgs g{T, d, V, R, dt, H, W, y, mask, cu_seqlens, a,
+             dH, dW, Jobj, logp_seq, dev_err};
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // Forward, then the surrogate's coefficients (they depend on this call's
+  // log-probabilities), then the backward with those coefficients.
+  pair_status st = grad_prepare(g, w, s);
+  if (st == PAIR_OK) st = dt == PAIR_BF16 ? grad_lse_tc(g, w, s) : grad_lse_simt(g, w, s);
+  if (st == PAIR_OK) st = grad_ppo_coefficients(g, w, logp_old, clip_eps, coef, s);
+  if (st == PAIR_OK) st = dt == PAIR_BF16 ? grad_bwd_tc(g, w, s) : grad_bwd_simt(g, w, s);
+  if (st == PAIR_OK && dt == PAIR_BF16) st = grad_onehot(g, w, s);
+  if (st == PAIR_OK) st = grad_ppo_finalize(g, w, s);
+  return st;
+}
+
 size_t pair_grad_workspace_size(int64_t T, int32_t d, int32_t V, int32_t R,
                                 pair_dtype dt) {
   if (T < 1 || R < 1 || V < 1 || d < 16 || (d % 16) != 0) return 0;

@@ -65,6 +65,8 @@ struct GradWorkspace {
   float *zy;           // [Tpad] target logit
   float2 *part;        // [nsplit][Tpad] partial (max, sum-exp) per split
   double *seg_logp;    // [R] per-rollout sum of logp (fp64)
+  float *ppo_c;        // [R] clipped-surrogate coefficients (pair_grad_clipped)
+  double *ppo_L;       // [R] clipped-surrogate terms (pair_grad_clipped)
   void *Hc;            // [Tpad][d] compacted hidden rows (dt), zero tail
   void *gring;         // per-cluster ring of published Gs tiles
   int64_t Tpad;
@@ -97,6 +99,16 @@ pair_status grad_head_simt(const GradArgs &g, const GradWorkspace &w,
                            cudaStream_t s);
 pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
                          cudaStream_t s);
+// Forward (log-sum-exp) and backward halves of the two head paths.
+pair_status grad_lse_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
+pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
+pair_status grad_lse_simt(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
+pair_status grad_bwd_simt(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
+// Clipped trajectory-ratio surrogate between the two halves (pair_grad_prep.cu).
+pair_status grad_ppo_coefficients(const GradArgs &g, const GradWorkspace &w,
+                                  const float *logp_old, float eps, float *coef_out,
+                                  cudaStream_t s);
+pair_status grad_ppo_finalize(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
 // Exact one-hot parts (added after the tensor-core softmax parts).
 pair_status grad_onehot(const GradArgs &g, const GradWorkspace &w,
                         cudaStream_t s);

@@ -310,6 +310,63 @@ __global__ void onehot_dw_kernel(int d, int V, int bucket,
   }
 }
 
+// Clipped trajectory-ratio surrogate of the practical PPO epochs (Sec. 4.5,
+// App. "Practical departures"): for rollout i with detached coefficient
+// A_i = a_i and ratio rho_i = exp(logp_seq_i - logp_old_i),
+//   L_i = min(rho_i A_i, clip(rho_i, 1 - eps, 1 + eps) A_i),
+// and the gradient coefficient c_i = A_i rho_i where the unclipped term is the
+// minimum (A_i > 0: rho_i <= 1 + eps; A_i < 0: rho_i >= 1 - eps), else 0.
+// The ratio is formed in fp64 from the fp64 per-rollout log-probability.
+__global__ void ppo_coef_kernel(int R, const float *a, const double *seg_logp,
+                                const float *logp_old, float eps, float *c, double *L,
+                                float *coef_out) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < R; i += gridDim.x * blockDim.x) {
+    const double A = (double)a[i];
+    float ci = 0.f;
+    double li = 0.0;
+    if (coef_nonzero(a[i])) {
+      const double ratio = exp(seg_logp[i] - (double)logp_old[i]);
+      const double lo = 1.0 - (double)eps, hi = 1.0 + (double)eps;
+      const double clipped = ratio < lo ? lo : (ratio > hi ? hi : ratio);
+      const double u = ratio * A, v = clipped * A;
+      li = u < v ? u : v;
+      const bool unclipped = A > 0.0 ? ratio <= hi : ratio >= lo;
+      ci = unclipped ? (float)(A * ratio) : 0.f;
+    }
+    c[i] = ci;
+    L[i] = li;
+    if (coef_out) coef_out[i] = ci;
+  }
+}
+
+// tok_c[p] = c_i for every compacted token p of rollout i.
+__global__ void retarget_c_kernel(int R, const int32_t *seg_off, const float *c, float *tok_c) {
+  const int i = blockIdx.x;
+  const int beg = seg_off[i], end = seg_off[i + 1];
+  const float ci = c[i];
+  for (int p = beg + threadIdx.x; p < end; p += blockDim.x) tok_c[p] = ci;
+}
+
+// Jobj = sum_i L_i (fp64, fixed order); logp_seq out as in objective_kernel.
+__global__ void ppo_objective_kernel(int R, const float *a, const double *seg_logp,
+                                     const double *L, double *Jobj, float *logp_seq) {
+  __shared__ double red[32];
+  double s = 0.0;
+  for (int i = threadIdx.x; i < R; i += blockDim.x) {
+    const bool on = coef_nonzero(a[i]);
+    if (logp_seq) logp_seq[i] = on ? (float)seg_logp[i] : 0.f;
+    s += L[i];
+  }
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) t += red[k];
+    *Jobj = t;
+  }
+}
+
 }  // namespace
 
 size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
@@ -332,6 +389,8 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   const size_t o_zy = take((size_t)Tpad * 4);
   const size_t o_part = take((size_t)kNSplit * Tpad * sizeof(float2));
   const size_t o_segl = take((size_t)R * 8);
+  const size_t o_ppoc = take((size_t)R * 4);
+  const size_t o_ppol = take((size_t)R * 8);
   const size_t o_hc = take((size_t)Tpad * d * esz);
   const size_t o_ring = dt == PAIR_BF16 ? take((size_t)kMaxClusters * kRingBytesPerCluster) : off;
   if (out) {
@@ -346,6 +405,8 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->zy = reinterpret_cast<float *>(b + o_zy);
     out->part = reinterpret_cast<float2 *>(b + o_part);
     out->seg_logp = reinterpret_cast<double *>(b + o_segl);
+    out->ppo_c = reinterpret_cast<float *>(b + o_ppoc);
+    out->ppo_L = reinterpret_cast<double *>(b + o_ppol);
     out->Hc = b + o_hc;
     out->gring = b + o_ring;
     out->Tpad = Tpad;
@@ -394,6 +455,29 @@ pair_status grad_finalize(const GradArgs &g, const GradWorkspace &w,
   PAIR_BEGIN("objective", s);
   objective_kernel<<<1, 1024, 0, s>>>(g.R, g.a, w.seg_logp, g.Jobj,
                                       g.logp_seq);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+pair_status grad_ppo_coefficients(const GradArgs &g, const GradWorkspace &w,
+                                  const float *logp_old, float eps, float *coef_out,
+                                  cudaStream_t s) {
+  PAIR_BEGIN("seg_logp", s);
+  seg_logp_kernel<<<g.R, 256, 0, s>>>(g.R, w.seg_off, w.zy, w.lse, w.seg_logp);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("ppo_coef", s);
+  ppo_coef_kernel<<<(int)ceil_div(g.R, 256), 256, 0, s>>>(g.R, g.a, w.seg_logp, logp_old, eps,
+                                                          w.ppo_c, w.ppo_L, coef_out);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("retarget_c", s);
+  retarget_c_kernel<<<g.R, 256, 0, s>>>(g.R, w.seg_off, w.ppo_c, w.tok_c);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+pair_status grad_ppo_finalize(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  PAIR_BEGIN("ppo_objective", s);
+  ppo_objective_kernel<<<1, 1024, 0, s>>>(g.R, g.a, w.seg_logp, w.ppo_L, g.Jobj, g.logp_seq);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }

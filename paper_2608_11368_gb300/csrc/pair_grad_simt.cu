@@ -134,33 +134,44 @@ __global__ void __launch_bounds__(kWarps * 32) simt_dw_kernel(
 
 }  // namespace
 
-pair_status grad_head_simt(const GradArgs &g, const GradWorkspace &w,
-                           cudaStream_t s) {
+pair_status grad_lse_simt(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
   const float *Hc = static_cast<const float *>(w.Hc);
   const float *W = static_cast<const float *>(g.W);
   const int grid = 152 * 8;
-  const size_t sm1 = (size_t)g.d * 4, sm2 = (size_t)(kWarps + 1) * g.d * 4;
+  const size_t sm1 = (size_t)g.d * 4;
   PAIR_CUDA_TRY(cudaFuncSetAttribute(simt_lse_kernel,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1));
+  PAIR_BEGIN("simt_lse", s);
+  simt_lse_kernel<<<grid, kWarps * 32, sm1, s>>>(g.d, g.V, w.counters, Hc, W, w.tok_y, w.lse,
+                                                 w.zy);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+pair_status grad_bwd_simt(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  const float *Hc = static_cast<const float *>(w.Hc);
+  const float *W = static_cast<const float *>(g.W);
+  const int grid = 152 * 8;
+  const size_t sm2 = (size_t)(kWarps + 1) * g.d * 4;
   PAIR_CUDA_TRY(cudaFuncSetAttribute(simt_dh_kernel,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2));
   PAIR_CUDA_TRY(cudaFuncSetAttribute(simt_dw_kernel,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2));
-  PAIR_BEGIN("simt_lse", s);
-  simt_lse_kernel<<<grid, kWarps * 32, sm1, s>>>(g.d, g.V, w.counters, Hc, W,
-                                                 w.tok_y, w.lse, w.zy);
-  PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("simt_dh", s);
-  simt_dh_kernel<<<grid, kWarps * 32, sm2, s>>>(g.d, g.V, w.counters,
-                                                w.tok_idx, Hc, W, w.tok_y,
+  simt_dh_kernel<<<grid, kWarps * 32, sm2, s>>>(g.d, g.V, w.counters, w.tok_idx, Hc, W, w.tok_y,
                                                 w.tok_c, w.lse, g.dH);
   PAIR_LAUNCH_CHECK(s);
   const int gridv = (int)(g.V < 152 * 16 ? g.V : 152 * 16);
   PAIR_BEGIN("simt_dw", s);
-  simt_dw_kernel<<<gridv, kWarps * 32, sm2, s>>>(g.d, g.V, w.counters, Hc, W,
-                                                 w.tok_y, w.tok_c, w.lse, g.dW);
+  simt_dw_kernel<<<gridv, kWarps * 32, sm2, s>>>(g.d, g.V, w.counters, Hc, W, w.tok_y, w.tok_c,
+                                                 w.lse, g.dW);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
+}
+
+pair_status grad_head_simt(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  const pair_status st = grad_lse_simt(g, w, s);
+  return st != PAIR_OK ? st : grad_bwd_simt(g, w, s);
 }
 
 }  // namespace pairk

@@ -1309,32 +1309,31 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
 
 }  // namespace
 
-pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
-                         cudaStream_t s) {
-  CUtensorMap mH, mW128, mW256;
-  if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) ||
-      !make_map(&mW128, g.W, g.V, g.d, 128) ||
-      !make_map(&mW256, g.W, g.V, g.d, 256))
+// Forward half: per-token log-sum-exp and target logit.
+pair_status grad_lse_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  CUtensorMap mH, mW128;
+  if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) || !make_map(&mW128, g.W, g.V, g.d, 128))
     return PAIR_ERR_CUDA;
   const int nsm = num_sms();
   const size_t lse_smem = sizeof(LseSmem) + 1024;
-  const size_t bwd_smem = sizeof(BwdSmem) + 1024;
   PAIR_CUDA_TRY(cudaFuncSetAttribute(lse_kernel,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)lse_smem));
-  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_kernel<true>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bwd_smem));
-  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_kernel<false>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bwd_smem));
-
   PAIR_BEGIN("lse_tc", s);
   lse_kernel<<<lse_grid(lse_smem), kThreads, lse_smem, s>>>(mH, mW128, g.d, g.V, w.nsplit,
-                                             w.Tpad, w.counters, w.tok_y,
-                                             w.part, w.zy, g.dev_err);
+                                                           w.Tpad, w.counters, w.tok_y,
+                                                           w.part, w.zy, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("lse_combine", s);
-  lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters,
-                                             w.part, w.lse);
+  lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters, w.part, w.lse);
   PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+// Backward half: softmax parts of dH and dW from the token coefficients.
+pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  CUtensorMap mH, mW128;
+  if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) || !make_map(&mW128, g.W, g.V, g.d, 128))
+    return PAIR_ERR_CUDA;
   if (use_cluster_path(g.d)) {
     switch (cluster_tile_width(g.d)) {
       case 128: return grad_bwd_cluster<128>(g, w, s, mH, mW128);
@@ -1342,17 +1341,26 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w,
       default: return grad_bwd_cluster<64>(g, w, s, mH, mW128);
     }
   }
+  const int nsm = num_sms();
+  const size_t bwd_smem = sizeof(BwdSmem) + 1024;
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_kernel<true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bwd_smem));
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_kernel<false>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bwd_smem));
   PAIR_BEGIN("bwd_dh_tc", s);
   bwd_kernel<true><<<nsm, kThreads, bwd_smem, s>>>(
-      mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
-      g.dev_err);
+      mH, mW128, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("bwd_dw_tc", s);
   bwd_kernel<false><<<nsm, kThreads, bwd_smem, s>>>(
-      mW128, mH, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
-      g.dev_err);
+      mW128, mH, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
+}
+
+pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  const pair_status st = grad_lse_tc(g, w, s);
+  return st != PAIR_OK ? st : grad_bwd_tc(g, w, s);
 }
 
 }  // namespace pairk
