@@ -41,7 +41,10 @@ METRIC = "pair_grad tokens/s (fwd+bwd) and % dense-BF16 peak; pair_coeffs GB/s v
 FLUSH_BYTES = 256 << 20          # > 129 MB L2
 CPU_SAMPLE_TOKENS = 256          # oracle sample for the CPU baseline
 REF_SAMPLE_TOKENS = 48           # oracle sample per --impl reference step
-TC_KERNELS = ("lse_tc", "bwd_dh_tc", "bwd_dw_tc")
+# Tensor-core kernels of one pair_grad call; each is charged one logit-sized
+# GEMM (2 T_eff V d FLOP) of algorithmic work per call, whatever the number of
+# token chunks it is launched for.
+TC_KERNELS = ("lse_tc", "bwd_dh_tc", "bwd_dw_tc", "dw_gemm_tc")
 
 
 def parse_args():
@@ -342,7 +345,10 @@ def main():
     flops_gemm = 2.0 * T_eff * V * d
     dominant = max(agg.items(), key=lambda kv: kv[1][1])[0]
     dn, dt_ms = agg[dominant]
-    dom_avg = dt_ms / dn
+    # One "launch" here is the kernel's whole share of one pair_grad call: the
+    # sum over its token-chunk launches (chunks past the last token exit at
+    # once), so per-call work divides per-call time.
+    dom_avg = dt_ms / args.steps
     dom_flops = flops_gemm if dominant in TC_KERNELS else None
     achieved = dom_flops / (dom_avg / 1e3) / 1e12 if dom_flops else None
     roofline = {"kernel": dominant, "bound": "tensor",
@@ -351,7 +357,7 @@ def main():
                 "traffic": traffic.get((dominant, args.workload)),
                 "peak_source": peaks["src"] + " sustained bf16 (kernel timed inside a long step)",
                 "algorithmic_flops_per_launch": dom_flops,
-                "avg_launch_ms": dom_avg}
+                "avg_launch_ms": dom_avg, "launches_per_call": dn / args.steps}
     tc_ms = sum(agg[k][1] for k in TC_KERNELS if k in agg) / args.steps
     grad_ms = sum(t for nm, (n, t) in agg.items() if nm not in ("coeffs",)) / args.steps
     pair_grad_info = {

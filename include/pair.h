@@ -246,12 +246,31 @@ PAIR_API pair_status pair_estimate_dense(int32_t B, int32_t G, int32_t D,
                                 pair_stream_t stream);
 
 /*
- * pair_grad_workspace_size -- bytes of device workspace pair_grad needs for
- * T packed tokens, hidden size d, vocabulary V, R rollouts and dtype dt.
- * Returns 0 for arguments pair_grad would reject.
+ * pair_grad_workspace_size -- bytes of device workspace pair_grad (and
+ * pair_grad_clipped) should be given for T packed tokens, hidden size d,
+ * vocabulary V, R rollouts and dtype dt. Returns 0 for arguments pair_grad
+ * would reject.
+ * For PAIR_BF16 with d in {512, 1024, 1536, 2048} this includes the
+ * logit-gradient image: the bf16 tiles Gs = -c_t softmax(z_t) the dH pass
+ * forms are kept, 32 KB per 128 tokens x 128 vocabulary rows, so that the dW
+ * pass reads them instead of recomputing the logits. It holds
+ * min(ceil(T/128), max(32, 2^33 / (ceil(V/128) * 32768))) token blocks of
+ * ceil(V/128) tiles (at most about 8 GiB); longer batches run the backward
+ * in token chunks of that many blocks.
  */
 PAIR_API size_t pair_grad_workspace_size(int64_t T, int32_t d, int32_t V, int32_t R,
                                 pair_dtype dt);
+
+/*
+ * pair_grad_workspace_min_size -- the smallest workspace pair_grad accepts:
+ * pair_grad_workspace_size without the logit-gradient image. Any size from
+ * here up to pair_grad_workspace_size is valid; the image then holds the
+ * token blocks that fit (more chunks), and with none the dW pass recomputes
+ * the logits. Results agree to fp32 rounding across sizes (the dW sums run
+ * in a different order), and are bit-identical for the same size.
+ */
+PAIR_API size_t pair_grad_workspace_min_size(int64_t T, int32_t d, int32_t V, int32_t R,
+                                    pair_dtype dt);
 
 /*
  * pair_grad -- the policy objective of Sec. 4.5, sum_i a_i log pi(o_i | q),
@@ -286,10 +305,11 @@ PAIR_API size_t pair_grad_workspace_size(int64_t T, int32_t d, int32_t V, int32_
  *      Jobj [1] double   (device pointer),
  *      logp_seq [R] float32 (nullable): sum of logp_t over the rollout's
  *                        mask = 1 tokens where a_i != 0, 0 elsewhere.
- * Workspace: ws (device, >= pair_grad_workspace_size bytes, any contents,
- *      256-byte aligned). dev_err as for pair_coeffs (target-range and
- *      pipeline-timeout errors).
- * Deterministic: repeated calls give bit-identical outputs.
+ * Workspace: ws (device, >= pair_grad_workspace_min_size bytes, normally
+ *      pair_grad_workspace_size; any contents, 256-byte aligned). dev_err as
+ *      for pair_coeffs (target-range and pipeline-timeout errors).
+ * Deterministic: repeated calls with the same ws_bytes give bit-identical
+ * outputs.
  */
 PAIR_API pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
                       const void *H, const void *W, const int32_t *y,
@@ -337,8 +357,9 @@ PAIR_API pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dty
  * Arguments, outputs and numerics are those of pair_grad, minus ws and
  * ws_bytes. The workspace is a file-scope device array of
  * PAIR_NOALLOC_MAX_WORKSPACE bytes that every GPU loading this library
- * holds until the process exits; problems whose
- * pair_grad_workspace_size(...) exceeds it are rejected with
+ * holds until the process exits. It keeps no logit-gradient image (the dW
+ * pass recomputes the logits); problems whose
+ * pair_grad_workspace_min_size(...) exceeds it are rejected with
  * PAIR_ERR_WORKSPACE before any launch. The call allocates nothing.
  * The first call on each device looks up the array's device address (with
  * that device current) and caches it; make that first call before any

@@ -55,6 +55,8 @@ def lib() -> ctypes.CDLL:
     L.pair_estimate_dense.restype = ctypes.c_int
     L.pair_grad_workspace_size.argtypes = [I64, I32, I32, I32, ctypes.c_int]
     L.pair_grad_workspace_size.restype = SZ
+    L.pair_grad_workspace_min_size.argtypes = [I64, I32, I32, I32, ctypes.c_int]
+    L.pair_grad_workspace_min_size.restype = SZ
     L.pair_grad.argtypes = [I64, I32, I32, ctypes.c_int, P, P, P, P, P, I32, P,
                             P, P, P, P, P, SZ, P, P]
     L.pair_grad.restype = ctypes.c_int
@@ -258,6 +260,11 @@ def pair_estimate_dense(r, J, rho, S, scale=1.0, g=None, a=None, dev_err=None,
 def pair_grad_workspace_size(T, d, V, R, dtype) -> int:
     return int(lib().pair_grad_workspace_size(int(T), int(d), int(V), int(R),
                                               int(dtype)))
+
+
+def pair_grad_workspace_min_size(T, d, V, R, dtype) -> int:
+    return int(lib().pair_grad_workspace_min_size(int(T), int(d), int(V), int(R),
+                                                  int(dtype)))
 
 
 def _pair_dtype(t):

@@ -155,7 +155,7 @@ pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dtype dt, co
   if (!(clip_eps >= 0.f && clip_eps <= 1.0e30f)) return PAIR_ERR_INVALID_ARG;
   if (!aligned16(H) || !aligned16(W) || !aligned16(dH) || !aligned16(dW))
     return PAIR_ERR_INVALID_ARG;
-  const size_t need = pair_grad_workspace_size(T, d, V, R, dt);
+  const size_t need = pair_grad_workspace_min_size(T, d, V, R, dt);
   if (need == 0) return (dt == PAIR_BF16 && d % 64 != 0 && d % 16 == 0)
                             ? PAIR_ERR_UNSUPPORTED
                             : PAIR_ERR_INVALID_ARG;
@@ -165,7 +165,7 @@ pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dtype dt, co
   if (dv != PAIR_OK) return dv;
 
   GradWorkspace w;
-  grad_workspace_bytes(T, d, V, R, dt, &w, ws);
+  grad_workspace_bytes(T, d, V, R, dt, &w, ws, grad_gimg_rows_fit(T, d, V, R, dt, ws_bytes));
   GradArgs g{T, d, V, R, dt, H, W, y, mask, cu_seqlens, a,
              dH, dW, Jobj, logp_seq, dev_err};
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
@@ -180,13 +180,25 @@ pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dtype dt, co
   return st;
 }
 
+namespace {
+bool grad_shape_ok(int64_t T, int32_t d, int32_t V, int32_t R, pair_dtype dt) {
+  if (T < 1 || R < 1 || V < 1 || d < 16 || (d % 16) != 0) return false;
+  if (dt != PAIR_F32 && dt != PAIR_BF16) return false;
+  if (dt == PAIR_BF16 && (d % 64) != 0) return false;
+  return T <= (int64_t)INT32_MAX - 1024;
+}
+}  // namespace
+
 size_t pair_grad_workspace_size(int64_t T, int32_t d, int32_t V, int32_t R,
                                 pair_dtype dt) {
-  if (T < 1 || R < 1 || V < 1 || d < 16 || (d % 16) != 0) return 0;
-  if (dt != PAIR_F32 && dt != PAIR_BF16) return 0;
-  if (dt == PAIR_BF16 && (d % 64) != 0) return 0;
-  if (T > (int64_t)INT32_MAX - 1024) return 0;
-  return grad_workspace_bytes(T, d, V, R, dt, nullptr, nullptr);
+  if (!grad_shape_ok(T, d, V, R, dt)) return 0;
+  return grad_workspace_bytes(T, d, V, R, dt, nullptr, nullptr, grad_gimg_rows(T, d, V, dt));
+}
+
+size_t pair_grad_workspace_min_size(int64_t T, int32_t d, int32_t V, int32_t R,
+                                    pair_dtype dt) {
+  if (!grad_shape_ok(T, d, V, R, dt)) return 0;
+  return grad_workspace_bytes(T, d, V, R, dt, nullptr, nullptr, 0);
 }
 
 pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
@@ -201,7 +213,7 @@ pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
     return PAIR_ERR_INVALID_ARG;
   if (!aligned16(H) || !aligned16(W) || !aligned16(dH) || !aligned16(dW))
     return PAIR_ERR_INVALID_ARG;
-  const size_t need = pair_grad_workspace_size(T, d, V, R, dt);
+  const size_t need = pair_grad_workspace_min_size(T, d, V, R, dt);
   if (need == 0) return (dt == PAIR_BF16 && d % 64 != 0 && d % 16 == 0)
                             ? PAIR_ERR_UNSUPPORTED
                             : PAIR_ERR_INVALID_ARG;
@@ -211,7 +223,7 @@ pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
   if (dv != PAIR_OK) return dv;
 
   GradWorkspace w;
-  grad_workspace_bytes(T, d, V, R, dt, &w, ws);
+  grad_workspace_bytes(T, d, V, R, dt, &w, ws, grad_gimg_rows_fit(T, d, V, R, dt, ws_bytes));
   GradArgs g{T, d, V, R, dt, H, W, y, mask, cu_seqlens, a,
              dH, dW, Jobj, logp_seq, dev_err};
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

@@ -69,12 +69,30 @@ struct GradWorkspace {
   double *ppo_L;       // [R] clipped-surrogate terms (pair_grad_clipped)
   void *Hc;            // [Tpad][d] compacted hidden rows (dt), zero tail
   void *gring;         // per-cluster ring of published Gs tiles
+  float *tailbuf;      // [kMaxClusters][2][128][d] partial tail units (cluster path)
+  void *gimg;          // bf16 logit-gradient tiles of gimg_rb token blocks, or null
+  int gimg_rb;         // token blocks (128 rows) per backward chunk; 0 = no image
   int64_t Tpad;
   int nsplit;
 };
 
+// Whether the bf16 backward runs as 8-CTA clusters: d = 512 A, 1 <= A <= 6.
+inline bool grad_cluster_path(int d) { return d % 512 == 0 && d >= 512 && d <= 3072; }
+
+// Token blocks of the logit-gradient image that the bf16 backward keeps for
+// its dW pass (0 where that path does not apply: fp32, or d outside the
+// 128-wide cluster tiles).
+int grad_gimg_rows(int64_t T, int32_t d, int32_t V, pair_dtype dt);
+constexpr uint32_t kGImgTileBytes = 128 * 128 * 2;  // one 128 x 128 bf16 tile
+
+// Workspace layout with gimg_rb token blocks of logit-gradient image (0 =
+// none; at most grad_gimg_rows). Returns its size in bytes.
 size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
-                            pair_dtype dt, GradWorkspace *out, void *base);
+                            pair_dtype dt, GradWorkspace *out, void *base, int gimg_rb);
+// Image token blocks that fit in ws_bytes (at most grad_gimg_rows), or -1 if
+// ws_bytes is below the size without an image.
+int grad_gimg_rows_fit(int64_t T, int32_t d, int32_t V, int32_t R, pair_dtype dt,
+                       size_t ws_bytes);
 
 struct GradArgs {
   int64_t T;

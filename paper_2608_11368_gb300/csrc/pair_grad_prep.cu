@@ -370,7 +370,7 @@ __global__ void ppo_objective_kernel(int R, const float *a, const double *seg_lo
 }  // namespace
 
 size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
-                            pair_dtype dt, GradWorkspace *out, void *base) {
+                            pair_dtype dt, GradWorkspace *out, void *base, int gimg_rb) {
   const int64_t Tpad = (T + 127) / 128 * 128 + 128;
   const size_t esz = dt == PAIR_BF16 ? 2 : 4;
   size_t off = 0;
@@ -393,6 +393,11 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   const size_t o_ppol = take((size_t)R * 8);
   const size_t o_hc = take((size_t)Tpad * d * esz);
   const size_t o_ring = dt == PAIR_BF16 ? take((size_t)kMaxClusters * kRingBytesPerCluster) : off;
+  const bool cl = dt == PAIR_BF16 && grad_cluster_path(d);
+  const size_t o_tail = cl ? take((size_t)kMaxClusters * 2 * 128 * d * sizeof(float)) : off;
+  // The image comes last, so that a larger workspace only adds token blocks.
+  const size_t o_gimg =
+      gimg_rb ? take((size_t)gimg_rb * (size_t)((V + 127) / 128) * kGImgTileBytes) : off;
   if (out) {
     char *b = static_cast<char *>(base);
     out->counters = reinterpret_cast<int32_t *>(b + o_cnt);
@@ -409,11 +414,23 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->ppo_L = reinterpret_cast<double *>(b + o_ppol);
     out->Hc = b + o_hc;
     out->gring = b + o_ring;
+    out->tailbuf = cl ? reinterpret_cast<float *>(b + o_tail) : nullptr;
+    out->gimg = gimg_rb ? b + o_gimg : nullptr;
+    out->gimg_rb = gimg_rb;
     out->Tpad = Tpad;
     out->nsplit = kNSplit;
   }
-  (void)V;
   return off;
+}
+
+int grad_gimg_rows_fit(int64_t T, int32_t d, int32_t V, int32_t R, pair_dtype dt,
+                       size_t ws_bytes) {
+  const size_t base = grad_workspace_bytes(T, d, V, R, dt, nullptr, nullptr, 0);
+  if (ws_bytes < base) return -1;
+  const int pref = grad_gimg_rows(T, d, V, dt);
+  if (pref == 0) return 0;
+  const size_t fit = (ws_bytes - base) / ((size_t)((V + 127) / 128) * kGImgTileBytes);
+  return fit < (size_t)pref ? (int)fit : pref;
 }
 
 pair_status grad_prepare(const GradArgs &g, const GradWorkspace &w,

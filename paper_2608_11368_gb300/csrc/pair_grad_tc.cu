@@ -652,10 +652,12 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 // The tiles of one cluster, in processing order: first its F = n_rb / ncl
 // full row blocks (cid, cid + ncl, ...), each with all n_ct column tiles;
 // then an even share [t0, t1) of the row-major tiles of the remaining
-// n_rb mod ncl row blocks, so that all clusters finish within a tile of each
-// other. A unit (run of tiles with one row block) in that tail may cover only
-// part of its row block; its rows are zeroed beforehand and its result is
-// added atomically.
+// R = n_rb mod ncl row blocks, so that all clusters finish within a tile of
+// each other. A unit (run of tiles with one row block) in that tail may cover
+// only part of its row block. Since R < ncl, a cluster's share has at most
+// n_ct tiles and so at most two tail units; each is stored to the cluster's
+// scratch slot (cid, u) and tail_reduce_kernel sums the slots of every tail
+// row in cluster order (deterministic, no atomics).
 struct TileMap {
   int n_ct, ncl, cid, gT, t0, rbT, N;
   __device__ void setup(int n_rb, int n_ct_, int cid_, int ncl_) {
@@ -705,21 +707,43 @@ struct TileCursor {
   __device__ bool unit_end(const TileMap &mp) const { return ct == mp.n_ct - 1 || g == mp.N - 1; }
 };
 
-// Zeroes the output rows of the tail row blocks (see TileMap) before the
-// cluster backward adds partial units into them.
-template <bool kTokenRows>
-__global__ void zero_tail_rows_kernel(int d, int V, int ncl, const int32_t *counters,
-                                      const int32_t *tok_idx, float *out) {
+// Final values of the tail rows (see TileMap) of the chunk of row blocks
+// [rb0, rb0 + cap): for each row, the sum in cluster order of the partial
+// units the clusters stored to their scratch slots.
+template <bool kTokenRows, int BN>
+__global__ void tail_reduce_kernel(int d, int V, int ncl, int rb0, int cap,
+                                   const int32_t *counters, const int32_t *tok_idx,
+                                   const float *tailbuf, float *out) {
   const int Teff = counters[0];
   const int n_rows = kTokenRows ? Teff : V;
-  const int n_rb = (n_rows + 127) / 128;
-  const int r0 = (n_rb / ncl) * ncl * 128;
+  const int n_ct = kTokenRows ? (V + BN - 1) / BN : (Teff + BN - 1) / BN;
+  const int n_rb = min(max((n_rows + 127) / 128 - rb0, 0), cap);
+  if (n_ct == 0) return;
+  const int F = n_rb / ncl, R = n_rb - F * ncl;
+  if (R == 0) return;
+  const int64_t Tt = (int64_t)R * n_ct;
+  const int r0 = (rb0 + F * ncl) * 128;
+  const int r1 = min(n_rows, (rb0 + n_rb) * 128);
   const int vec = d / 4;
+  const float4 *src = reinterpret_cast<const float4 *>(tailbuf);
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-       i < (int64_t)(n_rows - r0) * vec; i += (int64_t)gridDim.x * blockDim.x) {
-    const int rid = r0 + (int)(i / vec);
+       i < (int64_t)(r1 - r0) * vec; i += (int64_t)gridDim.x * blockDim.x) {
+    const int off = (int)(i / vec);           // row offset from r0
+    const int rl = off >> 7, rr = off & 127;  // tail row block, row within it
+    const int c4 = (int)(i % vec);
+    const int64_t lo = (int64_t)rl * n_ct, hi = lo + n_ct;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c = 0; c < ncl; ++c) {
+      const int64_t a = Tt * c / ncl, b = Tt * (c + 1) / ncl;
+      if ((a > lo ? a : lo) < (b < hi ? b : hi)) {
+        const int u = rl - (int)(a / n_ct);  // this row block's unit in cluster c
+        const float4 p = src[((int64_t)(c * 2 + u) * 128 + rr) * vec + c4];
+        acc.x += p.x; acc.y += p.y; acc.z += p.z; acc.w += p.w;
+      }
+    }
+    const int rid = r0 + off;
     const int64_t row = kTokenRows ? (int64_t)tok_idx[rid] : (int64_t)rid;
-    reinterpret_cast<float4 *>(out + row * d)[i % vec] = make_float4(0.f, 0.f, 0.f, 0.f);
+    reinterpret_cast<float4 *>(out + row * d)[c4] = acc;
   }
 }
 
@@ -730,7 +754,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
                        const __grid_constant__ CUtensorMap tmC64, int d, int V,
                        const int32_t *counters, const int32_t *tok_idx,
                        const float *tok_c, const float *lse, float *out,
-                       uint8_t *gring, int32_t *dev_err) {
+                       uint8_t *gring, uint8_t *gimg, float *tailbuf, int rb0, int cap,
+                       int32_t *dev_err) {
   extern __shared__ uint8_t smem_raw[];
   ClSmem<BN> &sm = *reinterpret_cast<ClSmem<BN> *>(align1k(smem_raw));
   using Tl = ClTile<BN>;
@@ -750,7 +775,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   // column parts of A0 and A - A0 atoms of the slice.
   const bool ksplit = BN == 128 && A <= 4;
   const int A0 = ksplit ? A : (A + 1) >> 1, A1 = ksplit ? A : A - A0;
-  const int n_rb = kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128;
+  // Row blocks [rb0, rb0 + n_rb) of this launch (one chunk); TileMap and
+  // TileCursor count them from 0.
+  const int n_rb = min(max((kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128) - rb0, 0), cap);
   const int n_ct = kTokenRows ? (V + BN - 1) / BN : (Teff + BN - 1) / BN;
   const int n_my = cid < n_rb ? (n_rb - cid + ncl - 1) / ncl : 0;
   TileMap mp;
@@ -758,8 +785,12 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   const int N = mp.N;                      // tiles of this cluster
   // Ring of published Gs tiles: [owner][job parity] for this cluster.
   uint8_t *ring = gring + (size_t)cid * kCl * 2 * kGsBytes;
-  auto ring_tile = [&](int g) {
-    return ring + ((size_t)(g & (kCl - 1)) * 2 + (size_t)((g >> 3) & 1)) * kGsBytes;
+  // Where tile g (chunk row block rb, column tile ct) is published: its own
+  // slot of the logit-gradient image when the launch keeps one (a later pass
+  // reads it again), else the ring slot.
+  auto gs_tile = [&](int g, int rb, int ct) {
+    return gimg ? gimg + ((size_t)rb * n_ct + ct) * kGsBytes
+                : ring + ((size_t)(g & (kCl - 1)) * 2 + (size_t)((g >> 3) & 1)) * kGsBytes;
   };
   // The tile whose S this CTA accumulates during slot s (may be < 0 or >= N).
   auto job_of = [&](int s) {
@@ -832,7 +863,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
           if (elect_one()) {
             mbar_expect_tx(&sm.full[stage], kAtom128 + kColAtom);
-            tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, job_rb * 128);
+            tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, (rb0 + job_rb) * 128);
             tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], a * 64, job_ct * BN);
           }
           __syncwarp();
@@ -867,7 +898,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
       };
       // K-split: part p = Gs atom p and rows [64p, 64p + 64) of every slice
       // atom, on one barrier.
-      auto load_khalf = [&](int p, int s, int ct) {
+      auto load_khalf = [&](int p, int s, int rb, int ct) {
         if (!(ok = wait(&sm.cs_empty[p], cs_ph[p] ^ 1, abort, dev_err))) return;
         if (p == 0) {
           // pub[o][b] completes once per two tiles of owner o: parity (m >> 1) & 1.
@@ -878,7 +909,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         }
         if (elect_one()) {
           mbar_expect_tx(&sm.cs_full[p], kAtom128 + (uint32_t)A * (kColAtom / 2));
-          bulk_load(sm.g[0][p], ring_tile(s) + p * kAtom128, kAtom128, &sm.cs_full[p]);
+          bulk_load(sm.g[0][p], gs_tile(s, rb, ct) + p * kAtom128, kAtom128, &sm.cs_full[p]);
           for (int j = 0; j < A; ++j)
             tma_load_2d(sm.cs[j] + p * (kColAtom / 2), &tmC64, &sm.cs_full[p], k * w + j * 64,
                         ct * BN + 64 * p);
@@ -888,9 +919,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         cs_ph[p] ^= 1;
       };
       for (int s = 0; s < N && ok && ksplit; ++s, cur.next(mp)) {
-        load_khalf(0, s, cur.ct);
+        load_khalf(0, s, cur.rb, cur.ct);
         if (!ok) break;
-        load_khalf(1, s, cur.ct);
+        load_khalf(1, s, cur.rb, cur.ct);
       }
       for (int s = 0; s < N && ok && !ksplit; ++s, cur.next(mp)) {
         load_cs(0, 0, A0, cur.ct);
@@ -905,7 +936,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         if (!(ok = wait(&sm.gs_empty[gb], ge_ph[gb] ^ 1, abort, dev_err))) break;
         if (elect_one()) {
           mbar_expect_tx(&sm.g_full[gb], kGsBytes);
-          bulk_load(sm.g[gb][0], ring_tile(s), kGsBytes, &sm.g_full[gb]);
+          bulk_load(sm.g[gb][0], gs_tile(s, cur.rb, cur.ct), kGsBytes, &sm.g_full[gb]);
         }
         __syncwarp();
         g_last[gb] = (int)ge_ph[gb];
@@ -1067,7 +1098,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         const int rb = gt.rb, ct = gt.ct;
         float rc = 0.f, rl = 0.f;
         if (kTokenRows) {
-          const int p = rb * 128 + row;
+          const int p = (rb0 + rb) * 128 + row;
           if (p < Teff) { rc = tok_c[p]; rl = lse[p] * kLog2e; }
         } else {
           epi_sync();
@@ -1087,7 +1118,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           free_ph[pb] ^= 1;
         }
         tc_fence_after();
-        uint8_t *dst_tile = ring_tile(g);
+        uint8_t *dst_tile = gs_tile(g, rb, ct);
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
           float v[32];
@@ -1136,29 +1167,28 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
       }
       if (s < 0) continue;
       const bool unit_end = cur.unit_end(mp);
-      const bool add = mp.tail(cur.g);
+      const bool tail = mp.tail(cur.g);
       const int rb = cur.rb;
+      // A tail unit's slot: its row block's place among this cluster's tail units.
+      const int tu = tail ? (rb - mp.rbT) - mp.t0 / mp.n_ct : 0;
       cur.next(mp);
       if (unit_end) {
         // Drain the finished unit: out[rows, k*w : (k+1)*w].
         if (!(ok = wait_sleepy(&sm.o_full, o_ph, abort, dev_err))) break;
         o_ph ^= 1;
         tc_fence_after();
-        const int rid = rb * 128 + row;
+        const int rid = (rb0 + rb) * 128 + row;
         const bool valid = kTokenRows ? (rid < Teff) : (rid < V);
         float *dst = nullptr;
-        if (valid)
+        if (tail)
+          dst = tailbuf + ((int64_t)(cid * 2 + tu) * 128 + row) * d + k * w;
+        else if (valid)
           dst = out + (kTokenRows ? (int64_t)tok_idx[rid] : (int64_t)rid) * d + k * w;
 #pragma unroll 1
         for (int c = 0; c < w / 32; ++c) {
           float v[32];
           tmem_ld32(tmem_o + lane_off + c * 32, v);
-          if (valid && add) {
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-              atomicAdd(reinterpret_cast<float4 *>(dst + c * 32) + q,
-                        make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
-          } else if (valid) {
+          if (dst) {
 #pragma unroll
             for (int q = 0; q < 8; ++q)
               reinterpret_cast<float4 *>(dst + c * 32)[q] =
@@ -1172,7 +1202,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
     // No column tiles at all (no active token): the slice is zero.
     if (ok && n_ct == 0) {
       for (int j = 0; j < n_my; ++j) {
-        const int rid = (cid + j * ncl) * 128 + row;
+        const int rid = (rb0 + cid + j * ncl) * 128 + row;
         if (!kTokenRows && rid < V)
           for (int c = 0; c < w; ++c) out[(int64_t)rid * d + k * w + c] = 0.f;
       }
@@ -1182,6 +1212,208 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   tc_fence_before();
   __syncthreads();
   cluster_sync();  // no CTA leaves while a peer may still signal its barriers
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ------------------------------------- dW from the stored logit gradient
+//
+// With 128-wide column tiles the dH pass keeps every bf16 tile Gs it forms
+// (128 tokens x 128 vocabulary rows, one 32 KB image per tile in the
+// K-major SWIZZLE_128B layout of its own MMA operand) for a chunk of token
+// blocks. Read with the token index as K, the same bytes are the MN-major
+// SWIZZLE_128B layout of Gs^T (64 vocabulary rows per 128-byte line, one
+// line per token), so the softmax part of dW is the plain GEMM
+//     dW[v, :] (+)= sum_t Gs[t, v] Hc[t, :]
+// with no logit recomputation.
+//
+// CTA pairs (2-CTA clusters) share one 512-column chunk of Hc: CTA r of the
+// pair fetches half of each Hc stage and multicasts it into both CTAs; each
+// CTA fetches the Gs^T stage of its own 128 vocabulary rows. Work unit =
+// (vocabulary block pair, 512-column chunk of d); CTA r accumulates
+// dW[block 2 p + r, chunk] (128 x 512 fp32 = all of TMEM) over the chunk's
+// tokens, 32 token rows per stage, and drains it with plain stores (first
+// chunk) or read-add-writes (later chunks; this CTA owns those rows).
+// An odd last block is computed twice (the pair's other CTA repeats the
+// last block) so both CTAs run the same stage sequence; only one stores it.
+constexpr int kDwKS = 32;                                 // token rows per stage
+constexpr int kDwStages = 5;
+constexpr int kDwN = 512;                                 // output columns per CTA
+constexpr uint32_t kDwGBytes = 2 * kDwKS * 128;           // 2 vocabulary atoms x 32 rows
+constexpr uint32_t kDwHBytes = (kDwN / 64) * kDwKS * 128; // 8 column atoms x 32 rows
+constexpr uint32_t kIdescDw = idesc_bf16(128, 256, 1, 1); // both operands MN-major
+
+struct DwSmem {
+  uint8_t g[kDwStages][kDwGBytes];  // Gs^T: MN-major A, atoms 4 KB apart
+  uint8_t h[kDwStages][kDwHBytes];  // Hc[t, chunk]: MN-major B, atoms 4 KB apart
+  uint64_t full[kDwStages], empty[kDwStages];
+  uint64_t acc_full, acc_empty, mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    dw_gemm_kernel(const __grid_constant__ CUtensorMap tmG,
+                   const __grid_constant__ CUtensorMap tmH, int d, int V, int rb0, int cap,
+                   int accumulate, const int32_t *counters, float *dW, int32_t *dev_err) {
+  const int Teff = counters[0];
+  const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  // A chunk past the last token adds nothing (the first chunk always runs:
+  // with no tokens at all it writes the zero softmax part).
+  if (nrb == 0 && accumulate) return;
+  extern __shared__ uint8_t smem_raw[];
+  DwSmem &sm = *reinterpret_cast<DwSmem *>(align1k(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = (int)cluster_rank();
+  const int pid = (int)cluster_id_x(), npairs = (int)num_clusters_x();
+  const int n_vb = (V + 127) / 128;
+  const int nq = d / kDwN;
+  const int n_units = (n_vb + 1) / 2 * nq;
+  const int nks = nrb * (128 / kDwKS);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kDwStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 2);  // both CTAs' MMAs done with the stage
+    }
+    mbar_init(&sm.acc_full, 1);
+    mbar_init(&sm.acc_empty, 128);
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmG);
+    prefetch_tmap(&tmH);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the peer's barriers exist before any multicast lands
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  volatile int *abort = &sm.abort;
+
+  if (warp == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
+      int stage = 0;
+      uint32_t ph = 0;
+      int last_ph[kDwStages];
+      for (int s = 0; s < kDwStages; ++s) last_ph[s] = -1;
+      bool ok = true;
+      for (int u = pid; u < n_units && ok; u += npairs) {
+        const int vp = u / nq, q = u - vp * nq;
+        const int vb = min(2 * vp + r, n_vb - 1);
+        for (int ks = 0; ks < nks; ++ks) {
+          const int rbl = ks >> 2, j = ks & 3;
+          if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+          if (elect_one()) {
+            mbar_expect_tx(&sm.full[stage], kDwGBytes + kDwHBytes);
+            tma_load_3d(sm.g[stage], &tmG, &sm.full[stage], 0, kDwKS * j,
+                        2 * (rbl * n_vb + vb));
+            tma_load_3d_mc(sm.h[stage] + r * (kDwHBytes / 2), &tmH, &sm.full[stage], 0,
+                           (rb0 + rbl) * 128 + kDwKS * j, q * (kDwN / 64) + r * (kDwN / 128),
+                           (uint16_t)3);
+          }
+          __syncwarp();
+          last_ph[stage] = (int)ph;
+          if (++stage == kDwStages) { stage = 0; ph ^= 1; }
+        }
+      }
+      // Never leave a copy in flight: wait (bounded) for the last one issued
+      // on every stage.
+      for (int s = 0; s < kDwStages; ++s)
+        if (last_ph[s] >= 0) {
+          volatile int never = 0;
+          wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+        }
+    }
+  } else if (warp == 1) {
+    {  // whole warp: uniform loop state; elected lane issues
+      // A: 2 vocabulary atoms (LBO 4 KB), token groups of 8 rows (SBO 1 KB);
+      // B: 8 column atoms (LBO 4 KB), the same token groups. One K step of 16
+      // tokens advances both by 2 KB; B's second 256-column half is 16 KB on.
+      const uint64_t dg0 = sdesc_sw128(smem_u32(sm.g[0]), kDwKS * 128, 1024);
+      const uint64_t dh0 = sdesc_sw128(smem_u32(sm.h[0]), kDwKS * 128, 1024);
+      int stage = 0;
+      uint32_t ph = 0, acc_ph = 0;
+      bool ok = true;
+      for (int u = pid; u < n_units && ok && nks > 0; u += npairs) {
+        if (!(ok = wait(&sm.acc_empty, acc_ph ^ 1, abort, dev_err))) break;
+        acc_ph ^= 1;
+        tc_fence_after();
+        for (int ks = 0; ks < nks; ++ks) {
+          if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+          const uint64_t dg = dg0 + (uint64_t)stage * (kDwGBytes >> 4);
+          const uint64_t dh = dh0 + (uint64_t)stage * (kDwHBytes >> 4);
+          if (elect_one()) {
+#pragma unroll
+            for (int kk = 0; kk < kDwKS / 16; ++kk)
+#pragma unroll
+              for (int nh = 0; nh < 2; ++nh)
+                mma_bf16(tmem + nh * 256, dg + kk * (2048 >> 4),
+                         dh + nh * ((kDwHBytes / 2) >> 4) + kk * (2048 >> 4), kIdescDw,
+                         (ks | kk) != 0);
+            mma_commit_multicast(&sm.empty[stage], (uint16_t)3);
+          }
+          __syncwarp();
+          if (++stage == kDwStages) { stage = 0; ph ^= 1; }
+        }
+        if (!ok) break;
+        if (elect_one()) mma_commit(&sm.acc_full);
+        __syncwarp();
+      }
+      if (elect_one()) mma_commit(&sm.mma_done);
+      __syncwarp();
+      volatile int never = 0;
+      wait(&sm.mma_done, 0, &never, dev_err);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    uint32_t acc_ph = 0;
+    bool ok = true;
+    for (int u = pid; u < n_units && ok; u += npairs) {
+      const int vp = u / nq, q = u - vp * nq;
+      const int v = (2 * vp + r) * 128 + row;
+      const bool valid = 2 * vp + r < n_vb && v < V;
+      float4 *dst = valid ? reinterpret_cast<float4 *>(dW + (int64_t)v * d + q * kDwN) : nullptr;
+      if (nks == 0) {
+        if (valid)
+          for (int c = 0; c < kDwN / 4; ++c) dst[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+        continue;
+      }
+      if (!(ok = wait_sleepy(&sm.acc_full, acc_ph, abort, dev_err))) break;
+      acc_ph ^= 1;
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < kDwN / 32; ++c) {
+        float x[32];
+        tmem_ld32(tmem + lane_off + c * 32, x);
+        if (valid) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            float4 o = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+            if (accumulate) {
+              const float4 p = dst[c * 8 + e];
+              o.x += p.x; o.y += p.y; o.z += p.z; o.w += p.w;
+            }
+            dst[c * 8 + e] = o;
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&sm.acc_empty);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still signal or fill it
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
@@ -1217,6 +1449,22 @@ bool make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t cols,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D bf16 map: dims (innermost first) with byte strides of dims 1 and 2,
+// box `box`, swizzle `sw`.
+bool make_map3(CUtensorMap *m, const void *ptr, const cuuint64_t (&dims)[3],
+               const cuuint64_t (&strides)[2], const cuuint32_t (&box)[3],
+               CUtensorMapSwizzle sw) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t d[3] = {dims[0], dims[1], dims[2]};
+  cuuint64_t st[2] = {strides[0], strides[1]};
+  cuuint32_t b[3] = {box[0], box[1], box[2]};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), d, st, b, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int num_sms();
 
 // CTAs of the LSE grid: every 2-CTA cluster that fits at once (persistent).
@@ -1247,10 +1495,28 @@ int num_sms() {
   return n;
 }
 
+// CTAs of the dW GEMM grid: every CTA pair that fits at once (persistent).
+int dw_grid(size_t smem) {
+  static int cached = 0;
+  if (cached) return cached;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * 64, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, (const void *)dw_gemm_kernel, &cfg) != cudaSuccess ||
+      n <= 0) {
+    cudaGetLastError();
+    n = num_sms() / 2;
+  }
+  cached = 2 * (n > 0 ? n : 1);
+  return cached;
+}
+
 // The cluster backward needs d = 8 * 64 * A with 1 <= A <= 6: each CTA's
 // output slice of 64 * A columns stays in TMEM beside two S buffers of the
 // column-tile width BN (2 BN + 64 A <= 512).
-bool use_cluster_path(int d) { return d % 512 == 0 && d >= 512 && d <= 3072; }
+bool use_cluster_path(int d) { return grad_cluster_path(d); }
 int cluster_tile_width(int d) { return d <= 2048 ? 128 : d <= 2560 ? 96 : 64; }
 
 // Clusters that fit at once (persistent grid), from the occupancy API.
@@ -1288,21 +1554,62 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
   PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<false, BN>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
   const int ncl = cluster_grid<BN>((const void *)bwd_cluster_kernel<true, BN>, cl_smem);
-  PAIR_BEGIN("zero_tail_dh", s);
-  zero_tail_rows_kernel<true><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, w.counters, w.tok_idx, g.dH);
-  PAIR_LAUNCH_CHECK(s);
+  uint8_t *gring = static_cast<uint8_t *>(w.gring);
+  if (BN == 128 && w.gimg && w.gimg_rb > 0) {
+    // Token blocks in chunks of w.gimg_rb: the dH pass keeps the chunk's
+    // logit-gradient tiles, the dW GEMM reads them (first chunk stores dW,
+    // later chunks add to it). Chunks past the last active token exit at
+    // once; their number is fixed by T so the launch sequence needs no
+    // device-to-host read.
+    const int cap = w.gimg_rb;
+    const int n_vb = (g.V + 127) / 128;
+    CUtensorMap mG, mH3;
+    if (!make_map3(&mG, w.gimg, {64, 128, (cuuint64_t)2 * cap * n_vb}, {128, 16384}, {64, 32, 2},
+                   CU_TENSOR_MAP_SWIZZLE_NONE) ||
+        !make_map3(&mH3, w.Hc, {64, (cuuint64_t)w.Tpad, (cuuint64_t)g.d / 64},
+                   {(cuuint64_t)g.d * 2, 128}, {64, (cuuint32_t)kDwKS, 4},
+                   CU_TENSOR_MAP_SWIZZLE_128B))
+      return PAIR_ERR_CUDA;
+    const size_t dw_smem = sizeof(DwSmem) + 1024;
+    PAIR_CUDA_TRY(cudaFuncSetAttribute(dw_gemm_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dw_smem));
+    const int64_t n_chunks = ((g.T + 127) / 128 + cap - 1) / cap;
+    for (int64_t c = 0; c < n_chunks; ++c) {
+      const int rb0 = (int)(c * cap);
+      PAIR_BEGIN("bwd_dh_tc", s);
+      bwd_cluster_kernel<true, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
+          mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH, gring,
+          static_cast<uint8_t *>(w.gimg), w.tailbuf, rb0, cap, g.dev_err);
+      PAIR_LAUNCH_CHECK(s);
+      PAIR_BEGIN("tail_dh", s);
+      tail_reduce_kernel<true, BN><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, rb0, cap, w.counters,
+                                                       w.tok_idx, w.tailbuf, g.dH);
+      PAIR_LAUNCH_CHECK(s);
+      PAIR_BEGIN("dw_gemm_tc", s);
+      dw_gemm_kernel<<<dw_grid(dw_smem), kThreads, dw_smem, s>>>(
+          mG, mH3, g.d, g.V, rb0, cap, c > 0 ? 1 : 0, w.counters, g.dW, g.dev_err);
+      PAIR_LAUNCH_CHECK(s);
+    }
+    return PAIR_OK;
+  }
+  constexpr int kAll = 0x7fffffff;
   PAIR_BEGIN("bwd_dh_tc", s);
   bwd_cluster_kernel<true, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-      mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH,
-      static_cast<uint8_t *>(w.gring), g.dev_err);
+      mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH, gring, nullptr,
+      w.tailbuf, 0, kAll, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
-  PAIR_BEGIN("zero_tail_dw", s);
-  zero_tail_rows_kernel<false><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, w.counters, w.tok_idx, g.dW);
+  PAIR_BEGIN("tail_dh", s);
+  tail_reduce_kernel<true, BN><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, 0, kAll, w.counters,
+                                                   w.tok_idx, w.tailbuf, g.dH);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("bwd_dw_tc", s);
   bwd_cluster_kernel<false, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-      mW128, mHc, mHc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW,
-      static_cast<uint8_t *>(w.gring), g.dev_err);
+      mW128, mHc, mHc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW, gring, nullptr,
+      w.tailbuf, 0, kAll, g.dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("tail_dw", s);
+  tail_reduce_kernel<false, BN><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, 0, kAll, w.counters,
+                                                    w.tok_idx, w.tailbuf, g.dW);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
@@ -1356,6 +1663,20 @@ pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t 
       mW128, mH, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
+}
+
+// Device memory the dW pass may use for kept logit-gradient tiles; larger
+// problems run in several token chunks.
+constexpr int64_t kGImgBudget = int64_t(8) << 30;
+
+int grad_gimg_rows(int64_t T, int32_t d, int32_t V, pair_dtype dt) {
+  if (dt != PAIR_BF16 || !use_cluster_path(d) || cluster_tile_width(d) != 128 || d % kDwN != 0)
+    return 0;
+  const int64_t n_rb = (T + 127) / 128;
+  const int64_t per_rb = (int64_t)((V + 127) / 128) * kGImgTileBytes;
+  int64_t cap = kGImgBudget / per_rb;
+  if (cap < 32) cap = 32;
+  return (int)(n_rb < cap ? n_rb : cap);
 }
 
 pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {

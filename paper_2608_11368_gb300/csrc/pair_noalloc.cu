@@ -51,7 +51,9 @@ extern "C" pair_status pair_grad_noalloc(
   reset_launches();
   if (!H || !W || !y || !mask || !cu_seqlens || !a || !dH || !dW || !Jobj)
     return PAIR_ERR_INVALID_ARG;
-  const size_t need = pair_grad_workspace_size(T, d, V, R, dt);
+  // This path keeps no logit-gradient image (its dW pass recomputes the
+  // logits), so it needs the workspace without one.
+  const size_t need = pair_grad_workspace_min_size(T, d, V, R, dt);
   if (need == 0)
     return (dt == PAIR_BF16 && d % 64 != 0 && d % 16 == 0)
                ? PAIR_ERR_UNSUPPORTED
@@ -73,7 +75,7 @@ extern "C" pair_status pair_grad_noalloc(
   // The workspace needs no initial contents: every kernel writes the parts
   // it later reads within the same call.
   GradWorkspace w;
-  grad_workspace_bytes(T, d, V, R, dt, &w, ws);
+  grad_workspace_bytes(T, d, V, R, dt, &w, ws, 0);
   GradArgs g{T, d, V, R, dt, H, W, y, mask, cu_seqlens, a,
              dH, dW, Jobj, logp_seq, dev_err};
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

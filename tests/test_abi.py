@@ -23,7 +23,7 @@ def L():
 def test_exports_every_header_function(L):
     names = L.header_functions()
     assert {"pair_coeffs", "pair_grad", "pair_estimate_dense",
-            "pair_grad_workspace_size", "pair_status_sync",
+            "pair_grad_workspace_size", "pair_grad_workspace_min_size", "pair_status_sync",
             "pair_status_string", "pair_last_launch_count"} <= set(names)
     lib = L.lib()
     for n in names:
@@ -40,16 +40,31 @@ def test_status_strings(L):
 def test_workspace_size_rules(L):
     ws = L.pair_grad_workspace_size
     assert ws(1000, 2048, 151936, 64, L.PAIR_BF16) > 1000 * 2048 * 2
+    wmin = L.pair_grad_workspace_min_size
     # The fp32 path stages 4-byte hidden rows; bf16 stages 2-byte rows plus a
-    # fixed ring of logit-gradient tiles, so fp32 needs more once T is large.
-    assert (ws(100000, 2048, 151936, 64, L.PAIR_F32) - ws(100000, 2048, 151936, 64, L.PAIR_BF16)
-            > 100000 * 2048 * 2 - (16 << 20))
+    # fixed ring of logit-gradient tiles and the clusters' tail scratch
+    # (24 x 2 x 128 x d fp32), so fp32 needs more once T is large.
+    fixed = (12 << 20) + 24 * 2 * 128 * 2048 * 4 + (1 << 20)
+    assert (wmin(100000, 2048, 151936, 64, L.PAIR_F32)
+            - wmin(100000, 2048, 151936, 64, L.PAIR_BF16) > 100000 * 2048 * 2 - fixed)
+    # With 128-wide tiles (d in {512, ..., 2048}) bf16 also keeps the
+    # logit-gradient image: min(ceil(T/128), max(32, 2^33 // per_block)) token
+    # blocks of ceil(V/128) 32 KB tiles; other widths and fp32 keep none.
+    for T, d, V in [(100000, 2048, 151936), (1000, 512, 1000), (10 ** 6, 1024, 10 ** 6),
+                    (5000, 1536, 300)]:
+        per_block = (V + 127) // 128 * 32768
+        blocks = min((T + 127) // 128, max(32, (8 << 30) // per_block))
+        assert ws(T, d, V, 64, L.PAIR_BF16) - wmin(T, d, V, 64, L.PAIR_BF16) == blocks * per_block
+    for d, dt in [(2560, L.PAIR_BF16), (3072, L.PAIR_BF16), (640, L.PAIR_BF16),
+                  (2048, L.PAIR_F32)]:
+        assert ws(5000, d, 1000, 8, dt) == wmin(5000, d, 1000, 8, dt)
     assert ws(1000, 96, 100, 4, L.PAIR_BF16) == 0      # bf16 needs d % 64 == 0
     assert ws(1000, 96, 100, 4, L.PAIR_F32) > 0
     assert ws(1000, 20, 100, 4, L.PAIR_F32) == 0       # d % 16 != 0
     assert ws(0, 64, 100, 4, L.PAIR_F32) == 0
     assert ws(10, 64, 100, 0, L.PAIR_F32) == 0
     assert ws(10, 64, 0, 1, L.PAIR_F32) == 0
+    assert wmin(1000, 96, 100, 4, L.PAIR_BF16) == 0
 
 
 def test_host_validation_without_device():

@@ -32,9 +32,20 @@ def _coeffs(inp, scale=1.0):
     return c["a"].reshape(-1).astype(np.float32)
 
 
-def _run(inp, a, **kw):
+def _run(inp, a, image_blocks=None, **kw):
+    """image_blocks: size the workspace to hold that many token blocks of the
+    logit-gradient image (0 = none, recomputing dW pass); None = the default
+    pair_grad_workspace_size."""
     B = _binding()
     t = head_inputs(inp, a)
+    if image_blocks is not None:
+        T, d = t["H"].shape
+        V, R = t["W"].shape[0], inp["R"]
+        dt = B.PAIR_BF16 if t["H"].dtype == torch.bfloat16 else B.PAIR_F32
+        nbytes = (B.pair_grad_workspace_min_size(T, d, V, R, dt)
+                  + image_blocks * ((V + 127) // 128) * 32768)
+        assert nbytes <= B.pair_grad_workspace_size(T, d, V, R, dt)
+        kw["ws"] = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
     err = dev_err_word()
     Jo, dH, dW, lps = B.pair_grad(t["H"], t["W"], t["y"], t["mask"],
                                   t["cu_seqlens"], t["a"], dev_err=err, **kw)
@@ -42,8 +53,8 @@ def _run(inp, a, **kw):
     return st, Jo.item(), dH, dW, lps, t
 
 
-def _full_check(inp, a):
-    st, J, dH, dW, lps, t = _run(inp, a)
+def _full_check(inp, a, image_blocks=None):
+    st, J, dH, dW, lps, t = _run(inp, a, image_blocks)
     assert st == 0
     ref = oracle.pair_grad_ref(inp, a.astype(np.float64), full=True)
     dHn, dWn = dH.cpu().numpy(), dW.cpu().numpy()
@@ -102,14 +113,43 @@ def test_grad_bf16_full_parity(case):
     _full_check(inp, a)
 
 
+CHUNKED = [
+    # name, d, V, B, G, len_scale, w_mult, image token blocks per chunk
+    ("qwen3_1p7b_head", 512, 1000, 3, 8, 0.3, 4.0, 0),      # no image: dW recomputes
+    ("qwen3_1p7b_head", 512, 1000, 3, 8, 0.3, 4.0, 1),      # 128-token chunks
+    ("longctx_skew", 1024, 5003, 2, 8, 0.15, 2.0, 3),       # ragged V, 3-block chunks
+    ("qwen3_1p7b_head", 2048, 20000, 2, 8, 0.15, 1.0, 2),   # d = 2048, 2-block chunks
+    ("qwen3_4b_head", 1536, 777, 2, 6, 0.08, 8.0, 1),
+]
+
+
+@pytest.mark.parametrize("case", CHUNKED,
+                         ids=[f"d{c[1]}_V{c[2]}_blocks{c[7]}" for c in CHUNKED])
+def test_grad_bf16_backward_chunks(case):
+    """Workspaces below pair_grad_workspace_size: the backward runs in token
+    chunks (dW stored by the first, added by later ones), or with no image at
+    all; each against the oracle."""
+    name, d, V, B, G, ls, wm, blocks = case
+    inp = synth.make_head_workload(synth.WORKLOADS[name], 5, B=B, G=G, d=d, V=V,
+                                   len_scale=ls, w_std_mult=wm)
+    a = _coeffs(inp)
+    if not (a != 0).any():
+        a[0] = 0.75
+    idx, _, _ = oracle.compact_tokens(inp["cu_seqlens"], inp["mask"], a)
+    if blocks:
+        assert idx.size > 128 * blocks   # several chunks
+    _full_check(inp, a, image_blocks=blocks)
+
+
 def test_grad_no_active_rollout():
     inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 1, B=2,
-                                   G=2, d=128, V=520, len_scale=0.05)
+                                   G=2, d=512, V=520, len_scale=0.05)
     a = np.zeros(inp["R"], np.float32)
     a[1] = -0.0
-    st, J, dH, dW, lps, _ = _run(inp, a)
-    assert st == 0 and J == 0.0
-    assert (dH == 0).all() and (dW == 0).all() and (lps == 0).all()
+    for blocks in (None, 0, 1):
+        st, J, dH, dW, lps, _ = _run(inp, a, blocks)
+        assert st == 0 and J == 0.0
+        assert (dH == 0).all() and (dW == 0).all() and (lps == 0).all()
 
 
 def test_grad_nan_padding_is_ignored_and_deterministic():
@@ -124,6 +164,19 @@ def test_grad_nan_padding_is_ignored_and_deterministic():
     for x, y in ((r0, r1), (r0, r2)):
         assert x[1] == y[1]
         assert torch.equal(x[2], y[2]) and torch.equal(x[3], y[3])
+
+
+@pytest.mark.parametrize("blocks", [None, 0, 2])
+def test_grad_cluster_path_deterministic(blocks):
+    """Cluster backward with tail row blocks split across clusters (and, for
+    blocks = 2, several token chunks): reruns are bit-identical."""
+    inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 5, B=3, G=8, d=512,
+                                   V=1000, len_scale=0.3, w_std_mult=4.0)
+    a = _coeffs(inp)
+    r0 = _run(inp, a, blocks)
+    r1 = _run(inp, a, blocks)
+    assert r0[0] == 0 and r1[0] == 0 and r0[1] == r1[1]
+    assert torch.equal(r0[2], r1[2]) and torch.equal(r0[3], r1[3])
 
 
 def test_grad_target_out_of_range_flagged():
