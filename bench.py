@@ -44,7 +44,7 @@ REF_SAMPLE_TOKENS = 48           # oracle sample per --impl reference step
 # Tensor-core kernels of one pair_grad call; each is charged one logit-sized
 # GEMM (2 T_eff V d FLOP) of algorithmic work per call, whatever the number of
 # token chunks it is launched for.
-TC_KERNELS = ("lse_tc", "bwd_dh_tc", "bwd_dw_tc", "dw_gemm_tc")
+TC_KERNELS = ("lse_tc", "bwd_dh_tc", "bwd_dw_tc", "dh_gemm_tc", "dw_gemm_tc")
 
 
 def parse_args():

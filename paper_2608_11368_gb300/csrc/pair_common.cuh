@@ -71,6 +71,7 @@ struct GradWorkspace {
   void *gring;         // per-cluster ring of published Gs tiles
   float *tailbuf;      // [kMaxClusters][2][128][d] partial tail units (cluster path)
   void *gimg;          // bf16 logit-gradient tiles of gimg_rb token blocks, or null
+  float *sbuf;         // fp32 logit tiles of the same blocks (kept by the LSE pass)
   int gimg_rb;         // token blocks (128 rows) per backward chunk; 0 = no image
   int64_t Tpad;
   int nsplit;
@@ -79,10 +80,12 @@ struct GradWorkspace {
 // Whether the bf16 backward runs as 8-CTA clusters: d = 512 A, 1 <= A <= 6.
 inline bool grad_cluster_path(int d) { return d % 512 == 0 && d >= 512 && d <= 3072; }
 
-// Token blocks of the logit-gradient image that the bf16 backward keeps for
-// its dW pass (0 where that path does not apply: fp32, or d outside the
-// 128-wide cluster tiles).
+// Token blocks per backward chunk for which the bf16 path keeps the fp32
+// logits and the bf16 logit-gradient image (0 where that path does not
+// apply: fp32, or d not a multiple of 512), and the bytes one block of both
+// takes.
 int grad_gimg_rows(int64_t T, int32_t d, int32_t V, pair_dtype dt);
+size_t grad_image_block_bytes(int32_t V);
 constexpr uint32_t kGImgTileBytes = 128 * 128 * 2;  // one 128 x 128 bf16 tile
 
 // Workspace layout with gimg_rb token blocks of logit-gradient image (0 =

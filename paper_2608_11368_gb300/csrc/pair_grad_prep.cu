@@ -396,8 +396,9 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   const bool cl = dt == PAIR_BF16 && grad_cluster_path(d);
   const size_t o_tail = cl ? take((size_t)kMaxClusters * 2 * 128 * d * sizeof(float)) : off;
   // The image comes last, so that a larger workspace only adds token blocks.
-  const size_t o_gimg =
-      gimg_rb ? take((size_t)gimg_rb * (size_t)((V + 127) / 128) * kGImgTileBytes) : off;
+  const size_t n_vt = (size_t)((V + 127) / 128);
+  const size_t o_gimg = gimg_rb ? take((size_t)gimg_rb * n_vt * kGImgTileBytes) : off;
+  const size_t o_sbuf = gimg_rb ? take((size_t)gimg_rb * n_vt * 128 * 128 * sizeof(float)) : off;
   if (out) {
     char *b = static_cast<char *>(base);
     out->counters = reinterpret_cast<int32_t *>(b + o_cnt);
@@ -416,6 +417,7 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->gring = b + o_ring;
     out->tailbuf = cl ? reinterpret_cast<float *>(b + o_tail) : nullptr;
     out->gimg = gimg_rb ? b + o_gimg : nullptr;
+    out->sbuf = gimg_rb ? reinterpret_cast<float *>(b + o_sbuf) : nullptr;
     out->gimg_rb = gimg_rb;
     out->Tpad = Tpad;
     out->nsplit = kNSplit;
@@ -429,7 +431,7 @@ int grad_gimg_rows_fit(int64_t T, int32_t d, int32_t V, int32_t R, pair_dtype dt
   if (ws_bytes < base) return -1;
   const int pref = grad_gimg_rows(T, d, V, dt);
   if (pref == 0) return 0;
-  const size_t fit = (ws_bytes - base) / ((size_t)((V + 127) / 128) * kGImgTileBytes);
+  const size_t fit = (ws_bytes - base) / grad_image_block_bytes(V);
   return fit < (size_t)pref ? (int)fit : pref;
 }
 

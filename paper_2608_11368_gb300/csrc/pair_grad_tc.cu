@@ -72,13 +72,18 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
     lse_kernel(const __grid_constant__ CUtensorMap tmH,
                const __grid_constant__ CUtensorMap tmW, int d, int V,
                int nsplit, int64_t Tpad, const int32_t *counters,
-               const int32_t *tok_y, float2 *part, float *zy,
-               int32_t *dev_err) {
+               const int32_t *tok_y, float2 *part, float *zy, int rb0, int cap,
+               float *sbuf, int s_blocks, int32_t *dev_err) {
   extern __shared__ uint8_t smem_raw[];
   LseSmem &sm = *reinterpret_cast<LseSmem *>(align1k(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int Teff = counters[0];
-  const int n_tb = (Teff + 127) / 128;
+  // Token blocks [rb0, rb0 + n_tb) of this launch; with sbuf, the fp32
+  // logits of its first s_blocks blocks are also stored (128 x 128 tiles,
+  // tile (b, vt) at ((b * n_vt128 + vt) * 128 + row) * 128 + col).
+  const int n_tb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  const int n_vt128 = (V + 127) / 128;
+  const int s_lim = min(n_tb, s_blocks);
   const int n_vt = (V + kLseBN - 1) / kLseBN;
   // Work unit = (pair of token blocks, vocabulary split); CTA r of the pair
   // takes token block 2 * pair + r (past the last block for an odd count:
@@ -122,7 +127,7 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
       for (int s = 0; s < kLseStages; ++s) last_ph[s] = -1;
       bool ok = true;
       for (int u = pid; u < n_units && ok; u += npairs) {
-        const int tb = 2 * (u / nsplit) + r, sp = u % nsplit;
+        const int tb = rb0 + 2 * (u / nsplit) + r, sp = u % nsplit;
         const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
         const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
         for (int vt = vt0; vt < vt1 && ok; ++vt) {
@@ -195,11 +200,16 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
     uint32_t acc_ph = 0;
     bool ok = true;
     for (int u = pid; u < n_units && ok; u += npairs) {
-      const int tb = 2 * (u / nsplit) + r, sp = u % nsplit;
+      const int tbl = 2 * (u / nsplit) + r, sp = u % nsplit;
+      const int tb = rb0 + tbl;
       const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
       const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
       const int p = tb * 128 + row;
       const bool valid = p < Teff;
+      // This row's fp32 logits, when this block's tiles are kept.
+      float *srow = (sbuf && tbl < s_lim)
+                        ? sbuf + ((int64_t)tbl * n_vt128 * 128 + row) * 128
+                        : nullptr;
       const int yt = valid ? tok_y[p] : -1;
       float m2 = -INFINITY, l = 0.f, zt = 0.f;
       bool found = false;
@@ -211,6 +221,13 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
           float v[32];
           tmem_ld32(lane_addr + acc * kLseBN + c * 32, v);
           const int col0 = vt * kLseBN + c * 32;
+          if (srow && col0 < V) {
+            float4 *dst = reinterpret_cast<float4 *>(
+                srow + (int64_t)(col0 >> 7) * (128 * 128) + (col0 & 127));
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+              dst[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+          }
           const int off = yt - col0;
           if (off >= 0 && off < 32) {
             found = true;
@@ -257,11 +274,14 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
 }
 
 // lse_t = ln 2 * (M + log2 sum_s l_s 2^(m_s - M)) over the vocabulary splits.
+// Tokens [128 rb0, 128 (rb0 + cap)) of the active ones.
 __global__ void lse_combine_kernel(int nsplit, int64_t Tpad,
                                    const int32_t *counters, const float2 *part,
-                                   float *lse) {
+                                   float *lse, int rb0, int cap) {
   const int Teff = counters[0];
-  for (int p = blockIdx.x * blockDim.x + threadIdx.x; p < Teff;
+  const int64_t hi64 = (int64_t)(rb0 + (int64_t)cap) * 128;
+  const int p1 = (int)(hi64 < Teff ? hi64 : Teff);
+  for (int p = rb0 * 128 + blockIdx.x * blockDim.x + threadIdx.x; p < p1;
        p += gridDim.x * blockDim.x) {
     float M = -INFINITY;
     for (int s = 0; s < nsplit; ++s) M = fmaxf(M, part[(int64_t)s * Tpad + p].x);
@@ -1218,6 +1238,230 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   }
 }
 
+// ------------------------------------------ logit-gradient image from S
+//
+// Gs_tv = -c_t exp(z_tv - lse_t) in bf16 for every tile of a chunk of token
+// blocks, from the fp32 logit tiles the LSE pass kept: one 32 KB image tile
+// per 128 tokens x 128 vocabulary rows, two K-major SWIZZLE_128B atoms of 64
+// vocabulary columns (the layout both backward GEMMs read). Columns >= V,
+// rows >= T_eff and tokens with c_t = 0 give exact zeros. Streaming kernel:
+// 64 KB read and 32 KB written per tile.
+__global__ void __launch_bounds__(256) g_image_kernel(int V, int rb0, int cap,
+                                                      const int32_t *counters,
+                                                      const float *tok_c, const float *lse,
+                                                      const float *sbuf, uint8_t *gimg) {
+  const int Teff = counters[0];
+  const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  const int n_vt = (V + 127) / 128;
+  const int64_t n_tiles = (int64_t)nrb * n_vt;
+  for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+    const int b = (int)(tile / n_vt), vt = (int)(tile - (int64_t)b * n_vt);
+    const float *src = sbuf + tile * (128 * 128);
+    uint8_t *dst = gimg + tile * kGImgTileBytes;
+    for (int i = threadIdx.x; i < 128 * 16; i += blockDim.x) {
+      const int row = i >> 4, ch = i & 15;  // 8-column chunk ch of the row
+      const int p = (rb0 + b) * 128 + row;
+      const float cc = p < Teff ? tok_c[p] : 0.f;
+      const float ll = p < Teff ? lse[p] * kLog2e : 0.f;
+      const float4 s0 = reinterpret_cast<const float4 *>(src + row * 128 + ch * 8)[0];
+      const float4 s1 = reinterpret_cast<const float4 *>(src + row * 128 + ch * 8)[1];
+      const float v[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+      const int col0 = vt * 128 + ch * 8;
+      uint32_t pk[4];
+#pragma unroll
+      for (int j = 0; j < 8; j += 2) {
+        float g2[2];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const bool live = cc != 0.f && col0 + j + e < V;
+          g2[e] = live ? -cc * ex2_approx(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
+        }
+        __nv_bfloat162 b2 = __floats2bfloat162_rn(g2[0], g2[1]);
+        pk[j >> 1] = *reinterpret_cast<uint32_t *>(&b2);
+      }
+      *reinterpret_cast<uint4 *>(dst + (ch >> 3) * kAtom128 + sw128_offset(row, (ch & 7) * 8)) =
+          make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    }
+  }
+}
+
+// ---------------------------------------------- dH from the stored image
+//
+// Softmax part of dH as the plain GEMM dH[t, :] = sum_v Gs[t, v] W[v, :],
+// with the image tiles as the K-major A operand (64 vocabulary rows per
+// stage, one 16 KB atom, copied verbatim) and W as the MN-major B operand.
+// CTA pairs (2-CTA clusters) take two token blocks of the same 256-column
+// chunk of d and share its W stage by multicast (each CTA fetches two of the
+// four 64-column atoms). Work unit = (token block pair, 256-column chunk);
+// the fp32 accumulator (128 x 256) is double-buffered in TMEM so the drain of
+// one unit overlaps the next. Each (token, column) is owned by one CTA and
+// summed over all of V in one fixed order: deterministic, no atomics. An odd
+// last block is computed twice (the pair's other CTA repeats it) and stored
+// once.
+constexpr int kDhN = 256;                              // output columns per unit
+constexpr int kDhStages = 4;
+constexpr uint32_t kDhABytes = kAtom128;               // 128 tokens x 64 vocabulary
+constexpr uint32_t kDhBBytes = (kDhN / 64) * 64 * 128; // 4 column atoms x 64 rows
+constexpr uint32_t kIdescDh = idesc_bf16(128, kDhN, 0, 1);
+
+struct DhSmem {
+  uint8_t a[kDhStages][kDhABytes];
+  uint8_t b[kDhStages][kDhBBytes];
+  uint64_t full[kDhStages], empty[kDhStages];
+  uint64_t acc_full[2], acc_empty[2], mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    dh_gemm_kernel(const __grid_constant__ CUtensorMap tmW, int d, int V, int rb0, int cap,
+                   const int32_t *counters, const int32_t *tok_idx, const uint8_t *gimg,
+                   float *dH, int32_t *dev_err) {
+  const int Teff = counters[0];
+  const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  if (nrb == 0) return;  // no token in this chunk
+  extern __shared__ uint8_t smem_raw[];
+  DhSmem &sm = *reinterpret_cast<DhSmem *>(align1k(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = (int)cluster_rank();
+  const int pid = (int)cluster_id_x(), npairs = (int)num_clusters_x();
+  const int n_vt = (V + 127) / 128;
+  const int nks = 2 * n_vt;  // 64-wide vocabulary steps (image atoms)
+  const int nq = d / kDhN;
+  const int n_units = (nrb + 1) / 2 * nq;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kDhStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 2);  // both CTAs' MMAs done with the stage
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.acc_full[s], 1);
+      mbar_init(&sm.acc_empty[s], 128);
+    }
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmW);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the peer's barriers exist before any multicast lands
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  volatile int *abort = &sm.abort;
+
+  if (warp == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
+      int stage = 0;
+      uint32_t ph = 0;
+      int last_ph[kDhStages];
+      for (int s = 0; s < kDhStages; ++s) last_ph[s] = -1;
+      bool ok = true;
+      for (int u = pid; u < n_units && ok; u += npairs) {
+        const int tp = u / nq, q = u - tp * nq;
+        const int b = min(2 * tp + r, nrb - 1);
+        const uint8_t *arow = gimg + (size_t)b * n_vt * kGImgTileBytes;
+        for (int ks = 0; ks < nks; ++ks) {
+          if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+          if (elect_one()) {
+            mbar_expect_tx(&sm.full[stage], kDhABytes + kDhBBytes);
+            bulk_load(sm.a[stage], arow + (size_t)ks * kAtom128, kAtom128, &sm.full[stage]);
+            tma_load_3d_mc(sm.b[stage] + r * (kDhBBytes / 2), &tmW, &sm.full[stage], 0, 64 * ks,
+                           q * (kDhN / 64) + r * (kDhN / 128), (uint16_t)3);
+          }
+          __syncwarp();
+          last_ph[stage] = (int)ph;
+          if (++stage == kDhStages) { stage = 0; ph ^= 1; }
+        }
+      }
+      for (int s = 0; s < kDhStages; ++s)
+        if (last_ph[s] >= 0) {
+          volatile int never = 0;
+          wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+        }
+    }
+  } else if (warp == 1) {
+    {  // whole warp: uniform loop state; elected lane issues
+      // A: K-major atom, 16 tokens of K = 32 bytes along the swizzled row.
+      // B: 4 column atoms of 64 vocabulary rows (LBO 8 KB), row groups of 8
+      // (SBO 1 KB); 16 vocabulary rows = 2 KB.
+      const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
+      const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 64 * 128, 1024);
+      int stage = 0, acc = 0;
+      uint32_t ph = 0, acc_ph = 0;
+      bool ok = true;
+      for (int u = pid; u < n_units && ok; u += npairs) {
+        if (!(ok = wait(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
+        tc_fence_after();
+        const uint32_t dt = tmem + acc * kDhN;
+        for (int ks = 0; ks < nks; ++ks) {
+          if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+          const uint64_t da = da0 + (uint64_t)stage * (kDhABytes >> 4);
+          const uint64_t db = db0 + (uint64_t)stage * (kDhBBytes >> 4);
+          if (elect_one()) {
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_bf16(dt, da + 2 * kk, db + kk * (2048 >> 4), kIdescDh, (ks | kk) != 0);
+            mma_commit_multicast(&sm.empty[stage], (uint16_t)3);
+          }
+          __syncwarp();
+          if (++stage == kDhStages) { stage = 0; ph ^= 1; }
+        }
+        if (!ok) break;
+        if (elect_one()) mma_commit(&sm.acc_full[acc]);
+        __syncwarp();
+        if (++acc == 2) { acc = 0; acc_ph ^= 1; }
+      }
+      if (elect_one()) mma_commit(&sm.mma_done);
+      __syncwarp();
+      volatile int never = 0;
+      wait(&sm.mma_done, 0, &never, dev_err);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    int acc = 0;
+    uint32_t acc_ph = 0;
+    bool ok = true;
+    for (int u = pid; u < n_units && ok; u += npairs) {
+      const int tp = u / nq, q = u - tp * nq;
+      const int t = (rb0 + 2 * tp + r) * 128 + row;
+      const bool valid = 2 * tp + r < nrb && t < Teff;
+      float4 *dst =
+          valid ? reinterpret_cast<float4 *>(dH + (int64_t)tok_idx[t] * d + q * kDhN) : nullptr;
+      if (!(ok = wait_sleepy(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < kDhN / 32; ++c) {
+        float x[32];
+        tmem_ld32(tmem + lane_off + acc * kDhN + c * 32, x);
+        if (valid) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            dst[c * 8 + e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&sm.acc_empty[acc]);
+      if (++acc == 2) { acc = 0; acc_ph ^= 1; }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still signal or fill it
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
 // ------------------------------------- dW from the stored logit gradient
 //
 // With 128-wide column tiles the dH pass keeps every bf16 tile Gs it forms
@@ -1495,22 +1739,21 @@ int num_sms() {
   return n;
 }
 
-// CTAs of the dW GEMM grid: every CTA pair that fits at once (persistent).
-int dw_grid(size_t smem) {
-  static int cached = 0;
-  if (cached) return cached;
+// CTAs of a persistent grid of 2-CTA clusters: every pair that fits at once
+// (from the occupancy API; cached per kernel in *cache).
+int pair_grid(const void *kernel, size_t smem, int *cache) {
+  if (*cache) return *cache;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * 64, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, (const void *)dw_gemm_kernel, &cfg) != cudaSuccess ||
-      n <= 0) {
+  if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess || n <= 0) {
     cudaGetLastError();
     n = num_sms() / 2;
   }
-  cached = 2 * (n > 0 ? n : 1);
-  return cached;
+  *cache = 2 * (n > 0 ? n : 1);
+  return *cache;
 }
 
 // The cluster backward needs d = 8 * 64 * A with 1 <= A <= 6: each CTA's
@@ -1555,43 +1798,6 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
   const int ncl = cluster_grid<BN>((const void *)bwd_cluster_kernel<true, BN>, cl_smem);
   uint8_t *gring = static_cast<uint8_t *>(w.gring);
-  if (BN == 128 && w.gimg && w.gimg_rb > 0) {
-    // Token blocks in chunks of w.gimg_rb: the dH pass keeps the chunk's
-    // logit-gradient tiles, the dW GEMM reads them (first chunk stores dW,
-    // later chunks add to it). Chunks past the last active token exit at
-    // once; their number is fixed by T so the launch sequence needs no
-    // device-to-host read.
-    const int cap = w.gimg_rb;
-    const int n_vb = (g.V + 127) / 128;
-    CUtensorMap mG, mH3;
-    if (!make_map3(&mG, w.gimg, {64, 128, (cuuint64_t)2 * cap * n_vb}, {128, 16384}, {64, 32, 2},
-                   CU_TENSOR_MAP_SWIZZLE_NONE) ||
-        !make_map3(&mH3, w.Hc, {64, (cuuint64_t)w.Tpad, (cuuint64_t)g.d / 64},
-                   {(cuuint64_t)g.d * 2, 128}, {64, (cuuint32_t)kDwKS, 4},
-                   CU_TENSOR_MAP_SWIZZLE_128B))
-      return PAIR_ERR_CUDA;
-    const size_t dw_smem = sizeof(DwSmem) + 1024;
-    PAIR_CUDA_TRY(cudaFuncSetAttribute(dw_gemm_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dw_smem));
-    const int64_t n_chunks = ((g.T + 127) / 128 + cap - 1) / cap;
-    for (int64_t c = 0; c < n_chunks; ++c) {
-      const int rb0 = (int)(c * cap);
-      PAIR_BEGIN("bwd_dh_tc", s);
-      bwd_cluster_kernel<true, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-          mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH, gring,
-          static_cast<uint8_t *>(w.gimg), w.tailbuf, rb0, cap, g.dev_err);
-      PAIR_LAUNCH_CHECK(s);
-      PAIR_BEGIN("tail_dh", s);
-      tail_reduce_kernel<true, BN><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, rb0, cap, w.counters,
-                                                       w.tok_idx, w.tailbuf, g.dH);
-      PAIR_LAUNCH_CHECK(s);
-      PAIR_BEGIN("dw_gemm_tc", s);
-      dw_gemm_kernel<<<dw_grid(dw_smem), kThreads, dw_smem, s>>>(
-          mG, mH3, g.d, g.V, rb0, cap, c > 0 ? 1 : 0, w.counters, g.dW, g.dev_err);
-      PAIR_LAUNCH_CHECK(s);
-    }
-    return PAIR_OK;
-  }
   constexpr int kAll = 0x7fffffff;
   PAIR_BEGIN("bwd_dh_tc", s);
   bwd_cluster_kernel<true, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
@@ -1614,10 +1820,13 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
   return PAIR_OK;
 }
 
-}  // namespace
+constexpr int kAllBlocks = 0x7fffffff;
 
-// Forward half: per-token log-sum-exp and target logit.
-pair_status grad_lse_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+// Log-sum-exp pass over token blocks [rb0, rb0 + cap) (clipped to the active
+// ones), then lse for those tokens. With sbuf, the fp32 logit tiles of the
+// first s_blocks of those blocks are kept.
+pair_status launch_lse(const GradArgs &g, const GradWorkspace &w, cudaStream_t s, int rb0,
+                       int cap, float *sbuf, int s_blocks) {
   CUtensorMap mH, mW128;
   if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) || !make_map(&mW128, g.W, g.V, g.d, 128))
     return PAIR_ERR_CUDA;
@@ -1626,18 +1835,93 @@ pair_status grad_lse_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t 
   PAIR_CUDA_TRY(cudaFuncSetAttribute(lse_kernel,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)lse_smem));
   PAIR_BEGIN("lse_tc", s);
-  lse_kernel<<<lse_grid(lse_smem), kThreads, lse_smem, s>>>(mH, mW128, g.d, g.V, w.nsplit,
-                                                           w.Tpad, w.counters, w.tok_y,
-                                                           w.part, w.zy, g.dev_err);
+  lse_kernel<<<lse_grid(lse_smem), kThreads, lse_smem, s>>>(
+      mH, mW128, g.d, g.V, w.nsplit, w.Tpad, w.counters, w.tok_y, w.part, w.zy, rb0, cap, sbuf,
+      s_blocks, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("lse_combine", s);
-  lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters, w.part, w.lse);
+  lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters, w.part, w.lse, rb0,
+                                             cap);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
 
-// Backward half: softmax parts of dH and dW from the token coefficients.
+// The backward through the logit-gradient image runs whenever the workspace
+// holds one: token blocks in chunks of w.gimg_rb, and for each chunk
+//   g_image   Gs (bf16 tiles) from the kept fp32 logits, lse and c_t,
+//   dh_gemm   dH rows of the chunk = Gs . W,
+//   dw_gemm   dW (+)= Gs^T . Hc (the first chunk stores, later ones add).
+// The number of chunks follows from T, so the launch sequence needs no
+// device-to-host read; chunks past the last active token exit at once.
+bool image_path(const GradWorkspace &w) { return w.gimg && w.sbuf && w.gimg_rb > 0; }
+
+int64_t image_chunks(const GradArgs &g, const GradWorkspace &w) {
+  return ((g.T + 127) / 128 + w.gimg_rb - 1) / w.gimg_rb;
+}
+
+pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStream_t s,
+                             int64_t c) {
+  const int cap = w.gimg_rb;
+  const int rb0 = (int)(c * cap);
+  const int n_vt = (g.V + 127) / 128;
+  CUtensorMap mG, mH3, mW3;
+  if (!make_map3(&mG, w.gimg, {64, 128, (cuuint64_t)2 * cap * n_vt}, {128, 16384}, {64, 32, 2},
+                 CU_TENSOR_MAP_SWIZZLE_NONE) ||
+      !make_map3(&mH3, w.Hc, {64, (cuuint64_t)w.Tpad, (cuuint64_t)g.d / 64},
+                 {(cuuint64_t)g.d * 2, 128}, {64, (cuuint32_t)kDwKS, 4},
+                 CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map3(&mW3, g.W, {64, (cuuint64_t)g.V, (cuuint64_t)g.d / 64},
+                 {(cuuint64_t)g.d * 2, 128}, {64, 64, 2}, CU_TENSOR_MAP_SWIZZLE_128B))
+    return PAIR_ERR_CUDA;
+  const size_t dh_smem = sizeof(DhSmem) + 1024, dw_smem = sizeof(DwSmem) + 1024;
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(dh_gemm_kernel,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dh_smem));
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(dw_gemm_kernel,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dw_smem));
+  static int dh_cache = 0, dw_cache = 0;
+  uint8_t *gimg = static_cast<uint8_t *>(w.gimg);
+  PAIR_BEGIN("g_image", s);
+  g_image_kernel<<<num_sms() * 4, 256, 0, s>>>(g.V, rb0, cap, w.counters, w.tok_c, w.lse, w.sbuf,
+                                               gimg);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("dh_gemm_tc", s);
+  dh_gemm_kernel<<<pair_grid((const void *)dh_gemm_kernel, dh_smem, &dh_cache), kThreads,
+                   dh_smem, s>>>(mW3, g.d, g.V, rb0, cap, w.counters, w.tok_idx, gimg, g.dH,
+                                 g.dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("dw_gemm_tc", s);
+  dw_gemm_kernel<<<pair_grid((const void *)dw_gemm_kernel, dw_smem, &dw_cache), kThreads,
+                   dw_smem, s>>>(mG, mH3, g.d, g.V, rb0, cap, c > 0 ? 1 : 0, w.counters, g.dW,
+                                 g.dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+}  // namespace
+
+// Forward half: per-token log-sum-exp and target logit over every active
+// token (with an image, the first chunk's logits are kept for the backward).
+pair_status grad_lse_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  if (image_path(w)) return launch_lse(g, w, s, 0, kAllBlocks, w.sbuf, w.gimg_rb);
+  return launch_lse(g, w, s, 0, kAllBlocks, nullptr, 0);
+}
+
+// Backward half: softmax parts of dH and dW from the token coefficients,
+// after grad_lse_tc (chunks after the first recompute their logits).
 pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  if (image_path(w)) {
+    const int64_t nc = image_chunks(g, w);
+    for (int64_t c = 0; c < nc; ++c) {
+      if (c > 0) {
+        const pair_status st = launch_lse(g, w, s, (int)(c * w.gimg_rb), w.gimg_rb, w.sbuf,
+                                          w.gimg_rb);
+        if (st != PAIR_OK) return st;
+      }
+      const pair_status st = launch_chunk_bwd(g, w, s, c);
+      if (st != PAIR_OK) return st;
+    }
+    return PAIR_OK;
+  }
   CUtensorMap mH, mW128;
   if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) || !make_map(&mW128, g.W, g.V, g.d, 128))
     return PAIR_ERR_CUDA;
@@ -1665,21 +1949,37 @@ pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t 
   return PAIR_OK;
 }
 
-// Device memory the dW pass may use for kept logit-gradient tiles; larger
-// problems run in several token chunks.
-constexpr int64_t kGImgBudget = int64_t(8) << 30;
+// Memory the backward may use for kept fp32 logits and bf16 logit-gradient
+// tiles (96 KB per 128 x 128 tile); larger problems run in token chunks.
+constexpr int64_t kImageBudget = int64_t(24) << 30;
+constexpr size_t kImageTileBytes = kGImgTileBytes + 128 * 128 * sizeof(float);
 
 int grad_gimg_rows(int64_t T, int32_t d, int32_t V, pair_dtype dt) {
-  if (dt != PAIR_BF16 || !use_cluster_path(d) || cluster_tile_width(d) != 128 || d % kDwN != 0)
-    return 0;
+  if (dt != PAIR_BF16 || d < 512 || d % kDwN != 0) return 0;
   const int64_t n_rb = (T + 127) / 128;
-  const int64_t per_rb = (int64_t)((V + 127) / 128) * kGImgTileBytes;
-  int64_t cap = kGImgBudget / per_rb;
+  const int64_t per_rb = (int64_t)((V + 127) / 128) * (int64_t)kImageTileBytes;
+  int64_t cap = kImageBudget / per_rb;
   if (cap < 32) cap = 32;
   return (int)(n_rb < cap ? n_rb : cap);
 }
 
+size_t grad_image_block_bytes(int32_t V) {
+  return (size_t)((V + 127) / 128) * kImageTileBytes;
+}
+
+// Whole head: with an image, each chunk's log-sum-exp pass keeps its logits
+// for that chunk's backward (no recomputation); otherwise forward, then the
+// recomputing backward.
 pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  if (image_path(w)) {
+    const int64_t nc = image_chunks(g, w);
+    for (int64_t c = 0; c < nc; ++c) {
+      pair_status st = launch_lse(g, w, s, (int)(c * w.gimg_rb), w.gimg_rb, w.sbuf, w.gimg_rb);
+      if (st == PAIR_OK) st = launch_chunk_bwd(g, w, s, c);
+      if (st != PAIR_OK) return st;
+    }
+    return PAIR_OK;
+  }
   const pair_status st = grad_lse_tc(g, w, s);
   return st != PAIR_OK ? st : grad_bwd_tc(g, w, s);
 }

@@ -33,9 +33,9 @@ def _coeffs(inp, scale=1.0):
 
 
 def _run(inp, a, image_blocks=None, **kw):
-    """image_blocks: size the workspace to hold that many token blocks of the
-    logit-gradient image (0 = none, recomputing dW pass); None = the default
-    pair_grad_workspace_size."""
+    """image_blocks: size the workspace to hold that many token blocks of
+    kept logits and logit-gradient image (0 = none: the recomputing
+    backward); None = the default pair_grad_workspace_size."""
     B = _binding()
     t = head_inputs(inp, a)
     if image_blocks is not None:
@@ -43,7 +43,7 @@ def _run(inp, a, image_blocks=None, **kw):
         V, R = t["W"].shape[0], inp["R"]
         dt = B.PAIR_BF16 if t["H"].dtype == torch.bfloat16 else B.PAIR_F32
         nbytes = (B.pair_grad_workspace_min_size(T, d, V, R, dt)
-                  + image_blocks * ((V + 127) // 128) * 32768)
+                  + image_blocks * ((V + 127) // 128) * (65536 + 32768))
         assert nbytes <= B.pair_grad_workspace_size(T, d, V, R, dt)
         kw["ws"] = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
     err = dev_err_word()
