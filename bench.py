@@ -50,7 +50,7 @@ TC_KERNELS = ("lse_tc", "bwd_dh_tc", "bwd_dw_tc", "dh_gemm_tc", "dw_gemm_tc")
 def parse_args():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--steps", type=int, default=80)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     p.add_argument("--seed", type=int, default=0)
@@ -60,6 +60,12 @@ def parse_args():
     p.add_argument("--workload", default=WORKLOAD,
                    choices=["qwen3_1p7b_head", "qwen3_4b_head", "longctx_skew"])
     p.add_argument("--len-scale", type=float, default=1.0)
+    p.add_argument("--vocab", type=int, default=0,
+                   help="override the head's vocabulary size (0 = the workload's)")
+    p.add_argument("--ws-exact", action="store_true",
+                   help="size the pair_grad workspace for the active tokens (kept logits "
+                        "and logit-gradient image for ceil(T_eff/128) token blocks) instead "
+                        "of pair_grad_workspace_size, which sizes it for the packed length")
     return p.parse_args()
 
 
@@ -265,7 +271,8 @@ def main():
     peaks = load_peaks()
     traffic = load_traffic()
     wl = synth.WORKLOADS[args.workload]
-    inp = synth.make_head_workload(wl, args.seed + rank, len_scale=args.len_scale)
+    kw = {"V": args.vocab} if args.vocab else {}
+    inp = synth.make_head_workload(wl, args.seed + rank, len_scale=args.len_scale, **kw)
     T, d, V, R = inp["T"], inp["d"], inp["V"], inp["R"]
 
     def pinned(x):
@@ -289,9 +296,19 @@ def main():
     dW = torch.empty((V, d), dtype=torch.float32, device="cuda")
     Jobj = torch.empty(1, dtype=torch.float64, device="cuda")
     lps = torch.empty(R, dtype=torch.float32, device="cuda")
-    ws = torch.empty(B.pair_grad_workspace_size(T, d, V, R, B.PAIR_BF16),
-                     dtype=torch.uint8, device="cuda")
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    if args.ws_exact:
+        # The coefficients fix which rollouts are active; kept logits and
+        # image for exactly their token blocks (96 KB per 128 x 128 tile).
+        B.pair_coeffs(devb["r"], devb["J"], devb["rho"], a=a, active=active, edges=edges,
+                      contrast_edges=contrast, dev_err=err)
+        blocks = (count_active_tokens(inp, a.view(-1).cpu().numpy()) + 127) // 128
+        ws_bytes = min(B.pair_grad_workspace_min_size(T, d, V, R, B.PAIR_BF16)
+                       + blocks * ((V + 127) // 128) * (65536 + 32768),
+                       B.pair_grad_workspace_size(T, d, V, R, B.PAIR_BF16))
+    else:
+        ws_bytes = B.pair_grad_workspace_size(T, d, V, R, B.PAIR_BF16)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     launches = [0]
 
