@@ -298,13 +298,15 @@ def main():
     lps = torch.empty(R, dtype=torch.float32, device="cuda")
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
     if args.ws_exact:
-        # The coefficients fix which rollouts are active; kept logits and
-        # image for exactly their token blocks (96 KB per 128 x 128 tile).
+        # The coefficients fix which rollouts are active; kept logit terms and
+        # image for exactly their token blocks (one block's bytes: the size
+        # difference at T = 128).
         B.pair_coeffs(devb["r"], devb["J"], devb["rho"], a=a, active=active, edges=edges,
                       contrast_edges=contrast, dev_err=err)
         blocks = (count_active_tokens(inp, a.view(-1).cpu().numpy()) + 127) // 128
-        ws_bytes = min(B.pair_grad_workspace_min_size(T, d, V, R, B.PAIR_BF16)
-                       + blocks * ((V + 127) // 128) * (65536 + 32768),
+        block = (B.pair_grad_workspace_size(128, d, V, R, B.PAIR_BF16)
+                 - B.pair_grad_workspace_min_size(128, d, V, R, B.PAIR_BF16))
+        ws_bytes = min(B.pair_grad_workspace_min_size(T, d, V, R, B.PAIR_BF16) + blocks * block,
                        B.pair_grad_workspace_size(T, d, V, R, B.PAIR_BF16))
     else:
         ws_bytes = B.pair_grad_workspace_size(T, d, V, R, B.PAIR_BF16)

@@ -71,7 +71,8 @@ struct GradWorkspace {
   void *gring;         // per-cluster ring of published Gs tiles
   float *tailbuf;      // [kMaxClusters][2][128][d] partial tail units (cluster path)
   void *gimg;          // bf16 logit-gradient tiles of gimg_rb token blocks, or null
-  float *sbuf;         // fp32 logit tiles of the same blocks (kept by the LSE pass)
+  void *sbuf;          // fp16 chunk-relative logit terms of the same blocks (LSE pass)
+  float4 *mbuf;        // fp32 maxima of their 32-column chunks, one float4 per tile row
   int gimg_rb;         // token blocks (128 rows) per backward chunk; 0 = no image
   int64_t Tpad;
   int nsplit;

@@ -398,7 +398,8 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   // The image comes last, so that a larger workspace only adds token blocks.
   const size_t n_vt = (size_t)((V + 127) / 128);
   const size_t o_gimg = gimg_rb ? take((size_t)gimg_rb * n_vt * kGImgTileBytes) : off;
-  const size_t o_sbuf = gimg_rb ? take((size_t)gimg_rb * n_vt * 128 * 128 * sizeof(float)) : off;
+  const size_t o_sbuf = gimg_rb ? take((size_t)gimg_rb * n_vt * 128 * 128 * 2) : off;
+  const size_t o_mbuf = gimg_rb ? take((size_t)gimg_rb * n_vt * 128 * 16) : off;
   if (out) {
     char *b = static_cast<char *>(base);
     out->counters = reinterpret_cast<int32_t *>(b + o_cnt);
@@ -417,7 +418,8 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->gring = b + o_ring;
     out->tailbuf = cl ? reinterpret_cast<float *>(b + o_tail) : nullptr;
     out->gimg = gimg_rb ? b + o_gimg : nullptr;
-    out->sbuf = gimg_rb ? reinterpret_cast<float *>(b + o_sbuf) : nullptr;
+    out->sbuf = gimg_rb ? b + o_sbuf : nullptr;
+    out->mbuf = gimg_rb ? reinterpret_cast<float4 *>(b + o_mbuf) : nullptr;
     out->gimg_rb = gimg_rb;
     out->Tpad = Tpad;
     out->nsplit = kNSplit;

@@ -27,6 +27,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include "pair_common.cuh"
 #include "tc_ptx.cuh"
@@ -80,17 +81,20 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
                const __grid_constant__ CUtensorMap tmS, int d, int V,
                int nsplit, int64_t Tpad, const int32_t *counters,
                const int32_t *tok_y, float2 *part, float *zy, int rb0, int cap,
-               float *sbuf, int s_blocks, int32_t *dev_err) {
+               const void *sbuf, float4 *mbuf, int s_blocks, int32_t *dev_err) {
   extern __shared__ uint8_t smem_raw[];
   LseSmem &sm = *reinterpret_cast<LseSmem *>(align1k(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int Teff = counters[0];
-  // Token blocks [rb0, rb0 + n_tb) of this launch; with sbuf, the fp32
-  // logits of its first s_blocks blocks are also stored (128 x 128 tiles,
-  // tile (b, vt) at ((b * n_vt128 + vt) * 128 + row) * 128 + col) through
-  // tmS, a [rows][128] fp32 view of sbuf: each epilogue warp stages its 32
-  // rows of a 32-column chunk in shared memory and writes them with one TMA
-  // store (full 128-byte lines).
+  // Token blocks [rb0, rb0 + n_tb) of this launch. With sbuf, the logits of
+  // its first s_blocks blocks are also kept, per 32-column chunk c of a row
+  // as P_j = 2^(z_j log2 e - m_c) in fp16 (in [0, 1]) with the chunk maximum
+  // m_c = max_j z_j log2 e in fp32: 128 x 128 tiles, tile (b, vt) at
+  // ((b * n_vt128 + vt) * 128 + row) * 128 + col of sbuf (written through
+  // tmS, a [rows][128] fp16 view: each epilogue warp stages its 32 rows of
+  // two chunks in shared memory and writes them with one TMA store), and
+  // the row's four maxima as one float4 at mbuf[(b * n_vt128 + vt) * 128 +
+  // row]. The same per-chunk terms P_j make up the log-sum-exp sum.
   const int n_tb = min(max((Teff + 127) / 128 - rb0, 0), cap);
   const int n_vt128 = (V + 127) / 128;
   const int s_lim = min(n_tb, s_blocks);
@@ -221,6 +225,7 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
       const int p = tb * 128 + row;
       const bool valid = p < Teff;
       const bool keep = sbuf && tbl < s_lim;  // uniform over the CTA
+      float mrow[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
       const int yt = valid ? tok_y[p] : -1;
       float m2 = -INFINITY, l = 0.f, zt = 0.f;
       bool found = false;
@@ -232,26 +237,6 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
           float v[32];
           tmem_ld32(lane_addr + acc * kLseBN + c * 32, v);
           const int col0 = vt * kLseBN + c * 32;
-          if (keep && col0 < V) {
-            // Per warp: its 32 rows x 32 columns, staged in its own buffer
-            // and stored by its lane 0. The store that last read this
-            // buffer (two chunks back) is done first.
-            if (lane == 0) bulk_wait_group_read<1>();
-            __syncwarp();
-            uint8_t *buf = sm.stg[sbuf_i] + quad * 4096;
-#pragma unroll
-            for (int e = 0; e < 8; ++e)
-              *reinterpret_cast<float4 *>(buf + lane * 128 + ((e ^ (lane & 7)) << 4)) =
-                  make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
-            fence_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-              tma_store_2d_evict_first(&tmS, buf, col0 & 127,
-                                       (tbl * n_vt128 + (col0 >> 7)) * 128 + quad * 32);
-              bulk_commit_group();
-            }
-            sbuf_i ^= 1;
-          }
           const int off = yt - col0;
           if (off >= 0 && off < 32) {
             found = true;
@@ -266,15 +251,61 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
             v[j] = (j < nvalid) ? v[j] * kLog2e : -INFINITY;
             mc = fmaxf(mc, v[j]);
           }
-          if (mc == -INFINITY) continue;
-          if (mc > m2) {
-            l *= ex2_approx(m2 - mc);
-            m2 = mc;
-          }
+          if (mc == -INFINITY) continue;  // the whole chunk lies past V
+          // Chunk terms relative to the chunk maximum, then folded into the
+          // running (max, sum): v[j] becomes P_j.
           float s = 0.f;
 #pragma unroll
-          for (int j = 0; j < 32; ++j) s += ex2_approx(v[j] - m2);
-          l += s;
+          for (int j = 0; j < 32; ++j) {
+            v[j] = ex2_approx(v[j] - mc);
+            s += v[j];
+          }
+          if (mc > m2) {
+            l = l * ex2_approx(m2 - mc) + s;
+            m2 = mc;
+          } else {
+            l += s * ex2_approx(mc - m2);
+          }
+          if (keep) {
+            // Per warp: its 32 rows x 64 columns (two chunks) in fp16, in its
+            // own 4 KB buffer, stored by its lane 0 once both halves (or the
+            // last chunk before V) are in. The store that last read this
+            // buffer is done before the first half is written.
+            const int half = c & 1;
+            if (half == 0) {
+              if (lane == 0) bulk_wait_group_read<1>();
+              __syncwarp();
+            }
+            uint8_t *buf = sm.stg[sbuf_i] + quad * 4096;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              uint32_t pk[4];
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                __half2 h2 = __floats2half2_rn(v[8 * e + 2 * q], v[8 * e + 2 * q + 1]);
+                pk[q] = *reinterpret_cast<uint32_t *>(&h2);
+              }
+              *reinterpret_cast<uint4 *>(buf + lane * 128 + (((half * 4 + e) ^ (lane & 7)) << 4)) =
+                  make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            }
+            mrow[c & 3] = mc;
+            const bool last = col0 + 32 >= V;
+            if (half == 1 || last) {
+              fence_async_smem();
+              __syncwarp();
+              if (lane == 0) {
+                tma_store_2d_evict_first(&tmS, buf, col0 & 64,
+                                         (tbl * n_vt128 + (col0 >> 7)) * 128 + quad * 32);
+                bulk_commit_group();
+              }
+              sbuf_i ^= 1;
+            }
+            if ((c & 3) == 3 || last) {
+              mbuf[((int64_t)tbl * n_vt128 + (col0 >> 7)) * 128 + row] =
+                  make_float4(mrow[0], mrow[1], mrow[2], mrow[3]);
+              mrow[0] = mrow[1] = mrow[2] = mrow[3] = -INFINITY;
+            }
+          }
         }
         tc_fence_before();
         mbar_arrive(&sm.acc_empty[acc]);
@@ -1264,43 +1295,61 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
 // ------------------------------------------ logit-gradient image from S
 //
 // Gs_tv = -c_t exp(z_tv - lse_t) in bf16 for every tile of a chunk of token
-// blocks, from the fp32 logit tiles the LSE pass kept: one 32 KB image tile
-// per 128 tokens x 128 vocabulary rows, two K-major SWIZZLE_128B atoms of 64
-// vocabulary columns (the layout both backward GEMMs read). Columns >= V,
-// rows >= T_eff and tokens with c_t = 0 give exact zeros. Streaming kernel:
-// 64 KB read and 32 KB written per tile.
+// blocks, from the chunk-relative terms the LSE pass kept (fp16 P_v =
+// 2^(z_v log2 e - m) and the fp32 chunk maximum m, per 32 columns):
+// Gs = -c_t 2^(m - lse_t log2 e) P_v, one exponential per 8 columns. One
+// 32 KB image tile per 128 tokens x 128 vocabulary rows, two K-major
+// SWIZZLE_128B atoms of 64 vocabulary columns (the layout both backward
+// GEMMs read). Columns >= V, rows >= T_eff and tokens with c_t = 0 give
+// exact zeros. Streaming kernel: 34 KB read and 32 KB written per tile.
 __global__ void __launch_bounds__(256) g_image_kernel(int V, int rb0, int cap,
                                                       const int32_t *counters,
-                                                      const float *tok_c, const float *lse,
-                                                      const float *sbuf, uint8_t *gimg) {
+                                                      const float *__restrict__ tok_c,
+                                                      const float *__restrict__ lse,
+                                                      const __half *__restrict__ sbuf,
+                                                      const float4 *__restrict__ mbuf,
+                                                      uint8_t *__restrict__ gimg) {
   const int Teff = counters[0];
   const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
   const int n_vt = (V + 127) / 128;
   const int64_t n_tiles = (int64_t)nrb * n_vt;
+  // Thread t of the block handles 8-column chunk (t & 15) of rows
+  // (t >> 4) + 16 k, k < 8; all eight loads are issued before any use.
+  const int ch = threadIdx.x & 15, r0 = threadIdx.x >> 4;
   for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
     const int b = (int)(tile / n_vt), vt = (int)(tile - (int64_t)b * n_vt);
-    const float *src = sbuf + tile * (128 * 128);
+    const __half *src = sbuf + tile * (128 * 128);
+    const float4 *mt = mbuf + tile * 128;
     uint8_t *dst = gimg + tile * kGImgTileBytes;
-    for (int i = threadIdx.x; i < 128 * 16; i += blockDim.x) {
-      const int row = i >> 4, ch = i & 15;  // 8-column chunk ch of the row
+    const int col0 = vt * 128 + ch * 8;
+    uint4 h[8];
+    float4 m4[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int row = r0 + 16 * k;
+      h[k] = *reinterpret_cast<const uint4 *>(src + row * 128 + ch * 8);
+      m4[k] = mt[row];
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int row = r0 + 16 * k;
       const int p = (rb0 + b) * 128 + row;
-      const float cc = p < Teff ? tok_c[p] : 0.f;
-      const float ll = p < Teff ? lse[p] * kLog2e : 0.f;
-      const float4 s0 = reinterpret_cast<const float4 *>(src + row * 128 + ch * 8)[0];
-      const float4 s1 = reinterpret_cast<const float4 *>(src + row * 128 + ch * 8)[1];
-      const float v[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-      const int col0 = vt * 128 + ch * 8;
+      float sc = 0.f;
+      if (p < Teff && col0 < V) {
+        const float cc = tok_c[p];
+        const int q = ch >> 2;
+        const float m = q == 0 ? m4[k].x : q == 1 ? m4[k].y : q == 2 ? m4[k].z : m4[k].w;
+        if (cc != 0.f) sc = -cc * ex2_approx(m - lse[p] * kLog2e);
+      }
+      const uint32_t hw[4] = {h[k].x, h[k].y, h[k].z, h[k].w};
       uint32_t pk[4];
 #pragma unroll
-      for (int j = 0; j < 8; j += 2) {
-        float g2[2];
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const bool live = cc != 0.f && col0 + j + e < V;
-          g2[e] = live ? -cc * ex2_approx(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
-        }
-        __nv_bfloat162 b2 = __floats2bfloat162_rn(g2[0], g2[1]);
-        pk[j >> 1] = *reinterpret_cast<uint32_t *>(&b2);
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&hw[e]));
+        const float g0 = col0 + 2 * e < V ? sc * f.x : 0.f;
+        const float g1 = col0 + 2 * e + 1 < V ? sc * f.y : 0.f;
+        __nv_bfloat162 b2 = __floats2bfloat162_rn(g0, g1);
+        pk[e] = *reinterpret_cast<uint32_t *>(&b2);
       }
       *reinterpret_cast<uint4 *>(dst + (ch >> 3) * kAtom128 + sw128_offset(row, (ch & 7) * 8)) =
           make_uint4(pk[0], pk[1], pk[2], pk[3]);
@@ -1732,16 +1781,17 @@ bool make_map3(CUtensorMap *m, const void *ptr, const cuuint64_t (&dims)[3],
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// fp32 [rows][128] map with 32-column x 32-row SWIZZLE_128B boxes (the
-// kept-logit tiles, stored by the LSE pass one warp's rows at a time).
+// fp16 [rows][128] map with 64-column x 32-row SWIZZLE_128B boxes (the
+// kept chunk-relative terms, stored by the LSE pass one warp's rows at a
+// time).
 bool make_map_s(CUtensorMap *m, const void *ptr, int64_t rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {128, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {128 * sizeof(float)};
-  cuuint32_t box[2] = {32, 32};
+  cuuint64_t strides[1] = {128 * 2};
+  cuuint32_t box[2] = {64, 32};
   cuuint32_t estr[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void *>(ptr), dims, strides, box,
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(ptr), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -1860,10 +1910,11 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
 constexpr int kAllBlocks = 0x7fffffff;
 
 // Log-sum-exp pass over token blocks [rb0, rb0 + cap) (clipped to the active
-// ones), then lse for those tokens. With sbuf, the fp32 logit tiles of the
-// first s_blocks of those blocks are kept.
+// ones), then lse for those tokens. With keep, the chunk-relative logit terms
+// of the first s_blocks of those blocks are kept in w.sbuf / w.mbuf.
 pair_status launch_lse(const GradArgs &g, const GradWorkspace &w, cudaStream_t s, int rb0,
-                       int cap, float *sbuf, int s_blocks) {
+                       int cap, bool keep, int s_blocks) {
+  void *sbuf = keep ? w.sbuf : nullptr;
   CUtensorMap mH, mW128, mS = {};
   if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) || !make_map(&mW128, g.W, g.V, g.d, 128))
     return PAIR_ERR_CUDA;
@@ -1876,7 +1927,7 @@ pair_status launch_lse(const GradArgs &g, const GradWorkspace &w, cudaStream_t s
   PAIR_BEGIN("lse_tc", s);
   lse_kernel<<<lse_grid(lse_smem), kThreads, lse_smem, s>>>(
       mH, mW128, mS, g.d, g.V, w.nsplit, w.Tpad, w.counters, w.tok_y, w.part, w.zy, rb0, cap, sbuf,
-      s_blocks, g.dev_err);
+      keep ? w.mbuf : nullptr, s_blocks, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("lse_combine", s);
   lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters, w.part, w.lse, rb0,
@@ -1920,8 +1971,8 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
   static int dh_cache = 0, dw_cache = 0;
   uint8_t *gimg = static_cast<uint8_t *>(w.gimg);
   PAIR_BEGIN("g_image", s);
-  g_image_kernel<<<num_sms() * 4, 256, 0, s>>>(g.V, rb0, cap, w.counters, w.tok_c, w.lse, w.sbuf,
-                                               gimg);
+  g_image_kernel<<<num_sms() * 3, 256, 0, s>>>(g.V, rb0, cap, w.counters, w.tok_c, w.lse,
+                                               static_cast<const __half *>(w.sbuf), w.mbuf, gimg);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("dh_gemm_tc", s);
   dh_gemm_kernel<<<pair_grid((const void *)dh_gemm_kernel, dh_smem, &dh_cache), kThreads,
@@ -1941,8 +1992,8 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
 // Forward half: per-token log-sum-exp and target logit over every active
 // token (with an image, the first chunk's logits are kept for the backward).
 pair_status grad_lse_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
-  if (image_path(w)) return launch_lse(g, w, s, 0, kAllBlocks, w.sbuf, w.gimg_rb);
-  return launch_lse(g, w, s, 0, kAllBlocks, nullptr, 0);
+  if (image_path(w)) return launch_lse(g, w, s, 0, kAllBlocks, true, w.gimg_rb);
+  return launch_lse(g, w, s, 0, kAllBlocks, false, 0);
 }
 
 // Backward half: softmax parts of dH and dW from the token coefficients,
@@ -1952,7 +2003,7 @@ pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t 
     const int64_t nc = image_chunks(g, w);
     for (int64_t c = 0; c < nc; ++c) {
       if (c > 0) {
-        const pair_status st = launch_lse(g, w, s, (int)(c * w.gimg_rb), w.gimg_rb, w.sbuf,
+        const pair_status st = launch_lse(g, w, s, (int)(c * w.gimg_rb), w.gimg_rb, true,
                                           w.gimg_rb);
         if (st != PAIR_OK) return st;
       }
@@ -1988,10 +2039,11 @@ pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t 
   return PAIR_OK;
 }
 
-// Memory the backward may use for kept fp32 logits and bf16 logit-gradient
-// tiles (96 KB per 128 x 128 tile); larger problems run in token chunks.
+// Memory the backward may use for kept logit terms (fp16 terms and fp32
+// chunk maxima) and bf16 logit-gradient tiles, 66 KB per 128 x 128 tile;
+// larger problems run in token chunks.
 constexpr int64_t kImageBudget = int64_t(24) << 30;
-constexpr size_t kImageTileBytes = kGImgTileBytes + 128 * 128 * sizeof(float);
+constexpr size_t kImageTileBytes = kGImgTileBytes + 128 * 128 * 2 + 128 * 16;
 
 int grad_gimg_rows(int64_t T, int32_t d, int32_t V, pair_dtype dt) {
   if (dt != PAIR_BF16 || d < 512 || d % kDwN != 0) return 0;
@@ -2013,7 +2065,7 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t
   if (image_path(w)) {
     const int64_t nc = image_chunks(g, w);
     for (int64_t c = 0; c < nc; ++c) {
-      pair_status st = launch_lse(g, w, s, (int)(c * w.gimg_rb), w.gimg_rb, w.sbuf, w.gimg_rb);
+      pair_status st = launch_lse(g, w, s, (int)(c * w.gimg_rb), w.gimg_rb, true, w.gimg_rb);
       if (st == PAIR_OK) st = launch_chunk_bwd(g, w, s, c);
       if (st != PAIR_OK) return st;
     }

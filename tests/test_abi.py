@@ -47,13 +47,14 @@ def test_workspace_size_rules(L):
     fixed = (12 << 20) + 24 * 2 * 128 * 2048 * 4 + (1 << 20)
     assert (wmin(100000, 2048, 151936, 64, L.PAIR_F32)
             - wmin(100000, 2048, 151936, 64, L.PAIR_BF16) > 100000 * 2048 * 2 - fixed)
-    # For d a multiple of 512, bf16 also keeps the fp32 logits and the bf16
-    # logit-gradient image of min(ceil(T/128), max(32, 24 GiB // per_block))
-    # token blocks, per_block = ceil(V/128) tiles of 64 + 32 KB; other widths
-    # and fp32 keep none.
+    # For d a multiple of 512, bf16 also keeps the logit terms (fp16 per
+    # element, an fp32 maximum per 32 columns) and the bf16 logit-gradient
+    # image of min(ceil(T/128), max(32, 24 GiB // per_block)) token blocks,
+    # per_block = ceil(V/128) tiles of 32 + 2 + 32 KB; other widths and fp32
+    # keep none.
     for T, d, V in [(100000, 2048, 151936), (1000, 512, 1000), (10 ** 6, 1024, 10 ** 6),
                     (5000, 1536, 300), (70000, 2560, 151936), (3000, 3072, 4099)]:
-        per_block = (V + 127) // 128 * (65536 + 32768)
+        per_block = (V + 127) // 128 * (32768 + 2048 + 32768)
         blocks = min((T + 127) // 128, max(32, (24 << 30) // per_block))
         assert ws(T, d, V, 64, L.PAIR_BF16) - wmin(T, d, V, 64, L.PAIR_BF16) == blocks * per_block
     for d, dt in [(640, L.PAIR_BF16), (256, L.PAIR_BF16), (2048, L.PAIR_F32)]:

@@ -42,8 +42,10 @@ def _run(inp, a, image_blocks=None, **kw):
         T, d = t["H"].shape
         V, R = t["W"].shape[0], inp["R"]
         dt = B.PAIR_BF16 if t["H"].dtype == torch.bfloat16 else B.PAIR_F32
-        nbytes = (B.pair_grad_workspace_min_size(T, d, V, R, dt)
-                  + image_blocks * ((V + 127) // 128) * (65536 + 32768))
+        # One token block's kept terms and image: the size difference at T = 128.
+        block = (B.pair_grad_workspace_size(128, d, V, R, dt)
+                 - B.pair_grad_workspace_min_size(128, d, V, R, dt))
+        nbytes = B.pair_grad_workspace_min_size(T, d, V, R, dt) + image_blocks * block
         assert nbytes <= B.pair_grad_workspace_size(T, d, V, R, dt)
         kw["ws"] = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
     err = dev_err_word()
