@@ -79,10 +79,23 @@ def load_peaks():
         return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
 
 
-def load_traffic():
-    """Per-launch DRAM bytes from the committed ncu summary, keyed by kernel,
-    valid only while the kernel source is unchanged (hash recorded there)."""
+def code_hash(path):
+    """sha256[:16] of a source file's code: every line with its // comment
+    removed and trailing space stripped, blank lines dropped (comment edits
+    leave it unchanged, any code change alters it)."""
     import hashlib
+    lines = []
+    for line in open(path, encoding="utf-8"):
+        code = line.split("//", 1)[0].rstrip()
+        if code:
+            lines.append(code)
+    return hashlib.sha256("\n".join(lines).encode()).hexdigest()[:16]
+
+
+def load_traffic():
+    """Per-call DRAM bytes from the committed ncu summary, keyed by kernel,
+    valid only while the kernel source code is unchanged (hash recorded
+    there, see code_hash)."""
     path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
     out = {}
     if not os.path.exists(path):
@@ -93,7 +106,7 @@ def load_traffic():
             continue
         name, wl, bytes_, src, sha = parts[:5]
         try:
-            cur = hashlib.sha256(open(os.path.join(ROOT, src), "rb").read()).hexdigest()[:16]
+            cur = code_hash(os.path.join(ROOT, src))
         except OSError:
             continue
         if cur == sha:

@@ -283,8 +283,10 @@ PAIR_API size_t pair_grad_workspace_min_size(int64_t T, int32_t d, int32_t V, in
  * The sequence score of Sec. 3.1 is the per-rollout sum over tokens (no
  * length normalisation). Rollouts with a_i == 0 (+0 or -0) are skipped
  * entirely; their tokens' dH rows, like those of mask = 0 tokens, are
- * written as exact zeros. Logits never leave the chip (vocabulary-tiled
- * on-chip softmax).
+ * written as exact zeros. No logit-sized tensor is written in fp32: the
+ * log-sum-exp pass keeps the logits as fp16 terms relative to each
+ * 32-column chunk maximum, from which the bf16 logit gradient is formed
+ * once and read by the dH and dW GEMMs (see pair_grad_workspace_size).
  *
  * In:  T >= 1 packed tokens; d hidden size; V vocabulary size; dt dtype of
  *      H and W (PAIR_BF16: fp32 accumulation on the tensor cores, requires

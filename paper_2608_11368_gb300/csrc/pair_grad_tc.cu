@@ -4,26 +4,28 @@
 // Objective (Sec. 4.5): J = sum_t c_t logp_t over compacted active tokens,
 // logp_t = z_{t,y_t} - lse_t, z = W h. Its gradients split into an exact
 // one-hot part (added in fp32 by grad_onehot) and a softmax part that is a
-// pair of dense contractions through the logit-gradient tile
-//     Gs_tv = -c_t exp(z_tv - lse_t)      (bf16 on chip, never in HBM):
+// pair of dense contractions through the logit gradient
+//     Gs_tv = -c_t exp(z_tv - lse_t)      (bf16):
 //     dH_t += sum_v Gs_tv W_v,     dW_v += sum_t Gs_tv h_t.
 //
-// Kernels (all persistent, one 192-thread CTA per SM, warp-specialised:
-// warp 0 = TMA producer, warp 1 = TMEM owner + single-thread MMA issuer,
-// warps 2..5 = epilogue, one TMEM lane / tile row per thread):
-//   lse_kernel  : 128-token x 256-vocab tiles, K = d streamed in 64-wide
-//                 SWIZZLE_128B atoms; fp32 accumulators double-buffered in
-//                 TMEM (2 x 256 columns); the epilogue folds each tile into
-//                 an online (max, sum-exp) per token and picks the target
-//                 logit. Work unit = (token block, vocabulary split).
-//   bwd_kernel  : rows x 128-column S tiles recomputed from the operands,
-//                 Gs formed in registers and written to shared memory as a
-//                 K-major SWIZZLE_128B bf16 tile, then a second MMA
-//                 out[rows, slice] += Gs . C[cols, slice] with the column
-//                 operand's d-slice read MN-major. Token rows give dH,
-//                 vocabulary rows give dW. The output slice (<= 256 fp32
-//                 columns) stays in TMEM for the whole unit, beside the two
-//                 128-column S buffers.
+// Kernels (persistent, warp-specialised: a TMA producer warp, a TMEM-owning
+// warp whose elected thread issues the MMAs, four epilogue warps on the four
+// TMEM lane quadrants, one tile row per thread):
+//   lse_kernel     : 128-token x 256-vocab tiles, K = d in 64-wide
+//                    SWIZZLE_128B atoms, fp32 accumulators double-buffered in
+//                    TMEM; the epilogue folds each 32-column chunk into an
+//                    online (max, sum-exp) per token, picks the target logit
+//                    and keeps the chunk's terms 2^(z log2 e - m_c) in fp16
+//                    with m_c for the backward.
+//   g_image_kernel : the bf16 Gs tiles (the logit-gradient image) from the
+//                    kept terms, once, in the swizzled MMA-operand layout.
+//   dh_gemm_kernel : dH = Gs . W, image tiles as the K-major A operand.
+//   dw_gemm_kernel : dW = Gs^T . Hc, the same tiles read as the MN-major A
+//                    operand.
+// Without room for the image (no-alloc path, minimum workspace) the logits
+// are recomputed: bwd_cluster_kernel (8-CTA clusters sharing each Gs tile
+// through an L2 ring) for d = 512 A, else bwd_kernel (one CTA per row
+// block and 256-wide d-slice).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -50,7 +52,7 @@ constexpr uint32_t kIdescLse = idesc_bf16(128, kLseBN, 0, 0);
 struct LseSmem {
   uint8_t a[kLseStages][kAtom128];
   uint8_t b[kLseStages][2 * kAtom128];
-  uint8_t stg[2][128 * 128];  // kept-logit staging: per warp 32 rows x 32 fp32, SWIZZLE_128B
+  uint8_t stg[2][128 * 128];  // kept-term staging: per warp 32 rows x 64 fp16, SWIZZLE_128B
   uint64_t full[kLseStages], empty[kLseStages];
   uint64_t acc_full[2], acc_empty[2];
   uint64_t mma_done;
