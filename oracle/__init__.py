@@ -19,6 +19,10 @@ Contents, each following the paper's definitions literally:
   target gather, and the exact gradients of the objective w.r.t. the hidden
   states and the head weight, in fp64 numpy (matmul as a library step).
 
+* ``allocation`` (submodule): the contrast graph, the shared-vertex
+  surrogate and the convex continuation design of Sec. 4.3-4.4, solved with
+  SLSQP in fp64 and certified by its KKT conditions.
+
 Parity status: the coefficient, dense and head functions are pinned by the
 paper's identities (Thm. 1, Thm. 2, Prop. bias/covariance, the edge-sum /
 coefficient-collapse identity) and by library/brute-force checks in
