@@ -524,6 +524,23 @@ def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
     Ma = Ga * (Ga - 1) // 2
     t_a = timed(lambda: B.pair_audit(ra, rhoa, Sa, Jda, scale=1.0 / Ma, stats=st_a, bias=bias_a,
                                      ws=ws_a), max(5, min(reps, 10)))
+    # Allocation step (Sec. 4.3-4.4): the paper's group size (G = 16) for 64
+    # prompts of one RL step, and the 4096 x 64 stress size. Latency bound
+    # (a fixed number of small fp64 Newton systems per group).
+    alloc = {}
+    for nb, ga in ((64, 16), (4096, 64)):
+        ai = synth.make_alloc_inputs(77 + rank, nb, ga)
+        c_al, b_al, p_al = dv(ai["c_hat"]), dv(ai["budget"]), dv(ai["p_hat"])
+        pi_al = torch.empty((nb, ga), dtype=torch.float32, device="cuda")
+        st_al = torch.empty((nb, 5), dtype=torch.float64, device="cuda")
+        t_al = timed(lambda: B.pair_allocate(c_al, b_al, float(ai["pi_min"]), p_hat=p_al,
+                                             pi=pi_al, stats=st_al), 3)
+        s_al = st_al.cpu().numpy()
+        alloc["%dx%d" % (nb, ga)] = {
+            "ms": t_al, "groups_per_s": nb / (t_al / 1e3),
+            "newton_mean": float(s_al[:, 3].mean()), "newton_max": int(s_al[:, 3].max()),
+            "solved": int((s_al[:, 4] == 0).sum()),
+            "bound": "latency (fp64 log-barrier Newton, one CTA per group)"}
     bytes_p = Bn * (4 * G + G + 4 * G + 4 * G + G + 16)
     bytes_d = 4 * D * n_act + Bn * (4 * G * (G - 1) // 2 + 4 * G + G) + 4 * Bn * D + 4 * Bn * G
     gbs_c = bytes_c / (t_c / 1e3) / 1e9
@@ -543,6 +560,7 @@ def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
                        "draws_per_s": Na / (t_a / 1e3),
                        "stats": dict(zip(B.AUDIT_STATS, st_a.cpu().tolist())),
                        "bound": "latency (per-draw coefficient collapse and quadratic forms)"},
+        "pair_allocate": alloc,
         "pair_coeffs_product": {"bound": "hbm", "achieved": bytes_p / (t_p / 1e3) / 1e9,
                                 "peak": peaks["hbm"], "unit": "GB/s",
                                 "frac": bytes_p / (t_p / 1e3) / 1e9 / peaks["hbm"],

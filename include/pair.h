@@ -63,8 +63,10 @@ typedef enum {
   PAIR_ERR_NONPOSITIVE_INCLUSION = 4, /* rho_ij <= 0 or NaN, completed edge */
   PAIR_ERR_TARGET_RANGE = 5,          /* y_t outside [0, V) at a mask=1 token */
   PAIR_ERR_CUDA = 6,                  /* a CUDA runtime call failed         */
-  PAIR_ERR_DEVICE_TIMEOUT = 7         /* a bounded on-device wait gave up;
+  PAIR_ERR_DEVICE_TIMEOUT = 7,        /* a bounded on-device wait gave up;
                                          outputs of that call are invalid  */
+  PAIR_ERR_ALLOC_INPUT = 8,           /* pair_allocate: invalid input value */
+  PAIR_ERR_ALLOC_INFEASIBLE = 9       /* pair_allocate: budget < pi_min sum c */
 } pair_status;
 
 typedef enum { PAIR_F32 = 0, PAIR_BF16 = 1 } pair_dtype;
@@ -73,6 +75,8 @@ typedef enum { PAIR_F32 = 0, PAIR_BF16 = 1 } pair_dtype;
 #define PAIR_DEV_ERR_NONPOSITIVE_INCLUSION 1
 #define PAIR_DEV_ERR_TARGET_RANGE 2
 #define PAIR_DEV_ERR_TIMEOUT 4 /* a pipeline wait exceeded its limit (~2 s) */
+#define PAIR_DEV_ERR_ALLOC_INPUT 8       /* pair_allocate: invalid input value */
+#define PAIR_DEV_ERR_ALLOC_INFEASIBLE 16 /* pair_allocate: budget < pi_min sum c */
 
 /* pair_coeffs flags. */
 #define PAIR_CENTER 1u /* subtract the mean of a over completed vertices
@@ -244,6 +248,59 @@ PAIR_API pair_status pair_estimate_dense(int32_t B, int32_t G, int32_t D,
                                 const float *rho, const float *S, float scale,
                                 float *g, float *a, int32_t *dev_err,
                                 pair_stream_t stream);
+
+/*
+ * pair_allocate -- the allocation step before the path (Sec. 4.3-4.4): for
+ * each of B groups of G candidates, the contrast graph, the shared-vertex
+ * surrogate and the continuation probabilities pi of the convex program of
+ * Eqs. (convex-objective)-(budget):
+ *     min_x  sum_{i<j} a_ij e^(x_i + x_j) + sum_i b_i e^(x_i)
+ *     s.t.   sum_i c_i e^(-x_i) <= budget,  0 <= x_i <= -log pi_min,
+ * pi_i = e^(-x_i), b_i = (sum_{j != i} sqrt a_ij)^2 - sum_{j != i} a_ij.
+ * The edge proxy a_ij (Eq. edge-proxy) is the explicit a when given, else
+ * the disagreement p_i (1 - p_j) + (1 - p_i) p_j of the predicted success
+ * probabilities (Eq. disagreement), times ((m_i + m_j) / 2)^2 when score-norm
+ * predictions m are given. Solved per group in fp64 to a duality-gap bound
+ * of 1e-12 Phi (log-barrier Newton, one CTA per group); the group's case is
+ * classified first from the fp64 sum of c in index order:
+ *     PAIR_ALLOC_SLACK       budget >= sum c: pi = 1 (x = 0 minimises Phi)
+ *     PAIR_ALLOC_FLOOR       budget == pi_min sum c: pi = pi_min
+ *     PAIR_ALLOC_INFEASIBLE  budget < pi_min sum c: pi = pi_min, and
+ *                            PAIR_DEV_ERR_ALLOC_INFEASIBLE is raised
+ *     PAIR_ALLOC_FLAT        every a_ij and b_i is 0: pi = budget / sum c
+ *     PAIR_ALLOC_OK          solved
+ *     PAIR_ALLOC_FALLBACK    Newton did not converge: pi = budget / sum c
+ *                            (uniform, same expected cost; App. C)
+ *     PAIR_ALLOC_INVALID     a non-finite or out-of-range input: pi = NaN,
+ *                            PAIR_DEV_ERR_ALLOC_INPUT is raised.
+ * In:  B >= 1, 2 <= G <= PAIR_MAX_G; p_hat [B][G] float in [0, 1] (nullable
+ *      when a is given); m_hat [B][G] float >= 0 (nullable); a [B][G][G]
+ *      float >= 0, symmetric, diagonal ignored (nullable); c_hat [B][G]
+ *      float > 0 (predicted suffix costs); budget [B] float > 0 (budget on
+ *      the expected suffix cost); 0 < pi_min <= 1. All device pointers.
+ * Out: pi [B][G] float; stats [B][PAIR_ALLOC_NSTATS] double (nullable):
+ *      [PAIR_ALLOC_PHI] objective at pi, [PAIR_ALLOC_SPENT] sum c pi,
+ *      [PAIR_ALLOC_GAP] duality-gap bound (2G + 1) / t, [PAIR_ALLOC_NEWTON]
+ *      Newton steps, [PAIR_ALLOC_STATUS] the status above.
+ * dev_err required. Deterministic. No workspace, no allocation.
+ */
+#define PAIR_ALLOC_OK 0
+#define PAIR_ALLOC_SLACK 1
+#define PAIR_ALLOC_FLOOR 2
+#define PAIR_ALLOC_INFEASIBLE 3
+#define PAIR_ALLOC_FALLBACK 4
+#define PAIR_ALLOC_FLAT 5
+#define PAIR_ALLOC_INVALID 6
+#define PAIR_ALLOC_PHI 0
+#define PAIR_ALLOC_SPENT 1
+#define PAIR_ALLOC_GAP 2
+#define PAIR_ALLOC_NEWTON 3
+#define PAIR_ALLOC_STATUS 4
+#define PAIR_ALLOC_NSTATS 5
+PAIR_API pair_status pair_allocate(int32_t B, int32_t G, const float *p_hat, const float *m_hat,
+                                   const float *a, const float *c_hat, const float *budget,
+                                   float pi_min, float *pi, double *stats, int32_t *dev_err,
+                                   pair_stream_t stream);
 
 /*
  * pair_grad_workspace_size -- bytes of device workspace pair_grad (and

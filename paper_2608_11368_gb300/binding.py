@@ -86,6 +86,8 @@ def lib() -> ctypes.CDLL:
     L.pair_audit.argtypes = [I32, I32, I32, P, P, P, P, P, F32, U32, ctypes.c_int, F32, P, P,
                              P, SZ, P, P]
     L.pair_audit.restype = ctypes.c_int
+    L.pair_allocate.argtypes = [I32, I32, P, P, P, P, P, F32, P, P, P, P]
+    L.pair_allocate.restype = ctypes.c_int
     L.pair_selftest_wait_timeout.argtypes = [I64, P, P, P]
     L.pair_selftest_wait_timeout.restype = ctypes.c_int
     _lib = L
@@ -239,6 +241,37 @@ def pair_audit(r, rho, S, Jdraws, draw_weight=None, wmode=PAIR_W_HT, w_max=0.0, 
                           _p(bias), _p(ws), ws.numel(), _p(dev_err), _stream(stream))
     _check(st, "pair_audit")
     return stats, bias
+
+
+ALLOC_OK, ALLOC_SLACK, ALLOC_FLOOR, ALLOC_INFEASIBLE, ALLOC_FALLBACK, ALLOC_FLAT, \
+    ALLOC_INVALID = range(7)
+ALLOC_STATS = ("phi", "spent", "gap", "newton", "status")
+
+
+def pair_allocate(c_hat, budget, pi_min, p_hat=None, m_hat=None, a=None, pi=None, stats=None,
+                  dev_err=None, stream=None):
+    """Continuation probabilities of the convex design (see pair.h).
+    c_hat [B, G], budget [B], p_hat [B, G] (or a [B, G, G]), m_hat [B, G] or
+    None. Returns (pi [B, G] f32, stats [B, 5] f64: phi, spent, gap, newton,
+    status)."""
+    B, G = c_hat.shape
+    _need(c_hat, "c_hat", torch.float32, (B, G))
+    _need(budget, "budget", torch.float32, (B,))
+    if p_hat is not None:
+        _need(p_hat, "p_hat", torch.float32, (B, G))
+    if m_hat is not None:
+        _need(m_hat, "m_hat", torch.float32, (B, G))
+    if a is not None:
+        _need(a, "a", torch.float32, (B, G, G))
+    dev = c_hat.device
+    pi = torch.empty((B, G), dtype=torch.float32, device=dev) if pi is None else pi
+    stats = torch.empty((B, 5), dtype=torch.float64, device=dev) if stats is None else stats
+    if dev_err is None:
+        dev_err = torch.zeros(1, dtype=torch.int32, device=dev)
+    st = lib().pair_allocate(B, G, _p(p_hat), _p(m_hat), _p(a), _p(c_hat), _p(budget),
+                             float(pi_min), _p(pi), _p(stats), _p(dev_err), _stream(stream))
+    _check(st, "pair_allocate")
+    return pi, stats
 
 
 def pair_estimate_dense(r, J, rho, S, scale=1.0, g=None, a=None, dev_err=None,

@@ -252,6 +252,8 @@ pair_status pair_status_sync(pair_stream_t stream, int32_t *dev_err) {
   if (h & PAIR_DEV_ERR_TIMEOUT) return PAIR_ERR_DEVICE_TIMEOUT;
   if (h & PAIR_DEV_ERR_NONPOSITIVE_INCLUSION) return PAIR_ERR_NONPOSITIVE_INCLUSION;
   if (h & PAIR_DEV_ERR_TARGET_RANGE) return PAIR_ERR_TARGET_RANGE;
+  if (h & PAIR_DEV_ERR_ALLOC_INPUT) return PAIR_ERR_ALLOC_INPUT;
+  if (h & PAIR_DEV_ERR_ALLOC_INFEASIBLE) return PAIR_ERR_ALLOC_INFEASIBLE;
   return PAIR_OK;
 }
 
@@ -266,6 +268,8 @@ const char *pair_status_string(pair_status st) {
     case PAIR_ERR_TARGET_RANGE: return "target id outside [0, V) at a mask=1 token";
     case PAIR_ERR_CUDA: return "CUDA runtime error";
     case PAIR_ERR_DEVICE_TIMEOUT: return "device pipeline wait timed out";
+    case PAIR_ERR_ALLOC_INPUT: return "allocation input out of range or not finite";
+    case PAIR_ERR_ALLOC_INFEASIBLE: return "allocation budget below pi_min times the summed cost";
   }
   return "unknown status";
 }

@@ -238,3 +238,20 @@ def make_dense_workload(wl: Workload, seed: int, B: Optional[int] = None,
 def as_float(x: np.ndarray, dtype: str) -> np.ndarray:
     """float32 view of stored H or W values (exact upcast for bf16)."""
     return bf16_bits_to_f32(x) if dtype == "bf16" else np.asarray(x, np.float32)
+
+
+def make_alloc_inputs(seed: int, B: int, G: int, budget_frac: float = 0.5,
+                      pi_min: float = 0.08, score_norms: bool = False):
+    """Inputs of the allocation step (Sec. 4.3-4.4) for B groups of G
+    candidates: predicted success probabilities p_hat ~ U(0.02, 0.98),
+    predicted suffix costs c_hat ~ lognormal(ln 1, 0.6) (relative units),
+    optionally score-norm predictions m_hat ~ U(0.3, 3), and a budget of
+    budget_frac of each group's summed cost (the paper's 50 % default);
+    float32 like the library's arguments. Returns a dict."""
+    g = _streams(seed, 3)
+    p_hat = g[0].uniform(0.02, 0.98, (B, G)).astype(np.float32)
+    c_hat = g[1].lognormal(0.0, 0.6, (B, G)).astype(np.float32)
+    m_hat = g[2].uniform(0.3, 3.0, (B, G)).astype(np.float32) if score_norms else None
+    budget = (budget_frac * c_hat.astype(np.float64).sum(1)).astype(np.float32)
+    return {"p_hat": p_hat, "c_hat": c_hat, "m_hat": m_hat, "budget": budget,
+            "pi_min": np.float32(pi_min)}
