@@ -104,7 +104,7 @@ __device__ void eval(const AllocIn &in, AllocSmem<GP> &sm, bool act, double x, d
 }
 
 template <int GP>
-__global__ void __launch_bounds__(GP) alloc_kernel(int G, const float *p_hat, const float *m_hat,
+__global__ void __launch_bounds__(GP, 1) alloc_kernel(int G, const float *p_hat, const float *m_hat,
                                                    const float *a, const float *c_hat,
                                                    const float *budget_in, float pi_min,
                                                    float *pi_out, double *stats,
