@@ -44,14 +44,25 @@ def _case(inp, deltas=DELTAS):
     return a, lo
 
 
-def _check(inp, a, lo):
+def _check(inp, a, lo, image_blocks=None):
+    """image_blocks: size the workspace for that many token blocks of kept
+    logit terms and image (several backward chunks, later ones recomputing
+    their log-sum-exp); None = pair_grad_workspace_size."""
     B = _binding()
     t = head_inputs(inp, a)
     err = dev_err_word()
+    kw = {}
+    if image_blocks is not None:
+        T, d = t["H"].shape
+        V, R = t["W"].shape[0], inp["R"]
+        block = (B.pair_grad_workspace_size(128, d, V, R, B.PAIR_BF16)
+                 - B.pair_grad_workspace_min_size(128, d, V, R, B.PAIR_BF16))
+        kw["ws"] = torch.empty(B.pair_grad_workspace_min_size(T, d, V, R, B.PAIR_BF16)
+                               + image_blocks * block, dtype=torch.uint8, device="cuda")
     J, dH, dW, lps, coef = B.pair_grad_clipped(t["H"], t["W"], t["y"], t["mask"],
                                                t["cu_seqlens"], t["a"],
                                                torch.from_numpy(lo).cuda(), clip_eps=EPS,
-                                               dev_err=err)
+                                               dev_err=err, **kw)
     assert B.pair_status_sync(err) == 0
     ref = oracle.pair_grad_clipped_ref(inp, a.astype(np.float64), lo.astype(np.float64), EPS)
     lps_n = lps.cpu().numpy().astype(np.float64)
@@ -99,6 +110,16 @@ def test_clipped_bf16_parity(case):
                                    len_scale=ls, w_std_mult=wm)
     a, lo = _case(inp)
     _check(inp, a, lo)
+
+
+@pytest.mark.parametrize("blocks", [1, 2])
+def test_clipped_backward_chunks(blocks):
+    """Several backward chunks: the first uses the logit terms the full
+    log-sum-exp pass kept, later chunks recompute theirs."""
+    inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 7, B=3, G=8, d=512,
+                                   V=1000, len_scale=0.3, w_std_mult=4.0)
+    a, lo = _case(inp)
+    _check(inp, a, lo, image_blocks=blocks)
 
 
 def test_clipped_on_policy_equals_pair_grad():
