@@ -232,7 +232,7 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
       float m2 = -INFINITY, l = 0.f, zt = 0.f;
       bool found = false;
       for (int vt = vt0; vt < vt1; ++vt) {
-        if (!(ok = wait(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
+        if (!(ok = wait_sleepy(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
         tc_fence_after();
 #pragma unroll 1
         for (int c = 0; c < kLseBN / 32; ++c) {
