@@ -394,7 +394,10 @@ PAIR_API pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
  *      and clip_eps >= 0 (finite).
  * Out: as pair_grad (Jobj = the surrogate J); coef [R] float32 (nullable):
  *      the c_i used.
- * Workspace: pair_grad_workspace_size. Errors: as pair_grad.
+ * Workspace: as pair_grad (>= pair_grad_workspace_min_size, normally
+ * pair_grad_workspace_size). With more than one token chunk, chunks after
+ * the first recompute their log-sum-exp pass (the first keeps its logit
+ * terms from the full pass that forms the ratios). Errors: as pair_grad.
  */
 PAIR_API pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dtype dt,
                                        const void *H, const void *W, const int32_t *y,
