@@ -122,6 +122,10 @@ CHUNKED = [
     ("longctx_skew", 1024, 5003, 2, 8, 0.15, 2.0, 3),       # ragged V, 3-block chunks
     ("qwen3_1p7b_head", 2048, 20000, 2, 8, 0.15, 1.0, 2),   # d = 2048, 2-block chunks
     ("qwen3_4b_head", 1536, 777, 2, 6, 0.08, 8.0, 1),
+    # No image: the cluster backward with its narrower column tiles (96 wide
+    # for d = 2560, 64 wide for d = 3072).
+    ("qwen3_4b_head", 2560, 4099, 2, 3, 0.05, 3.0, 0),
+    ("longctx_skew", 3072, 2011, 2, 4, 0.04, 3.0, 0),
 ]
 
 
