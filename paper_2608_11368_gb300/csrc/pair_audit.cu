@@ -102,6 +102,9 @@ __global__ void __launch_bounds__(GP, 1) audit_draws_kernel(
     sm.grp.pi[tid] = (in && wmode == PAIR_W_MARGINAL) ? rho[(size_t)tid * G + tid] : 1.f;
   }
   const double gg = *gg_p;
+  // rho is the same for every draw: its triangle is read once per block.
+  float v[GP / 2];
+  load_upper<GP>(rho, G, weighting_reads_rho(wmode), v);
   double acc[6] = {0, 0, 0, 0, 0, 0};  // mse, cos, vertices, edges, ess, weight
   double a_acc = 0.0;
   for (int b = blockIdx.x; b < N; b += gridDim.x) {
@@ -109,7 +112,7 @@ __global__ void __launch_bounds__(GP, 1) audit_draws_kernel(
     sm.grp.J[tid] = (tid < G) ? (Jd[(size_t)b * G + tid] != 0) : 0;
     __syncthreads();
     const WeightedOut o =
-        group_coeffs_w<GP>(sm.grp, rho, G, scale, (uint32_t)center, wmode, w_max, dev_err);
+        group_coeffs_w<GP>(sm.grp, v, G, scale, (uint32_t)center, wmode, w_max, dev_err);
     const double ai = (double)o.a;
     const double ei = ai - sm.abar[tid];
     sm.e[tid] = ei;

@@ -36,6 +36,23 @@ __device__ void group_coeffs(GroupSmem<GP> &sm, int b, int G, const float *r,
                              int &contrast_out, uint8_t &active_out) {
   const int tid = threadIdx.x;
   const size_t gbase = (size_t)b * G;
+  const float *rho_g = rho + (size_t)b * G * G;
+  // Load phase: every upper entry this thread owns, issued together with r
+  // and J so the group pays one memory latency (the lines of the triangle
+  // are fetched in any case; entries of edges that are not completed are
+  // loaded but never used). Step k covers rows k (first GP-1-k threads) and
+  // GP-1-k (the rest).
+  float v[GP / 2];
+  if (tid < GP - 1) {
+#pragma unroll
+    for (int k = 0; k < GP / 2; ++k) {
+      const int n1 = GP - 1 - k;
+      int i, j;
+      if (tid < n1) { i = k; j = k + 1 + tid; }
+      else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
+      v[k] = (j < G) ? __ldg(rho_g + (size_t)i * G + j) : 1.f;
+    }
+  }
   if (tid < GP) {
     const bool in = tid < G;
     sm.r[tid] = in ? r[gbase + tid] : 0.f;
@@ -43,21 +60,8 @@ __device__ void group_coeffs(GroupSmem<GP> &sm, int b, int G, const float *r,
   }
   __syncthreads();
 
-  const float *rho_g = rho + (size_t)b * G * G;
   int my_contrast = 0, bad = 0;
   if (tid < GP - 1) {
-    // Load phase: every upper entry this thread owns, all loads in flight.
-    // Step k covers rows k (first GP-1-k threads) and GP-1-k (the rest).
-    float v[GP / 2];
-#pragma unroll
-    for (int k = 0; k < GP / 2; ++k) {
-      const int n1 = GP - 1 - k;
-      int i, j;
-      if (tid < n1) { i = k; j = k + 1 + tid; }
-      else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
-      const bool live = (j < G) && sm.J[i] && sm.J[j];
-      v[k] = live ? __ldg(rho_g + (size_t)i * G + j) : 1.f;
-    }
 #pragma unroll
     for (int k = 0; k < GP / 2; ++k) {
       const int n1 = GP - 1 - k;
@@ -247,6 +251,8 @@ __global__ void __launch_bounds__(GP, 1024 / GP) coeffs_w_kernel(
   const int b = blockIdx.x, tid = threadIdx.x;
   const size_t gbase = (size_t)b * G;
   const float *rho_g = rho + (size_t)b * G * G;
+  float v[GP / 2];
+  load_upper<GP>(rho_g, G, weighting_reads_rho(wmode), v);
   {
     const bool in = tid < G;
     sm.r[tid] = in ? r[gbase + tid] : 0.f;
@@ -254,7 +260,7 @@ __global__ void __launch_bounds__(GP, 1024 / GP) coeffs_w_kernel(
     sm.pi[tid] = (in && wmode == PAIR_W_MARGINAL) ? rho_g[(size_t)tid * G + tid] : 1.f;
   }
   __syncthreads();
-  const WeightedOut o = group_coeffs_w<GP>(sm, rho_g, G, scale, (uint32_t)center, wmode, w_max,
+  const WeightedOut o = group_coeffs_w<GP>(sm, v, G, scale, (uint32_t)center, wmode, w_max,
                                            dev_err);
   if (tid < G) {
     a[gbase + tid] = o.a;

@@ -99,30 +99,41 @@ struct WeightedOut {
   float W, W2, Wmax;  // sum, sum of squares and max of the completed-edge weights
 };
 
-// Coefficients of one group under a weighting variant (see
-// pair_coeffs_weighted). The caller has placed r, J (and, for the marginal
-// weighting, the marginals) in shared memory; rho_g is the group's G x G
-// matrix. The upper triangle is read by row pairs as in coeffs_kernel, every
-// term placed once, every vertex summed by the fixed pairwise tree. All GP
-// threads call.
+// The upper-triangle entries of rho_g that thread tid owns, read by row
+// pairs (step k covers rows k and GP-1-k), all loads in flight at once; every
+// entry with j < G is loaded (its line is fetched anyway), so the loads need
+// not wait for J. Entries of edges that are not completed are never used.
 template <int GP>
-__device__ WeightedOut group_coeffs_w(GroupSmemW<GP> &sm, const float *rho_g, int G, float scale,
-                                      uint32_t flags, int wmode, float w_max, int32_t *dev_err) {
+__device__ __forceinline__ void load_upper(const float *rho_g, int G, bool needs_rho,
+                                           float (&v)[GP / 2]) {
   const int tid = threadIdx.x;
-  const bool needs_rho = wmode == PAIR_W_HT || wmode == PAIR_W_CLIPPED || wmode == PAIR_W_HAJEK;
+#pragma unroll
+  for (int k = 0; k < GP / 2; ++k) {
+    const int n1 = GP - 1 - k;
+    int i, j;
+    if (tid < n1) { i = k; j = k + 1 + tid; }
+    else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
+    v[k] = (needs_rho && tid < GP - 1 && j < G) ? __ldg(rho_g + (size_t)i * G + j) : 1.f;
+  }
+}
+
+__device__ __forceinline__ bool weighting_reads_rho(int wmode) {
+  return wmode == PAIR_W_HT || wmode == PAIR_W_CLIPPED || wmode == PAIR_W_HAJEK;
+}
+
+// Coefficients of one group under a weighting variant (see
+// pair_coeffs_weighted), from the entries load_upper fetched. The caller has
+// placed r, J (and, for the marginal weighting, the marginals) in shared
+// memory. Every term is placed once, every vertex summed by the fixed
+// pairwise tree. All GP threads call.
+template <int GP>
+__device__ WeightedOut group_coeffs_w(GroupSmemW<GP> &sm, const float (&v)[GP / 2], int G,
+                                      float scale, uint32_t flags, int wmode, float w_max,
+                                      int32_t *dev_err) {
+  const int tid = threadIdx.x;
   int my_contrast = 0, bad = 0;
   float sw = 0.f, sw2 = 0.f, mw = 0.f;
   if (tid < GP - 1) {
-    float v[GP / 2];
-#pragma unroll
-    for (int k = 0; k < GP / 2; ++k) {
-      const int n1 = GP - 1 - k;
-      int i, j;
-      if (tid < n1) { i = k; j = k + 1 + tid; }
-      else { i = GP - 1 - k; j = i + 1 + (tid - n1); }
-      const bool live = (j < G) && sm.J[i] && sm.J[j];
-      v[k] = (live && needs_rho) ? __ldg(rho_g + (size_t)i * G + j) : 1.f;
-    }
 #pragma unroll
     for (int k = 0; k < GP / 2; ++k) {
       const int n1 = GP - 1 - k;
