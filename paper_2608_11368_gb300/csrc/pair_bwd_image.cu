@@ -1,0 +1,521 @@
+// Backward of the bf16 LM-head path through the logit-gradient image: the
+// bf16 tiles Gs = -c_t softmax(z_t) formed once from the kept logit terms,
+// then dH = Gs W and dW = Gs^T Hc as plain tcgen05 GEMMs (no logit
+// recomputation), one token chunk at a time.
+#include "tc_kernels.cuh"
+
+namespace pairk {
+namespace {
+
+using namespace tc;
+using namespace tck;
+
+// ------------------------------------------ logit-gradient image from S
+//
+// Gs_tv = -c_t exp(z_tv - lse_t) in bf16 for every tile of a chunk of token
+// blocks, from the chunk-relative terms the LSE pass kept (fp16 P_v =
+// 2^(z_v log2 e - m) and the fp32 chunk maximum m, per 32 columns):
+// Gs = -c_t 2^(m - lse_t log2 e) P_v, one exponential per 8 columns. One
+// 32 KB image tile per 128 tokens x 128 vocabulary rows, two K-major
+// SWIZZLE_128B atoms of 64 vocabulary columns (the layout both backward
+// GEMMs read). Columns >= V, rows >= T_eff and tokens with c_t = 0 give
+// exact zeros. Streaming kernel: 34 KB read and 32 KB written per tile.
+__global__ void __launch_bounds__(256) g_image_kernel(int V, int rb0, int cap,
+                                                      const int32_t *counters,
+                                                      const float *__restrict__ tok_c,
+                                                      const float *__restrict__ lse,
+                                                      const __half *__restrict__ sbuf,
+                                                      const float4 *__restrict__ mbuf,
+                                                      uint8_t *__restrict__ gimg) {
+  const int Teff = counters[0];
+  const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  const int n_vt = (V + 127) / 128;
+  const int64_t n_tiles = (int64_t)nrb * n_vt;
+  // Thread t of the block handles 8-column chunk (t & 15) of rows
+  // (t >> 4) + 16 k, k < 8; all eight loads are issued before any use.
+  const int ch = threadIdx.x & 15, r0 = threadIdx.x >> 4;
+  for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+    const int b = (int)(tile / n_vt), vt = (int)(tile - (int64_t)b * n_vt);
+    const __half *src = sbuf + tile * (128 * 128);
+    const float4 *mt = mbuf + tile * 128;
+    uint8_t *dst = gimg + tile * kGImgTileBytes;
+    const int col0 = vt * 128 + ch * 8;
+    uint4 h[8];
+    float4 m4[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int row = r0 + 16 * k;
+      h[k] = *reinterpret_cast<const uint4 *>(src + row * 128 + ch * 8);
+      m4[k] = mt[row];
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int row = r0 + 16 * k;
+      const int p = (rb0 + b) * 128 + row;
+      float sc = 0.f;
+      if (p < Teff && col0 < V) {
+        const float cc = tok_c[p];
+        const int q = ch >> 2;
+        const float m = q == 0 ? m4[k].x : q == 1 ? m4[k].y : q == 2 ? m4[k].z : m4[k].w;
+        if (cc != 0.f) sc = -cc * ex2_approx(m - lse[p] * kLog2e);
+      }
+      const uint32_t hw[4] = {h[k].x, h[k].y, h[k].z, h[k].w};
+      uint32_t pk[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&hw[e]));
+        const float g0 = col0 + 2 * e < V ? sc * f.x : 0.f;
+        const float g1 = col0 + 2 * e + 1 < V ? sc * f.y : 0.f;
+        __nv_bfloat162 b2 = __floats2bfloat162_rn(g0, g1);
+        pk[e] = *reinterpret_cast<uint32_t *>(&b2);
+      }
+      *reinterpret_cast<uint4 *>(dst + (ch >> 3) * kAtom128 + sw128_offset(row, (ch & 7) * 8)) =
+          make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    }
+  }
+}
+
+// ---------------------------------------------- dH from the stored image
+//
+// Softmax part of dH as the plain GEMM dH[t, :] = sum_v Gs[t, v] W[v, :],
+// with the image tiles as the K-major A operand (64 vocabulary rows per
+// stage, one 16 KB atom, copied verbatim) and W as the MN-major B operand.
+// CTA pairs (2-CTA clusters) take two token blocks of the same 256-column
+// chunk of d and share its W stage by multicast (each CTA fetches two of the
+// four 64-column atoms). Work unit = (token block pair, 256-column chunk);
+// the fp32 accumulator (128 x 256) is double-buffered in TMEM so the drain of
+// one unit overlaps the next. Each (token, column) is owned by one CTA and
+// summed over all of V in one fixed order: deterministic, no atomics. An odd
+// last block is computed twice (the pair's other CTA repeats it) and stored
+// once.
+constexpr int kDhN = 256;                              // output columns per unit
+constexpr int kDhStages = 4;
+constexpr uint32_t kDhABytes = kAtom128;               // 128 tokens x 64 vocabulary
+constexpr uint32_t kDhBBytes = (kDhN / 64) * 64 * 128; // 4 column atoms x 64 rows
+constexpr uint32_t kIdescDh = idesc_bf16(128, kDhN, 0, 1);
+
+struct DhSmem {
+  uint8_t a[kDhStages][kDhABytes];
+  uint8_t b[kDhStages][kDhBBytes];
+  uint64_t full[kDhStages], empty[kDhStages];
+  uint64_t acc_full[2], acc_empty[2], mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    dh_gemm_kernel(const __grid_constant__ CUtensorMap tmW, int d, int V, int rb0, int cap,
+                   const int32_t *counters, const int32_t *tok_idx, const uint8_t *gimg,
+                   float *dH, int32_t *dev_err) {
+  const int Teff = counters[0];
+  const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  if (nrb == 0) return;  // no token in this chunk
+  extern __shared__ uint8_t smem_raw[];
+  DhSmem &sm = *reinterpret_cast<DhSmem *>(align1k(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = (int)cluster_rank();
+  const int pid = (int)cluster_id_x(), npairs = (int)num_clusters_x();
+  const int n_vt = (V + 127) / 128;
+  const int nks = 2 * n_vt;  // 64-wide vocabulary steps (image atoms)
+  const int nq = d / kDhN;
+  const int n_units = (nrb + 1) / 2 * nq;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kDhStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 2);  // both CTAs' MMAs done with the stage
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.acc_full[s], 1);
+      mbar_init(&sm.acc_empty[s], 128);
+    }
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmW);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the peer's barriers exist before any multicast lands
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  volatile int *abort = &sm.abort;
+
+  if (warp == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
+      int stage = 0;
+      uint32_t ph = 0;
+      int last_ph[kDhStages];
+      for (int s = 0; s < kDhStages; ++s) last_ph[s] = -1;
+      bool ok = true;
+      for (int u = pid; u < n_units && ok; u += npairs) {
+        const int tp = u / nq, q = u - tp * nq;
+        const int b = min(2 * tp + r, nrb - 1);
+        const uint8_t *arow = gimg + (size_t)b * n_vt * kGImgTileBytes;
+        for (int ks = 0; ks < nks; ++ks) {
+          if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+          if (elect_one()) {
+            mbar_expect_tx(&sm.full[stage], kDhABytes + kDhBBytes);
+            bulk_load(sm.a[stage], arow + (size_t)ks * kAtom128, kAtom128, &sm.full[stage]);
+            tma_load_3d_mc(sm.b[stage] + r * (kDhBBytes / 2), &tmW, &sm.full[stage], 0, 64 * ks,
+                           q * (kDhN / 64) + r * (kDhN / 128), (uint16_t)3);
+          }
+          __syncwarp();
+          last_ph[stage] = (int)ph;
+          if (++stage == kDhStages) { stage = 0; ph ^= 1; }
+        }
+      }
+      for (int s = 0; s < kDhStages; ++s)
+        if (last_ph[s] >= 0) {
+          volatile int never = 0;
+          wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+        }
+    }
+  } else if (warp == 1) {
+    {  // whole warp: uniform loop state; elected lane issues
+      // A: K-major atom, 16 tokens of K = 32 bytes along the swizzled row.
+      // B: 4 column atoms of 64 vocabulary rows (LBO 8 KB), row groups of 8
+      // (SBO 1 KB); 16 vocabulary rows = 2 KB.
+      const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
+      const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 64 * 128, 1024);
+      int stage = 0, acc = 0;
+      uint32_t ph = 0, acc_ph = 0;
+      bool ok = true;
+      for (int u = pid; u < n_units && ok; u += npairs) {
+        if (!(ok = wait(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
+        tc_fence_after();
+        const uint32_t dt = tmem + acc * kDhN;
+        for (int ks = 0; ks < nks; ++ks) {
+          if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+          const uint64_t da = da0 + (uint64_t)stage * (kDhABytes >> 4);
+          const uint64_t db = db0 + (uint64_t)stage * (kDhBBytes >> 4);
+          if (elect_one()) {
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_bf16(dt, da + 2 * kk, db + kk * (2048 >> 4), kIdescDh, (ks | kk) != 0);
+            mma_commit_multicast(&sm.empty[stage], (uint16_t)3);
+          }
+          __syncwarp();
+          if (++stage == kDhStages) { stage = 0; ph ^= 1; }
+        }
+        if (!ok) break;
+        if (elect_one()) mma_commit(&sm.acc_full[acc]);
+        __syncwarp();
+        if (++acc == 2) { acc = 0; acc_ph ^= 1; }
+      }
+      if (elect_one()) mma_commit(&sm.mma_done);
+      __syncwarp();
+      volatile int never = 0;
+      wait(&sm.mma_done, 0, &never, dev_err);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    int acc = 0;
+    uint32_t acc_ph = 0;
+    bool ok = true;
+    for (int u = pid; u < n_units && ok; u += npairs) {
+      const int tp = u / nq, q = u - tp * nq;
+      const int t = (rb0 + 2 * tp + r) * 128 + row;
+      const bool valid = 2 * tp + r < nrb && t < Teff;
+      float4 *dst =
+          valid ? reinterpret_cast<float4 *>(dH + (int64_t)tok_idx[t] * d + q * kDhN) : nullptr;
+      if (!(ok = wait_sleepy(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < kDhN / 32; ++c) {
+        float x[32];
+        tmem_ld32(tmem + lane_off + acc * kDhN + c * 32, x);
+        if (valid) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            dst[c * 8 + e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&sm.acc_empty[acc]);
+      if (++acc == 2) { acc = 0; acc_ph ^= 1; }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still signal or fill it
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ------------------------------------- dW from the stored logit gradient
+//
+// With 128-wide column tiles the dH pass keeps every bf16 tile Gs it forms
+// (128 tokens x 128 vocabulary rows, one 32 KB image per tile in the
+// K-major SWIZZLE_128B layout of its own MMA operand) for a chunk of token
+// blocks. Read with the token index as K, the same bytes are the MN-major
+// SWIZZLE_128B layout of Gs^T (64 vocabulary rows per 128-byte line, one
+// line per token), so the softmax part of dW is the plain GEMM
+//     dW[v, :] (+)= sum_t Gs[t, v] Hc[t, :]
+// with no logit recomputation.
+//
+// CTA pairs (2-CTA clusters) share one 512-column chunk of Hc: CTA r of the
+// pair fetches half of each Hc stage and multicasts it into both CTAs; each
+// CTA fetches the Gs^T stage of its own 128 vocabulary rows. Work unit =
+// (vocabulary block pair, 512-column chunk of d); CTA r accumulates
+// dW[block 2 p + r, chunk] (128 x 512 fp32 = all of TMEM) over the chunk's
+// tokens, 32 token rows per stage, and drains it with plain stores (first
+// chunk) or read-add-writes (later chunks; this CTA owns those rows).
+// An odd last block is computed twice (the pair's other CTA repeats the
+// last block) so both CTAs run the same stage sequence; only one stores it.
+constexpr int kDwKS = 32;                                 // token rows per stage
+constexpr int kDwStages = 5;
+constexpr int kDwN = 512;                                 // output columns per CTA
+constexpr uint32_t kDwGBytes = 2 * kDwKS * 128;           // 2 vocabulary atoms x 32 rows
+constexpr uint32_t kDwHBytes = (kDwN / 64) * kDwKS * 128; // 8 column atoms x 32 rows
+constexpr uint32_t kIdescDw = idesc_bf16(128, 256, 1, 1); // both operands MN-major
+
+struct DwSmem {
+  uint8_t g[kDwStages][kDwGBytes];  // Gs^T: MN-major A, atoms 4 KB apart
+  uint8_t h[kDwStages][kDwHBytes];  // Hc[t, chunk]: MN-major B, atoms 4 KB apart
+  uint64_t full[kDwStages], empty[kDwStages];
+  uint64_t acc_full, acc_empty, mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    dw_gemm_kernel(const __grid_constant__ CUtensorMap tmG,
+                   const __grid_constant__ CUtensorMap tmH, int d, int V, int rb0, int cap,
+                   int accumulate, const int32_t *counters, float *dW, int32_t *dev_err) {
+  const int Teff = counters[0];
+  const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  // A chunk past the last token adds nothing (the first chunk always runs:
+  // with no tokens at all it writes the zero softmax part).
+  if (nrb == 0 && accumulate) return;
+  extern __shared__ uint8_t smem_raw[];
+  DwSmem &sm = *reinterpret_cast<DwSmem *>(align1k(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = (int)cluster_rank();
+  const int pid = (int)cluster_id_x(), npairs = (int)num_clusters_x();
+  const int n_vb = (V + 127) / 128;
+  const int nq = d / kDwN;
+  const int n_units = (n_vb + 1) / 2 * nq;
+  const int nks = nrb * (128 / kDwKS);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kDwStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 2);  // both CTAs' MMAs done with the stage
+    }
+    mbar_init(&sm.acc_full, 1);
+    mbar_init(&sm.acc_empty, 128);
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmG);
+    prefetch_tmap(&tmH);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the peer's barriers exist before any multicast lands
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  volatile int *abort = &sm.abort;
+
+  if (warp == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
+      int stage = 0;
+      uint32_t ph = 0;
+      int last_ph[kDwStages];
+      for (int s = 0; s < kDwStages; ++s) last_ph[s] = -1;
+      bool ok = true;
+      for (int u = pid; u < n_units && ok; u += npairs) {
+        const int vp = u / nq, q = u - vp * nq;
+        const int vb = min(2 * vp + r, n_vb - 1);
+        for (int ks = 0; ks < nks; ++ks) {
+          const int rbl = ks >> 2, j = ks & 3;
+          if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+          if (elect_one()) {
+            mbar_expect_tx(&sm.full[stage], kDwGBytes + kDwHBytes);
+            tma_load_3d(sm.g[stage], &tmG, &sm.full[stage], 0, kDwKS * j,
+                        2 * (rbl * n_vb + vb));
+            tma_load_3d_mc(sm.h[stage] + r * (kDwHBytes / 2), &tmH, &sm.full[stage], 0,
+                           (rb0 + rbl) * 128 + kDwKS * j, q * (kDwN / 64) + r * (kDwN / 128),
+                           (uint16_t)3);
+          }
+          __syncwarp();
+          last_ph[stage] = (int)ph;
+          if (++stage == kDwStages) { stage = 0; ph ^= 1; }
+        }
+      }
+      // Never leave a copy in flight: wait (bounded) for the last one issued
+      // on every stage.
+      for (int s = 0; s < kDwStages; ++s)
+        if (last_ph[s] >= 0) {
+          volatile int never = 0;
+          wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+        }
+    }
+  } else if (warp == 1) {
+    {  // whole warp: uniform loop state; elected lane issues
+      // A: 2 vocabulary atoms (LBO 4 KB), token groups of 8 rows (SBO 1 KB);
+      // B: 8 column atoms (LBO 4 KB), the same token groups. One K step of 16
+      // tokens advances both by 2 KB; B's second 256-column half is 16 KB on.
+      const uint64_t dg0 = sdesc_sw128(smem_u32(sm.g[0]), kDwKS * 128, 1024);
+      const uint64_t dh0 = sdesc_sw128(smem_u32(sm.h[0]), kDwKS * 128, 1024);
+      int stage = 0;
+      uint32_t ph = 0, acc_ph = 0;
+      bool ok = true;
+      for (int u = pid; u < n_units && ok && nks > 0; u += npairs) {
+        if (!(ok = wait(&sm.acc_empty, acc_ph ^ 1, abort, dev_err))) break;
+        acc_ph ^= 1;
+        tc_fence_after();
+        for (int ks = 0; ks < nks; ++ks) {
+          if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+          const uint64_t dg = dg0 + (uint64_t)stage * (kDwGBytes >> 4);
+          const uint64_t dh = dh0 + (uint64_t)stage * (kDwHBytes >> 4);
+          if (elect_one()) {
+#pragma unroll
+            for (int kk = 0; kk < kDwKS / 16; ++kk)
+#pragma unroll
+              for (int nh = 0; nh < 2; ++nh)
+                mma_bf16(tmem + nh * 256, dg + kk * (2048 >> 4),
+                         dh + nh * ((kDwHBytes / 2) >> 4) + kk * (2048 >> 4), kIdescDw,
+                         (ks | kk) != 0);
+            mma_commit_multicast(&sm.empty[stage], (uint16_t)3);
+          }
+          __syncwarp();
+          if (++stage == kDwStages) { stage = 0; ph ^= 1; }
+        }
+        if (!ok) break;
+        if (elect_one()) mma_commit(&sm.acc_full);
+        __syncwarp();
+      }
+      if (elect_one()) mma_commit(&sm.mma_done);
+      __syncwarp();
+      volatile int never = 0;
+      wait(&sm.mma_done, 0, &never, dev_err);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    uint32_t acc_ph = 0;
+    bool ok = true;
+    for (int u = pid; u < n_units && ok; u += npairs) {
+      const int vp = u / nq, q = u - vp * nq;
+      const int v = (2 * vp + r) * 128 + row;
+      const bool valid = 2 * vp + r < n_vb && v < V;
+      float4 *dst = valid ? reinterpret_cast<float4 *>(dW + (int64_t)v * d + q * kDwN) : nullptr;
+      if (nks == 0) {
+        if (valid)
+          for (int c = 0; c < kDwN / 4; ++c) dst[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+        continue;
+      }
+      if (!(ok = wait_sleepy(&sm.acc_full, acc_ph, abort, dev_err))) break;
+      acc_ph ^= 1;
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = 0; c < kDwN / 32; ++c) {
+        float x[32];
+        tmem_ld32(tmem + lane_off + c * 32, x);
+        if (valid) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            float4 o = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+            if (accumulate) {
+              const float4 p = dst[c * 8 + e];
+              o.x += p.x; o.y += p.y; o.z += p.z; o.w += p.w;
+            }
+            dst[c * 8 + e] = o;
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&sm.acc_empty);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still signal or fill it
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+}  // namespace
+
+namespace tck {
+
+pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStream_t s,
+                             int64_t c) {
+  const int cap = w.gimg_rb;
+  const int rb0 = (int)(c * cap);
+  const int n_vt = (g.V + 127) / 128;
+  CUtensorMap mG, mH3, mW3;
+  if (!make_map3(&mG, w.gimg, {64, 128, (cuuint64_t)2 * cap * n_vt}, {128, 16384}, {64, 32, 2},
+                 CU_TENSOR_MAP_SWIZZLE_NONE) ||
+      !make_map3(&mH3, w.Hc, {64, (cuuint64_t)w.Tpad, (cuuint64_t)g.d / 64},
+                 {(cuuint64_t)g.d * 2, 128}, {64, (cuuint32_t)kDwKS, 4},
+                 CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !make_map3(&mW3, g.W, {64, (cuuint64_t)g.V, (cuuint64_t)g.d / 64},
+                 {(cuuint64_t)g.d * 2, 128}, {64, 64, 2}, CU_TENSOR_MAP_SWIZZLE_128B))
+    return PAIR_ERR_CUDA;
+  const size_t dh_smem = sizeof(DhSmem) + 1024, dw_smem = sizeof(DwSmem) + 1024;
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(dh_gemm_kernel,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dh_smem));
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(dw_gemm_kernel,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dw_smem));
+  static int dh_cache = 0, dw_cache = 0;
+  uint8_t *gimg = static_cast<uint8_t *>(w.gimg);
+  PAIR_BEGIN("g_image", s);
+  g_image_kernel<<<num_sms() * 3, 256, 0, s>>>(g.V, rb0, cap, w.counters, w.tok_c, w.lse,
+                                               static_cast<const __half *>(w.sbuf), w.mbuf, gimg);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("dh_gemm_tc", s);
+  dh_gemm_kernel<<<pair_grid((const void *)dh_gemm_kernel, dh_smem, &dh_cache), kThreads,
+                   dh_smem, s>>>(mW3, g.d, g.V, rb0, cap, w.counters, w.tok_idx, gimg, g.dH,
+                                 g.dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("dw_gemm_tc", s);
+  dw_gemm_kernel<<<pair_grid((const void *)dw_gemm_kernel, dw_smem, &dw_cache), kThreads,
+                   dw_smem, s>>>(mG, mH3, g.d, g.V, rb0, cap, c > 0 ? 1 : 0, w.counters, g.dW,
+                                 g.dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+
+}  // namespace tck
+
+// Memory the backward may use for kept logit terms (fp16 terms and fp32
+// chunk maxima) and bf16 logit-gradient tiles, 66 KB per 128 x 128 tile;
+// larger problems run in token chunks.
+constexpr int64_t kImageBudget = int64_t(24) << 30;
+constexpr size_t kImageTileBytes = kGImgTileBytes + 128 * 128 * 2 + 128 * 16;
+
+int grad_gimg_rows(int64_t T, int32_t d, int32_t V, pair_dtype dt) {
+  if (dt != PAIR_BF16 || d < 512 || d % kDwN != 0) return 0;
+  const int64_t n_rb = (T + 127) / 128;
+  const int64_t per_rb = (int64_t)((V + 127) / 128) * (int64_t)kImageTileBytes;
+  int64_t cap = kImageBudget / per_rb;
+  if (cap < 32) cap = 32;
+  return (int)(n_rb < cap ? n_rb : cap);
+}
+
+size_t grad_image_block_bytes(int32_t V) {
+  return (size_t)((V + 127) / 128) * kImageTileBytes;
+}
+
+}  // namespace pairk

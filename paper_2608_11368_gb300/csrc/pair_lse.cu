@@ -1,0 +1,365 @@
+// Log-sum-exp pass of the bf16 LM-head path (Sec. 4.5 forward): per active
+// token the log-sum-exp of its logits z = W h and its target logit, on the
+// 5th-generation tensor cores. With a workspace that keeps them, the logit
+// terms of a chunk of token blocks are stored for the backward (fp16 terms
+// relative to each 32-column chunk maximum, and the maxima).
+#include "tc_kernels.cuh"
+
+namespace pairk {
+namespace {
+
+using namespace tc;
+using namespace tck;
+
+// ------------------------------------------------------------------ LSE
+constexpr int kLseBN = 256;
+constexpr int kLseStages = 4;
+constexpr uint32_t kLseStageTx = (128 + kLseBN) * 64 * 2;
+constexpr int kLsePair = 2;  // CTAs per cluster sharing each vocabulary tile
+constexpr uint32_t kIdescLse = idesc_bf16(128, kLseBN, 0, 0);
+
+struct LseSmem {
+  uint8_t a[kLseStages][kAtom128];
+  uint8_t b[kLseStages][2 * kAtom128];
+  uint8_t stg[2][128 * 128];  // kept-term staging: per warp 32 rows x 64 fp16, SWIZZLE_128B
+  uint64_t full[kLseStages], empty[kLseStages];
+  uint64_t acc_full[2], acc_empty[2];
+  uint64_t mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+// CTA pairs (2-CTA clusters) work on two token blocks of the same vocabulary
+// split in lockstep: each CTA fetches its own token atom and one half (128
+// rows) of the shared 256-row vocabulary atom, multicast into both CTAs'
+// stage. A stage is refilled only after both CTAs' MMAs released it (each
+// MMA warp commits to the empty barrier of both CTAs). This halves the
+// vocabulary bytes each SM's copy engine requests, which is what limits the
+// loads here (the engine's outstanding requests wait on DRAM-latency tiles).
+__global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
+    lse_kernel(const __grid_constant__ CUtensorMap tmH,
+               const __grid_constant__ CUtensorMap tmW,
+               const __grid_constant__ CUtensorMap tmS, int d, int V,
+               int nsplit, int64_t Tpad, const int32_t *counters,
+               const int32_t *tok_y, float2 *part, float *zy, int rb0, int cap,
+               const void *sbuf, float4 *mbuf, int s_blocks, int32_t *dev_err) {
+  extern __shared__ uint8_t smem_raw[];
+  LseSmem &sm = *reinterpret_cast<LseSmem *>(align1k(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int Teff = counters[0];
+  // Token blocks [rb0, rb0 + n_tb) of this launch. With sbuf, the logits of
+  // its first s_blocks blocks are also kept, per 32-column chunk c of a row
+  // as P_j = 2^(z_j log2 e - m_c) in fp16 (in [0, 1]) with the chunk maximum
+  // m_c = max_j z_j log2 e in fp32: 128 x 128 tiles, tile (b, vt) at
+  // ((b * n_vt128 + vt) * 128 + row) * 128 + col of sbuf (written through
+  // tmS, a [rows][128] fp16 view: each epilogue warp stages its 32 rows of
+  // two chunks in shared memory and writes them with one TMA store), and
+  // the row's four maxima as one float4 at mbuf[(b * n_vt128 + vt) * 128 +
+  // row]. The same per-chunk terms P_j make up the log-sum-exp sum.
+  const int n_tb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  const int n_vt128 = (V + 127) / 128;
+  const int s_lim = min(n_tb, s_blocks);
+  const int n_vt = (V + kLseBN - 1) / kLseBN;
+  // Work unit = (pair of token blocks, vocabulary split); CTA r of the pair
+  // takes token block 2 * pair + r (past the last block for an odd count:
+  // in-bounds padding rows whose results are never written).
+  // Units (pair of token blocks, vocabulary split), split index fastest.
+  // (Split-major order, which lets the pairs running at once share each W
+  // split in L2, measured 4 % slower.)
+  const int n_pairs = (n_tb + 1) / 2;
+  const int n_units = n_pairs * nsplit;
+  const int nk = d / 64;
+  const int r = (int)cluster_rank();
+  const int pid = (int)cluster_id_x(), npairs = (int)num_clusters_x();
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kLseStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], kLsePair);  // both CTAs' MMAs done with the stage
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.acc_full[s], 1);
+      mbar_init(&sm.acc_empty[s], 128);
+    }
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmH);
+    prefetch_tmap(&tmW);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the peer's barriers exist before any multicast lands
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  volatile int *abort = &sm.abort;
+
+  if (warp == 0) {
+    {  // whole warp: uniform loop state; elected lane issues
+      int stage = 0;
+      uint32_t ph = 0;
+      int last_ph[kLseStages];
+      for (int s = 0; s < kLseStages; ++s) last_ph[s] = -1;
+      bool ok = true;
+      for (int u = pid; u < n_units && ok; u += npairs) {
+        const int tb = rb0 + 2 * (u / nsplit) + r, sp = u % nsplit;
+        const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
+        const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
+        for (int vt = vt0; vt < vt1 && ok; ++vt) {
+          for (int k = 0; k < nk; ++k) {
+            if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
+            if (elect_one()) {
+              mbar_expect_tx(&sm.full[stage], kLseStageTx);
+              tma_load_2d(sm.a[stage], &tmH, &sm.full[stage], k * 64, tb * 128);
+              tma_load_2d_mc(sm.b[stage] + r * (kLseBN / 2) * 128, &tmW, &sm.full[stage],
+                             k * 64, vt * kLseBN + r * (kLseBN / 2), (uint16_t)3);
+            }
+            __syncwarp();
+            last_ph[stage] = (int)ph;
+            if (++stage == kLseStages) { stage = 0; ph ^= 1; }
+          }
+        }
+      }
+      // Never leave a copy in flight: wait (bounded) for the last one issued
+      // on every stage.
+      for (int s = 0; s < kLseStages; ++s)
+        if (last_ph[s] >= 0) {
+          volatile int never = 0;
+          wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+        }
+    }
+  } else if (warp == 1) {
+    {  // whole warp: uniform loop state; elected lane issues
+      int stage = 0, acc = 0;
+      uint32_t ph = 0, acc_ph = 0;
+      const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
+      const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 16, 1024);
+      bool ok = true;
+      for (int u = pid; u < n_units && ok; u += npairs) {
+        const int sp = u % nsplit;
+        const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
+        const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
+        for (int vt = vt0; vt < vt1 && ok; ++vt) {
+          if (!(ok = wait(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
+          tc_fence_after();
+          const uint32_t dt = tmem + acc * kLseBN;
+          for (int k = 0; k < nk; ++k) {
+            if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+            const uint64_t da = da0 + (uint64_t)stage * (kAtom128 >> 4);
+            const uint64_t db = db0 + (uint64_t)stage * ((2 * kAtom128) >> 4);
+            if (elect_one()) {
+#pragma unroll
+              for (int kk = 0; kk < 4; ++kk)
+                mma_bf16(dt, da + 2 * kk, db + 2 * kk, kIdescLse, (k | kk) != 0);
+              mma_commit_multicast(&sm.empty[stage], (uint16_t)3);
+            }
+            __syncwarp();
+            if (++stage == kLseStages) { stage = 0; ph ^= 1; }
+          }
+          if (!ok) break;
+          if (elect_one()) mma_commit(&sm.acc_full[acc]);
+          __syncwarp();
+          if (++acc == 2) { acc = 0; acc_ph ^= 1; }
+        }
+      }
+      if (elect_one()) mma_commit(&sm.mma_done);
+      __syncwarp();
+      volatile int never = 0;
+      wait(&sm.mma_done, 0, &never, dev_err);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    int acc = 0, sbuf_i = 0;
+    uint32_t acc_ph = 0;
+    bool ok = true;
+    for (int u = pid; u < n_units && ok; u += npairs) {
+      const int tbl = 2 * (u / nsplit) + r, sp = u % nsplit;
+      const int tb = rb0 + tbl;
+      const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
+      const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
+      const int p = tb * 128 + row;
+      const bool valid = p < Teff;
+      const bool keep = sbuf && tbl < s_lim;  // uniform over the CTA
+      float mrow[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      const int yt = valid ? tok_y[p] : -1;
+      float m2 = -INFINITY, l = 0.f, zt = 0.f;
+      bool found = false;
+      for (int vt = vt0; vt < vt1; ++vt) {
+        if (!(ok = wait_sleepy(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < kLseBN / 32; ++c) {
+          float v[32];
+          tmem_ld32(lane_addr + acc * kLseBN + c * 32, v);
+          const int col0 = vt * kLseBN + c * 32;
+          const int off = yt - col0;
+          if (off >= 0 && off < 32) {
+            found = true;
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (j == off) zt = v[j];
+          }
+          const int nvalid = V - col0;  // columns >= V are padding
+          float mc = -INFINITY;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            v[j] = (j < nvalid) ? v[j] * kLog2e : -INFINITY;
+            mc = fmaxf(mc, v[j]);
+          }
+          if (mc == -INFINITY) continue;  // the whole chunk lies past V
+          // Chunk terms relative to the chunk maximum, then folded into the
+          // running (max, sum): v[j] becomes P_j.
+          float s = 0.f;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            v[j] = ex2_approx(v[j] - mc);
+            s += v[j];
+          }
+          if (mc > m2) {
+            l = l * ex2_approx(m2 - mc) + s;
+            m2 = mc;
+          } else {
+            l += s * ex2_approx(mc - m2);
+          }
+          if (keep) {
+            // Per warp: its 32 rows x 64 columns (two chunks) in fp16, in its
+            // own 4 KB buffer, stored by its lane 0 once both halves (or the
+            // last chunk before V) are in. The store that last read this
+            // buffer is done before the first half is written.
+            const int half = c & 1;
+            if (half == 0) {
+              if (lane == 0) bulk_wait_group_read<1>();
+              __syncwarp();
+            }
+            uint8_t *buf = sm.stg[sbuf_i] + quad * 4096;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              uint32_t pk[4];
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                __half2 h2 = __floats2half2_rn(v[8 * e + 2 * q], v[8 * e + 2 * q + 1]);
+                pk[q] = *reinterpret_cast<uint32_t *>(&h2);
+              }
+              *reinterpret_cast<uint4 *>(buf + lane * 128 + (((half * 4 + e) ^ (lane & 7)) << 4)) =
+                  make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            }
+            mrow[c & 3] = mc;
+            const bool last = col0 + 32 >= V;
+            if (half == 1 || last) {
+              fence_async_smem();
+              __syncwarp();
+              if (lane == 0) {
+                tma_store_2d_evict_first(&tmS, buf, col0 & 64,
+                                         (tbl * n_vt128 + (col0 >> 7)) * 128 + quad * 32);
+                bulk_commit_group();
+              }
+              sbuf_i ^= 1;
+            }
+            if ((c & 3) == 3 || last) {
+              mbuf[((int64_t)tbl * n_vt128 + (col0 >> 7)) * 128 + row] =
+                  make_float4(mrow[0], mrow[1], mrow[2], mrow[3]);
+              mrow[0] = mrow[1] = mrow[2] = mrow[3] = -INFINITY;
+            }
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(&sm.acc_empty[acc]);
+        if (++acc == 2) { acc = 0; acc_ph ^= 1; }
+      }
+      if (!ok) break;
+      if (valid) {
+        part[(int64_t)sp * Tpad + p] = make_float2(m2, l);
+        if (found) zy[p] = zt;
+      }
+    }
+    // Every kept-logit store has completed before the CTA leaves.
+    if (lane == 0) bulk_wait_group<0>();
+    __syncwarp();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still signal or fill it
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// lse_t = ln 2 * (M + log2 sum_s l_s 2^(m_s - M)) over the vocabulary splits.
+// Tokens [128 rb0, 128 (rb0 + cap)) of the active ones.
+__global__ void lse_combine_kernel(int nsplit, int64_t Tpad,
+                                   const int32_t *counters, const float2 *part,
+                                   float *lse, int rb0, int cap) {
+  const int Teff = counters[0];
+  const int64_t hi64 = (int64_t)(rb0 + (int64_t)cap) * 128;
+  const int p1 = (int)(hi64 < Teff ? hi64 : Teff);
+  for (int p = rb0 * 128 + blockIdx.x * blockDim.x + threadIdx.x; p < p1;
+       p += gridDim.x * blockDim.x) {
+    float M = -INFINITY;
+    for (int s = 0; s < nsplit; ++s) M = fmaxf(M, part[(int64_t)s * Tpad + p].x);
+    float L = 0.f;
+    for (int s = 0; s < nsplit; ++s) {
+      const float2 q = part[(int64_t)s * Tpad + p];
+      if (q.y > 0.f) L += q.y * exp2f(q.x - M);
+    }
+    lse[p] = (M + log2f(L)) * 0.6931471805599453f;
+  }
+}
+
+// CTAs of the LSE grid: every 2-CTA cluster that fits at once (persistent).
+int lse_grid(size_t smem) {
+  static int cached = 0;
+  if (cached) return cached;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kLsePair * 64, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, (const void *)lse_kernel, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    n = num_sms() / kLsePair;
+  }
+  cached = kLsePair * (n > 0 ? n : 1);
+  return cached;
+}
+
+}  // namespace
+
+namespace tck {
+
+// Log-sum-exp pass over token blocks [rb0, rb0 + cap) (clipped to the active
+// ones), then lse for those tokens. With keep, the chunk-relative logit terms
+// of the first s_blocks of those blocks are kept in w.sbuf / w.mbuf.
+pair_status launch_lse(const GradArgs &g, const GradWorkspace &w, cudaStream_t s, int rb0,
+                       int cap, bool keep, int s_blocks) {
+  void *sbuf = keep ? w.sbuf : nullptr;
+  CUtensorMap mH, mW128, mS = {};
+  if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) || !make_map(&mW128, g.W, g.V, g.d, 128))
+    return PAIR_ERR_CUDA;
+  if (sbuf && !make_map_s(&mS, sbuf, (int64_t)w.gimg_rb * ((g.V + 127) / 128) * 128))
+    return PAIR_ERR_CUDA;
+  const int nsm = num_sms();
+  const size_t lse_smem = sizeof(LseSmem) + 1024;
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(lse_kernel,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)lse_smem));
+  PAIR_BEGIN("lse_tc", s);
+  lse_kernel<<<lse_grid(lse_smem), kThreads, lse_smem, s>>>(
+      mH, mW128, mS, g.d, g.V, w.nsplit, w.Tpad, w.counters, w.tok_y, w.part, w.zy, rb0, cap, sbuf,
+      keep ? w.mbuf : nullptr, s_blocks, g.dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("lse_combine", s);
+  lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters, w.part, w.lse, rb0,
+                                             cap);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+}  // namespace tck
+}  // namespace pairk
