@@ -12,7 +12,7 @@
 // together hold exactly GP-1 upper entries, so a block of >= GP threads reads
 // them as two contiguous runs per step, fully unrolled to keep every load
 // of the group in flight at once.
-#include "pair_coeffs_dev.cuh"
+#include "pair_coeffs_stream.cuh"
 
 namespace pairk {
 namespace {
@@ -152,28 +152,21 @@ __global__ void __launch_bounds__(GP, 1024 / GP) coeffs_kernel(
   }
 }
 
-// One block per group: coefficients, then g_b = sum_i a_i s_{b,i} streamed
-// over D with 16-byte loads; rows with a_i == 0 are never read.
+// g_b = sum_i a_i s_{b,i} for one group, given its coefficients a_s[0..G) in
+// shared memory (block-wide call): the nonzero coefficients are listed, then
+// S is streamed over D with 16-byte loads; rows with a_i == 0 are never read.
 template <int GP>
-__global__ void __launch_bounds__(256, 4) dense_kernel(
-    int B, int G, int D, const float *__restrict__ r,
-    const uint8_t *__restrict__ J, const float *__restrict__ rho,
-    const float *__restrict__ S, float scale, float *__restrict__ g,
-    float *__restrict__ a_out, int32_t *dev_err) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  GroupSmem<GP> &sm = *reinterpret_cast<GroupSmem<GP> *>(smem_raw);
+__device__ __forceinline__ void dense_rows(int b, int G, int D, const float *a_s,
+                                           const float *__restrict__ S,
+                                           float *__restrict__ g) {
   __shared__ int rows[GP];
   __shared__ float coef[GP];
   __shared__ int n_rows;
-  const int b = blockIdx.x, tid = threadIdx.x;
-  int K, C;
-  uint8_t act;
-  group_coeffs<GP>(sm, b, G, r, J, rho, scale, false, dev_err, K, C, act);
-  if (a_out && tid < G) a_out[(size_t)b * G + tid] = sm.a[tid];
+  const int tid = threadIdx.x;
   if (tid == 0) {
     int n = 0;
     for (int i = 0; i < G; ++i)
-      if (sm.a[i] != 0.f) { rows[n] = i; coef[n] = sm.a[i]; ++n; }
+      if (a_s[i] != 0.f) { rows[n] = i; coef[n] = a_s[i]; ++n; }
     n_rows = n;
   }
   __syncthreads();
@@ -234,6 +227,70 @@ __global__ void __launch_bounds__(256, 4) dense_kernel(
       gb[c] = acc;
     }
   }
+}
+
+// One block per group: coefficients (general form), then dense_rows.
+template <int GP>
+__global__ void __launch_bounds__(256, 4) dense_kernel(
+    int B, int G, int D, const float *__restrict__ r,
+    const uint8_t *__restrict__ J, const float *__restrict__ rho,
+    const float *__restrict__ S, float scale, float *__restrict__ g,
+    float *__restrict__ a_out, int32_t *dev_err) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  GroupSmem<GP> &sm = *reinterpret_cast<GroupSmem<GP> *>(smem_raw);
+  const int b = blockIdx.x, tid = threadIdx.x;
+  int K, C;
+  uint8_t act;
+  group_coeffs<GP>(sm, b, G, r, J, rho, scale, false, dev_err, K, C, act);
+  if (a_out && tid < G) a_out[(size_t)b * G + tid] = sm.a[tid];
+  dense_rows<GP>(b, G, D, sm.a, S, g);
+}
+
+// The same for groups the streaming coefficient kernel takes (G <= 64, G a
+// multiple of 4, aligned inputs): warp 0 stages the group and collapses it
+// with warp_group_coeffs, so the coefficients are bit-identical to
+// pair_coeffs'.
+struct DenseStagedSmem {
+  int Qt[kGMax];
+  float a[kGMax];
+  __align__(16) unsigned char stage[kStageBytes];
+  __align__(16) unsigned char aux[kWarpAux];
+};
+
+__global__ void __launch_bounds__(256, 4) dense_staged_kernel(
+    int B, int G, int D, const float *__restrict__ r, const uint8_t *__restrict__ J,
+    const float *__restrict__ rho, const float *__restrict__ S, float scale,
+    float *__restrict__ g, float *__restrict__ a_out, int32_t *dev_err) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  DenseStagedSmem &sm = *reinterpret_cast<DenseStagedSmem *>(smem_raw);
+  const int b = blockIdx.x, tid = threadIdx.x;
+  stream_qt(G, sm.Qt);
+  __syncthreads();
+  if (tid < 32) {
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm.aux + 64 * 4 * 3);
+    volatile int *abort = reinterpret_cast<volatile int *>(bar + 2);
+    stream_init_gaps(sm.stage, G, sm.Qt);
+    if (tid == 0) {
+      tc::mbar_init(bar, 1);
+      *abort = 0;
+      tc::fence_mbar_init();
+    }
+    __syncwarp();
+    issue_group(sm.stage, bar, rho, r, J, b, G, stream_rows(G, sm.Qt));
+    const bool ok = __all_sync(0xffffffffu, tc::wait(bar, 0u, abort, dev_err));
+    if (!ok) drain_wait(bar, 0u);
+    cp_async_wait<0>();
+    __syncwarp();
+    WarpCoeffs o = {};
+    if (ok)
+      o = warp_group_coeffs<PAIR_W_HT, false>(sm.stage, sm.Qt, stream_diag(G, sm.Qt), G, scale,
+                                              0u, 0.f, sm.aux, dev_err);
+    sm.a[tid] = o.a0;
+    sm.a[tid + 32] = o.a1;
+  }
+  __syncthreads();
+  if (a_out && tid < G) a_out[(size_t)b * G + tid] = sm.a[tid];
+  dense_rows<kGMax>(b, G, D, sm.a, S, g);
 }
 
 // Coefficients under a weighting variant (see pair_coeffs_weighted), plus
@@ -415,6 +472,9 @@ pair_status launch_coeffs(int32_t B, int32_t G, const float *r,
                           uint32_t flags, float *a, uint8_t *active,
                           int32_t *edges, int32_t *contrast, int32_t *dev_err,
                           cudaStream_t s) {
+  if (coeffs_stream_applies(G, r, J, rho))
+    return launch_coeffs_stream(B, G, r, J, rho, scale, flags, PAIR_W_HT, false, 0.f, a, active,
+                                edges, contrast, nullptr, nullptr, dev_err, s);
   if (flags & PAIR_STANDARDIZE)  // HT through the weighted kernel (bit-identical HT terms)
     return launch_coeffs_weighted(B, G, r, J, rho, scale, flags, PAIR_W_HT, 0.f, a, active, edges,
                                   contrast, nullptr, nullptr, dev_err, s);
@@ -433,6 +493,10 @@ pair_status launch_coeffs_weighted(int32_t B, int32_t G, const float *r, const u
                                    float w_max, float *a, uint8_t *active, int32_t *edges,
                                    int32_t *contrast, float *ess, float *max_w,
                                    int32_t *dev_err, cudaStream_t s) {
+  if ((wmode == PAIR_W_HT || wmode == PAIR_W_CLIPPED || wmode == PAIR_W_HAJEK) &&
+      coeffs_stream_applies(G, r, J, rho))
+    return launch_coeffs_stream(B, G, r, J, rho, scale, flags, wmode, true, w_max, a, active,
+                                edges, contrast, ess, max_w, dev_err, s);
   if (G <= 32)
     return launch_coeffs_w_gp<32>(B, G, r, J, rho, scale, flags, wmode, w_max, a, active, edges,
                                   contrast, ess, max_w, dev_err, s);
@@ -462,6 +526,15 @@ pair_status launch_estimate_dense(int32_t B, int32_t G, int32_t D,
                                   const float *rho, const float *S,
                                   float scale, float *g, float *a,
                                   int32_t *dev_err, cudaStream_t s) {
+  if (coeffs_stream_applies(G, r, J, rho)) {
+    const size_t smem = sizeof(DenseStagedSmem);
+    PAIR_CUDA_TRY(cudaFuncSetAttribute(dense_staged_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    PAIR_BEGIN("dense", s);
+    dense_staged_kernel<<<B, 256, smem, s>>>(B, G, D, r, J, rho, S, scale, g, a, dev_err);
+    PAIR_LAUNCH_CHECK(s);
+    return PAIR_OK;
+  }
   if (G <= 32)
     return launch_dense_gp<32>(B, G, D, r, J, rho, S, scale, g, a, dev_err, s);
   if (G <= 64)

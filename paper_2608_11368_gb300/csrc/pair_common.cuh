@@ -48,6 +48,15 @@ pair_status launch_coeffs_weighted(int32_t B, int32_t G, const float *r, const u
                                    float w_max, float *a, uint8_t *active, int32_t *edges,
                                    int32_t *contrast, float *ess, float *max_w,
                                    int32_t *dev_err, cudaStream_t s);
+// Streaming coefficient kernel (pair_coeffs_stream.cu): G <= 64, G % 4 == 0,
+// 16-byte aligned r and rho, 4-byte aligned J. Weightings HT (diag = whether
+// ess / max_w are written), clipped and self-normalised.
+bool coeffs_stream_applies(int32_t G, const float *r, const uint8_t *J, const float *rho);
+pair_status launch_coeffs_stream(int32_t B, int32_t G, const float *r, const uint8_t *J,
+                                 const float *rho, float scale, uint32_t flags, int wmode,
+                                 bool diag, float w_max, float *a, uint8_t *active,
+                                 int32_t *edges, int32_t *contrast, float *ess, float *max_w,
+                                 int32_t *dev_err, cudaStream_t s);
 pair_status launch_coeffs_product(int32_t B, int32_t G, const float *r, const uint8_t *J,
                                   const float *p, float scale, uint32_t flags, float *a,
                                   uint8_t *active, int32_t *edges, int32_t *contrast, float *ess,

@@ -117,3 +117,67 @@ def test_coeffs_invalid_arguments():
     with pytest.raises(B.PairError):
         B.pair_coeffs(r, torch.zeros((2, 1), dtype=torch.uint8, device="cuda"),
                       torch.zeros((2, 1, 1), device="cuda"))
+
+
+def _boundary_inputs(seed, nb, G):
+    """Groups whose completed counts sit at the packing boundaries of the
+    streaming kernel (0, 1, 2, 31, 32, 33, 63, 64 completed, capped at G, at
+    random positions), the rest with a per-group completion rate; one group
+    carries NaN rewards on its incomplete rollouts, one signed-zero rewards,
+    one a zero diagonal of rho."""
+    rng = np.random.default_rng(seed)
+    r = rng.random((nb, G)).astype(np.float32)
+    r[::2] = (r[::2] < 0.5)
+    J = (rng.random((nb, G)) < rng.uniform(0.05, 1.0, (nb, 1))).astype(np.uint8)
+    for row, k in enumerate([0, 1, 2, 31, 32, 33, 63, 64]):
+        J[row] = 0
+        J[row, rng.permutation(G)[:min(k, G)]] = 1
+    r[8] = 1.0                      # equal rewards: no contrast edge
+    r[9][J[9] == 0] = np.nan        # rewards of rollouts that were not completed are unused
+    J[10] = 1
+    r[10, ::3] = -0.0               # -0 and +0 are equal rewards
+    r[10, 1::3] = 0.0
+    rho = rng.uniform(0.02, 1.0, (nb, G, G)).astype(np.float32)
+    rho[11, np.arange(G), np.arange(G)] = 0.0   # the diagonal is never read
+    return r, J, rho
+
+
+@pytest.mark.parametrize("G", [4, 8, 12, 16, 36, 60, 64])
+def test_coeffs_streaming_form(G):
+    """Groups of at most 64 candidates with G a multiple of 4 run as a
+    stream of groups per warp: completed counts at the packing boundaries,
+    4000 groups (more than the resident warps, so each warp runs several),
+    every flag combination, bit-identical reruns."""
+    B = _binding()
+    nb = 4000
+    r, J, rho = _boundary_inputs(600 + G, nb, G)
+    dr, dJ, drho = dev(r), dev(J), dev(rho)
+    for scale, flags in [(1.0, 0), (0.3, B.PAIR_CENTER), (1.0, B.PAIR_STANDARDIZE),
+                         (2.0, B.PAIR_STANDARDIZE | B.PAIR_CENTER)]:
+        err = dev_err_word()
+        out = B.pair_coeffs(dr, dJ, drho, scale=scale, flags=flags, dev_err=err)
+        assert B.pair_last_launch_count() == 1
+        assert B.pair_status_sync(err) == 0
+        center, std = bool(flags & B.PAIR_CENTER), bool(flags & B.PAIR_STANDARDIZE)
+        ref = oracle.coeffs_w(r, J, rho, scale=scale, center=center, standardize=std)
+        _check(ref, *out, tol=3e-6 if std else 1e-6, center=center)
+        again = B.pair_coeffs(dr, dJ, drho, scale=scale, flags=flags)
+        for x, y in zip(out, again):
+            assert torch.equal(x, y)
+
+
+def test_coeffs_misaligned_inputs_take_the_general_kernel():
+    """r four bytes off a 16-byte boundary: the general kernel runs, with
+    the same results up to rounding."""
+    B = _binding()
+    G, nb = 64, 300
+    r, J, rho = _boundary_inputs(77, nb, G)
+    store = torch.empty(nb * G + 1, dtype=torch.float32, device="cuda")
+    r_off = store[1:].view(nb, G)
+    r_off.copy_(torch.from_numpy(r).cuda())
+    assert r_off.data_ptr() % 16 != 0
+    out = B.pair_coeffs(r_off, dev(J), dev(rho))
+    _check(oracle.coeffs(r, J, rho), *out)
+    aligned = B.pair_coeffs(dev(r), dev(J), dev(rho))
+    for x, y in zip(out[1:], aligned[1:]):
+        assert torch.equal(x, y)

@@ -50,7 +50,7 @@ def _inputs(seed, B, G, pJ=0.6, lo=0.02):
     return r, J, p, rho
 
 
-@pytest.mark.parametrize("G", [2, 3, 17, 32, 33, 64, 65, 128])
+@pytest.mark.parametrize("G", [2, 3, 4, 12, 17, 32, 33, 36, 60, 64, 65, 128])
 @pytest.mark.parametrize("wmode", MODES)
 def test_weighted_parity(G, wmode):
     B = _binding()
@@ -137,7 +137,7 @@ def test_variant_host_validation():
     _check(ref, out)
 
 
-@pytest.mark.parametrize("G", [2, 9, 33, 64, 128])
+@pytest.mark.parametrize("G", [2, 8, 9, 33, 40, 64, 128])
 def test_standardised_parity(G):
     B = _binding()
     r, J, p, rho = _inputs(970 + G, 23, G)
