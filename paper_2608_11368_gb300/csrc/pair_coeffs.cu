@@ -260,11 +260,11 @@ struct DenseStagedSmem {
 __global__ void __launch_bounds__(256, 4) dense_staged_kernel(
     int B, int G, int D, const float *__restrict__ r, const uint8_t *__restrict__ J,
     const float *__restrict__ rho, const float *__restrict__ S, float scale,
-    float *__restrict__ g, float *__restrict__ a_out, int32_t *dev_err) {
+    float *__restrict__ g, float *__restrict__ a_out, int32_t *dev_err, const StreamGeom geom) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   DenseStagedSmem &sm = *reinterpret_cast<DenseStagedSmem *>(smem_raw);
   const int b = blockIdx.x, tid = threadIdx.x;
-  stream_qt(G, sm.Qt);
+  stream_qt(geom, sm.Qt);
   __syncthreads();
   if (tid < 32) {
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm.aux + 64 * 4 * 3);
@@ -276,7 +276,7 @@ __global__ void __launch_bounds__(256, 4) dense_staged_kernel(
       tc::fence_mbar_init();
     }
     __syncwarp();
-    issue_group(sm.stage, bar, rho, r, J, b, G, stream_rows(G, sm.Qt));
+    issue_group(sm.stage, bar, rho, r, J, b, G, stream_rows(G, sm.Qt, geom.group_bytes));
     const bool ok = __all_sync(0xffffffffu, tc::wait(bar, 0u, abort, dev_err));
     if (!ok) drain_wait(bar, 0u);
     cp_async_wait<0>();
@@ -531,7 +531,8 @@ pair_status launch_estimate_dense(int32_t B, int32_t G, int32_t D,
     PAIR_CUDA_TRY(cudaFuncSetAttribute(dense_staged_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     PAIR_BEGIN("dense", s);
-    dense_staged_kernel<<<B, 256, smem, s>>>(B, G, D, r, J, rho, S, scale, g, a, dev_err);
+    dense_staged_kernel<<<B, 256, smem, s>>>(B, G, D, r, J, rho, S, scale, g, a, dev_err,
+                                              make_stream_geom(G));
     PAIR_LAUNCH_CHECK(s);
     return PAIR_OK;
   }

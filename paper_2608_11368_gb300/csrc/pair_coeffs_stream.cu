@@ -18,7 +18,7 @@ namespace pairk {
 namespace {
 
 constexpr int kStages = 1;  // groups staged per warp
-constexpr int kSW = kStages == 1 ? 21 : 11;  // warps per block (as many as shared memory holds)
+constexpr int kSW = kStages == 1 ? 19 : 10;  // warps per block (as many as shared memory holds)
 
 static_assert(kStages == 1 || kStages == 2, "one or two stages per warp");
 
@@ -34,11 +34,11 @@ __global__ void __launch_bounds__(kSW * 32, 1) coeffs_stream_kernel(
     const float *__restrict__ rho, float scale, uint32_t flags, float w_max,
     float *__restrict__ a, uint8_t *__restrict__ active, int32_t *__restrict__ edges,
     int32_t *__restrict__ contrast, float *__restrict__ ess, float *__restrict__ max_w,
-    int32_t *dev_err) {
+    int32_t *dev_err, const StreamGeom geom) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   StreamSmem &sm = *reinterpret_cast<StreamSmem *>(smem_raw);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  stream_qt(G, sm.Qt);
+  stream_qt(geom, sm.Qt);
   __syncthreads();
 
   unsigned char *wbase = sm.warp[warp];
@@ -46,7 +46,7 @@ __global__ void __launch_bounds__(kSW * 32, 1) coeffs_stream_kernel(
   uint64_t *bar = reinterpret_cast<uint64_t *>(aux + 64 * 4 * 3);  // one per stage
   volatile int *abort = reinterpret_cast<volatile int *>(bar + kStages);
   const int2 dg = stream_diag(G, sm.Qt);
-  const RowCopies rc = stream_rows(G, sm.Qt);
+  const RowCopies rc = stream_rows(G, sm.Qt, geom.group_bytes);
 #pragma unroll
   for (int s = 0; s < kStages; ++s) stream_init_gaps(wbase + s * kStageBytes, G, sm.Qt);
   if (lane == 0) {
@@ -137,7 +137,8 @@ pair_status launch_stream(int32_t B, int32_t G, const float *r, const uint8_t *J
   const int blocks = (int)std::min<int64_t>(B, nsm > 0 ? nsm : 1);
   PAIR_BEGIN(DIAG ? "coeffs_w" : "coeffs", s);
   coeffs_stream_kernel<WM, DIAG><<<blocks, kSW * 32, smem, s>>>(
-      B, G, r, J, rho, scale, flags, w_max, a, active, edges, contrast, ess, max_w, dev_err);
+      B, G, r, J, rho, scale, flags, w_max, a, active, edges, contrast, ess, max_w, dev_err,
+      make_stream_geom(G));
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }

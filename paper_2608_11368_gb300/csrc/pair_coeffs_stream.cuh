@@ -9,9 +9,11 @@
 //
 // Staging: the strict upper triangle of rho_g is copied by bulk copies (one
 // per row) completing on an mbarrier, row i from column (i + 1) rounded down
-// to a multiple of 4 up to G - 1; each row is preceded by a 4-float gap.
-// Entry (i, j) then sits at float Qt[i] + j of the stage. Gap cells hold +inf
-// (written once), and
+// to a multiple of 4 up to G - 1; each row is preceded by a gap of at least
+// 4 floats, widened so that row bases fall in different shared-memory banks
+// (lanes reading one column of many rows then conflict less). Entry (i, j)
+// sits at float Qt[i] + j of the stage. Gap cells hold +inf (written once),
+// and
 // after each copy the staged diagonal cells are set to +inf too, so a read
 // of the diagonal, or of column G of any row (the next gap), gives weight
 // 1/inf = 0. Rewards and completion flags follow the triangle.
@@ -34,7 +36,7 @@ namespace pairk {
 namespace {
 
 constexpr int kGMax = 64;                               // largest group of this form
-constexpr int kTriFloats = 2112 + 4 * 65;               // G = 64 triangle rows and their gaps
+constexpr int kTriFloats = 2620;                        // largest staged triangle (G = 64)
 constexpr int kTriBytes = kTriFloats * 4;
 constexpr int kStageBytes = kTriBytes + 256 + 64;       // triangle, r[64], J[64]
 constexpr int kWarpAux = 64 * 4 * 3 + 32;               // packed r, column, Q; 2 barriers; abort
@@ -71,29 +73,53 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
-// Row geometry of this G. Row i (i <= G - 2) holds columns row_col0(i) ..
-// G - 1 and starts at float D_i, with D_0 = 4 and D_{i+1} = D_i + (its
-// length) + 4; row G - 1 has no entries (length 0), and 4 gap floats follow
-// it. Qt[v] = D_v - row_col0(v) (v <= G - 2), D_{G-1} - G (v = G - 1), so
-// column G of every row and the diagonal of row G - 1 land in a gap.
-__device__ __forceinline__ int row_start(int G, int v) {
-  int P = 0;
-  for (int i = 0; i < v && i < G - 1; ++i) P += G - row_col0(i);
-  return 4 * (v + 1) + P;
+// Row geometry of this G (host-computed once per G, passed by value). Row i
+// (i <= G - 2) holds columns row_col0(i) .. G - 1 and starts at float D_i;
+// row G - 1 has no entries and 4 gap floats follow it. Between rows there
+// are at least 4 gap floats, more where needed so that the bank of Q_i =
+// D_i - row_col0(i) (mod 32 words) differs from the previous three rows'.
+// Qt[v] = Q_v (v <= G - 2), D_{G-1} - G (v = G - 1), 0 (v >= G): column G
+// of every row, and the diagonal of a row whose staging starts at column
+// i + 1, then land in a gap.
+struct StreamGeom {
+  int Qt[kGMax];
+  uint32_t group_bytes;  // bulk-copied bytes of one group: triangle rows + rewards
+};
+
+inline StreamGeom make_stream_geom(int G) {
+  StreamGeom g = {};
+  int d = 4, recent[3] = {-1, -1, -1}, nrec = 0;
+  uint32_t tri = 0;
+  for (int i = 0; i < G; ++i) {
+    if (i <= G - 2) {
+      auto used = [&](int res) {
+        for (int k = 0; k < 3 && k < nrec; ++k)
+          if (recent[k] == res) return true;
+        return false;
+      };
+      while (used((d - row_col0(i)) & 31)) d += 4;
+      recent[nrec % 3] = (d - row_col0(i)) & 31;
+      ++nrec;
+      g.Qt[i] = d - row_col0(i);
+      tri += (uint32_t)(G - row_col0(i));
+      d += G - row_col0(i) + 4;
+    } else {
+      g.Qt[i] = d - G;
+    }
+  }
+  g.group_bytes = 4u * (tri + (uint32_t)G);
+  return g;
 }
 
-// Qt[v] for v < 64 (0 for v >= G); threads 0..63 of the block call, the
-// caller synchronises before use.
-__device__ __forceinline__ void stream_qt(int G, int *Qt) {
-  const int v = threadIdx.x;
-  if (v < kGMax) {
-    const int D = row_start(G, v);
-    Qt[v] = (v <= G - 2) ? D - row_col0(v) : (v == G - 1 ? D - G : 0);
-  }
+// Copies Qt into shared memory (threads 0..63 of the block; the caller
+// synchronises before use).
+__device__ __forceinline__ void stream_qt(const StreamGeom &geom, int *Qt) {
+  if (threadIdx.x < kGMax) Qt[threadIdx.x] = geom.Qt[threadIdx.x];
 }
 
 // Sets the gap cells of a stage to +inf (once per stage; copies never write
-// them). Whole warp calls.
+// them): the cells before each row and the 4 after row G - 1. Whole warp
+// calls.
 __device__ __forceinline__ void stream_init_gaps(unsigned char *stage, int G, const int *Qt) {
   float *tri = reinterpret_cast<float *>(stage);
   const int lane = threadIdx.x & 31;
@@ -102,8 +128,9 @@ __device__ __forceinline__ void stream_init_gaps(unsigned char *stage, int G, co
   for (int h = 0; h < 2; ++h) {
     const int i = lane + 32 * h;
     if (i < G) {
+      const int start = (i == 0) ? 0 : Qt[i - 1] + G;  // end of row i - 1
       const int D = (i <= G - 2) ? Qt[i] + row_col0(i) : Qt[i] + G;
-      for (int e = 1; e <= 4; ++e) tri[D - e] = inf;
+      for (int e = start; e < D; ++e) tri[e] = inf;
       if (i == G - 1)
         for (int e = 0; e < 4; ++e) tri[D + e] = inf;
     }
@@ -129,7 +156,7 @@ struct RowCopies {
   uint32_t group_bytes; // bytes of all bulk copies of one group (triangle + rewards)
 };
 
-__device__ __forceinline__ RowCopies stream_rows(int G, const int *Qt) {
+__device__ __forceinline__ RowCopies stream_rows(int G, const int *Qt, uint32_t group_bytes) {
   const int lane = threadIdx.x & 31;
   RowCopies rc;
   const int i0 = lane, i1 = lane + 32;
@@ -139,8 +166,7 @@ __device__ __forceinline__ RowCopies stream_rows(int G, const int *Qt) {
   rc.dst1 = (i1 <= G - 2) ? Qt[i1] + row_col0(i1) : 0;
   rc.by0 = (i0 <= G - 2) ? 4u * (uint32_t)(G - row_col0(i0)) : 0u;
   rc.by1 = (i1 <= G - 2) ? 4u * (uint32_t)(G - row_col0(i1)) : 0u;
-  // D_{G-1} = 4 G + (floats of all rows), and D_{G-1} = Qt[G-1] + G.
-  rc.group_bytes = 4u * (uint32_t)(Qt[G - 1] + G - 4 * G) + 4u * (uint32_t)G;
+  rc.group_bytes = group_bytes;
   return rc;
 }
 
@@ -327,6 +353,7 @@ __device__ WarpCoeffs warp_group_coeffs(unsigned char *stage, const int *Qt, int
   {
     const float ra = cr[lane], rb = cr[lane + 32];
     const int ob = co[lane + 32], qa = cq[lane], qb = cq[lane + 32];
+#pragma unroll 2
     for (int cx = 32; cx < K; ++cx) {
       const float rx = cr[cx];
       const int ox = co[cx], Qx = cq[cx];
