@@ -92,6 +92,18 @@ def code_hash(path):
     return hashlib.sha256("\n".join(lines).encode()).hexdigest()[:16]
 
 
+def sources_hash(src):
+    """code_hash of one file, or for a comma-separated list of files the
+    sha256[:16] of their code_hash values joined by commas (a kernel whose
+    code spans several files)."""
+    files = src.split(",")
+    if len(files) == 1:
+        return code_hash(os.path.join(ROOT, files[0]))
+    import hashlib
+    joined = ",".join(code_hash(os.path.join(ROOT, f)) for f in files)
+    return hashlib.sha256(joined.encode()).hexdigest()[:16]
+
+
 def load_traffic():
     """Per-call DRAM bytes from the committed ncu summary, keyed by kernel,
     valid only while the kernel source code is unchanged (hash recorded
@@ -106,7 +118,7 @@ def load_traffic():
             continue
         name, wl, bytes_, src, sha = parts[:5]
         try:
-            cur = code_hash(os.path.join(ROOT, src))
+            cur = sources_hash(src)
         except OSError:
             continue
         if cur == sha:

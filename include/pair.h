@@ -112,8 +112,14 @@ typedef enum { PAIR_F32 = 0, PAIR_BF16 = 1 } pair_dtype;
  *      contrast_edges [B] int32 observed edges with r_i != r_j (nullable).
  *      dev_err: device int32 error word (nullable; if null, device data
  *               errors are not reported).
- * Arithmetic: fp32, IEEE division, tree summation over the partners (a
- * relative error of a few ulp of sum_j |term_j|); deterministic.
+ * Arithmetic: fp32, fixed-order tree summation over the partners;
+ * deterministic (bit-identical reruns). For G <= 64 with G a multiple of 4
+ * and 16-byte aligned r and rho (4-byte aligned J) each term is
+ * (r_i - r_j) times the hardware reciprocal of rho_ij (within 1.5 ulp of the
+ * quotient; exactly 0 when r_i = r_j and exactly antisymmetric), and a rho
+ * below 2^-126 on a completed edge is reported like rho <= 0; otherwise the
+ * term is the IEEE quotient. Either way the error of a_i is a few ulp of
+ * 1/2 sum_j |term_j|.
  */
 PAIR_API pair_status pair_coeffs(int32_t B, int32_t G, const float *r, const uint8_t *J,
                         const float *rho, float scale, uint32_t flags,
@@ -160,7 +166,9 @@ typedef enum {
  *      wmode, or a non-positive / non-finite w_max with PAIR_W_CLIPPED;
  *      device: rho_ij <= 0 or NaN on a completed edge (pi_i, pi_j for
  *      PAIR_W_MARGINAL) -> PAIR_DEV_ERR_NONPOSITIVE_INCLUSION.
- * Arithmetic: fp32, IEEE division and reciprocal, fixed tree sums.
+ * Arithmetic: fp32, fixed tree sums; the weights of HT, clipped and
+ * self-normalised weighting as pair_coeffs' terms (the hardware reciprocal
+ * where pair_coeffs uses it, IEEE division and reciprocal otherwise).
  */
 PAIR_API pair_status pair_coeffs_weighted(int32_t B, int32_t G, const float *r,
                                           const uint8_t *J, const float *rho, float scale,

@@ -23,7 +23,7 @@
 // c then sums packed row c: per term one shared-memory load of rho, one
 // hardware reciprocal, one subtract, one multiply and one tree addition, with
 // no mask (the diagonal and the slots past K read +inf), and a running check
-// that rho > 0. Rows 32..K-1 (K > 32) are summed by the whole warp. Contrast
+// that rho >= 2^-126 (so a subnormal rho is reported like rho <= 0). Rows 32..K-1 (K > 32) are summed by the whole warp. Contrast
 // edges and active flags follow from the rewards alone (warp match on equal
 // rewards). Every sum has a fixed order (bit-identical reruns): a lane's row
 // is a pairwise tree of 8-term blocks, a warp-summed row a butterfly.
@@ -40,6 +40,7 @@ constexpr int kTriFloats = 2620;                        // largest staged triang
 constexpr int kTriBytes = kTriFloats * 4;
 constexpr int kStageBytes = kTriBytes + 256 + 64;       // triangle, r[64], J[64]
 constexpr int kWarpAux = 64 * 4 * 3 + 32;               // packed r, column, Q; 2 barriers; abort
+constexpr float kRhoMin = 1.17549435e-38f;              // 2^-126, smallest normal float
 
 using tc::smem_u32;
 __device__ __forceinline__ void cp_async16(void *dst, const void *src) {
@@ -215,7 +216,8 @@ __device__ __forceinline__ void issue_group(unsigned char *stage, uint64_t *bar,
 }
 
 // Reciprocal by the hardware approximation (PTX rcp.approx.ftz.f32: at most
-// 1 ulp, one instruction; 1/inf = 0; an input below 2^-126 counts as 0). A term (r_i - r_j) *
+// 1 ulp, one instruction; 1/inf = 0; an input below 2^-126 counts as 0,
+// which is why a completed edge's rho must be at least kRhoMin). A term (r_i - r_j) *
 // rcp(rho_ij) is then within 1.5 ulp of the quotient, is exactly 0 when
 // r_i = r_j, and is exactly antisymmetric (both directions use the same
 // weight).
@@ -247,7 +249,8 @@ __device__ __forceinline__ float weight_of(float rho, float w_max) {
 // copies completed and the warp synchronised; `dg` from stream_diag; `aux` is
 // the warp's kWarpAux bytes, 16-byte aligned). WM is the weighting, DIAG
 // whether the weight sums are wanted. Flags: PAIR_CENTER, PAIR_STANDARDIZE.
-// A device error bit is set for rho <= 0 or NaN on a completed edge.
+// A device error bit is set for rho < 2^-126 (zero, negative, subnormal) or NaN
+// on a completed edge.
 template <int WM, bool DIAG>
 __device__ WarpCoeffs warp_group_coeffs(unsigned char *stage, const int *Qt, int2 dg, int G,
                                         float scale, uint32_t flags, float w_max,
@@ -292,7 +295,7 @@ __device__ WarpCoeffs warp_group_coeffs(unsigned char *stage, const int *Qt, int
 
   // Sweep, rows 0..31: lane c sums row c over 8-term blocks (fixed 3-level
   // tree), the 8 block sums combined by a pairwise tree.
-  bool ok0 = true;  // every rho read by row c is > 0 (+inf cells pass)
+  bool ok0 = true;  // every rho read by row c is >= kRhoMin (+inf cells pass)
   float sw0 = 0.f, sq0 = 0.f, mw0 = 0.f, sum0;
   {
     float p[4];
@@ -314,7 +317,7 @@ __device__ WarpCoeffs warp_group_coeffs(unsigned char *stage, const int *Qt, int
         for (int u = 0; u < 8; ++u) {
           const int cp = blk * 8 + u;
           const float rho = tri[(cp < c) ? qv[u] + oc : Qc + ov[u]];
-          ok0 = ok0 && (rho > 0.f);
+          ok0 = ok0 && (rho >= kRhoMin);
           const float w = weight_of<WM>(rho, w_max);
           x[u] = (rc - rv[u]) * w;
           if (DIAG) {
@@ -359,7 +362,7 @@ __device__ WarpCoeffs warp_group_coeffs(unsigned char *stage, const int *Qt, int
       const int ox = co[cx], Qx = cq[cx];
       const float rho_a = tri[qa + ox];  // lane < 32 <= cx
       const float rho_b = tri[(lane + 32 < cx) ? qb + ox : Qx + ob];
-      okx = okx && (rho_a > 0.f) && (rho_b > 0.f);
+      okx = okx && (rho_a >= kRhoMin) && (rho_b >= kRhoMin);
       const float wa = weight_of<WM>(rho_a, w_max), wb = weight_of<WM>(rho_b, w_max);
       if (DIAG) {
         swx += wa + wb;

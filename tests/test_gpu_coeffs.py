@@ -181,3 +181,22 @@ def test_coeffs_misaligned_inputs_take_the_general_kernel():
     aligned = B.pair_coeffs(dev(r), dev(J), dev(rho))
     for x, y in zip(out[1:], aligned[1:]):
         assert torch.equal(x, y)
+
+
+def test_coeffs_streaming_form_reports_subnormal_rho():
+    """The streaming form (G a multiple of 4, at most 64) takes the hardware
+    reciprocal, so a completed edge's rho below 2^-126 is reported like
+    rho <= 0; on an edge that was not observed it is never read."""
+    B = _binding()
+    G = 8
+    r = np.tile(np.array([1, 0, 1, 0, 1, 0, 1, 0], np.float32), (2, 1))
+    rho = np.full((2, G, G), 0.5, np.float32)
+    rho[:, 0, 1] = np.float32(1e-39)          # subnormal
+    J = np.ones((2, G), np.uint8)
+    err = dev_err_word()
+    B.pair_coeffs(dev(r), dev(J), dev(rho), dev_err=err)
+    assert B.pair_status_sync(err) == 4
+    J[:, 1] = 0
+    out = B.pair_coeffs(dev(r), dev(J), dev(rho), dev_err=err)
+    assert B.pair_status_sync(err) == 0
+    _check(oracle.coeffs(r, J, rho), *out)
