@@ -39,9 +39,15 @@ constexpr double kTMul = 16.0;          // barrier parameter growth per centring
 // of F_t ~ t Phi near the end of the path.
 constexpr double kCentred = 1e-6;
 
+// Groups of up to 64 keep the edge proxies a_ij in shared memory (fp64, as
+// computed on the fly otherwise); the 128-candidate form has no room for them.
+template <int GP>
+constexpr bool kEdgeTable = GP <= 64;
+
 template <int GP>
 struct AllocSmem {
   double H[GP][GP + 1];  // Newton system, factorised in place (lower triangle)
+  double A[kEdgeTable<GP> ? GP : 1][kEdgeTable<GP> ? GP + 1 : 1];  // a_ij (see kEdgeTable)
   double c[GP], b[GP], dx[GP];
   double dinv[GP];       // 1 / L_kk of the current factorisation
   float p[GP], m[GP];
@@ -86,6 +92,14 @@ __device__ __forceinline__ double edge(const AllocIn &in, const AllocSmem<GP> &s
   return d;
 }
 
+// a_ij from the table where there is one (same fp64 value as edge()).
+template <int GP>
+__device__ __forceinline__ double edge_at(const AllocIn &in, const AllocSmem<GP> &sm, int i,
+                                          int j) {
+  if constexpr (kEdgeTable<GP>) return sm.A[i][j];
+  else return edge<GP>(in, sm, i, j);
+}
+
 // Phi, the budget slack and this coordinate's S_i = sum_j a_ij u_j at x_i
 // (u_i = e^x_i held by thread i, shared through sm.dx as scratch).
 template <int GP>
@@ -98,7 +112,7 @@ __device__ void eval(const AllocIn &in, AllocSmem<GP> &sm, bool act, double x, d
   __syncthreads();
   S = 0.0;
   if (act)
-    for (int j = 0; j < in.G; ++j) S += edge<GP>(in, sm, threadIdx.x, j) * sm.dx[j];
+    for (int j = 0; j < in.G; ++j) S += edge_at<GP>(in, sm, threadIdx.x, j) * sm.dx[j];
   phi = block_sum<GP>(sm, act ? u * (0.5 * S + sm.b[threadIdx.x]) : 0.0);
   slack = budget - block_sum<GP>(sm, e);
 }
@@ -153,13 +167,18 @@ __global__ void __launch_bounds__(GP, 1) alloc_kernel(int G, const float *p_hat,
   __syncthreads();
   const bool invalid = sm.any != 0;
   const double sc = sm.sum_c, pmin = (double)pi_min, X = -log(pmin);
+  if constexpr (kEdgeTable<GP>) {
+    if (act && !invalid)
+      for (int j = 0; j < G; ++j) sm.A[i][j] = edge<GP>(in, sm, i, j);
+    __syncthreads();
+  }
 
   // ---- b_i = (sum_{j != i} sqrt a_ij)^2 - sum_{j != i} a_ij
   double bi = 0.0, asum = 0.0;
   if (act && !invalid) {
     double sq = 0.0;
     for (int j = 0; j < G; ++j) {
-      const double v = edge<GP>(in, sm, i, j);
+      const double v = edge_at<GP>(in, sm, i, j);
       sq += sqrt(v);
       asum += v;
     }
@@ -210,20 +229,21 @@ __global__ void __launch_bounds__(GP, 1) alloc_kernel(int G, const float *p_hat,
           if (j == i)
             h += t * u * (S + sm.b[i]) + e / slack + bnd_lo * bnd_lo + bnd_hi * bnd_hi;
           else
-            h += t * edge<GP>(in, sm, i, j) * u * sm.dx[j];
+            h += t * edge_at<GP>(in, sm, i, j) * u * sm.dx[j];
           sm.H[i][j] = h;
         }
       }
       // Cholesky (lower triangle, in place); each pivot's inverse is formed
-      // once, so the column scaling and both substitutions multiply.
+      // once, so the column scaling and both substitutions multiply. One
+      // reciprocal square root per pivot gives both 1/L_kk and L_kk = d/sqrt(d).
       bool spd = true;
       for (int k = 0; k < G; ++k) {
         __syncthreads();
         if (i == k) {
           const double d = sm.H[k][k];
-          const double l = d > 0.0 ? sqrt(d) : 0.0;
-          sm.H[k][k] = l;
-          sm.dinv[k] = l > 0.0 ? 1.0 / l : 0.0;
+          const double rs = d > 0.0 ? rsqrt(d) : 0.0;
+          sm.H[k][k] = d * rs;
+          sm.dinv[k] = rs;
         }
         __syncthreads();
         if (sm.H[k][k] == 0.0) spd = false;
