@@ -39,7 +39,12 @@ __global__ void __launch_bounds__(kSW * 32, 1) coeffs_stream_kernel(
   StreamSmem &sm = *reinterpret_cast<StreamSmem *>(smem_raw);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   stream_qt(geom, sm.Qt);
-  __syncthreads();
+  __syncthreads();  // the only block-wide barrier: warps are independent after it
+  // Groups dealt warp-major (b = warp * blocks + block, stride all warps),
+  // so every SM gets the same number of groups to within one per warp row.
+  const int nw = gridDim.x * kSW;
+  const int b0 = warp * gridDim.x + blockIdx.x;
+  if (b0 >= B) return;  // no group for this warp (small batches)
 
   unsigned char *wbase = sm.warp[warp];
   unsigned char *aux = wbase + kStages * kStageBytes;
@@ -56,10 +61,6 @@ __global__ void __launch_bounds__(kSW * 32, 1) coeffs_stream_kernel(
   }
   __syncwarp();
 
-  // Groups dealt warp-major (b = warp * blocks + block, stride all warps),
-  // so every SM gets the same number of groups to within one per warp row.
-  const int nw = gridDim.x * kSW;
-  const int b0 = warp * gridDim.x + blockIdx.x;
   uint32_t ph = 0;       // bit s: parity of the next completion of stage s
   uint32_t pending = 0;  // bit s: stage s has copies issued and not yet waited for
 #pragma unroll
