@@ -38,6 +38,11 @@ constexpr double kTMul = 16.0;          // barrier parameter growth per centring
 // bound (2G + 1) / t; a tighter threshold would sit under fp64 resolution
 // of F_t ~ t Phi near the end of the path.
 constexpr double kCentred = 1e-6;
+// A line search stops once the decrease its step could bring, step * lambda^2,
+// is below this many fp64 units of |F_t|: such a decrease cannot be told from
+// rounding, so halving further only repeats function evaluations (the point
+// is then treated as centred, as after a failed search).
+constexpr double kResolution = 16.0 * 2.220446049250313e-16;
 
 // Groups of up to 64 keep the edge proxies a_ij in shared memory (fp64, as
 // computed on the fly otherwise); the 128-candidate form has no room for them.
@@ -301,6 +306,8 @@ __global__ void __launch_bounds__(GP, 1) alloc_kernel(int G, const float *p_hat,
                         block_sum<GP>(sm, act ? log(x) + log(X - x) : 0.0);
       bool moved = false;
       for (int ls = 0; ls < kAllocMaxBacktrack; ++ls) {
+        // step, lam2 and F0 are the same in every thread: the exit is uniform.
+        if (step * lam2 < kResolution * fabs(F0)) break;
         const double xt = x + step * d;
         double ut, et, St, phit, slackt;
         eval<GP>(in, sm, act, xt, budget, ut, et, St, phit, slackt);
