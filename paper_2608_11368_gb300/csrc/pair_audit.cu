@@ -18,7 +18,7 @@
 namespace pairk {
 namespace {
 
-constexpr int kAuditBlocks = 1024;  // partial-sum slots (draw b -> block b mod grid)
+constexpr int kAuditBlocks = 4096;  // partial-sum slots (draw b -> block b mod grid), at most
 constexpr int kAuditStats = 8;
 
 // Deterministic block sum of one double per thread (all threads call).
@@ -154,18 +154,23 @@ __global__ void audit_finish_kernel(int nblk, int G, int GP, int D, const float 
   __shared__ double red[32];
   __shared__ double tot[6];
   const int tid = threadIdx.x;
-  if (tid < 6) {
+  // Each column of the partials (6 statistics, then G coefficient sums) is
+  // summed by every thread over a strided share of the blocks, then by the
+  // block reduction: a fixed order, and the loads of a column in flight
+  // together.
+  for (int k = 0; k < 6 + G; ++k) {
+    const int col = k < 6 ? k : kAuditStats + (k - 6);
     double s = 0.0;
-    for (int q = 0; q < nblk; ++q) s += part[(size_t)q * (kAuditStats + GP) + tid];
-    tot[tid] = s;
+    for (int q = tid; q < nblk; q += blockDim.x) s += part[(size_t)q * (kAuditStats + GP) + col];
+    const double t = block_sum_double(s, red);
+    if (tid == 0) {
+      if (k < 6) tot[k] = t;
+      else em[k - 6] = t;
+    }
   }
   __syncthreads();
   const double W = tot[5];
-  if (tid < G) {
-    double s = 0.0;
-    for (int q = 0; q < nblk; ++q) s += part[(size_t)q * (kAuditStats + GP) + kAuditStats + tid];
-    em[tid] = (W > 0.0 ? s / W : 0.0) - abar[tid];
-  }
+  if (tid < G) em[tid] = (W > 0.0 ? em[tid] / W : 0.0) - abar[tid];
   __syncthreads();
   double Ke = 0.0;
   if (tid < G)
@@ -198,10 +203,19 @@ pair_status launch_audit_gp(int N, int G, int D, const float *r, const float *rh
   PAIR_BEGIN("audit_target", s);
   audit_target_kernel<<<1, 128, 0, s>>>(G, r, scale, K, abar, u, gg);
   PAIR_LAUNCH_CHECK(s);
-  const int nblk = N < kAuditBlocks ? N : kAuditBlocks;
+  // As many blocks as the SMs hold at once (the draws loop is latency bound,
+  // one group per block), at most the kAuditBlocks partial slots.
   const size_t smem = sizeof(AuditSmem<GP>);
   PAIR_CUDA_TRY(cudaFuncSetAttribute(audit_draws_kernel<GP>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  int dev = 0, nsm = 0, per_sm = 0;
+  PAIR_CUDA_TRY(cudaGetDevice(&dev));
+  PAIR_CUDA_TRY(cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev));
+  PAIR_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, audit_draws_kernel<GP>, GP,
+                                                              smem));
+  int nblk = (nsm > 0 ? nsm : 1) * (per_sm > 0 ? per_sm : 1);
+  if (nblk > kAuditBlocks) nblk = kAuditBlocks;
+  if (nblk > N) nblk = N;
   PAIR_BEGIN("audit_draws", s);
   audit_draws_kernel<GP><<<nblk, GP, smem, s>>>(N, G, r, rho, Jd, wd, scale,
                                                 (int)flags, wmode, w_max, K,
