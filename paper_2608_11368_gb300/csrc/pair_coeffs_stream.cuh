@@ -13,20 +13,20 @@
 // 4 floats, widened so that row bases fall in different shared-memory banks
 // (lanes reading one column of many rows then conflict less). Entry (i, j)
 // sits at float Qt[i] + j of the stage. Gap cells hold +inf (written once),
-// and
-// after each copy the staged diagonal cells are set to +inf too, so a read
-// of the diagonal, or of column G of any row (the next gap), gives weight
-// 1/inf = 0. Rewards and completion flags follow the triangle.
+// and after each copy the staged diagonal cells are set to +inf too, so a
+// read of the diagonal, or of column G of any row (the next gap), gives
+// weight 1/inf = 0. Rewards and completion flags follow the triangle.
 //
 // Collapse: only completed vertices take part in an edge, so the warp packs
 // them to the front (K of G, vertex order); slots past K name column G. Lane
 // c then sums packed row c: per term one shared-memory load of rho, one
 // hardware reciprocal, one subtract, one multiply and one tree addition, with
 // no mask (the diagonal and the slots past K read +inf), and a running check
-// that rho >= 2^-126 (so a subnormal rho is reported like rho <= 0). Rows 32..K-1 (K > 32) are summed by the whole warp. Contrast
-// edges and active flags follow from the rewards alone (warp match on equal
-// rewards). Every sum has a fixed order (bit-identical reruns): a lane's row
-// is a pairwise tree of 8-term blocks, a warp-summed row a butterfly.
+// that rho >= 2^-126 (so a subnormal rho is reported like rho <= 0). Rows
+// 32..K-1 (K > 32) are summed by the whole warp. Contrast edges and active
+// flags follow from the rewards alone (warp match on equal rewards). Every
+// sum has a fixed order (bit-identical reruns): a lane's row is a pairwise
+// tree of 8-term blocks, a warp-summed row a butterfly.
 #pragma once
 
 #include "pair_coeffs_dev.cuh"
@@ -43,10 +43,6 @@ constexpr int kWarpAux = 64 * 4 * 3 + 32;               // packed r, column, Q; 
 constexpr float kRhoMin = 1.17549435e-38f;              // 2^-126, smallest normal float
 
 using tc::smem_u32;
-__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src)
-               : "memory");
-}
 __device__ __forceinline__ void cp_async4(void *dst, const void *src) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src)
                : "memory");
@@ -74,7 +70,7 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
-// Row geometry of this G (host-computed once per G, passed by value). Row i
+// Row geometry of this G (built on the host at each launch, passed by value). Row i
 // (i <= G - 2) holds columns row_col0(i) .. G - 1 and starts at float D_i;
 // row G - 1 has no entries and 4 gap floats follow it. Between rows there
 // are at least 4 gap floats, more where needed so that the bank of Q_i =
