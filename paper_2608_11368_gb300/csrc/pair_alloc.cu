@@ -115,7 +115,7 @@ template <int GP>
 __device__ void eval(const AllocIn &in, AllocSmem<GP> &sm, bool act, double x, double budget,
                      double &u, double &e, double &S, double &phi, double &slack) {
   u = act ? exp(x) : 0.0;
-  e = act ? sm.c[threadIdx.x] * exp(-x) : 0.0;
+  e = act ? sm.c[threadIdx.x] / u : 0.0;  // c e^-x without a second exp
   __syncthreads();
   sm.dx[threadIdx.x] = u;
   __syncthreads();
@@ -224,20 +224,23 @@ __global__ void __launch_bounds__(GP, 1) alloc_kernel(int G, const float *p_hat,
     while (newton < kAllocMaxNewton && !done) {
       ++newton;
       // Gradient and Hessian of F_t at x.
-      const double bnd_lo = act ? 1.0 / x : 0.0, bnd_hi = act ? 1.0 / (X - x) : 0.0;
+      // 1/x and 1/(X - x) from one division; 1/slack once per step.
+      const double rr = act ? 1.0 / (x * (X - x)) : 0.0;
+      const double bnd_lo = act ? (X - x) * rr : 0.0, bnd_hi = act ? x * rr : 0.0;
+      const double inv_s = 1.0 / slack;
       const double gi =
-          act ? t * u * (S + sm.b[i]) - e / slack - bnd_lo + bnd_hi : 0.0;
+          act ? t * u * (S + sm.b[i]) - e * inv_s - bnd_lo + bnd_hi : 0.0;
       // u_j and e_j for the Hessian rows (e_j in H's spare column).
       __syncthreads();
       sm.dx[i] = u;
       if (act) sm.H[i][GP] = e;
       __syncthreads();
       if (act) {
-        const double inv_s2 = 1.0 / (slack * slack);
+        const double inv_s2 = inv_s * inv_s;
         for (int j = 0; j <= i; ++j) {
           double h = e * sm.H[j][GP] * inv_s2;
           if (j == i)
-            h += t * u * (S + sm.b[i]) + e / slack + bnd_lo * bnd_lo + bnd_hi * bnd_hi;
+            h += t * u * (S + sm.b[i]) + e * inv_s + bnd_lo * bnd_lo + bnd_hi * bnd_hi;
           else
             h += t * edge_at<GP>(in, sm, i, j) * u * sm.dx[j];
           sm.H[i][j] = h;
@@ -308,7 +311,7 @@ __global__ void __launch_bounds__(GP, 1) alloc_kernel(int G, const float *p_hat,
       __syncthreads();
       double step = fmin(1.0, 0.99 * sm.red[0]);
       const double F0 = t * phi - log(slack) -
-                        block_sum<GP>(sm, act ? log(x) + log(X - x) : 0.0);
+                        block_sum<GP>(sm, act ? log(x * (X - x)) : 0.0);
       bool moved = false;
       for (int ls = 0; ls < kAllocMaxBacktrack; ++ls) {
         // step, lam2 and F0 are the same in every thread: the exit is uniform.
@@ -319,7 +322,7 @@ __global__ void __launch_bounds__(GP, 1) alloc_kernel(int G, const float *p_hat,
         bool ok = slackt > 0.0;
         if (ok) {
           const double Ft = t * phit - log(slackt) -
-                            block_sum<GP>(sm, act ? log(xt) + log(X - xt) : 0.0);
+                            block_sum<GP>(sm, act ? log(xt * (X - xt)) : 0.0);
           // Strict decrease as well: at fp64 resolution of F_t a step can
           // pass Armijo without changing anything.
           ok = Ft < F0 && Ft <= F0 - 0.01 * step * lam2;
