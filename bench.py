@@ -11,9 +11,12 @@ pair_grad tokens/s (packed tokens per second, forward + backward); the JSON
 line also carries pair_coeffs / pair_estimate_dense GB/s on the
 4096 x 64 coefficient stress workload.
 
-Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
-For N > 1 launch with torch.distributed.run; each rank runs its own batch
-(groups are independent: weak scaling, no data-path collective).
+Usage: python bench.py [--steps K] [--warmup W] [--impl gb300|reference]
+The library is single-GPU: its tensor-core kernels multicast TMA tiles within
+a thread-block cluster of this GPU, and every call runs on the current device
+alone. --gpus N with N > 1 (or a torchrun launch with WORLD_SIZE > 1) exits
+with an error for the GPU arm; the reference arm (the fp64 CPU oracle) runs
+on rank 0 only.
 """
 from __future__ import annotations
 
@@ -39,12 +42,14 @@ WORKLOAD = "qwen3_1p7b_head"
 STRESS = "coeffs_dense_stress"
 METRIC = "pair_grad tokens/s (fwd+bwd) and % dense-BF16 peak; pair_coeffs GB/s vs HBM"
 FLUSH_BYTES = 256 << 20          # > 129 MB L2
-CPU_SAMPLE_TOKENS = 256          # oracle sample for the CPU baseline
-REF_SAMPLE_TOKENS = 48           # oracle sample per --impl reference step
-# Tensor-core kernels of one pair_grad call; each is charged one logit-sized
-# GEMM (2 T_eff V d FLOP) of algorithmic work per call, whatever the number of
-# token chunks it is launched for.
-TC_KERNELS = ("lse_tc", "bwd_dh_tc", "bwd_dw_tc", "dh_gemm_tc", "dw_gemm_tc")
+ORACLE_SAMPLE_TOKENS = 256       # active tokens of the oracle sample (both CPU legs)
+EXTRA_WORKLOADS = ("qwen3_4b_head", "longctx_skew")
+EXTRA_STEPS, EXTRA_WARMUP = 3, 3
+# Tensor-core kernels of one pair_grad call and the logit-sized GEMMs
+# (2 T_eff V d FLOP each) of algorithmic work each is charged per call,
+# whatever the number of token chunks it is launched for.
+TC_KERNELS = {"lse_tc": 1, "bwd_dh_tc": 1, "bwd_dw_tc": 1, "dh_gemm_tc": 1, "dw_gemm_tc": 1,
+              "lse_dh_tc": 2}
 
 
 def parse_args():
@@ -56,6 +61,8 @@ def parse_args():
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-stress", action="store_true")
+    p.add_argument("--no-onchip", action="store_true")
+    p.add_argument("--no-extra", action="store_true")
     # Smaller variants of the workload, for profiling captures only.
     p.add_argument("--workload", default=WORKLOAD,
                    choices=["qwen3_1p7b_head", "qwen3_4b_head", "longctx_skew"])
@@ -196,67 +203,99 @@ def cores():
 
 # ------------------------------------------------------------- CPU oracle leg
 
-def oracle_sample_time(inp, n_tok):
-    """Time the fp64 oracle (as it stands) on the coefficients of every group
-    plus the complete head work (lse, logp, dH rows, dW contribution over all
-    V rows) of the first n_tok active tokens. Returns (seconds for the sample,
-    seconds for the coefficients, T_eff)."""
-    import oracle
-    t0 = time.perf_counter()
-    c = oracle.coeffs(inp["r"], inp["J"], inp["rho"])
-    t_coef = time.perf_counter() - t0
-    a = c["a"].reshape(-1)
-    idx, cc, _ = oracle.compact_tokens(inp["cu_seqlens"], inp["mask"], a)
-    sub = idx[:n_tok]
-    W64 = synth.as_float(inp["W"], inp["dtype"]).astype(np.float64)
-    Hs = synth.as_float(inp["H"][sub], inp["dtype"]).astype(np.float64)
-    ys = inp["y"][sub]
-    t0 = time.perf_counter()
-    lse, zy = oracle.head_lse(Hs, W64, ys)
-    oracle.head_dh_rows(Hs, W64, ys, cc[:sub.size], lse)
-    oracle.head_dw_rows(Hs, W64, ys, cc[:sub.size], lse, np.arange(inp["V"]))
-    t_head = time.perf_counter() - t0
-    return t_head, t_coef, int(idx.size), int(sub.size)
+class OracleSample:
+    """The fp64 oracle (as it stands) on a bounded sample of one step: the
+    coefficients of every group plus the complete head work (lse, logp, dH
+    rows, dW contribution over all V rows) of the first n_tok active tokens.
+    Both CPU legs (cpu_baseline and --impl reference) time this same sample;
+    the full step is extrapolated by T_eff / n_tok."""
+
+    def __init__(self, inp, n_tok):
+        import oracle
+        self.oracle = oracle
+        self.inp = inp
+        c = oracle.coeffs(inp["r"], inp["J"], inp["rho"])
+        idx, cc, _ = oracle.compact_tokens(inp["cu_seqlens"], inp["mask"], c["a"].reshape(-1))
+        self.T_eff = int(idx.size)
+        sub = idx[:n_tok]
+        self.n = int(sub.size)
+        # Upcasts (untimed): the oracle works on fp64 copies of the bf16 inputs.
+        self.W64 = synth.as_float(inp["W"], inp["dtype"]).astype(np.float64)
+        self.Hs = synth.as_float(inp["H"][sub], inp["dtype"]).astype(np.float64)
+        self.ys = inp["y"][sub]
+        self.cs = cc[:sub.size]
+
+    def run(self):
+        """Seconds of (coefficients, head sample)."""
+        o, inp = self.oracle, self.inp
+        t0 = time.perf_counter()
+        o.coeffs(inp["r"], inp["J"], inp["rho"])
+        t_coef = time.perf_counter() - t0
+        t0 = time.perf_counter()
+        lse, _ = o.head_lse(self.Hs, self.W64, self.ys)
+        o.head_dh_rows(self.Hs, self.W64, self.ys, self.cs, lse)
+        o.head_dw_rows(self.Hs, self.W64, self.ys, self.cs, lse, np.arange(inp["V"]))
+        return t_coef, time.perf_counter() - t0
+
+    def full_step_s(self, t_coef, t_head):
+        return t_coef + t_head * self.T_eff / max(self.n, 1)
+
+    def describe(self, measured_s):
+        return ("fp64 oracle: coefficients of all %d groups + full head work (lse, dH rows, "
+                "dW over all V) of %d of %d active tokens; measured %.2f s per sample, step "
+                "time extrapolated by T_eff/%d" % (self.inp["B"], self.n, self.T_eff, measured_s,
+                                                   self.n))
 
 
 def cpu_baseline(inp):
-    t_head, t_coef, T_eff, n = oracle_sample_time(inp, CPU_SAMPLE_TOKENS)
-    est = t_coef + t_head * T_eff / max(n, 1)
-    return {"value": inp["T"] / est, "unit": "tokens/s", "cores": cores(),
-            "kind": "oracle",
-            "sample": ("fp64 oracle: coefficients of all %d groups + full head "
-                       "work (lse, dH rows, dW over all V) of %d of %d active "
-                       "tokens, %.1f s; step time extrapolated by T_eff/%d"
-                       % (inp["B"], n, T_eff, t_head + t_coef, n))}
+    smp = OracleSample(inp, ORACLE_SAMPLE_TOKENS)
+    t_coef, t_head = smp.run()
+    est = smp.full_step_s(t_coef, t_head)
+    return {"value": inp["T"] / est, "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+            "measured_sample_s": t_coef + t_head, "extrapolated_step_s": est,
+            "sample": smp.describe(t_coef + t_head)}
 
 
-def run_reference(args, rank, world):
+def bench_config(args, wl, inp, T_eff):
+    """The `config` object of both arms' JSON lines."""
+    return {"workload": args.workload, "len_scale": args.len_scale, "d": inp["d"],
+            "V": inp["V"], "global_batch": wl.B * wl.G, "prompts": wl.B,
+            "rollouts_per_prompt": wl.G, "tokens_packed": inp["T"], "tokens_active": T_eff,
+            "l2": "flushed between timed steps (256 MiB write); inputs exceed L2",
+            "parallelism": "single GPU"}
+
+
+def run_reference(args, rank):
+    """The reference arm: the fp64 oracle as it stands on the host cores, one
+    bounded sample per step (the same sample as the GPU arm's cpu_baseline);
+    ms_per_step is the measured time of that sample, value the packed tokens
+    of the full step over its extrapolated time."""
     if rank != 0:
         return 0
-    wl = synth.WORKLOADS[WORKLOAD]
-    inp = synth.make_head_workload(wl, args.seed)
-    times = []
-    T_eff = n = 0
-    t_coef = 0.0
+    wl = synth.WORKLOADS[args.workload]
+    kw = {"V": args.vocab} if args.vocab else {}
+    inp = synth.make_head_workload(wl, args.seed, len_scale=args.len_scale, **kw)
+    smp = OracleSample(inp, ORACLE_SAMPLE_TOKENS)
+    measured, full = [], []
     for k in range(args.warmup + args.steps):
-        t_head, t_coef, T_eff, n = oracle_sample_time(inp, REF_SAMPLE_TOKENS)
+        t_coef, t_head = smp.run()
         if k >= args.warmup:
-            times.append(t_coef + t_head * T_eff / max(n, 1))
-    step_s = statistics.mean(times)
-    value = inp["T"] * world / step_s
+            measured.append(t_coef + t_head)
+            full.append(smp.full_step_s(t_coef, t_head))
+    meas_s = statistics.mean(measured)
+    step_s = statistics.mean(full)
+    value = inp["T"] / step_s
     line = {"impl": "reference", "metric": METRIC, "value": value,
-            "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+            "unit": "tokens/s", "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": meas_s * 1e3,
+            "extrapolated_full_step_ms": step_s * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "global_batch": wl.B * wl.G * world,
-                       "tokens_packed": inp["T"], "tokens_active": T_eff,
-                       "parallelism": "replicas"},
+            "dtype": "f64", "data": "synthetic (seeded; Qwen3-1.7B head shapes, random-init weights)",
+            "config": bench_config(args, wl, inp, smp.T_eff),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores(),
-                             "kind": "oracle",
-                             "sample": "per step: coefficients of all groups + "
-                                       "full head work of %d active tokens, "
-                                       "extrapolated to T_eff=%d" % (n, T_eff)},
+                             "kind": "oracle", "measured_sample_s": meas_s,
+                             "extrapolated_step_s": step_s,
+                             "sample": "per step: " + smp.describe(meas_s)},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -265,39 +304,98 @@ def run_reference(args, rank, world):
 
 # ----------------------------------------------------------------- GPU leg
 
+def timed_steps(B, torch, step, steps, flush):
+    """Per-step device times (CUDA events on the current stream, L2 flushed
+    before each step) and the library's per-kernel event timings."""
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    torch.cuda.synchronize()
+    B.pair_timing_enable(True)
+    for k in range(steps):
+        flush.zero_()
+        ev[k][0].record()
+        step()
+        ev[k][1].record()
+    torch.cuda.synchronize()
+    kern = B.pair_timing_read()
+    B.pair_timing_enable(False)
+    return [s.elapsed_time(e) for s, e in ev], kern
+
+
+def kernel_report(kern, steps, T_eff, V, d, peaks, traffic, workload):
+    """Roofline of the dominant kernel and the per-kernel breakdown of one
+    pair_grad call. Each tensor-core kernel is charged its algorithmic share of
+    the head's three logit-sized GEMMs (2 T_eff V d FLOP each): one, or two for
+    the fused log-sum-exp + dH pass. One "launch" is the kernel's whole share of
+    one call (the sum over its token-chunk launches)."""
+    agg = {}
+    for name, ms in kern:
+        n, tot = agg.get(name, (0, 0.0))
+        agg[name] = (n + 1, tot + ms)
+    flops_gemm = 2.0 * T_eff * V * d
+    dominant = max(agg.items(), key=lambda kv: kv[1][1])[0]
+    dn, dt_ms = agg[dominant]
+    dom_avg = dt_ms / steps
+    dom_flops = flops_gemm * TC_KERNELS[dominant] if dominant in TC_KERNELS else None
+    achieved = dom_flops / (dom_avg / 1e3) / 1e12 if dom_flops else None
+    roofline = {"kernel": dominant, "bound": "tensor",
+                "achieved": achieved, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
+                "frac": (achieved / peaks["bf16_sus"]) if achieved else None,
+                "traffic": traffic.get((dominant, workload)),
+                "peak_source": peaks["src"] + " sustained bf16 (kernel timed inside a long step)",
+                "algorithmic_flops_per_launch": dom_flops,
+                "avg_launch_ms": dom_avg, "launches_per_call": dn / steps}
+    tc_ms = sum(agg[k][1] for k in TC_KERNELS if k in agg) / steps
+    grad_ms = sum(t for nm, (n, t) in agg.items() if nm not in ("coeffs",)) / steps
+    total = sum(x[1] for x in agg.values())
+    info = {
+        "algorithmic_tflops": 3 * flops_gemm / (grad_ms / 1e3) / 1e12,
+        "frac_of_sustained_bf16": 3 * flops_gemm / (grad_ms / 1e3) / 1e12 / peaks["bf16_sus"],
+        "ms_per_call": grad_ms, "tensor_kernels_ms": tc_ms,
+        "tokens_active_per_s": T_eff / (grad_ms / 1e3),
+        "kernels": {k: {"launches": n, "total_ms": t, "share": t / total}
+                    for k, (n, t) in sorted(agg.items(), key=lambda kv: -kv[1][1])}}
+    return roofline, info
+
+
+def device_head_workload(torch, wl, seed):
+    """A head workload for a throughput line: rewards, masks, lengths and
+    targets from the seeded generator, H ~ N(0, 1) and W ~ N(0, 1/d) drawn on
+    the device by torch's seeded generator and rounded to bf16 (the same
+    distributions; the timing does not depend on the values)."""
+    inp = synth.make_head_workload(wl, seed, draw_hw=False)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(1000003 * (seed + 1))
+    T, d, V = inp["T"], inp["d"], inp["V"]
+    H = torch.empty((T, d), dtype=torch.bfloat16, device="cuda")
+    for s in range(0, T, 65536):
+        e = min(T, s + 65536)
+        H[s:e] = torch.randn((e - s, d), generator=g, device="cuda").to(torch.bfloat16)
+    H[torch.from_numpy(inp["mask"] == 0).cuda()] = 0
+    W = (torch.randn((V, d), generator=g, device="cuda") / math.sqrt(d)).to(torch.bfloat16)
+    return inp, H, W
+
+
 def main():
     args = parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
-        return run_reference(args, rank, world)
+        return run_reference(args, rank)
+    if args.gpus != 1 or world != 1:
+        print("bench.py: single-GPU library (the head kernels multicast TMA tiles within a "
+              "cluster of one GPU); run it with --gpus 1", file=sys.stderr)
+        return 2
 
     import torch
-    import torch.distributed as dist
     from paper_2608_11368_gb300 import binding as B
 
-    torch.cuda.set_device(local)
-    if world > 1:
-        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-
-    def barrier():
-        if world > 1:
-            dist.barrier()
-
-    def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
-
+    torch.cuda.set_device(0)
     peaks = load_peaks()
     traffic = load_traffic()
     wl = synth.WORKLOADS[args.workload]
     kw = {"V": args.vocab} if args.vocab else {}
-    inp = synth.make_head_workload(wl, args.seed + rank, len_scale=args.len_scale, **kw)
+    inp = synth.make_head_workload(wl, args.seed, len_scale=args.len_scale, **kw)
     T, d, V, R = inp["T"], inp["d"], inp["V"], inp["R"]
 
     def pinned(x):
@@ -311,8 +409,6 @@ def main():
         "J": pinned(inp["J"]), "rho": pinned(inp["rho"]),
     }
     devb = {k: v.to("cuda", non_blocking=False) for k, v in host.items()}
-    H = devb["H"].view(torch.bfloat16)
-    W = devb["W"].view(torch.bfloat16)
     a = torch.empty((wl.B, wl.G), dtype=torch.float32, device="cuda")
     active = torch.empty((wl.B, wl.G), dtype=torch.uint8, device="cuda")
     edges = torch.empty(wl.B, dtype=torch.int32, device="cuda")
@@ -339,14 +435,15 @@ def main():
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     launches = [0]
 
-    def step(bufs=None):
+    def step(bufs=None, wsp=None):
         bufs = devb if bufs is None else bufs
         B.pair_coeffs(bufs["r"], bufs["J"], bufs["rho"], a=a, active=active,
                       edges=edges, contrast_edges=contrast, dev_err=err)
         n = B.pair_last_launch_count()
         B.pair_grad(bufs["H"].view(torch.bfloat16), bufs["W"].view(torch.bfloat16), bufs["y"],
                     bufs["mask"], bufs["cu"], a.view(-1),
-                    dH=dH, dW=dW, Jobj=Jobj, logp_seq=lps, ws=ws, dev_err=err)
+                    dH=dH, dW=dW, Jobj=Jobj, logp_seq=lps, ws=ws if wsp is None else wsp,
+                    dev_err=err)
         launches[0] += n + B.pair_last_launch_count()
 
     for _ in range(args.warmup):
@@ -357,62 +454,46 @@ def main():
     T_eff = count_active_tokens(inp, a.view(-1).cpu().numpy())
 
     # ---- timed region: inputs resident in HBM, L2 flushed between steps.
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(args.steps)]
-    sampler = ClockSampler(local)
+    sampler = ClockSampler(0)
     sampler.start()
-    barrier()
-    torch.cuda.synchronize()
     launches[0] = 0
-    B.pair_timing_enable(True)
-    for k in range(args.steps):
-        flush.zero_()
-        ev[k][0].record()
-        step()
-        ev[k][1].record()
-    torch.cuda.synchronize()
-    barrier()
-    kern = B.pair_timing_read()
-    B.pair_timing_enable(False)
+    step_ms, kern = timed_steps(B, torch, step, args.steps, flush)
     clocks = sampler.stop()
     gpu_launches = launches[0]
-    step_ms = [s.elapsed_time(e) for s, e in ev]
-    total_ms = max_over_ranks(sum(step_ms))
+    total_ms = sum(step_ms)
     if B.pair_status_sync(err) != 0:
         raise SystemExit("timed steps reported a device error")
-    value = T * world * args.steps / (total_ms / 1e3)
+    value = T * args.steps / (total_ms / 1e3)
+    roofline, pair_grad_info = kernel_report(kern, args.steps, T_eff, V, d, peaks, traffic,
+                                             args.workload)
 
-    # Per-kernel durations over the timed region (CUDA events on the library's
-    # launch stream).
-    agg = {}
-    for name, ms in kern:
-        n, tot = agg.get(name, (0, 0.0))
-        agg[name] = (n + 1, tot + ms)
-    flops_gemm = 2.0 * T_eff * V * d
-    dominant = max(agg.items(), key=lambda kv: kv[1][1])[0]
-    dn, dt_ms = agg[dominant]
-    # One "launch" here is the kernel's whole share of one pair_grad call: the
-    # sum over its token-chunk launches (chunks past the last token exit at
-    # once), so per-call work divides per-call time.
-    dom_avg = dt_ms / args.steps
-    dom_flops = flops_gemm if dominant in TC_KERNELS else None
-    achieved = dom_flops / (dom_avg / 1e3) / 1e12 if dom_flops else None
-    roofline = {"kernel": dominant, "bound": "tensor",
-                "achieved": achieved, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
-                "frac": (achieved / peaks["bf16_sus"]) if achieved else None,
-                "traffic": traffic.get((dominant, args.workload)),
-                "peak_source": peaks["src"] + " sustained bf16 (kernel timed inside a long step)",
-                "algorithmic_flops_per_launch": dom_flops,
-                "avg_launch_ms": dom_avg, "launches_per_call": dn / args.steps}
-    tc_ms = sum(agg[k][1] for k in TC_KERNELS if k in agg) / args.steps
-    grad_ms = sum(t for nm, (n, t) in agg.items() if nm not in ("coeffs",)) / args.steps
-    pair_grad_info = {
-        "algorithmic_tflops": 3 * flops_gemm / (grad_ms / 1e3) / 1e12,
-        "frac_of_sustained_bf16": 3 * flops_gemm / (grad_ms / 1e3) / 1e12 / peaks["bf16_sus"],
-        "ms_per_call": grad_ms, "tensor_kernels_ms": tc_ms,
-        "tokens_active_per_s": T_eff * world / (grad_ms / 1e3),
-        "kernels": {k: {"launches": n, "total_ms": t, "share": t / sum(x[1] for x in agg.values())}
-                    for k, (n, t) in sorted(agg.items(), key=lambda kv: -kv[1][1])}}
+    # ---- the on-chip form: the same step with pair_grad_workspace_min_size,
+    # so no logit-sized tensor (logit terms or logit-gradient image) is kept
+    # in HBM; the backward recomputes the logits in clusters.
+    onchip = None
+    if not args.no_onchip:
+        ws_min = torch.empty(B.pair_grad_workspace_min_size(T, d, V, R, B.PAIR_BF16),
+                             dtype=torch.uint8, device="cuda")
+        oc_step = lambda: step(wsp=ws_min)
+        for _ in range(args.warmup):
+            oc_step()
+        if B.pair_status_sync(err) != 0:
+            raise SystemExit("on-chip warm-up step failed")
+        oc_steps = max(3, min(args.steps, 20))
+        sampler_oc = ClockSampler(0)
+        sampler_oc.start()
+        oc_ms, oc_kern = timed_steps(B, torch, oc_step, oc_steps, flush)
+        oc_clocks = sampler_oc.stop()
+        if B.pair_status_sync(err) != 0:
+            raise SystemExit("on-chip steps reported a device error")
+        oc_roof, oc_info = kernel_report(oc_kern, oc_steps, T_eff, V, d, peaks, traffic,
+                                         args.workload + ":onchip")
+        onchip = {"ms_per_step": sum(oc_ms) / oc_steps, "steps": oc_steps,
+                  "warmup": args.warmup,
+                  "value": T * oc_steps / (sum(oc_ms) / 1e3), "unit": "tokens/s",
+                  "workspace_bytes": ws_min.numel(), "roofline": oc_roof, "pair_grad": oc_info,
+                  "clocks": oc_clocks}
+        del ws_min
 
     # ---- end-to-end through the C-ABI with host buffers: every step copies
     # all of its inputs from pinned host memory and reads J and logp back.
@@ -440,7 +521,6 @@ def main():
 
     for j in range(2):
         consumed[j].record(main_s)
-    barrier()
     torch.cuda.synchronize()
     e2e_ev[0].record(main_s)
     copy_s.wait_event(e2e_ev[0])
@@ -456,46 +536,96 @@ def main():
         lps_h.copy_(lps, non_blocking=True)
     e2e_ev[1].record(main_s)
     torch.cuda.synchronize()
-    e2e_ms = max_over_ranks(e2e_ev[0].elapsed_time(e2e_ev[1]))
-    e2e = {"value": T * world * args.steps / (e2e_ms / 1e3), "unit": "tokens/s",
+    e2e_ms = e2e_ev[0].elapsed_time(e2e_ev[1])
+    e2e = {"value": T * args.steps / (e2e_ms / 1e3), "unit": "tokens/s",
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+    del sets
+
+    # ---- the other head workloads (Qwen3-4B head; heavy-tailed long context).
+    extra = None
+    if not args.no_extra:
+        extra = {}
+        del dH, dW, ws
+        torch.cuda.empty_cache()
+        for name in EXTRA_WORKLOADS:
+            extra[name] = bench_extra(B, torch, name, args.seed, peaks, traffic, flush)
+            torch.cuda.empty_cache()
 
     # ---- pair_coeffs / pair_estimate_dense on the 4096 x 64 stress workload.
     stress = None
     if not args.no_stress:
-        stress = bench_stress(B, torch, peaks, flush, args.steps, rank, traffic)
+        stress = bench_stress(B, torch, peaks, flush, args.steps, traffic)
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if not args.no_cpu_baseline:
         cpu = cpu_baseline(inp)
 
     line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": 1,
         "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": total_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; Qwen3-1.7B head shapes, random-init weights)",
-        "config": {"workload": args.workload, "len_scale": args.len_scale,
-                   "d": d, "V": V,
-                   "global_batch": wl.B * wl.G * world, "prompts": wl.B * world,
-                   "rollouts_per_prompt": wl.G, "tokens_packed": T,
-                   "tokens_active": T_eff,
-                   "l2": "flushed between timed steps (256 MiB write); inputs exceed L2",
-                   "parallelism": "replicas" if world == 1 else "dp%d weak (independent groups)" % world},
-        "roofline": roofline, "pair_grad": pair_grad_info,
-        "stress": stress, "cpu_baseline": cpu, "e2e": e2e,
+        "config": bench_config(args, wl, inp, T_eff),
+        "roofline": roofline, "pair_grad": pair_grad_info, "pair_grad_onchip": onchip,
+        "configs": extra, "stress": stress, "cpu_baseline": cpu, "e2e": e2e,
         "clocks": clocks, "gpu_launches": gpu_launches,
     }
-    if rank == 0:
-        print(json.dumps(line), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
+    print(json.dumps(line), flush=True)
     return 0
 
 
-def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
+def bench_extra(B, torch, name, seed, peaks, traffic, flush):
+    """Throughput of the default pair_coeffs + pair_grad step on another head
+    workload (inputs resident in HBM, L2 flushed between steps)."""
+    wl = synth.WORKLOADS[name]
+    inp, H, W = device_head_workload(torch, wl, seed)
+    T, d, V, R = inp["T"], inp["d"], inp["V"], inp["R"]
+    dv = lambda x: torch.from_numpy(np.ascontiguousarray(x)).cuda()
+    r, J, rho = dv(inp["r"]), dv(inp["J"]), dv(inp["rho"])
+    y, mask, cu = dv(inp["y"]), dv(inp["mask"]), dv(inp["cu_seqlens"])
+    a = torch.empty((wl.B, wl.G), dtype=torch.float32, device="cuda")
+    dH = torch.empty((T, d), dtype=torch.float32, device="cuda")
+    dW = torch.empty((V, d), dtype=torch.float32, device="cuda")
+    Jobj = torch.empty(1, dtype=torch.float64, device="cuda")
+    lps = torch.empty(R, dtype=torch.float32, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ws = torch.empty(B.pair_grad_workspace_size(T, d, V, R, B.PAIR_BF16), dtype=torch.uint8,
+                     device="cuda")
+
+    def step():
+        B.pair_coeffs(r, J, rho, a=a, dev_err=err)
+        B.pair_grad(H, W, y, mask, cu, a.view(-1), dH=dH, dW=dW, Jobj=Jobj, logp_seq=lps,
+                    ws=ws, dev_err=err)
+
+    for _ in range(EXTRA_WARMUP):
+        step()
+    if B.pair_status_sync(err) != 0:
+        raise SystemExit("%s warm-up step failed" % name)
+    T_eff = count_active_tokens(inp, a.view(-1).cpu().numpy())
+    sampler = ClockSampler(0)
+    sampler.start()
+    ms, kern = timed_steps(B, torch, step, EXTRA_STEPS, flush)
+    clocks = sampler.stop()
+    if B.pair_status_sync(err) != 0:
+        raise SystemExit("%s timed steps reported a device error" % name)
+    roof, info = kernel_report(kern, EXTRA_STEPS, T_eff, V, d, peaks, traffic, name)
+    step_ms = sum(ms) / EXTRA_STEPS
+    out = {"ms_per_step": step_ms, "steps": EXTRA_STEPS, "warmup": EXTRA_WARMUP,
+           "tokens_packed": T, "tokens_active": T_eff, "d": d, "V": V,
+           "prompts": wl.B, "rollouts_per_prompt": wl.G,
+           "value": T / (step_ms / 1e3), "unit": "tokens/s",
+           "tokens_active_per_s": T_eff / (step_ms / 1e3),
+           "roofline": roof, "pair_grad": info, "clocks": clocks,
+           "data": "group inputs, lengths and targets from the seeded generator; H, W drawn "
+                   "on the device (same distributions)"}
+    del H, W, dH, dW, ws
+    return out
+
+
+def bench_stress(B, torch, peaks, flush, steps, traffic):
     wl = synth.WORKLOADS[STRESS]
-    inp = synth.make_dense_workload(wl, 100 + rank)
+    inp = synth.make_dense_workload(wl, 100)
     dv = lambda x: torch.from_numpy(np.ascontiguousarray(x)).cuda()
     r, J, rho, S = dv(inp["r"]), dv(inp["J"]), dv(inp["rho"]), dv(inp["S"])
     Bn, G, D = wl.B, wl.G, wl.d
@@ -546,7 +676,7 @@ def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
                                               contrast_edges=e2, ess=ess, max_w=mw), reps)
     # Frozen-population audit at the paper's audit scale: one 16-candidate
     # group, 50,000 independent-design draws, scores of dimension 4096.
-    rng = np.random.default_rng(1234 + rank)
+    rng = np.random.default_rng(1234)
     Ga, Da, Na = 16, 4096, 50000
     pa = rng.uniform(0.1, 0.95, Ga)
     ra = dv((rng.random(Ga) < 0.5).astype(np.float32))
@@ -567,7 +697,7 @@ def bench_stress(B, torch, peaks, flush, steps, rank, traffic):
     # (a fixed number of small fp64 Newton systems per group).
     alloc = {}
     for nb, ga in ((64, 16), (4096, 64)):
-        ai = synth.make_alloc_inputs(77 + rank, nb, ga)
+        ai = synth.make_alloc_inputs(77, nb, ga)
         c_al, b_al, p_al = dv(ai["c_hat"]), dv(ai["budget"]), dv(ai["p_hat"])
         pi_al = torch.empty((nb, ga), dtype=torch.float32, device="cuda")
         st_al = torch.empty((nb, 5), dtype=torch.float64, device="cuda")

@@ -35,6 +35,14 @@
  *    the caller's device word `dev_err`, which `pair_status_sync` decodes.
  *  - Requires a compute capability 10.3 device (GB300). Other devices get
  *    PAIR_ERR_UNSUPPORTED.
+ *  - Single-GPU library: every call runs on the current device only, and
+ *    every array it is given must live on that device. The tensor-core head
+ *    kernels (the log-sum-exp pass and the two backward GEMMs) load tiles
+ *    with TMA multicast to the CTAs of one thread-block cluster; their tensor
+ *    maps cover only the caller's buffers and the workspace on the current
+ *    device, never another GPU's memory. A multi-GPU trainer runs one
+ *    independent call per GPU (whole prompt groups per GPU) and does its own
+ *    exchange of dW outside the library.
  */
 #ifndef PAIR_H_
 #define PAIR_H_
@@ -386,6 +394,25 @@ PAIR_API pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
                       size_t ws_bytes, int32_t *dev_err, pair_stream_t stream);
 
 /*
+ * pair_grad_token_logp -- the per-token log-probabilities of the most recent
+ * pair_grad (or pair_grad_clipped) call that used workspace ws:
+ *     logp_tok[t] = z_t[y_t] - logsumexp(z_t)        (Sec. 4.5, log pi per token)
+ * for every token t with mask_t = 1 in a rollout with a_i != 0, and 0 at every
+ * other token. This is what a PPO trainer keeps as the old log-probabilities
+ * of the next epochs (App. "Practical departures"); summed over a rollout it
+ * is that call's logp_seq. The workspace holds them until the next call that
+ * uses it.
+ * In:  T, d, V, R, dt, ws and ws_bytes exactly as given to that call, on the
+ *      same stream after it (stream order is the only synchronisation).
+ * Out: logp_tok [T] float32 (device).
+ * Errors: PAIR_ERR_INVALID_ARG (null logp_tok or shapes pair_grad rejects),
+ *      PAIR_ERR_WORKSPACE (ws null, misaligned or below the minimum size).
+ */
+PAIR_API pair_status pair_grad_token_logp(int64_t T, int32_t d, int32_t V, int32_t R,
+                                          pair_dtype dt, const void *ws, size_t ws_bytes,
+                                          float *logp_tok, pair_stream_t stream);
+
+/*
  * pair_grad_clipped -- the clipped trajectory-ratio surrogate of the practical
  * PPO epochs (Sec. 4.5; App. "Practical departures"), on the same LM-head
  * realisation as pair_grad. With the detached coefficients A_i = a[i] and the
@@ -427,13 +454,24 @@ PAIR_API pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dty
  * Arguments, outputs and numerics are those of pair_grad, minus ws and
  * ws_bytes. The workspace is a file-scope device array of
  * PAIR_NOALLOC_MAX_WORKSPACE bytes that every GPU loading this library
- * holds until the process exits. It keeps no logit-gradient image (the dW
- * pass recomputes the logits); problems whose
- * pair_grad_workspace_min_size(...) exceeds it are rejected with
- * PAIR_ERR_WORKSPACE before any launch. The call allocates nothing.
+ * holds until the process exits. It keeps no logit-gradient image (the
+ * backward recomputes the logits); a problem is accepted iff
+ * pair_grad_workspace_min_size(T, d, V, R, dt) <= PAIR_NOALLOC_MAX_WORKSPACE
+ * and rejected with PAIR_ERR_WORKSPACE before any launch otherwise. That
+ * size grows with T * d (the compacted hidden rows) plus, for bf16, a fixed
+ * exchange buffer and, for d a multiple of 512, per-cluster partial rows of
+ * width d. In this build the accepted range is, roughly: PAIR_F32, T (4 d +
+ * 148) <= 33 MB (T <= 32,000 at d = 256); PAIR_BF16 with d a multiple of 512,
+ * only d = 512 with T <= 7,000 (larger d need more than the array for the
+ * partial rows alone); other PAIR_BF16 d, T (2 d + 148) <= 20.9 MB. Larger
+ * heads (the Qwen3 shapes) need pair_grad with a caller-provided workspace.
+ * The call allocates nothing.
  * The first call on each device looks up the array's device address (with
- * that device current) and caches it; make that first call before any
- * stream capture. All calls on a device share the one array, which keeps
+ * that device current) and caches it per device and CUDA context; make that
+ * first call before any stream capture. A device reset (cudaDeviceReset)
+ * unloads the array but may leave the context handle unchanged, so a process
+ * that resets a device must not call pair_grad_noalloc on it afterwards.
+ * All calls on a device share the one array, which keeps
  * the previous call's contents (pair_grad needs no zeroed workspace): calls
  * whose executions overlap on the GPU (different streams, or host threads
  * without ordering) race on it and must be serialised by the caller.

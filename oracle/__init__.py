@@ -291,19 +291,43 @@ def head_logits(Hrows, W):
     return np.asarray(Hrows, np.float64) @ np.asarray(W, np.float64).T
 
 
-def head_lse(Hrows, W, y, chunk=256):
+def head_lse(Hrows, W, y, chunk=256, threads=1):
     """Per token: log-sum-exp over the vocabulary (max-shifted) and the
-    target logit. Returns (lse, z_target), fp64."""
+    target logit. Returns (lse, z_target), fp64.
+
+    threads > 1 splits each chunk's rows over that many threads for the
+    per-row steps (max, shift, exp, sum, log); every row's arithmetic and its
+    order are the same as with one thread. The logit matmul stays one library
+    call per chunk."""
     W64 = np.asarray(W, np.float64)
     n = Hrows.shape[0]
     lse = np.empty(n, np.float64)
     zy = np.empty(n, np.float64)
-    for s in range(0, n, chunk):
-        e = min(n, s + chunk)
-        Z = np.asarray(Hrows[s:e], np.float64) @ W64.T
-        m = Z.max(axis=1)
-        lse[s:e] = m + np.log(np.exp(Z - m[:, None]).sum(axis=1))
-        zy[s:e] = Z[np.arange(e - s), y[s:e]]
+
+    def rows(Z, s, a, b):
+        m = Z[a:b].max(axis=1)
+        lse[s + a:s + b] = m + np.log(np.exp(Z[a:b] - m[:, None]).sum(axis=1))
+        zy[s + a:s + b] = Z[np.arange(a, b), y[s + a:s + b]]
+
+    pool = None
+    if threads > 1:
+        import concurrent.futures as cf
+        pool = cf.ThreadPoolExecutor(threads)
+    try:
+        for s in range(0, n, chunk):
+            e = min(n, s + chunk)
+            Z = np.asarray(Hrows[s:e], np.float64) @ W64.T
+            if pool is None:
+                rows(Z, s, 0, e - s)
+            else:
+                step = -(-(e - s) // threads)
+                futs = [pool.submit(rows, Z, s, a, min(e - s, a + step))
+                        for a in range(0, e - s, step)]
+                for f in futs:
+                    f.result()
+    finally:
+        if pool is not None:
+            pool.shutdown()
     return lse, zy
 
 

@@ -88,6 +88,8 @@ def lib() -> ctypes.CDLL:
     L.pair_audit.restype = ctypes.c_int
     L.pair_allocate.argtypes = [I32, I32, P, P, P, P, P, F32, P, P, P, P]
     L.pair_allocate.restype = ctypes.c_int
+    L.pair_grad_token_logp.argtypes = [I64, I32, I32, I32, ctypes.c_int, P, SZ, P, P]
+    L.pair_grad_token_logp.restype = ctypes.c_int
     L.pair_selftest_wait_timeout.argtypes = [I64, P, P, P]
     L.pair_selftest_wait_timeout.restype = ctypes.c_int
     _lib = L
@@ -149,23 +151,39 @@ def _check(st, where):
         raise PairError(st, where)
 
 
+def _on_device(t):
+    """Context manager making t's device current for the call: the library
+    launches on the current device and takes its stream from there."""
+    return torch.cuda.device(t.device)
+
+
+def _out(t, name, shape, dtype, dev):
+    """Caller-passed output (checked) or a fresh torch allocation."""
+    if t is None:
+        return torch.empty(shape, dtype=dtype, device=dev)
+    _need(t, name, dtype, shape)
+    if t.device != dev:
+        raise ValueError("%s must be on %s, got %s" % (name, dev, t.device))
+    return t
+
+
 def pair_coeffs(r, J, rho, scale=1.0, flags=0, a=None, active=None, edges=None,
                 contrast_edges=None, dev_err=None, stream=None):
-    """Coefficients of Eq. (pair-advantage) (times `scale`, see pair.h).
-    Returns (a, active, edges, contrast_edges)."""
+    """Coefficients of Eq. (pair-advantage) (times `scale`, see pair.h), on
+    r's device. Returns (a, active, edges, contrast_edges)."""
     B, G = r.shape
     dev = r.device
     _need(r, "r", torch.float32)
     _need(J, "J", torch.uint8, (B, G))
     _need(rho, "rho", torch.float32, (B, G, G))
-    a = torch.empty((B, G), dtype=torch.float32, device=dev) if a is None else a
-    active = torch.empty((B, G), dtype=torch.uint8, device=dev) if active is None else active
-    edges = torch.empty(B, dtype=torch.int32, device=dev) if edges is None else edges
-    contrast_edges = (torch.empty(B, dtype=torch.int32, device=dev)
-                      if contrast_edges is None else contrast_edges)
-    st = lib().pair_coeffs(B, G, _p(r), _p(J), _p(rho), float(scale), int(flags),
-                           _p(a), _p(active), _p(edges), _p(contrast_edges),
-                           _p(dev_err), _stream(stream))
+    a = _out(a, "a", (B, G), torch.float32, dev)
+    active = _out(active, "active", (B, G), torch.uint8, dev)
+    edges = _out(edges, "edges", (B,), torch.int32, dev)
+    contrast_edges = _out(contrast_edges, "contrast_edges", (B,), torch.int32, dev)
+    with _on_device(r):
+        st = lib().pair_coeffs(B, G, _p(r), _p(J), _p(rho), float(scale), int(flags),
+                               _p(a), _p(active), _p(edges), _p(contrast_edges),
+                               _p(dev_err), _stream(stream))
     _check(st, "pair_coeffs")
     return a, active, edges, contrast_edges
 
@@ -174,10 +192,12 @@ PAIR_W_HT, PAIR_W_UNWEIGHTED, PAIR_W_MARGINAL, PAIR_W_CLIPPED, PAIR_W_HAJEK = 0,
 
 
 def _coeffs_outputs(B, G, dev, a, active, edges, contrast_edges, ess, max_w):
-    f = lambda t, shape, dt: torch.empty(shape, dtype=dt, device=dev) if t is None else t
-    return (f(a, (B, G), torch.float32), f(active, (B, G), torch.uint8),
-            f(edges, (B,), torch.int32), f(contrast_edges, (B,), torch.int32),
-            f(ess, (B,), torch.float32), f(max_w, (B,), torch.float32))
+    return (_out(a, "a", (B, G), torch.float32, dev),
+            _out(active, "active", (B, G), torch.uint8, dev),
+            _out(edges, "edges", (B,), torch.int32, dev),
+            _out(contrast_edges, "contrast_edges", (B,), torch.int32, dev),
+            _out(ess, "ess", (B,), torch.float32, dev),
+            _out(max_w, "max_w", (B,), torch.float32, dev))
 
 
 def pair_coeffs_weighted(r, J, rho, wmode=PAIR_W_HT, w_max=0.0, scale=1.0, flags=0, a=None,
@@ -191,9 +211,10 @@ def pair_coeffs_weighted(r, J, rho, wmode=PAIR_W_HT, w_max=0.0, scale=1.0, flags
     if rho is not None:
         _need(rho, "rho", torch.float32, (B, G, G))
     outs = _coeffs_outputs(B, G, r.device, a, active, edges, contrast_edges, ess, max_w)
-    st = lib().pair_coeffs_weighted(B, G, _p(r), _p(J), _p(rho), float(scale), int(flags),
-                                    int(wmode), float(w_max), *[_p(t) for t in outs],
-                                    _p(dev_err), _stream(stream))
+    with _on_device(r):
+        st = lib().pair_coeffs_weighted(B, G, _p(r), _p(J), _p(rho), float(scale), int(flags),
+                                        int(wmode), float(w_max), *[_p(t) for t in outs],
+                                        _p(dev_err), _stream(stream))
     _check(st, "pair_coeffs_weighted")
     return outs
 
@@ -207,8 +228,9 @@ def pair_coeffs_product(r, J, p, scale=1.0, flags=0, a=None, active=None, edges=
     _need(J, "J", torch.uint8, (B, G))
     _need(p, "p", torch.float32, (B, G))
     outs = _coeffs_outputs(B, G, r.device, a, active, edges, contrast_edges, ess, max_w)
-    st = lib().pair_coeffs_product(B, G, _p(r), _p(J), _p(p), float(scale), int(flags),
-                                   *[_p(t) for t in outs], _p(dev_err), _stream(stream))
+    with _on_device(r):
+        st = lib().pair_coeffs_product(B, G, _p(r), _p(J), _p(p), float(scale), int(flags),
+                                       *[_p(t) for t in outs], _p(dev_err), _stream(stream))
     _check(st, "pair_coeffs_product")
     return outs
 
@@ -231,14 +253,16 @@ def pair_audit(r, rho, S, Jdraws, draw_weight=None, wmode=PAIR_W_HT, w_max=0.0, 
     if draw_weight is not None:
         _need(draw_weight, "draw_weight", torch.float64, (N,))
     dev = r.device
-    stats = torch.empty(8, dtype=torch.float64, device=dev) if stats is None else stats
-    bias = torch.empty(D, dtype=torch.float64, device=dev) if bias is None else bias
+    stats = _out(stats, "stats", (8,), torch.float64, dev)
+    bias = _out(bias, "bias", (D,), torch.float64, dev)
     need = int(lib().pair_audit_workspace_size(N, G, D))
-    if ws is None:
-        ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
-    st = lib().pair_audit(N, G, D, _p(r), _p(rho), _p(S), _p(Jdraws), _p(draw_weight),
-                          float(scale), int(flags), int(wmode), float(w_max), _p(stats),
-                          _p(bias), _p(ws), ws.numel(), _p(dev_err), _stream(stream))
+    with _on_device(r):
+        if ws is None:
+            ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+        _need(ws, "ws", torch.uint8)
+        st = lib().pair_audit(N, G, D, _p(r), _p(rho), _p(S), _p(Jdraws), _p(draw_weight),
+                              float(scale), int(flags), int(wmode), float(w_max), _p(stats),
+                              _p(bias), _p(ws), ws.numel(), _p(dev_err), _stream(stream))
     _check(st, "pair_audit")
     return stats, bias
 
@@ -264,28 +288,33 @@ def pair_allocate(c_hat, budget, pi_min, p_hat=None, m_hat=None, a=None, pi=None
     if a is not None:
         _need(a, "a", torch.float32, (B, G, G))
     dev = c_hat.device
-    pi = torch.empty((B, G), dtype=torch.float32, device=dev) if pi is None else pi
-    stats = torch.empty((B, 5), dtype=torch.float64, device=dev) if stats is None else stats
+    pi = _out(pi, "pi", (B, G), torch.float32, dev)
+    stats = _out(stats, "stats", (B, 5), torch.float64, dev)
     if dev_err is None:
         dev_err = torch.zeros(1, dtype=torch.int32, device=dev)
-    st = lib().pair_allocate(B, G, _p(p_hat), _p(m_hat), _p(a), _p(c_hat), _p(budget),
-                             float(pi_min), _p(pi), _p(stats), _p(dev_err), _stream(stream))
+    with _on_device(c_hat):
+        st = lib().pair_allocate(B, G, _p(p_hat), _p(m_hat), _p(a), _p(c_hat), _p(budget),
+                                 float(pi_min), _p(pi), _p(stats), _p(dev_err),
+                                 _stream(stream))
     _check(st, "pair_allocate")
     return pi, stats
 
 
 def pair_estimate_dense(r, J, rho, S, scale=1.0, g=None, a=None, dev_err=None,
                         stream=None):
-    """Eq. (pair-ht) for explicit scores S [B,G,D]. Returns (g, a)."""
+    """Eq. (pair-ht) for explicit scores S [B,G,D], on S's device. Returns (g, a)."""
     B, G, D = S.shape
     _need(r, "r", torch.float32, (B, G))
     _need(J, "J", torch.uint8, (B, G))
     _need(rho, "rho", torch.float32, (B, G, G))
     _need(S, "S", torch.float32)
-    g = torch.empty((B, D), dtype=torch.float32, device=S.device) if g is None else g
-    st = lib().pair_estimate_dense(B, G, D, _p(r), _p(J), _p(rho), _p(S),
-                                   float(scale), _p(g), _p(a), _p(dev_err),
-                                   _stream(stream))
+    g = _out(g, "g", (B, D), torch.float32, S.device)
+    if a is not None:
+        a = _out(a, "a", (B, G), torch.float32, S.device)
+    with _on_device(S):
+        st = lib().pair_estimate_dense(B, G, D, _p(r), _p(J), _p(rho), _p(S),
+                                       float(scale), _p(g), _p(a), _p(dev_err),
+                                       _stream(stream))
     _check(st, "pair_estimate_dense")
     return g, a
 
@@ -308,64 +337,81 @@ def _pair_dtype(t):
     raise TypeError("H/W must be bfloat16 or float32")
 
 
-def pair_grad(H, W, y, mask, cu_seqlens, a, dH=None, dW=None, Jobj=None,
-              logp_seq=None, ws=None, dev_err=None, stream=None):
-    """LM-head realisation of sum_i a_i log pi(o_i|q) and its gradients.
-    Returns (Jobj [1] f64, dH [T,d] f32, dW [V,d] f32, logp_seq [R] f32)."""
+def _grad_inputs(H, W, y, mask, cu_seqlens, a):
     T, d = H.shape
     V = W.shape[0]
     R = cu_seqlens.numel() - 1
     dt = _pair_dtype(H)
-    _need(H, "H", H.dtype)
+    _need(H, "H", H.dtype, (T, d))
     _need(W, "W", H.dtype, (V, d))
     _need(y, "y", torch.int32, (T,))
     _need(mask, "mask", torch.uint8, (T,))
     _need(cu_seqlens, "cu_seqlens", torch.int32, (R + 1,))
     _need(a, "a", torch.float32, (R,))
+    for t, nm in ((W, "W"), (y, "y"), (mask, "mask"), (cu_seqlens, "cu_seqlens"), (a, "a")):
+        if t.device != H.device:
+            raise ValueError("%s must be on %s like H, got %s" % (nm, H.device, t.device))
+    return T, d, V, R, dt
+
+
+def _grad_outputs(T, d, V, R, dev, dH, dW, Jobj, logp_seq):
+    return (_out(dH, "dH", (T, d), torch.float32, dev), _out(dW, "dW", (V, d), torch.float32, dev),
+            _out(Jobj, "Jobj", (1,), torch.float64, dev),
+            _out(logp_seq, "logp_seq", (R,), torch.float32, dev))
+
+
+def pair_grad(H, W, y, mask, cu_seqlens, a, dH=None, dW=None, Jobj=None,
+              logp_seq=None, ws=None, dev_err=None, stream=None):
+    """LM-head realisation of sum_i a_i log pi(o_i|q) and its gradients.
+    Runs on H's device. Returns (Jobj [1] f64, dH [T,d] f32, dW [V,d] f32,
+    logp_seq [R] f32)."""
+    T, d, V, R, dt = _grad_inputs(H, W, y, mask, cu_seqlens, a)
     dev = H.device
-    dH = torch.empty((T, d), dtype=torch.float32, device=dev) if dH is None else dH
-    dW = torch.empty((V, d), dtype=torch.float32, device=dev) if dW is None else dW
-    Jobj = torch.empty(1, dtype=torch.float64, device=dev) if Jobj is None else Jobj
-    logp_seq = torch.empty(R, dtype=torch.float32, device=dev) if logp_seq is None else logp_seq
-    need = pair_grad_workspace_size(T, d, V, R, dt)
-    if ws is None:
-        ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
-    st = lib().pair_grad(T, d, V, dt, _p(H), _p(W), _p(y), _p(mask),
-                         _p(cu_seqlens), R, _p(a), _p(dH), _p(dW), _p(Jobj),
-                         _p(logp_seq), _p(ws), ws.numel(), _p(dev_err),
-                         _stream(stream))
+    dH, dW, Jobj, logp_seq = _grad_outputs(T, d, V, R, dev, dH, dW, Jobj, logp_seq)
+    with _on_device(H):
+        if ws is None:
+            need = pair_grad_workspace_size(T, d, V, R, dt)
+            ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+        _need(ws, "ws", torch.uint8)
+        st = lib().pair_grad(T, d, V, dt, _p(H), _p(W), _p(y), _p(mask),
+                             _p(cu_seqlens), R, _p(a), _p(dH), _p(dW), _p(Jobj),
+                             _p(logp_seq), _p(ws), ws.numel(), _p(dev_err),
+                             _stream(stream))
     _check(st, "pair_grad")
     return Jobj, dH, dW, logp_seq
 
 
+def pair_grad_token_logp(T, d, V, R, dtype, ws, logp_tok=None, stream=None):
+    """Per-token log-probabilities [T] left in `ws` by the last pair_grad (or
+    pair_grad_clipped) call with these shapes (see pair.h): logp_t for active
+    tokens, 0 elsewhere."""
+    _need(ws, "ws", torch.uint8)
+    logp_tok = _out(logp_tok, "logp_tok", (int(T),), torch.float32, ws.device)
+    with _on_device(ws):
+        st = lib().pair_grad_token_logp(int(T), int(d), int(V), int(R), int(dtype), _p(ws),
+                                        ws.numel(), _p(logp_tok), _stream(stream))
+    _check(st, "pair_grad_token_logp")
+    return logp_tok
+
+
 def pair_grad_clipped(H, W, y, mask, cu_seqlens, a, logp_old, clip_eps=0.2, dH=None, dW=None,
                       Jobj=None, logp_seq=None, coef=None, ws=None, dev_err=None, stream=None):
-    """Clipped trajectory-ratio surrogate (see pair.h). Returns
-    (Jobj [1] f64, dH [T,d] f32, dW [V,d] f32, logp_seq [R] f32, coef [R] f32)."""
-    T, d = H.shape
-    V = W.shape[0]
-    R = cu_seqlens.numel() - 1
-    dt = _pair_dtype(H)
-    _need(H, "H", H.dtype)
-    _need(W, "W", H.dtype, (V, d))
-    _need(y, "y", torch.int32, (T,))
-    _need(mask, "mask", torch.uint8, (T,))
-    _need(cu_seqlens, "cu_seqlens", torch.int32, (R + 1,))
-    _need(a, "a", torch.float32, (R,))
+    """Clipped trajectory-ratio surrogate (see pair.h). Runs on H's device.
+    Returns (Jobj [1] f64, dH [T,d] f32, dW [V,d] f32, logp_seq [R] f32, coef [R] f32)."""
+    T, d, V, R, dt = _grad_inputs(H, W, y, mask, cu_seqlens, a)
     _need(logp_old, "logp_old", torch.float32, (R,))
     dev = H.device
-    dH = torch.empty((T, d), dtype=torch.float32, device=dev) if dH is None else dH
-    dW = torch.empty((V, d), dtype=torch.float32, device=dev) if dW is None else dW
-    Jobj = torch.empty(1, dtype=torch.float64, device=dev) if Jobj is None else Jobj
-    logp_seq = torch.empty(R, dtype=torch.float32, device=dev) if logp_seq is None else logp_seq
-    coef = torch.empty(R, dtype=torch.float32, device=dev) if coef is None else coef
-    need = pair_grad_workspace_size(T, d, V, R, dt)
-    if ws is None:
-        ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
-    st = lib().pair_grad_clipped(T, d, V, dt, _p(H), _p(W), _p(y), _p(mask), _p(cu_seqlens), R,
-                                 _p(a), _p(logp_old), float(clip_eps), _p(dH), _p(dW), _p(Jobj),
-                                 _p(logp_seq), _p(coef), _p(ws), ws.numel(), _p(dev_err),
-                                 _stream(stream))
+    dH, dW, Jobj, logp_seq = _grad_outputs(T, d, V, R, dev, dH, dW, Jobj, logp_seq)
+    coef = _out(coef, "coef", (R,), torch.float32, dev)
+    with _on_device(H):
+        if ws is None:
+            need = pair_grad_workspace_size(T, d, V, R, dt)
+            ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+        _need(ws, "ws", torch.uint8)
+        st = lib().pair_grad_clipped(T, d, V, dt, _p(H), _p(W), _p(y), _p(mask), _p(cu_seqlens),
+                                     R, _p(a), _p(logp_old), float(clip_eps), _p(dH), _p(dW),
+                                     _p(Jobj), _p(logp_seq), _p(coef), _p(ws), ws.numel(),
+                                     _p(dev_err), _stream(stream))
     _check(st, "pair_grad_clipped")
     return Jobj, dH, dW, logp_seq, coef
 
@@ -376,28 +422,18 @@ NOALLOC_MAX_WORKSPACE = 32 << 20
 def pair_grad_noalloc(H, W, y, mask, cu_seqlens, a, dH=None, dW=None,
                       Jobj=None, logp_seq=None, dev_err=None, stream=None):
     """pair_grad on the library's fixed device workspace (no workspace
-    argument; see pair.h for the size limit and the sharing rules).
-    Output tensors not passed in are allocated here by torch, as in
-    pair_grad; pass them to keep the call allocation-free.
-    Returns (Jobj, dH, dW, logp_seq)."""
-    T, d = H.shape
-    V = W.shape[0]
-    R = cu_seqlens.numel() - 1
-    dt = _pair_dtype(H)
-    _need(W, "W", H.dtype, (V, d))
-    _need(y, "y", torch.int32, (T,))
-    _need(mask, "mask", torch.uint8, (T,))
-    _need(cu_seqlens, "cu_seqlens", torch.int32, (R + 1,))
-    _need(a, "a", torch.float32, (R,))
+    argument; see pair.h for the size limit and the sharing rules). Runs on
+    H's device. Output tensors not passed in are allocated here by torch, as
+    in pair_grad; pass all four (checked for shape, dtype and device) to keep
+    the call allocation-free. Returns (Jobj, dH, dW, logp_seq)."""
+    T, d, V, R, dt = _grad_inputs(H, W, y, mask, cu_seqlens, a)
     dev = H.device
-    dH = torch.empty((T, d), dtype=torch.float32, device=dev) if dH is None else dH
-    dW = torch.empty((V, d), dtype=torch.float32, device=dev) if dW is None else dW
-    Jobj = torch.empty(1, dtype=torch.float64, device=dev) if Jobj is None else Jobj
-    logp_seq = torch.empty(R, dtype=torch.float32, device=dev) if logp_seq is None else logp_seq
-    st = lib().pair_grad_noalloc(T, d, V, dt, _p(H), _p(W), _p(y), _p(mask),
-                                 _p(cu_seqlens), R, _p(a), _p(dH), _p(dW),
-                                 _p(Jobj), _p(logp_seq), _p(dev_err),
-                                 _stream(stream))
+    dH, dW, Jobj, logp_seq = _grad_outputs(T, d, V, R, dev, dH, dW, Jobj, logp_seq)
+    with _on_device(H):
+        st = lib().pair_grad_noalloc(T, d, V, dt, _p(H), _p(W), _p(y), _p(mask),
+                                     _p(cu_seqlens), R, _p(a), _p(dH), _p(dW),
+                                     _p(Jobj), _p(logp_seq), _p(dev_err),
+                                     _stream(stream))
     _check(st, "pair_grad_noalloc")
     return Jobj, dH, dW, logp_seq
 
@@ -412,5 +448,9 @@ def pair_selftest_wait_timeout(limit_cycles, dev_err, seen, stream=None):
 
 
 def pair_status_sync(dev_err=None, stream=None) -> int:
-    """Synchronise the stream and decode/reset the device error word."""
-    return int(lib().pair_status_sync(_stream(stream), _p(dev_err)))
+    """Synchronise the stream and decode/reset the device error word (on
+    dev_err's device when it is given)."""
+    if dev_err is None:
+        return int(lib().pair_status_sync(_stream(stream), None))
+    with _on_device(dev_err):
+        return int(lib().pair_status_sync(_stream(stream), _p(dev_err)))

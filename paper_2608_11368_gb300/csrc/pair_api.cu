@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "pair_common.cuh"
 
 namespace pairk {
@@ -50,23 +52,23 @@ void launch_end(cudaStream_t s) {
 
 void reset_launches() { g_log.launches = 0; }
 
-// Compute capability 10.3 (GB300) on the current device; cached per device.
+// Compute capability 10.3 (GB300) on the current device; the answer is
+// cached per device ordinal (0 = not yet known, 1 = supported, 2 = not), so
+// host threads working on different devices never share a slot.
 pair_status check_device() {
-  static int cached_dev = -1;
-  static pair_status cached = PAIR_OK;
+  constexpr int kMaxDev = 128;
+  static std::atomic<int> cache[kMaxDev];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return PAIR_ERR_CUDA;
-  if (dev != cached_dev) {
-    int major = 0, minor = 0;
-    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) !=
-            cudaSuccess ||
-        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) !=
-            cudaSuccess)
-      return PAIR_ERR_CUDA;
-    cached = (major == 10 && minor == 3) ? PAIR_OK : PAIR_ERR_UNSUPPORTED;
-    cached_dev = dev;
-  }
-  return cached;
+  const int known = (dev >= 0 && dev < kMaxDev) ? cache[dev].load(std::memory_order_relaxed) : 0;
+  if (known) return known == 1 ? PAIR_OK : PAIR_ERR_UNSUPPORTED;
+  int major = 0, minor = 0;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+    return PAIR_ERR_CUDA;
+  const bool ok = major == 10 && minor == 3;
+  if (dev >= 0 && dev < kMaxDev) cache[dev].store(ok ? 1 : 2, std::memory_order_relaxed);
+  return ok ? PAIR_OK : PAIR_ERR_UNSUPPORTED;
 }
 
 static bool aligned16(const void *p) {
@@ -238,6 +240,23 @@ pair_status pair_grad(int64_t T, int32_t d, int32_t V, pair_dtype dt,
   }
   if (st != PAIR_OK) return st;
   return grad_finalize(g, w, s);
+}
+
+pair_status pair_grad_token_logp(int64_t T, int32_t d, int32_t V, int32_t R, pair_dtype dt,
+                                 const void *ws, size_t ws_bytes, float *logp_tok,
+                                 pair_stream_t stream) {
+  reset_launches();
+  if (!logp_tok) return PAIR_ERR_INVALID_ARG;
+  const size_t need = pair_grad_workspace_min_size(T, d, V, R, dt);
+  if (need == 0) return PAIR_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return PAIR_ERR_WORKSPACE;
+  const pair_status dv = check_device();
+  if (dv != PAIR_OK) return dv;
+  GradWorkspace w;
+  grad_workspace_bytes(T, d, V, R, dt, &w, const_cast<void *>(ws),
+                       grad_gimg_rows_fit(T, d, V, R, dt, ws_bytes));
+  return grad_token_logp(T, w, logp_tok, reinterpret_cast<cudaStream_t>(stream));
 }
 
 pair_status pair_status_sync(pair_stream_t stream, int32_t *dev_err) {

@@ -140,6 +140,8 @@ pair_status grad_ppo_coefficients(const GradArgs &g, const GradWorkspace &w,
                                   const float *logp_old, float eps, float *coef_out,
                                   cudaStream_t s);
 pair_status grad_ppo_finalize(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
+// Per-token log-probabilities kept in the workspace, scattered to [T].
+pair_status grad_token_logp(int64_t T, const GradWorkspace &w, float *logp_tok, cudaStream_t s);
 // Exact one-hot parts (added after the tensor-core softmax parts).
 pair_status grad_onehot(const GradArgs &g, const GradWorkspace &w,
                         cudaStream_t s);

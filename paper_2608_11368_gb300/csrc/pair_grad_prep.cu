@@ -367,6 +367,22 @@ __global__ void ppo_objective_kernel(int R, const float *a, const double *seg_lo
   }
 }
 
+// logp_tok[t] = 0 for every packed token (the scatter below then fills the
+// active ones).
+__global__ void zero_f32_kernel(int64_t n, float *x) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    x[i] = 0.f;
+}
+
+// logp_tok[tok_idx[p]] = zy[p] - lse[p] for every compacted token p.
+__global__ void scatter_logp_kernel(const int32_t *counters, const int32_t *tok_idx,
+                                    const float *zy, const float *lse, float *logp_tok) {
+  const int Teff = counters[0];
+  for (int p = blockIdx.x * blockDim.x + threadIdx.x; p < Teff; p += gridDim.x * blockDim.x)
+    logp_tok[tok_idx[p]] = zy[p] - lse[p];
+}
+
 }  // namespace
 
 size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
@@ -476,6 +492,17 @@ pair_status grad_finalize(const GradArgs &g, const GradWorkspace &w,
   PAIR_BEGIN("objective", s);
   objective_kernel<<<1, 1024, 0, s>>>(g.R, g.a, w.seg_logp, g.Jobj,
                                       g.logp_seq);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+pair_status grad_token_logp(int64_t T, const GradWorkspace &w, float *logp_tok,
+                            cudaStream_t s) {
+  PAIR_BEGIN("zero_logp", s);
+  zero_f32_kernel<<<152 * 4, 256, 0, s>>>(T, logp_tok);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("scatter_logp", s);
+  scatter_logp_kernel<<<152 * 4, 256, 0, s>>>(w.counters, w.tok_idx, w.zy, w.lse, logp_tok);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }

@@ -2,6 +2,8 @@
 // memory. Its workspace is a fixed array in this library's device data
 // instead of a caller-provided buffer; everything else is the pair_grad
 // launch sequence, unchanged.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "pair_common.cuh"
@@ -17,23 +19,50 @@ static __device__ __align__(256) unsigned char g_scratch[kStaticScratchBytes];
 
 constexpr int kMaxDevices = 128;
 std::mutex g_scratch_mu;
-void *g_scratch_addr[kMaxDevices] = {};
+struct ScratchSlot {
+  CUcontext ctx;  // context the address was looked up in
+  void *addr;
+};
+ScratchSlot g_scratch_slot[kMaxDevices] = {};
+
+using CtxGetCurrentFn = CUresult (*)(CUcontext *);
+CtxGetCurrentFn ctx_get_current() {
+  static CtxGetCurrentFn fn = nullptr;
+  if (!fn) {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetCurrentFn>(p);
+  }
+  return fn;
+}
 
 // Device address of g_scratch on the current device. The host-side name of
-// a __device__ array is only a stand-in, so the address is looked up once
-// per device (with that device current) and cached.
+// a __device__ array is only a stand-in, so the address is looked up (with
+// the device current) the first time a device is used, and again whenever
+// the current context differs from the one it was looked up in.
 pair_status scratch_address(void **out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return PAIR_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return PAIR_ERR_UNSUPPORTED;
+  CtxGetCurrentFn get = ctx_get_current();
+  if (!get) return PAIR_ERR_CUDA;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_addr[dev]) {
+  ScratchSlot &slot = g_scratch_slot[dev];
+  CUcontext ctx = nullptr;
+  if (get(&ctx) != CUDA_SUCCESS) return PAIR_ERR_CUDA;
+  if (!slot.addr || !ctx || slot.ctx != ctx) {
     void *p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || !p)
-      return PAIR_ERR_CUDA;
-    g_scratch_addr[dev] = p;
+    // The lookup also makes the device's primary context current when no
+    // context is yet.
+    if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || !p) return PAIR_ERR_CUDA;
+    if (get(&ctx) != CUDA_SUCCESS || !ctx) return PAIR_ERR_CUDA;
+    slot.ctx = ctx;
+    slot.addr = p;
   }
-  *out = g_scratch_addr[dev];
+  *out = slot.addr;
   return PAIR_OK;
 }
 
@@ -62,12 +91,8 @@ extern "C" pair_status pair_grad_noalloc(
   if ((reinterpret_cast<uintptr_t>(H) & 15u) || (reinterpret_cast<uintptr_t>(W) & 15u) ||
       (reinterpret_cast<uintptr_t>(dH) & 15u) || (reinterpret_cast<uintptr_t>(dW) & 15u))
     return PAIR_ERR_INVALID_ARG;
-  int dev = 0, major = 0, minor = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
-    return PAIR_ERR_CUDA;
-  if (major != 10 || minor != 3) return PAIR_ERR_UNSUPPORTED;
+  const pair_status dv = check_device();
+  if (dv != PAIR_OK) return dv;
   void *ws = nullptr;
   const pair_status sa = scratch_address(&ws);
   if (sa != PAIR_OK) return sa;

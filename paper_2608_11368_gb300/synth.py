@@ -182,13 +182,15 @@ def _normal_bits(gen, rows, cols, std, as_bf16, chunk=8192):
 def make_head_workload(wl: Workload, seed: int, B: Optional[int] = None,
                        G: Optional[int] = None, len_scale: float = 1.0,
                        V: Optional[int] = None, d: Optional[int] = None,
-                       pad_fill: str = "zero", w_std_mult: float = 1.0):
+                       pad_fill: str = "zero", w_std_mult: float = 1.0,
+                       draw_hw: bool = True):
     """Complete input set for pair_coeffs + pair_grad.
 
     Optional overrides shrink a workload (fewer groups, shorter responses,
     smaller V or d) for tests; the draws keep the workload's distributions.
     pad_fill: "zero" or "nan" for the hidden rows of padding tokens.
     w_std_mult scales the head weight std (a peaky-softmax variant for tests).
+    draw_hw=False leaves H and W out (None): every other array is the same.
     """
     assert wl.kind == "head"
     B = wl.B if B is None else B
@@ -203,15 +205,16 @@ def make_head_workload(wl: Workload, seed: int, B: Optional[int] = None,
     T = int(cu[-1])
     st = _streams(seed)
     bf = wl.dtype == "bf16"
-    H = _normal_bits(st[_S_H], T, d, 1.0, bf)
-    W = _normal_bits(st[_S_W], V, d, w_std_mult / math.sqrt(d), bf)
+    H = _normal_bits(st[_S_H], T, d, 1.0, bf) if draw_hw else None
+    W = _normal_bits(st[_S_W], V, d, w_std_mult / math.sqrt(d), bf) if draw_hw else None
     y = st[_S_Y].integers(0, V, size=T).astype(np.int32)
     pad = mask == 0
     y[pad] = -100
-    if pad_fill == "nan":
-        H[pad] = 0x7FC0 if bf else np.float32(np.nan)
-    else:
-        H[pad] = 0
+    if H is not None:
+        if pad_fill == "nan":
+            H[pad] = 0x7FC0 if bf else np.float32(np.nan)
+        else:
+            H[pad] = 0
     out = dict(grp)
     out.update(name=wl.name, B=B, G=G, R=B * G, T=T, d=d, V=V,
                dtype=wl.dtype, H=H, W=W, y=y, mask=mask, cu_seqlens=cu,

@@ -109,3 +109,12 @@ def _host_validation_checks(L):
     assert lib.pair_grad(*bad) == 3          # workspace too small
     bad = list(args); bad[15] = P(16 + 128)
     assert lib.pair_grad(*bad) == 3          # workspace not 256-aligned
+    # pair_grad_token_logp: null output, bad shapes, workspace missing or small.
+    need = L.pair_grad_workspace_min_size(100, 128, 256, 2, L.PAIR_BF16)
+    ws_ok = P(1 << 20)
+    assert lib.pair_grad_token_logp(100, 128, 256, 2, L.PAIR_BF16, ws_ok, need, None,
+                                    None) == 1
+    assert lib.pair_grad_token_logp(100, 96, 256, 2, L.PAIR_BF16, ws_ok, need, one, None) == 1
+    assert lib.pair_grad_token_logp(100, 128, 256, 2, L.PAIR_BF16, None, need, one, None) == 3
+    assert lib.pair_grad_token_logp(100, 128, 256, 2, L.PAIR_BF16, ws_ok, need - 1, one,
+                                    None) == 3

@@ -201,32 +201,97 @@ def test_grad_target_out_of_range_flagged():
 FULL = ["qwen3_1p7b_head", "qwen3_4b_head", "longctx_skew"]
 
 
+def _logp_close(got, ref):
+    """Per-token log-probabilities: each within the loss tolerance relative
+    to its own magnitude."""
+    got = np.asarray(got, np.float64)
+    bad = np.abs(got - ref) > TOL * np.abs(ref)
+    assert not bad.any(), (int(bad.sum()), float(np.abs(got - ref).max()))
+
+
 @pytest.mark.parametrize("name", FULL)
-def test_grad_full_size_sampled(name):
-    """Full-size workload in the benchmark's launch configuration: sampled
-    rows against the oracle, and size-independent identities for the rest."""
+def test_grad_full_size_against_oracle(name):
+    """Full-size workload in the benchmark's launch configuration (default
+    workspace) against the fp64 oracle.
+    1.7B head (the benchmark workload): the oracle's lse and logp for every
+    active token, so J and every per-token log-probability are compared in
+    full, every rollout's logp_seq, dH on 1,024 sampled rows plus two whole
+    rollouts, and dW on 256 sampled vocabulary rows (half of them targeted).
+    4B and long-context heads: per-token logp on 4,096 sampled active tokens
+    and on 8 whole active rollouts (with their logp_seq), dH on 1,024 of those
+    rows. Identities that hold at any size cover the rest."""
+    B = _binding()
     wl = synth.WORKLOADS[name]
     inp = synth.make_head_workload(wl, 0)
     a = _coeffs(inp)
-    st, J, dH, dW, lps, t = _run(inp, a)
-    assert st == 0
+    t = head_inputs(inp, a)
+    T, d, V, R = inp["T"], inp["d"], inp["V"], inp["R"]
+    ws = torch.empty(B.pair_grad_workspace_size(T, d, V, R, B.PAIR_BF16), dtype=torch.uint8,
+                     device="cuda")
+    err = dev_err_word()
+    Jo, dH, dW, lps = B.pair_grad(t["H"], t["W"], t["y"], t["mask"], t["cu_seqlens"], t["a"],
+                                  ws=ws, dev_err=err)
+    assert B.pair_status_sync(err) == 0
+    lpt = B.pair_grad_token_logp(T, d, V, R, B.PAIR_BF16, ws).cpu().numpy()
+    J = Jo.item()
+    lps_n = lps.cpu().numpy()
+    del ws
     rng = np.random.default_rng(11)
     idx, c, seg = oracle.compact_tokens(inp["cu_seqlens"], inp["mask"], a)
     assert idx.size > 0
-    # dH: 1024 sampled active rows plus every row of the two shortest active
-    # rollouts (whose summed logp is checked too).
-    act_r = np.nonzero(a)[0]
-    L = np.diff(inp["cu_seqlens"])[act_r]
-    two = act_r[np.argsort(L)[:2]]
     cu = inp["cu_seqlens"]
-    whole = np.concatenate([np.arange(cu[i], cu[i + 1]) for i in two])
-    rows = np.unique(np.concatenate([rng.choice(idx, 1024, replace=False), whole]))
-    ref = oracle.pair_grad_ref(inp, a.astype(np.float64), dh_rows=rows,
-                               logp_rollouts=two)
-    dHn = dH.cpu().numpy()
-    assert rel_fro(dHn[rows], ref["dH_rows"]) <= TOL
-    lps_n = lps.cpu().numpy()
-    np.testing.assert_allclose(lps_n[two], ref["logp_seq_sel"], rtol=1e-4)
+    y = inp["y"]
+    Wf = synth.as_float(inp["W"], inp["dtype"]).astype(np.float64)
+    nthr = oracle.n_threads()
+    # Tokens outside the objective have logp 0.
+    keep = np.zeros(T, bool)
+    keep[idx] = True
+    assert (lpt[~keep] == 0).all()
+    act_r = np.nonzero(a)[0]
+
+    def hrows(tok):
+        return synth.as_float(inp["H"][tok], inp["dtype"]).astype(np.float64)
+
+    if name == "qwen3_1p7b_head":
+        Ha = hrows(idx)
+        lse, zy = oracle.head_lse(Ha, Wf, y[idx], threads=nthr)
+        logp = zy - lse
+        J_ref = float(np.sum(c * logp))
+        assert abs(J - J_ref) <= TOL * float(np.sum(np.abs(c * logp)))
+        _logp_close(lpt[idx], logp)
+        lps_ref = np.zeros(R, np.float64)
+        np.add.at(lps_ref, seg, logp)
+        np.testing.assert_allclose(lps_n, lps_ref, rtol=1e-4, atol=1e-3)
+        targeted = np.unique(y[idx])
+        vrows = np.unique(np.concatenate([
+            rng.choice(targeted, 128, replace=False),
+            rng.choice(V, 128, replace=False), [V - 1]]))
+        dW_ref = oracle.head_dw_rows(Ha, Wf, y[idx], c, lse, vrows)
+        assert rel_fro(dW.cpu().numpy()[vrows], dW_ref) <= TOL
+        # dH rows: 1,024 sampled active tokens plus the two shortest active
+        # rollouts, from the same lse.
+        L = np.diff(cu)[act_r]
+        two = act_r[np.argsort(L)[:2]]
+        pos = np.nonzero(np.isin(seg, two))[0]
+        pos = np.unique(np.concatenate([rng.choice(idx.size, 1024, replace=False), pos]))
+        dH_ref = oracle.head_dh_rows(Ha[pos], Wf, y[idx[pos]], c[pos], lse[pos])
+        assert rel_fro(dH.cpu().numpy()[idx[pos]], dH_ref) <= TOL
+    else:
+        eight = rng.choice(act_r, 8, replace=False)
+        whole = np.nonzero(np.isin(seg, eight))[0]
+        pos = np.unique(np.concatenate([rng.choice(idx.size, 4096, replace=False), whole]))
+        Hs = hrows(idx[pos])
+        lse, zy = oracle.head_lse(Hs, Wf, y[idx[pos]], threads=nthr)
+        logp = zy - lse
+        _logp_close(lpt[idx[pos]], logp)
+        for i in eight:
+            sel = seg[pos] == i
+            assert sel.sum() == (seg == i).sum()
+            ref_i = float(logp[sel].sum())
+            assert abs(lps_n[i] - ref_i) <= 1e-4 * abs(ref_i) + 1e-3
+        sub = rng.choice(pos.size, 1024, replace=False)
+        dH_ref = oracle.head_dh_rows(Hs[sub], Wf, y[idx[pos[sub]]], c[pos[sub]], lse[sub])
+        assert rel_fro(dH.cpu().numpy()[idx[pos[sub]]], dH_ref) <= TOL
     # J is the coefficient-weighted sum of the per-rollout log-probabilities.
     assert abs(J - float(np.dot(a.astype(np.float64), lps_n.astype(np.float64)))) \
         <= 1e-4 * float(np.abs(a).dot(np.abs(lps_n)))
@@ -264,3 +329,41 @@ def test_grad_full_head_single_rollout_dw(name):
         [inp["V"] - 1]]))
     ref = oracle.pair_grad_ref(inp, a.astype(np.float64), dw_rows=vrows)
     assert rel_fro(dW.cpu().numpy()[vrows], ref["dW_rows"]) <= TOL
+
+
+@pytest.mark.parametrize("case", [("pr1_ref_fp32", None, None, None, None), 
+                                  ("qwen3_1p7b_head", 512, 1000, "default", 4.0),
+                                  ("qwen3_1p7b_head", 512, 1000, "min", 4.0),
+                                  ("longctx_skew", 256, 3000, "default", 2.0)],
+                         ids=["fp32", "bf16_image", "bf16_min_ws", "bf16_d256"])
+def test_token_logp_matches_oracle(case):
+    """pair_grad_token_logp returns every active token's logp (0 elsewhere),
+    for each head path, and sums to logp_seq per rollout."""
+    B = _binding()
+    name, d, V, ws_kind, wm = case
+    kw = {} if d is None else dict(B=3, G=8, d=d, V=V, len_scale=0.2, w_std_mult=wm)
+    inp = synth.make_head_workload(synth.WORKLOADS[name], 2, **kw)
+    a = _coeffs(inp)
+    if not (a != 0).any():
+        a[0] = 0.5
+    t = head_inputs(inp, a)
+    T, dd, VV, R = inp["T"], inp["d"], inp["V"], inp["R"]
+    dt = B.PAIR_BF16 if inp["dtype"] == "bf16" else B.PAIR_F32
+    size = (B.pair_grad_workspace_min_size if ws_kind == "min"
+            else B.pair_grad_workspace_size)(T, dd, VV, R, dt)
+    ws = torch.empty(size, dtype=torch.uint8, device="cuda")
+    err = dev_err_word()
+    _, _, _, lps = B.pair_grad(t["H"], t["W"], t["y"], t["mask"], t["cu_seqlens"], t["a"],
+                               ws=ws, dev_err=err)
+    assert B.pair_status_sync(err) == 0
+    lpt = B.pair_grad_token_logp(T, dd, VV, R, dt, ws).cpu().numpy()
+    ref = oracle.pair_grad_ref(inp, a.astype(np.float64), full=True)
+    idx = ref["active_tokens"]
+    _logp_close(lpt[idx], ref["logp"])
+    keep = np.zeros(T, bool)
+    keep[idx] = True
+    assert (lpt[~keep] == 0).all()
+    seg = oracle.segment_ids(inp["cu_seqlens"])
+    sums = np.zeros(R, np.float64)
+    np.add.at(sums, seg, lpt.astype(np.float64))
+    np.testing.assert_allclose(lps.cpu().numpy(), sums, rtol=1e-5, atol=1e-4)

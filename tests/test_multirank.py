@@ -2,8 +2,8 @@
 prompt groups (groups are independent: no data-path exchange). Each rank
 computes its groups' coefficients and head gradients with the fp64 oracle;
 the dW contributions are summed with an all-reduce, as a data-parallel
-trainer would, and must equal the single-process result over all groups.
-The timing reduction (max over ranks) used by bench.py is exercised too."""
+trainer would, and must equal the single-process result over all groups
+(the library itself is single-GPU; this exchange belongs to a trainer)."""
 import os
 import socket
 
