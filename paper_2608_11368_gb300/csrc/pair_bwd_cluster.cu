@@ -466,7 +466,174 @@ __global__ void tail_reduce_kernel(int d, int V, int ncl, int rb0, int cap,
   }
 }
 
-template <bool kTokenRows, int BN>
+// State of the fused log-sum-exp + dH pass (kFused; null otherwise).
+//
+// Every active token t gets a fixed reference R_t (log2 units) before the
+// pass: its target logit z_t[y_t] log2 e (target_logit_kernel), or, for the
+// row blocks the fix-up pass redoes, the row maximum found by the first pass.
+// The owner of a tile converts S to P = 2^(S log2 e - R_t) (bf16 operand of
+// the output MMA, which accumulates O_t = sum_v P_tv W_v) and adds the fp32 P
+// to its running l_t = sum_v P_tv; at the end of every unit each CTA writes
+// its l and row-maximum partials to lpart[slot][k] and counts itself into
+// ready[slot]; the drain waits for all kCl partials, sums them in CTA order
+// and writes dH_t = -c_t O_t / l_t and lse_t = (R_t + log2 l_t) ln 2. Since
+// z_t[y_t] <= max_v z_tv, P never underflows where it matters; a row whose
+// maximum exceeds R_t by more than kFixLog2 (P would approach the fp32 range)
+// flags its row block, and the fix-up pass redoes those blocks with R_t = the
+// row maximum. Tail units keep O, l and the maximum unscaled for
+// tail_fused_kernel.
+struct FusedArgs {
+  const float *ref;      // [Tpad] R_t, log2 units
+  float *lse;            // [Tpad] out: log-sum-exp (natural units)
+  float *mrow;           // [Tpad] out: row maximum of the logits, log2 units
+  int *rbflag;           // [n_rb] out: 1 = the row block needs the fix-up pass
+  float *lpart;          // [slots][kCl][2][128] per-CTA partials (l, max)
+  int *ready;            // [slots] CTAs that published their partials (zeroed)
+  float *tail_l;         // [kMaxClusters][2][2][128] cluster sums of tail units
+  const int *rb_list;    // row blocks to process (fix-up pass), or null
+  const int *n_list;     // their count (device), with rb_list
+};
+constexpr float kFixLog2 = 64.f;
+constexpr float kLn2 = 0.69314718055994531f;
+
+// Bounded wait until *ctr >= target (acquire at GPU scope).
+__device__ __forceinline__ bool wait_count(const int *ctr, int target, volatile int *abort,
+                                           int32_t *dev_err) {
+  const long long t0 = clock64();
+  while (true) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+    if (v >= target) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *abort = 1;
+      flag_error(dev_err, PAIR_DEV_ERR_TIMEOUT);
+      return false;
+    }
+    __nanosleep(64);
+  }
+}
+
+// z_t[y_t] = <Hc_p, W_{y_p}> for every compacted token p (fp32 sums of bf16
+// products, a fixed order per token: lane-strided 8-element pieces, then the
+// warp's butterfly) and its log2-unit reference R_p = z log2 e for the fused
+// pass; also zeroes the fused pass's counters and row-block flags.
+__global__ void target_logit_kernel(int d, const int32_t *counters, const int32_t *tok_y,
+                                    const __nv_bfloat16 *Hc, const __nv_bfloat16 *W,
+                                    float *zy, float *ref, int *ready, int n_ready, int *rbflag,
+                                    int n_rbflag) {
+  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int nth = gridDim.x * blockDim.x;
+  for (int i = tid; i < n_ready; i += nth) ready[i] = 0;
+  for (int i = tid; i < n_rbflag; i += nth) rbflag[i] = 0;
+  const int Teff = counters[0];
+  const int lane = threadIdx.x & 31;
+  for (int p = tid >> 5; p < Teff; p += nth >> 5) {
+    const __nv_bfloat16 *h = Hc + (int64_t)p * d;
+    const __nv_bfloat16 *w = W + (int64_t)tok_y[p] * d;
+    float acc = 0.f;
+    for (int k = lane * 8; k < d; k += 256) {
+      const uint4 hu = *reinterpret_cast<const uint4 *>(h + k);
+      const uint4 wu = *reinterpret_cast<const uint4 *>(w + k);
+      const __nv_bfloat162 *hb = reinterpret_cast<const __nv_bfloat162 *>(&hu);
+      const __nv_bfloat162 *wb = reinterpret_cast<const __nv_bfloat162 *>(&wu);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 hf = __bfloat1622float2(hb[i]), wf = __bfloat1622float2(wb[i]);
+        acc = fmaf(hf.x, wf.x, acc);
+        acc = fmaf(hf.y, wf.y, acc);
+      }
+    }
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) {
+      zy[p] = acc;
+      ref[p] = acc * kLog2e;
+    }
+  }
+}
+
+// Tail rows of the fused pass (see TileMap and FusedArgs): O, l and the row
+// maximum summed (maximum taken) in cluster order over the partial units that
+// cover the row, then dH_t = -c_t O_t / l_t, lse_t and the fix-up flag.
+template <int BN>
+__global__ void tail_fused_kernel(int d, int V, int ncl, const int32_t *counters,
+                                  const int32_t *tok_idx, const float *tok_c,
+                                  const float *tailbuf, FusedArgs fa, float *out) {
+  const int Teff = counters[0];
+  const int n_ct = (V + BN - 1) / BN;
+  const int n_rb = fa.rb_list ? *fa.n_list : (Teff + 127) / 128;
+  const int F = n_rb / ncl, R = n_rb - F * ncl;
+  if (R == 0) return;
+  const int64_t Tt = (int64_t)R * n_ct;
+  const int vec = d / 4;
+  const float4 *src = reinterpret_cast<const float4 *>(tailbuf);
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < (int64_t)R * 128 * vec;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int off = (int)(i / vec);
+    const int rl = off >> 7, rr = off & 127;
+    const int c4 = (int)(i % vec);
+    const int prb = fa.rb_list ? fa.rb_list[F * ncl + rl] : F * ncl + rl;
+    const int rid = prb * 128 + rr;
+    if (rid >= Teff) continue;
+    const int64_t lo = (int64_t)rl * n_ct, hi = lo + n_ct;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float L = 0.f, M = -INFINITY;
+    for (int c = 0; c < ncl; ++c) {
+      const int64_t a = Tt * c / ncl, b = Tt * (c + 1) / ncl;
+      if ((a > lo ? a : lo) < (b < hi ? b : hi)) {
+        const int u = rl - (int)(a / n_ct);
+        const float4 p = src[((int64_t)(c * 2 + u) * 128 + rr) * vec + c4];
+        acc.x += p.x; acc.y += p.y; acc.z += p.z; acc.w += p.w;
+        L += fa.tail_l[(c * 2 + u) * 256 + rr];
+        M = fmaxf(M, fa.tail_l[(c * 2 + u) * 256 + 128 + rr]);
+      }
+    }
+    const float R2 = fa.ref[rid];
+    const float scale = -tok_c[rid] / L;
+    reinterpret_cast<float4 *>(out + (int64_t)tok_idx[rid] * d)[c4] =
+        make_float4(acc.x * scale, acc.y * scale, acc.z * scale, acc.w * scale);
+    if (c4 == 0) {
+      const float M2 = M * kLog2e;
+      fa.lse[rid] = (R2 + log2f(L)) * kLn2;
+      fa.mrow[rid] = M2;
+      if (!(L > 0.f) || !(L < INFINITY) || !(M2 - R2 <= kFixLog2)) fa.rbflag[prb] = 1;
+    }
+  }
+}
+
+// Between the fused pass and its fix-up: the flagged row blocks, in order,
+// become the fix-up pass's list (count in *n_list), their rows' reference
+// becomes the row maximum the first pass found, and the pass counters are
+// zeroed again. One block.
+__global__ void fixup_prep_kernel(const int32_t *counters, const int *rbflag, int *rb_list,
+                                  int *n_list, float *ref, const float *mrow, int *ready,
+                                  int n_ready) {
+  __shared__ int count;
+  const int Teff = counters[0];
+  const int n_rb = (Teff + 127) / 128;
+  for (int i = threadIdx.x; i < n_ready; i += blockDim.x) ready[i] = 0;
+  if (threadIdx.x < 32) {
+    int base = 0;
+    for (int r0 = 0; r0 < n_rb; r0 += 32) {
+      const int r = r0 + (int)threadIdx.x;
+      const bool f = r < n_rb && rbflag[r] != 0;
+      const unsigned bal = __ballot_sync(0xffffffffu, f);
+      if (f) rb_list[base + __popc(bal & ((1u << threadIdx.x) - 1u))] = r;
+      base += __popc(bal);
+    }
+    if (threadIdx.x == 0) {
+      count = base;
+      *n_list = base;
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < count * 128; i += blockDim.x) {
+    const int p = rb_list[i >> 7] * 128 + (i & 127);
+    if (p < Teff) ref[p] = mrow[p];
+  }
+}
+
+template <bool kTokenRows, int BN, bool kFused = false>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
     bwd_cluster_kernel(const __grid_constant__ CUtensorMap tmR,
                        const __grid_constant__ CUtensorMap tmC,
@@ -474,7 +641,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
                        const int32_t *counters, const int32_t *tok_idx,
                        const float *tok_c, const float *lse, float *out,
                        uint8_t *gring, uint8_t *gimg, float *tailbuf, int rb0, int cap,
-                       int32_t *dev_err) {
+                       FusedArgs fa, int32_t *dev_err) {
   extern __shared__ uint8_t smem_raw[];
   ClSmem<BN> &sm = *reinterpret_cast<ClSmem<BN> *>(align1k(smem_raw));
   using Tl = ClTile<BN>;
@@ -496,8 +663,13 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   const int A0 = ksplit ? A : (A + 1) >> 1, A1 = ksplit ? A : A - A0;
   // Row blocks [rb0, rb0 + n_rb) of this launch (one chunk); TileMap and
   // TileCursor count them from 0.
-  const int n_rb = min(max((kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128) - rb0, 0), cap);
+  const int n_rb = (kFused && fa.rb_list)
+                       ? min(*fa.n_list, cap)
+                       : min(max((kTokenRows ? (Teff + 127) / 128 : (V + 127) / 128) - rb0, 0), cap);
   const int n_ct = kTokenRows ? (V + BN - 1) / BN : (Teff + BN - 1) / BN;
+  // Row block of the launch's row-block index rb (TileMap counts from 0): the
+  // chunk's rb0 + rb, or the fix-up pass's list entry.
+  auto phys_rb = [&](int rb) { return (kFused && fa.rb_list) ? fa.rb_list[rb] : rb0 + rb; };
   const int n_my = cid < n_rb ? (n_rb - cid + ncl - 1) / ncl : 0;
   TileMap mp;
   mp.setup(n_rb, n_ct, cid, ncl);
@@ -582,7 +754,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           if (!(ok = wait(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
           if (elect_one()) {
             mbar_expect_tx(&sm.full[stage], kAtom128 + kColAtom);
-            tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, (rb0 + job_rb) * 128);
+            tma_load_2d(sm.a[stage], &tmR, &sm.full[stage], a * 64, phys_rb(job_rb) * 128);
             tma_load_2d(sm.b[stage], &tmC, &sm.full[stage], a * 64, job_ct * BN);
           }
           __syncwarp();
@@ -807,6 +979,17 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
     bool ok = true;
     TileCursor cur;  // tile of slot s (s >= 0), for unit drains
     cur.init(mp, 0);
+    // kFused: this thread's row partials (sum of P, maximum logit) over the
+    // tiles this CTA owns in the current unit, and the tile of the
+    // conversion phase (to find unit ends).
+    float lacc = 0.f, macc = -INFINITY;
+    TileCursor cg;
+    cg.init(mp, 0);
+    // Slot of the fused partials of the unit holding a tile: full units by
+    // row block, tail units after them by (cluster, tail unit).
+    auto fused_slot = [&](const TileCursor &t) {
+      return mp.tail(t.g) ? n_rb + 2 * cid + ((t.rb - mp.rbT) - mp.t0 / mp.n_ct) : t.rb;
+    };
     for (int s = -kClJ; s < N && ok; ++s) {
       const int g = s + kClLag + 1;  // tile whose S completes in slot s
       if (g >= 0 && g < N && (g & (kCl - 1)) == k) {
@@ -817,8 +1000,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         const int rb = gt.rb, ct = gt.ct;
         float rc = 0.f, rl = 0.f;
         if (kTokenRows) {
-          const int p = (rb0 + rb) * 128 + row;
-          if (p < Teff) { rc = tok_c[p]; rl = lse[p] * kLog2e; }
+          const int p = phys_rb(rb) * 128 + row;
+          if (p < Teff) { rc = tok_c[p]; rl = kFused ? fa.ref[p] : lse[p] * kLog2e; }
         } else {
           epi_sync();
           const int p = ct * BN + row;
@@ -838,6 +1021,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         }
         tc_fence_after();
         uint8_t *dst_tile = gs_tile(g, rb, ct);
+        float tsum = 0.f, tmax = -INFINITY;
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
           float v[32];
@@ -858,7 +1042,14 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
                 cc = sm.col_c[col]; ll = sm.col_l[col];
                 live = cc != 0.f;
               }
-              g2[e] = live ? -cc * ex2_approx(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
+              if (kFused) {
+                // P = 2^(z log2 e - R_t); l and the maximum from the fp32 values.
+                g2[e] = live ? ex2_approx(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
+                tsum += g2[e];
+                if (live) tmax = fmaxf(tmax, v[j + e]);
+              } else {
+                g2[e] = live ? -cc * ex2_approx(fmaf(v[j + e], kLog2e, -ll)) : 0.f;
+              }
             }
             __nv_bfloat162 b2 = __floats2bfloat162_rn(g2[0], g2[1]);
             pk[j >> 1] = *reinterpret_cast<uint32_t *>(&b2);
@@ -870,6 +1061,10 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
                                        sw128_offset(row, kc & 63)) =
                 make_uint4(pk[q * 4], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
           }
+        }
+        if (kFused) {
+          lacc += tsum;
+          macc = fmaxf(macc, tmax);
         }
         tc_fence_before();
         mbar_arrive(&sm.s_empty[buf]);
@@ -884,20 +1079,69 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           mbar_arrive_cluster_relaxed(mapa(smem_u32(&sm.pub[k][m & 1]), (uint32_t)lane));
         }
       }
+      if (kFused && g >= 0 && g < N) {
+        // Every CTA passes every tile g in order; at the last tile of a unit
+        // it has converted all of its own tiles of that unit and publishes
+        // its row partials (a CTA owning none of them publishes zeros).
+        if (cg.unit_end(mp)) {
+          const int slot = fused_slot(cg);
+          float *lp = fa.lpart + ((size_t)slot * kCl + k) * 256;
+          lp[row] = lacc;
+          lp[128 + row] = macc;
+          __threadfence();
+          epi_sync();
+          if (warp == 2 && lane == 0) {
+            __threadfence();
+            atomicAdd(&fa.ready[slot], 1);
+          }
+          lacc = 0.f;
+          macc = -INFINITY;
+        }
+        cg.next(mp);
+      }
       if (s < 0) continue;
       const bool unit_end = cur.unit_end(mp);
       const bool tail = mp.tail(cur.g);
       const int rb = cur.rb;
       // A tail unit's slot: its row block's place among this cluster's tail units.
       const int tu = tail ? (rb - mp.rbT) - mp.t0 / mp.n_ct : 0;
+      const int fslot = kFused ? fused_slot(cur) : 0;
       cur.next(mp);
       if (unit_end) {
         // Drain the finished unit: out[rows, k*w : (k+1)*w].
         if (!(ok = wait_sleepy(&sm.o_full, o_ph, abort, dev_err))) break;
         o_ph ^= 1;
         tc_fence_after();
-        const int rid = (rb0 + rb) * 128 + row;
+        const int rid = phys_rb(rb) * 128 + row;
         const bool valid = kTokenRows ? (rid < Teff) : (rid < V);
+        float scale = 1.f;
+        if (kFused) {
+          // The unit's l and maximum: all kCl CTAs' partials, in CTA order.
+          if (!(ok = wait_count(&fa.ready[fslot], kCl, abort, dev_err))) break;
+          const float *lp = fa.lpart + (size_t)fslot * kCl * 256;
+          float L = 0.f, M = -INFINITY;
+#pragma unroll 1
+          for (int j = 0; j < kCl; ++j) {
+            L += __ldcg(lp + j * 256 + row);
+            M = fmaxf(M, __ldcg(lp + j * 256 + 128 + row));
+          }
+          if (tail) {
+            if (k == 0) {
+              fa.tail_l[(cid * 2 + tu) * 256 + row] = L;
+              fa.tail_l[(cid * 2 + tu) * 256 + 128 + row] = M;
+            }
+          } else if (valid) {
+            const float R = fa.ref[rid];
+            scale = -tok_c[rid] / L;
+            if (k == 0) {
+              const float M2 = M * kLog2e;
+              fa.lse[rid] = (R + log2f(L)) * kLn2;
+              fa.mrow[rid] = M2;
+              if (!(L > 0.f) || !(L < INFINITY) || !(M2 - R <= kFixLog2))
+                fa.rbflag[phys_rb(rb)] = 1;
+            }
+          }
+        }
         float *dst = nullptr;
         if (tail)
           dst = tailbuf + ((int64_t)(cid * 2 + tu) * 128 + row) * d + k * w;
@@ -911,7 +1155,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
 #pragma unroll
             for (int q = 0; q < 8; ++q)
               reinterpret_cast<float4 *>(dst + c * 32)[q] =
-                  make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                  make_float4(v[4 * q] * scale, v[4 * q + 1] * scale, v[4 * q + 2] * scale,
+                              v[4 * q + 3] * scale);
           }
         }
         tc_fence_before();
@@ -983,7 +1228,7 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
   PAIR_BEGIN("bwd_dh_tc", s);
   bwd_cluster_kernel<true, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
       mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH, gring, nullptr,
-      w.tailbuf, 0, kAll, g.dev_err);
+      w.tailbuf, 0, kAll, FusedArgs{}, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("tail_dh", s);
   tail_reduce_kernel<true, BN><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, 0, kAll, w.counters,
@@ -992,7 +1237,64 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
   PAIR_BEGIN("bwd_dw_tc", s);
   bwd_cluster_kernel<false, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
       mW128, mHc, mHc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW, gring, nullptr,
-      w.tailbuf, 0, kAll, g.dev_err);
+      w.tailbuf, 0, kAll, FusedArgs{}, g.dev_err);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("tail_dw", s);
+  tail_reduce_kernel<false, BN><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, 0, kAll, w.counters,
+                                                    w.tok_idx, w.tailbuf, g.dW);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
+// The whole bf16 head without keeping any logit-sized tensor: target logits,
+// the fused log-sum-exp + dH pass (and its fix-up for flagged row blocks),
+// then dW by the recomputing cluster kernel. 4 logit-sized GEMMs per call.
+template <int BN>
+pair_status grad_head_fused(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  CUtensorMap mH, mW128, mHc, mWc, mHc64, mWc64;
+  if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) || !make_map(&mW128, g.W, g.V, g.d, 128) ||
+      !make_map(&mHc, w.Hc, w.Tpad, g.d, BN) || !make_map(&mWc, g.W, g.V, g.d, BN) ||
+      !make_map(&mHc64, w.Hc, w.Tpad, g.d, 64) || !make_map(&mWc64, g.W, g.V, g.d, 64))
+    return PAIR_ERR_CUDA;
+  const int nsm = num_sms();
+  const size_t cl_smem = sizeof(ClSmem<BN>) + 1024;
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<true, BN, true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(bwd_cluster_kernel<false, BN>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cl_smem));
+  const int ncl = cluster_grid<BN>((const void *)bwd_cluster_kernel<false, BN>, cl_smem);
+  uint8_t *gring = static_cast<uint8_t *>(w.gring);
+  constexpr int kAll = 0x7fffffff;
+  const __nv_bfloat16 *Hc = static_cast<const __nv_bfloat16 *>(w.Hc);
+  const __nv_bfloat16 *W = static_cast<const __nv_bfloat16 *>(g.W);
+  PAIR_BEGIN("target_logit", s);
+  target_logit_kernel<<<nsm * 8, 256, 0, s>>>(g.d, w.counters, w.tok_y, Hc, W, w.zy, w.ref,
+                                              w.ready, w.n_slots, w.rbflag, w.n_rbmax);
+  PAIR_LAUNCH_CHECK(s);
+  FusedArgs fa{w.ref, w.lse, w.mrow, w.rbflag, w.lpart, w.ready, w.tail_l, nullptr, nullptr};
+  for (int pass = 0; pass < 2; ++pass) {
+    if (pass == 1) {
+      PAIR_BEGIN("fixup_prep", s);
+      fixup_prep_kernel<<<1, 1024, 0, s>>>(w.counters, w.rbflag, w.rb_list, w.counters + 1,
+                                           w.ref, w.mrow, w.ready, w.n_slots);
+      PAIR_LAUNCH_CHECK(s);
+      fa.rb_list = w.rb_list;
+      fa.n_list = w.counters + 1;
+    }
+    PAIR_BEGIN(pass == 0 ? "lse_dh_tc" : "lse_dh_fixup", s);
+    bwd_cluster_kernel<true, BN, true><<<ncl * kCl, kClThreads, cl_smem, s>>>(
+        mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, nullptr, g.dH, gring, nullptr,
+        w.tailbuf, 0, kAll, fa, g.dev_err);
+    PAIR_LAUNCH_CHECK(s);
+    PAIR_BEGIN("tail_lse_dh", s);
+    tail_fused_kernel<BN><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, w.counters, w.tok_idx, w.tok_c,
+                                               w.tailbuf, fa, g.dH);
+    PAIR_LAUNCH_CHECK(s);
+  }
+  PAIR_BEGIN("bwd_dw_tc", s);
+  bwd_cluster_kernel<false, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
+      mW128, mHc, mHc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW, gring, nullptr,
+      w.tailbuf, 0, kAll, FusedArgs{}, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("tail_dw", s);
   tail_reduce_kernel<false, BN><<<nsm, 256, 0, s>>>(g.d, g.V, ncl, 0, kAll, w.counters,
@@ -1004,6 +1306,19 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
 }  // namespace
 
 namespace tck {
+
+// The bf16 head without a logit-gradient image: the fused log-sum-exp + dH
+// pass and the recomputing dW pass (cluster form), for the hidden sizes the
+// cluster kernels take; false elsewhere (the caller runs the three passes).
+bool onchip_fused_applies(int d) { return use_cluster_path(d); }
+
+pair_status grad_head_onchip(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  switch (cluster_tile_width(g.d)) {
+    case 128: return grad_head_fused<128>(g, w, s);
+    case 96: return grad_head_fused<96>(g, w, s);
+    default: return grad_head_fused<64>(g, w, s);
+  }
+}
 
 // Softmax parts of dH and dW, recomputing the logits.
 pair_status grad_bwd_recompute(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {

@@ -79,6 +79,15 @@ struct GradWorkspace {
   void *Hc;            // [Tpad][d] compacted hidden rows (dt), zero tail
   void *gring;         // per-cluster ring of published Gs tiles
   float *tailbuf;      // [kMaxClusters][2][128][d] partial tail units (cluster path)
+  // Fused log-sum-exp + dH pass (cluster path; null otherwise).
+  float *ref;          // [Tpad] per-token reference of the softmax terms (log2 units)
+  float *mrow;         // [Tpad] row maximum of the logits (log2 units)
+  int32_t *rbflag;     // [n_rbmax] row block needs the fix-up pass
+  int32_t *rb_list;    // [n_rbmax] row blocks of the fix-up pass (count in counters[1])
+  int32_t *ready;      // [n_slots] per-unit publication counters
+  float *lpart;        // [n_slots][8][2][128] per-CTA row partials (l, maximum)
+  float *tail_l;       // [kMaxClusters][2][2][128] tail units' row partials
+  int n_rbmax, n_slots;
   void *gimg;          // bf16 logit-gradient tiles of gimg_rb token blocks, or null
   void *sbuf;          // fp16 chunk-relative logit terms of the same blocks (LSE pass)
   float4 *mbuf;        // fp32 maxima of their 32-column chunks, one float4 per tile row

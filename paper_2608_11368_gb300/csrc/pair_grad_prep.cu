@@ -411,6 +411,15 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   const size_t o_ring = dt == PAIR_BF16 ? take((size_t)kMaxClusters * kRingBytesPerCluster) : off;
   const bool cl = dt == PAIR_BF16 && grad_cluster_path(d);
   const size_t o_tail = cl ? take((size_t)kMaxClusters * 2 * 128 * d * sizeof(float)) : off;
+  const int n_rbmax = (int)(Tpad / 128);
+  const int n_slots = n_rbmax + 2 * kMaxClusters;
+  const size_t o_ref = cl ? take((size_t)Tpad * 4) : off;
+  const size_t o_mrow = cl ? take((size_t)Tpad * 4) : off;
+  const size_t o_rbflag = cl ? take((size_t)n_rbmax * 4) : off;
+  const size_t o_rblist = cl ? take((size_t)n_rbmax * 4) : off;
+  const size_t o_ready = cl ? take((size_t)n_slots * 4) : off;
+  const size_t o_lpart = cl ? take((size_t)n_slots * 8 * 256 * 4) : off;
+  const size_t o_taill = cl ? take((size_t)kMaxClusters * 2 * 256 * 4) : off;
   // The image comes last, so that a larger workspace only adds token blocks.
   const size_t n_vt = (size_t)((V + 127) / 128);
   const size_t o_gimg = gimg_rb ? take((size_t)gimg_rb * n_vt * kGImgTileBytes) : off;
@@ -433,6 +442,15 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->Hc = b + o_hc;
     out->gring = b + o_ring;
     out->tailbuf = cl ? reinterpret_cast<float *>(b + o_tail) : nullptr;
+    out->ref = cl ? reinterpret_cast<float *>(b + o_ref) : nullptr;
+    out->mrow = cl ? reinterpret_cast<float *>(b + o_mrow) : nullptr;
+    out->rbflag = cl ? reinterpret_cast<int32_t *>(b + o_rbflag) : nullptr;
+    out->rb_list = cl ? reinterpret_cast<int32_t *>(b + o_rblist) : nullptr;
+    out->ready = cl ? reinterpret_cast<int32_t *>(b + o_ready) : nullptr;
+    out->lpart = cl ? reinterpret_cast<float *>(b + o_lpart) : nullptr;
+    out->tail_l = cl ? reinterpret_cast<float *>(b + o_taill) : nullptr;
+    out->n_rbmax = n_rbmax;
+    out->n_slots = n_slots;
     out->gimg = gimg_rb ? b + o_gimg : nullptr;
     out->sbuf = gimg_rb ? b + o_sbuf : nullptr;
     out->mbuf = gimg_rb ? reinterpret_cast<float4 *>(b + o_mbuf) : nullptr;

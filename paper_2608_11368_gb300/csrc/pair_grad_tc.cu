@@ -149,8 +149,10 @@ pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t 
 // device-to-host read; chunks past the last active token exit at once.
 //
 // Whole head: with an image, each chunk's log-sum-exp pass keeps its logits
-// for that chunk's backward (no recomputation); otherwise forward, then the
-// recomputing backward.
+// for that chunk's backward (no recomputation); otherwise, where the cluster
+// kernels apply, the fused log-sum-exp + dH pass and the recomputing dW pass
+// (no logit-sized tensor in HBM), else forward, then the recomputing
+// backward.
 pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
   if (image_path(w)) {
     const int64_t nc = image_chunks(g, w);
@@ -161,6 +163,7 @@ pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t
     }
     return PAIR_OK;
   }
+  if (onchip_fused_applies(g.d)) return grad_head_onchip(g, w, s);
   const pair_status st = grad_lse_tc(g, w, s);
   return st != PAIR_OK ? st : grad_bwd_tc(g, w, s);
 }

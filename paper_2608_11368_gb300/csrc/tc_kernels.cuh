@@ -75,6 +75,11 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
                              int64_t c);
 // Backward without an image, recomputing the logits (pair_bwd_cluster.cu).
 pair_status grad_bwd_recompute(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
+// Whole head without an image: fused log-sum-exp + dH, then dW (cluster
+// form; d = 512 A, A <= 6). lse, zy and dH, dW softmax parts as the
+// three-pass sequence leaves them.
+bool onchip_fused_applies(int d);
+pair_status grad_head_onchip(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
 
 inline bool image_path(const GradWorkspace &w) { return w.gimg && w.sbuf && w.gimg_rb > 0; }
 inline int64_t image_chunks(const GradArgs &g, const GradWorkspace &w) {
