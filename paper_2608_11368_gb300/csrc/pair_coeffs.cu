@@ -276,10 +276,10 @@ __global__ void __launch_bounds__(256, 4) dense_staged_kernel(
       tc::fence_mbar_init();
     }
     __syncwarp();
-    issue_group(sm.stage, bar, rho, r, J, b, G, stream_rows(G, sm.Qt, geom.group_bytes));
+    issue_group(sm.stage, bar, rho, r, load_j_word(J, b, B, G), b, G,
+                stream_rows(G, sm.Qt, geom.group_bytes));
     const bool ok = __all_sync(0xffffffffu, tc::wait(bar, 0u, abort, dev_err));
     if (!ok) drain_wait(bar, 0u);
-    cp_async_wait<0>();
     __syncwarp();
     WarpCoeffs o = {};
     if (ok)

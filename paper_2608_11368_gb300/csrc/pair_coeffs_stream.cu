@@ -38,6 +38,11 @@ __global__ void __launch_bounds__(kSW * 32, 1) coeffs_stream_kernel(
   extern __shared__ __align__(16) unsigned char smem_raw[];
   StreamSmem &sm = *reinterpret_cast<StreamSmem *>(smem_raw);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  // Launched as a programmatic dependent of the previous kernel in the
+  // stream: a following launch of this kernel may be scheduled as soon as
+  // every block got here, and its prologue (which reads no global memory)
+  // overlaps this launch's tail.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   stream_qt(geom, sm.Qt);
   __syncthreads();  // the only block-wide barrier: warps are independent after it
   // Groups dealt warp-major (b = warp * blocks + block, stride all warps),
@@ -60,6 +65,9 @@ __global__ void __launch_bounds__(kSW * 32, 1) coeffs_stream_kernel(
     tc::fence_mbar_init();
   }
   __syncwarp();
+  // Every global read below happens after the previous grid in the stream
+  // has completed and its writes are visible.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 
   uint32_t ph = 0;       // bit s: parity of the next completion of stage s
   uint32_t pending = 0;  // bit s: stage s has copies issued and not yet waited for
@@ -67,12 +75,13 @@ __global__ void __launch_bounds__(kSW * 32, 1) coeffs_stream_kernel(
   for (int s = 0; s < kStages - 1; ++s) {
     const int b = b0 + s * nw;
     if (b < B) {
-      issue_group(wbase + s * kStageBytes, &bar[s], rho, r, J, b, G, rc);
+      issue_group(wbase + s * kStageBytes, &bar[s], rho, r, load_j_word(J, b, B, G), b, G, rc);
       pending |= 1u << s;
-    } else {
-      cp_async_commit();
     }
   }
+  // Completion flags of the next group to issue, loaded one group ahead (the
+  // row copies depend on them).
+  uint32_t jnext = load_j_word(J, b0 + (kStages - 1) * nw, B, G);
 
   int it = 0;
   for (int b = b0; b < B; b += nw, ++it) {
@@ -81,17 +90,15 @@ __global__ void __launch_bounds__(kSW * 32, 1) coeffs_stream_kernel(
       const int sn = (it + kStages - 1) % kStages;
       const int bn = b + (kStages - 1) * nw;
       if (bn < B) {
-        issue_group(wbase + sn * kStageBytes, &bar[sn], rho, r, J, bn, G, rc);
+        issue_group(wbase + sn * kStageBytes, &bar[sn], rho, r, jnext, bn, G, rc);
         pending |= 1u << sn;
-      } else {
-        cp_async_commit();
       }
+      jnext = load_j_word(J, bn + nw, B, G);
     }
     if (!__all_sync(0xffffffffu, tc::wait(&bar[s], (ph >> s) & 1u, abort, dev_err)))
       break;  // timed out (error flagged); warp-uniform
     ph ^= 1u << s;
     pending &= ~(1u << s);
-    cp_async_wait<kStages - 1>();
     __syncwarp();
     const WarpCoeffs o = warp_group_coeffs<WM, DIAG>(wbase + s * kStageBytes, sm.Qt, dg, G,
                                                      scale, flags, w_max, aux, dev_err);
@@ -119,7 +126,6 @@ __global__ void __launch_bounds__(kSW * 32, 1) coeffs_stream_kernel(
 #pragma unroll
   for (int s = 0; s < kStages; ++s)
     if (pending & (1u << s)) drain_wait(&bar[s], (ph >> s) & 1u);
-  cp_async_wait<0>();
 }
 
 template <int WM, bool DIAG>
@@ -136,10 +142,20 @@ pair_status launch_stream(int32_t B, int32_t G, const float *r, const uint8_t *J
   // One block per SM (groups are dealt warp-major, so a small batch still
   // spreads over the SMs).
   const int blocks = (int)std::min<int64_t>(B, nsm > 0 ? nsm : 1);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(blocks, 1, 1);
+  cfg.blockDim = dim3(kSW * 32, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
   PAIR_BEGIN(DIAG ? "coeffs_w" : "coeffs", s);
-  coeffs_stream_kernel<WM, DIAG><<<blocks, kSW * 32, smem, s>>>(
-      B, G, r, J, rho, scale, flags, w_max, a, active, edges, contrast, ess, max_w, dev_err,
-      make_stream_geom(G));
+  PAIR_CUDA_TRY(cudaLaunchKernelEx(&cfg, coeffs_stream_kernel<WM, DIAG>, B, G, r, J, rho, scale,
+                                   flags, w_max, a, active, edges, contrast, ess, max_w, dev_err,
+                                   make_stream_geom(G)));
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }

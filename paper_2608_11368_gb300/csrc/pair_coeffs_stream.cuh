@@ -7,9 +7,10 @@
 //
 // for groups of at most 64 candidates with G a multiple of 4.
 //
-// Staging: the strict upper triangle of rho_g is copied by bulk copies (one
-// per row) completing on an mbarrier, row i from column (i + 1) rounded down
-// to a multiple of 4 up to G - 1; each row is preceded by a gap of at least
+// Staging: the strict upper triangle rows of the group's completed vertices
+// (no other row is ever read) are copied by bulk copies (one per row)
+// completing on an mbarrier, row i from column (i + 1) rounded down to a
+// multiple of 4 up to G - 1; each row is preceded by a gap of at least
 // 4 floats, widened so that row bases fall in different shared-memory banks
 // (lanes reading one column of many rows then conflict less). Entry (i, j)
 // sits at float Qt[i] + j of the stage. Gap cells hold +inf (written once),
@@ -43,17 +44,6 @@ constexpr int kWarpAux = 64 * 4 * 3 + 32;               // packed r, column, Q; 
 constexpr float kRhoMin = 1.17549435e-38f;              // 2^-126, smallest normal float
 
 using tc::smem_u32;
-__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
 
 // First staged column of upper-triangle row i (i + 1 rounded down to 4).
 __host__ __device__ __forceinline__ int row_col0(int i) { return (i + 1) & ~3; }
@@ -189,26 +179,44 @@ __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
   }
 }
 
-// Issues group b into `stage` (whole warp): the expected bytes on `bar`, the
-// bulk copies of the triangle rows and rewards, and the completion flags as
-// 4-byte cp.async copies (one cp.async group per lane, possibly empty). The
-// warp's earlier reads and writes of the stage are ordered before the copies.
+// This lane's 4 completion flags of group b (lanes 0 .. G/4 - 1; 0 elsewhere
+// and past the last group). J is 4-byte aligned and G a multiple of 4.
+__device__ __forceinline__ uint32_t load_j_word(const uint8_t *J, int b, int B, int G) {
+  const int lane = threadIdx.x & 31;
+  if (b >= B || lane >= (G >> 2)) return 0u;
+  return __ldg(reinterpret_cast<const uint32_t *>(J + (size_t)b * G) + lane);
+}
+
+// Issues group b into `stage` (whole warp; jw = this lane's load_j_word of
+// group b): the expected bytes on `bar`, a bulk copy of the triangle row of
+// every completed vertex (the collapse reads no other row: an edge needs
+// both endpoints completed) and of the rewards, and the completion flags
+// stored from registers. The warp's earlier reads and writes of the stage
+// are ordered before the copies.
 __device__ __forceinline__ void issue_group(unsigned char *stage, uint64_t *bar,
-                                            const float *rho, const float *r, const uint8_t *J,
+                                            const float *rho, const float *r, uint32_t jw,
                                             int b, int G, const RowCopies &rc) {
   const int lane = threadIdx.x & 31;
+  // Flags of rows lane and lane + 32 (byte v & 3 of lane v >> 2's word).
+  const uint32_t w0 = __shfl_sync(0xffffffffu, jw, lane >> 2);
+  const uint32_t w1 = __shfl_sync(0xffffffffu, jw, (lane + 32) >> 2);
+  const int sh = 8 * (lane & 3);
+  const bool c0 = rc.src0 >= 0 && ((w0 >> sh) & 0xffu) != 0u;
+  const bool c1 = rc.src1 >= 0 && ((w1 >> sh) & 0xffu) != 0u;
+  uint32_t tx = (c0 ? rc.by0 : 0u) + (c1 ? rc.by1 : 0u);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) tx += __shfl_xor_sync(0xffffffffu, tx, o);
+  tx += 4u * (uint32_t)G;
   fence_proxy_async_smem();
   __syncwarp();
-  if (lane == 0) tc::mbar_expect_tx(bar, rc.group_bytes);
+  if (lane == 0) tc::mbar_expect_tx(bar, tx);
   __syncwarp();
   const float *rho_g = rho + (size_t)b * G * G;
   float *tri = reinterpret_cast<float *>(stage);
-  if (rc.src0 >= 0) bulk_g2s(tri + rc.dst0, rho_g + rc.src0, rc.by0, bar);
-  if (rc.src1 >= 0) bulk_g2s(tri + rc.dst1, rho_g + rc.src1, rc.by1, bar);
+  if (c0) bulk_g2s(tri + rc.dst0, rho_g + rc.src0, rc.by0, bar);
+  if (c1) bulk_g2s(tri + rc.dst1, rho_g + rc.src1, rc.by1, bar);
   if (lane == 31) bulk_g2s(stage + kTriBytes, r + (size_t)b * G, 4u * (uint32_t)G, bar);
-  if (lane < (G >> 2))
-    cp_async4(stage + kTriBytes + 256 + 4 * lane, J + (size_t)b * G + 4 * lane);
-  cp_async_commit();
+  if (lane < (G >> 2)) reinterpret_cast<uint32_t *>(stage + kTriBytes + 256)[lane] = jw;
 }
 
 // Reciprocal by the hardware approximation (PTX rcp.approx.ftz.f32: at most
