@@ -419,6 +419,125 @@ pair_status launch_coeffs_w_gp(int32_t B, int32_t G, const float *r, const uint8
   return PAIR_OK;
 }
 
+// Product design for G <= 64: one warp per group. Lane c holds vertices c
+// and c + 32; the completed ones are packed (vertex order) into the warp's
+// shared lists of r and q = 1/p (IEEE reciprocal, as the block form), and
+// each completed vertex i sums its terms (r_i - r_j) q_j over every packed
+// partner (its own slot adds an exact 0) in a fixed order: four interleaved
+// partial sums combined pairwise. a_i = 1/2 q_i sum; the weight diagnostics
+// sum q_i q_j over the pairs i < j of packed slots.
+template <bool DIAG>
+__global__ void __launch_bounds__(128) coeffs_product_warp_kernel(
+    int B, int G, const float *__restrict__ r, const uint8_t *__restrict__ J,
+    const float *__restrict__ p, float scale, uint32_t flags, float *__restrict__ a,
+    uint8_t *__restrict__ active, int32_t *__restrict__ edges, int32_t *__restrict__ contrast,
+    float *__restrict__ ess, float *__restrict__ max_w, int32_t *dev_err) {
+  __shared__ float pr[4][64], pq[4][64];
+  const int lane = threadIdx.x & 31, wi = threadIdx.x >> 5;
+  const int b = blockIdx.x * 4 + wi;
+  if (b >= B) return;  // warp-uniform; the warps of a block never synchronise
+  const size_t gb = (size_t)b * G;
+  float rv[2], qv[2];
+  bool cv[2];
+  int bad = 0;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int v = lane + 32 * h;
+    const bool in = v < G;
+    const bool j = in && J[gb + v] != 0;
+    const float pv = in ? p[gb + v] : 1.f;
+    if (j && !(pv > 0.f)) bad = 1;
+    cv[h] = j && pv > 0.f;
+    rv[h] = in ? r[gb + v] : 0.f;
+    qv[h] = cv[h] ? __frcp_rn(pv) : 0.f;
+  }
+  if (__any_sync(0xffffffffu, bad) && lane == 0)
+    flag_error(dev_err, PAIR_DEV_ERR_NONPOSITIVE_INCLUSION);
+  const unsigned m0 = __ballot_sync(0xffffffffu, cv[0]), m1 = __ballot_sync(0xffffffffu, cv[1]);
+  const unsigned lt = (1u << lane) - 1u;
+  const int K0 = __popc(m0), K = K0 + __popc(m1);
+  const int slot[2] = {__popc(m0 & lt), K0 + __popc(m1 & lt)};
+#pragma unroll
+  for (int h = 0; h < 2; ++h)
+    if (cv[h]) {
+      pr[wi][slot[h]] = rv[h];
+      pq[wi][slot[h]] = qv[h];
+    }
+  __syncwarp();
+  float av[2] = {0.f, 0.f};
+  int diff[2] = {0, 0};
+  float sw = 0.f, sw2 = 0.f, mw = 0.f;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    if (!cv[h]) continue;
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    int nd = 0;
+    int kk = 0;
+    for (; kk + 4 <= K; kk += 4) {
+      const float r0 = pr[wi][kk], r1 = pr[wi][kk + 1], r2 = pr[wi][kk + 2], r3 = pr[wi][kk + 3];
+      s0 += (rv[h] - r0) * pq[wi][kk];
+      s1 += (rv[h] - r1) * pq[wi][kk + 1];
+      s2 += (rv[h] - r2) * pq[wi][kk + 2];
+      s3 += (rv[h] - r3) * pq[wi][kk + 3];
+      nd += (r0 != rv[h]) + (r1 != rv[h]) + (r2 != rv[h]) + (r3 != rv[h]);
+    }
+    for (; kk < K; ++kk) {
+      const float rk = pr[wi][kk];
+      const float x = (rv[h] - rk) * pq[wi][kk];
+      if ((kk & 3) == 0) s0 += x; else if ((kk & 3) == 1) s1 += x; else s2 += x;
+      nd += rk != rv[h];
+    }
+    const float sum = (s0 + s1) + (s2 + s3);
+    av[h] = (sum == 0.f) ? 0.f : 0.5f * qv[h] * sum;
+    diff[h] = nd;
+    if (DIAG)
+      for (int k2 = slot[h] + 1; k2 < K; ++k2) {
+        const float w = qv[h] * pq[wi][k2];
+        sw += w;
+        sw2 = fmaf(w, w, sw2);
+        mw = fmaxf(mw, w);
+      }
+  }
+  if ((flags & PAIR_STANDARDIZE) && K >= 2) {
+    // Sample standard deviation (n - 1) of the completed rewards, two-pass.
+    const float mean = warp_sum((cv[0] ? rv[0] : 0.f) + (cv[1] ? rv[1] : 0.f)) / (float)K;
+    const float d0 = cv[0] ? rv[0] - mean : 0.f, d1 = cv[1] ? rv[1] - mean : 0.f;
+    const float sd = sqrtf(warp_sum(d0 * d0 + d1 * d1) / (float)(K - 1));
+    av[0] = sd > 0.f ? __fdiv_rn(av[0], sd) : 0.f;
+    av[1] = sd > 0.f ? __fdiv_rn(av[1], sd) : 0.f;
+  }
+  if ((flags & PAIR_CENTER) && K > 0) {
+    const float mean = warp_sum(av[0] + av[1]) / (float)K;
+    if (cv[0]) av[0] -= mean;
+    if (cv[1]) av[1] -= mean;
+  }
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int v = lane + 32 * h;
+    if (v < G) {
+      a[gb + v] = av[h] * scale;
+      if (active) active[gb + v] = (cv[h] && diff[h] > 0) ? 1 : 0;
+    }
+  }
+  int nd_all = diff[0] + diff[1];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) nd_all += __shfl_xor_sync(0xffffffffu, nd_all, o);
+  float W = 0.f, W2 = 0.f, Wmax = 0.f;
+  if (DIAG) {
+    W = warp_sum(sw);
+    W2 = warp_sum(sw2);
+    Wmax = warp_max(mw);
+  }
+  if (lane == 0) {
+    if (edges) edges[b] = K * (K - 1) / 2;
+    if (contrast) contrast[b] = nd_all / 2;
+    if (DIAG) {
+      if (ess) ess[b] = W2 > 0.f ? __fdiv_rn(W * W, W2) : 0.f;
+      if (max_w) max_w[b] = Wmax;
+    }
+  }
+}
+
 template <int GP>
 pair_status launch_coeffs_product_gp(int32_t B, int32_t G, const float *r, const uint8_t *J,
                                      const float *p, float scale, uint32_t flags, float *a,
@@ -511,12 +630,18 @@ pair_status launch_coeffs_product(int32_t B, int32_t G, const float *r, const ui
                                   const float *p, float scale, uint32_t flags, float *a,
                                   uint8_t *active, int32_t *edges, int32_t *contrast, float *ess,
                                   float *max_w, int32_t *dev_err, cudaStream_t s) {
-  if (G <= 32)
-    return launch_coeffs_product_gp<32>(B, G, r, J, p, scale, flags, a, active, edges, contrast,
-                                        ess, max_w, dev_err, s);
-  if (G <= 64)
-    return launch_coeffs_product_gp<64>(B, G, r, J, p, scale, flags, a, active, edges, contrast,
-                                        ess, max_w, dev_err, s);
+  if (G <= 64) {
+    const int blocks = (int)ceil_div(B, 4);
+    PAIR_BEGIN("coeffs_product", s);
+    if (ess || max_w)
+      coeffs_product_warp_kernel<true><<<blocks, 128, 0, s>>>(
+          B, G, r, J, p, scale, flags, a, active, edges, contrast, ess, max_w, dev_err);
+    else
+      coeffs_product_warp_kernel<false><<<blocks, 128, 0, s>>>(
+          B, G, r, J, p, scale, flags, a, active, edges, contrast, ess, max_w, dev_err);
+    PAIR_LAUNCH_CHECK(s);
+    return PAIR_OK;
+  }
   return launch_coeffs_product_gp<128>(B, G, r, J, p, scale, flags, a, active, edges, contrast,
                                        ess, max_w, dev_err, s);
 }

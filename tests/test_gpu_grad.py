@@ -126,6 +126,10 @@ CHUNKED = [
     # for d = 2560, 64 wide for d = 3072).
     ("qwen3_4b_head", 2560, 4099, 2, 3, 0.05, 3.0, 0),
     ("longctx_skew", 3072, 2011, 2, 4, 0.04, 3.0, 0),
+    # No image at d = 2048: 6-CTA clusters with 320- and 352-column slices,
+    # a ragged vocabulary and tail row blocks split across clusters.
+    ("qwen3_1p7b_head", 2048, 20000, 2, 8, 0.15, 1.0, 0),
+    ("longctx_skew", 2048, 5003, 4, 8, 0.12, 2.0, 0),
 ]
 
 
@@ -172,11 +176,12 @@ def test_grad_nan_padding_is_ignored_and_deterministic():
         assert torch.equal(x[2], y[2]) and torch.equal(x[3], y[3])
 
 
-@pytest.mark.parametrize("blocks", [None, 0, 2])
-def test_grad_cluster_path_deterministic(blocks):
+@pytest.mark.parametrize("blocks,d", [(None, 512), (0, 512), (2, 512), (0, 2048)])
+def test_grad_cluster_path_deterministic(blocks, d):
     """Cluster backward with tail row blocks split across clusters (and, for
-    blocks = 2, several token chunks): reruns are bit-identical."""
-    inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 5, B=3, G=8, d=512,
+    blocks = 2, several token chunks; at d = 2048 with 6-CTA clusters): reruns
+    are bit-identical."""
+    inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 5, B=3, G=8, d=d,
                                    V=1000, len_scale=0.3, w_std_mult=4.0)
     a = _coeffs(inp)
     r0 = _run(inp, a, blocks)
@@ -369,8 +374,9 @@ def test_token_logp_matches_oracle(case):
     np.testing.assert_allclose(lps.cpu().numpy(), sums, rtol=1e-5, atol=1e-4)
 
 
-@pytest.mark.parametrize("case", [(512, 1000, 0.3, 3), (1024, 3001, 0.2, 8)],
-                         ids=["d512_V1000", "d1024_V3001"])
+@pytest.mark.parametrize("case", [(512, 1000, 0.3, 3), (1024, 3001, 0.2, 8),
+                                  (2048, 2000, 0.15, 5)],
+                         ids=["d512_V1000", "d1024_V3001", "d2048_V2000"])
 def test_grad_onchip_fixup_rows(case):
     """The on-chip path (minimum workspace) takes each token's softmax terms
     relative to its target logit; a row whose maximum logit exceeds the
