@@ -10,8 +10,10 @@
 //     F_t(x) = t Phi(x) - log(budget - sum c e^-x) - sum log x_i - sum log(X - x_i),
 // Newton steps on F_t (gradient and Hessian in closed form, the G x G system
 // factorised by Cholesky in shared memory, backtracking line search kept
-// strictly feasible), t multiplied by 32 (G <= 24) or 16 after each centring, until the
-// duality-gap bound (2G + 1) / t is below 1e-12 Phi. The paper solves the
+// strictly feasible), t multiplied by 32 (G <= 24) or 16 after each centring,
+// with a predictor step along the central path's tangent from the factor of
+// the centred point, until the duality-gap bound (2G + 1) / t is below
+// 1e-12 Phi. The paper solves the
 // same program with SLSQP on the CPU (App. C); any method reaching its
 // unique optimum is equivalent, and a barrier method maps onto one CTA with
 // a fixed, small number of dense factorisations. Cases the program leaves
@@ -77,6 +79,50 @@ __device__ double block_sum(AllocSmem<GP> &sm, double v) {
 #pragma unroll
   for (int w = 0; w < GP / 32; ++w) t += sm.red[w];
   return t;
+}
+
+// Solves H y = r in place in sm.dx with the Cholesky factor in sm.H (lower
+// triangle) and the pivot inverses in sm.dinv (all GP threads call; thread i
+// holds r_i on entry and reads y_i after the call).
+template <int GP>
+__device__ void chol_solve(AllocSmem<GP> &sm, int G, bool act, double r) {
+  const int i = threadIdx.x;
+  __syncthreads();
+  sm.dx[i] = act ? r : 0.0;
+  for (int k = 0; k < G; ++k) {
+    __syncthreads();
+    if (i == k) sm.dx[k] *= sm.dinv[k];
+    __syncthreads();
+    if (i > k && act) sm.dx[i] -= sm.H[i][k] * sm.dx[k];
+  }
+  for (int k = G - 1; k >= 0; --k) {
+    __syncthreads();
+    if (i == k) sm.dx[k] *= sm.dinv[k];
+    __syncthreads();
+    if (i < k) sm.dx[i] -= sm.H[k][i] * sm.dx[k];
+  }
+  __syncthreads();
+}
+
+// Largest step along d keeping every coordinate strictly inside the box
+// (0, X), shared by all threads (min over the group, 1e300 if unbounded).
+template <int GP>
+__device__ double box_step(AllocSmem<GP> &sm, int G, bool act, double x, double d, double X) {
+  double smax = 1.0e300;
+  if (act && d < 0.0) smax = -x / d;
+  if (act && d > 0.0) smax = (X - x) / d;
+  __syncthreads();
+  sm.dx[threadIdx.x] = smax;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double mn = 1.0e300;
+    for (int k = 0; k < G; ++k) mn = fmin(mn, sm.dx[k]);
+    sm.red[0] = mn;
+  }
+  __syncthreads();
+  const double r = sm.red[0];
+  __syncthreads();
+  return r;
 }
 
 struct AllocIn {
@@ -270,21 +316,7 @@ __global__ void __launch_bounds__(GP, 1) alloc_kernel(int G, const float *p_hat,
       }
       if (!spd) break;
       // Solve H dx = -g (forward, then backward substitution).
-      __syncthreads();
-      sm.dx[i] = act ? -gi : 0.0;
-      for (int k = 0; k < G; ++k) {
-        __syncthreads();
-        if (i == k) sm.dx[k] *= sm.dinv[k];
-        __syncthreads();
-        if (i > k && act) sm.dx[i] -= sm.H[i][k] * sm.dx[k];
-      }
-      for (int k = G - 1; k >= 0; --k) {
-        __syncthreads();
-        if (i == k) sm.dx[k] *= sm.dinv[k];
-        __syncthreads();
-        if (i < k) sm.dx[i] -= sm.H[k][i] * sm.dx[k];
-      }
-      __syncthreads();
+      chol_solve<GP>(sm, G, act, -gi);
       const double d = act ? sm.dx[i] : 0.0;
       const double lam2 = -block_sum<GP>(sm, gi * d);
       if (lam2 * 0.5 <= kCentred) {
@@ -293,23 +325,29 @@ __global__ void __launch_bounds__(GP, 1) alloc_kernel(int G, const float *p_hat,
           done = true;
           break;
         }
+        // Predictor: the central path x*(t) has grad F_t = 0, so
+        // dx*/dt = -H^-1 grad Phi with the Hessian just factorised; move
+        // along it to the next t (kept strictly inside the box and the
+        // budget, halving the step otherwise), then let Newton correct.
+        chol_solve<GP>(sm, G, act, act ? -u * (S + sm.b[i]) : 0.0);
+        const double v = act ? (tmul - 1.0) * t * sm.dx[i] : 0.0;
+        double pstep = fmin(1.0, 0.99 * box_step<GP>(sm, G, act, x, v, X));
+        for (int ls = 0; ls < 8; ++ls) {
+          const double xt = x + pstep * v;
+          double ut, et, St, phit, slackt;
+          eval<GP>(in, sm, act, xt, budget, ut, et, St, phit, slackt);
+          // slackt is the same in every thread: the exit is uniform.
+          if (slackt > 0.0) {
+            x = xt; u = ut; e = et; S = St; phi = phit; slack = slackt;
+            break;
+          }
+          pstep *= 0.5;
+        }
         t *= tmul;
         continue;
       }
       // Largest step keeping every coordinate strictly inside the box.
-      double smax = 1.0e300;
-      if (act && d < 0.0) smax = -x / d;
-      if (act && d > 0.0) smax = (X - x) / d;
-      __syncthreads();
-      sm.dx[i] = smax;
-      __syncthreads();
-      if (i == 0) {
-        double mn = 1.0e300;
-        for (int k = 0; k < G; ++k) mn = fmin(mn, sm.dx[k]);
-        sm.red[0] = mn;
-      }
-      __syncthreads();
-      double step = fmin(1.0, 0.99 * sm.red[0]);
+      double step = fmin(1.0, 0.99 * box_step<GP>(sm, G, act, x, d, X));
       const double F0 = t * phi - log(slack) -
                         block_sum<GP>(sm, act ? log(x * (X - x)) : 0.0);
       bool moved = false;

@@ -640,7 +640,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
                        const __grid_constant__ CUtensorMap tmC64, int d, int V,
                        const int32_t *counters, const int32_t *tok_idx,
                        const float *tok_c, const float *lse, float *out,
-                       uint8_t *gring, uint8_t *gimg, float *tailbuf, int rb0, int cap,
+                       uint8_t *gring, float *tailbuf, int rb0, int cap,
                        FusedArgs fa, int32_t *dev_err) {
   extern __shared__ uint8_t smem_raw[];
   ClSmem<BN> &sm = *reinterpret_cast<ClSmem<BN> *>(align1k(smem_raw));
@@ -676,12 +676,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
   const int N = mp.N;                      // tiles of this cluster
   // Ring of published Gs tiles: [owner][job parity] for this cluster.
   uint8_t *ring = gring + (size_t)cid * kCl * 2 * kGsBytes;
-  // Where tile g (chunk row block rb, column tile ct) is published: its own
-  // slot of the logit-gradient image when the launch keeps one (a later pass
-  // reads it again), else the ring slot.
-  auto gs_tile = [&](int g, int rb, int ct) {
-    return gimg ? gimg + ((size_t)rb * n_ct + ct) * kGsBytes
-                : ring + ((size_t)(g & (kCl - 1)) * 2 + (size_t)((g >> 3) & 1)) * kGsBytes;
+  // Where tile g is published: its owner's ring slot for the tile's parity.
+  auto gs_tile = [&](int g) {
+    return ring + ((size_t)(g & (kCl - 1)) * 2 + (size_t)((g >> 3) & 1)) * kGsBytes;
   };
   // The tile whose S this CTA accumulates during slot s (may be < 0 or >= N).
   auto job_of = [&](int s) {
@@ -800,7 +797,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         }
         if (elect_one()) {
           mbar_expect_tx(&sm.cs_full[p], kAtom128 + (uint32_t)A * (kColAtom / 2));
-          bulk_load(sm.g[0][p], gs_tile(s, rb, ct) + p * kAtom128, kAtom128, &sm.cs_full[p]);
+          bulk_load(sm.g[0][p], gs_tile(s) + p * kAtom128, kAtom128, &sm.cs_full[p]);
           for (int j = 0; j < A; ++j)
             tma_load_2d(sm.cs[j] + p * (kColAtom / 2), &tmC64, &sm.cs_full[p], k * w + j * 64,
                         ct * BN + 64 * p);
@@ -827,7 +824,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
         if (!(ok = wait(&sm.gs_empty[gb], ge_ph[gb] ^ 1, abort, dev_err))) break;
         if (elect_one()) {
           mbar_expect_tx(&sm.g_full[gb], kGsBytes);
-          bulk_load(sm.g[gb][0], gs_tile(s, cur.rb, cur.ct), kGsBytes, &sm.g_full[gb]);
+          bulk_load(sm.g[gb][0], gs_tile(s), kGsBytes, &sm.g_full[gb]);
         }
         __syncwarp();
         g_last[gb] = (int)ge_ph[gb];
@@ -1020,7 +1017,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kClThreads, 1)
           free_ph[pb] ^= 1;
         }
         tc_fence_after();
-        uint8_t *dst_tile = gs_tile(g, rb, ct);
+        uint8_t *dst_tile = gs_tile(g);
         float tsum = 0.f, tmax = -INFINITY;
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
@@ -1227,7 +1224,7 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
   constexpr int kAll = 0x7fffffff;
   PAIR_BEGIN("bwd_dh_tc", s);
   bwd_cluster_kernel<true, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-      mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH, gring, nullptr,
+      mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dH, gring,
       w.tailbuf, 0, kAll, FusedArgs{}, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("tail_dh", s);
@@ -1236,7 +1233,7 @@ pair_status grad_bwd_cluster(const GradArgs &g, const GradWorkspace &w, cudaStre
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("bwd_dw_tc", s);
   bwd_cluster_kernel<false, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-      mW128, mHc, mHc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW, gring, nullptr,
+      mW128, mHc, mHc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW, gring,
       w.tailbuf, 0, kAll, FusedArgs{}, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("tail_dw", s);
@@ -1283,7 +1280,7 @@ pair_status grad_head_fused(const GradArgs &g, const GradWorkspace &w, cudaStrea
     }
     PAIR_BEGIN(pass == 0 ? "lse_dh_tc" : "lse_dh_fixup", s);
     bwd_cluster_kernel<true, BN, true><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-        mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, nullptr, g.dH, gring, nullptr,
+        mH, mWc, mWc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, nullptr, g.dH, gring,
         w.tailbuf, 0, kAll, fa, g.dev_err);
     PAIR_LAUNCH_CHECK(s);
     PAIR_BEGIN("tail_lse_dh", s);
@@ -1293,7 +1290,7 @@ pair_status grad_head_fused(const GradArgs &g, const GradWorkspace &w, cudaStrea
   }
   PAIR_BEGIN("bwd_dw_tc", s);
   bwd_cluster_kernel<false, BN><<<ncl * kCl, kClThreads, cl_smem, s>>>(
-      mW128, mHc, mHc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW, gring, nullptr,
+      mW128, mHc, mHc64, g.d, g.V, w.counters, w.tok_idx, w.tok_c, w.lse, g.dW, gring,
       w.tailbuf, 0, kAll, FusedArgs{}, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("tail_dw", s);
