@@ -42,9 +42,14 @@ def test_workspace_size_rules(L):
     assert ws(1000, 2048, 151936, 64, L.PAIR_BF16) > 1000 * 2048 * 2
     wmin = L.pair_grad_workspace_min_size
     # The fp32 path stages 4-byte hidden rows; bf16 stages 2-byte rows plus a
-    # fixed ring of logit-gradient tiles and the clusters' tail scratch
-    # (24 x 2 x 128 x d fp32), so fp32 needs more once T is large.
-    fixed = (12 << 20) + 24 * 2 * 128 * 2048 * 4 + (1 << 20)
+    # fixed ring of logit-gradient tiles, the clusters' tail scratch
+    # (24 x 2 x 128 x d fp32) and the fused LSE pass's per-token arrays
+    # (reference and row maximum, 2 x 4 bytes per padded token; one 8 x 256
+    # fp32 partial block per 128-token slot, ceil(T/128) + 48 slots), so fp32
+    # needs more once T is large.
+    tpad = (100000 + 127) // 128 * 128
+    fused = 2 * 4 * tpad + (tpad // 128 + 48) * 8 * 256 * 4 + (1 << 20)
+    fixed = (12 << 20) + 24 * 2 * 128 * 2048 * 4 + (1 << 20) + fused
     assert (wmin(100000, 2048, 151936, 64, L.PAIR_F32)
             - wmin(100000, 2048, 151936, 64, L.PAIR_BF16) > 100000 * 2048 * 2 - fixed)
     # For d a multiple of 512, bf16 also keeps the logit terms (fp16 per
