@@ -81,9 +81,11 @@ __global__ void __launch_bounds__(256) g_image_kernel(int V, int rb0, int cap,
 // with the image tiles as the K-major A operand (64 vocabulary rows per
 // stage, one 16 KB atom, copied verbatim) and W as the MN-major B operand.
 // CTA pairs (2-CTA clusters) take two token blocks of the same 256-column
-// chunk of d and share its W stage by multicast (each CTA fetches two of the
-// four 64-column atoms). Work unit = (token block pair, 256-column chunk);
-// the fp32 accumulator (128 x 256) is double-buffered in TMEM so the drain of
+// chunk of d as one M = 256 tile: the even CTA issues every MMA of the pair
+// (cta_group::2) over both CTAs' image atoms and the chunk's four W column
+// atoms, two in each CTA, and each CTA's TMEM receives its own token block's
+// rows. Work unit = (token block pair, 256-column chunk); the fp32
+// accumulator (128 x 256 per CTA) is double-buffered in TMEM so the drain of
 // one unit overlaps the next. Each (token, column) is owned by one CTA and
 // summed over all of V in one fixed order: deterministic, no atomics. An odd
 // last block is computed twice (the pair's other CTA repeats it) and stored
@@ -91,8 +93,8 @@ __global__ void __launch_bounds__(256) g_image_kernel(int V, int rb0, int cap,
 constexpr int kDhN = 256;                              // output columns per unit
 constexpr int kDhStages = 4;
 constexpr uint32_t kDhABytes = kAtom128;               // 128 tokens x 64 vocabulary
-constexpr uint32_t kDhBBytes = (kDhN / 64) * 64 * 128; // 4 column atoms x 64 rows
-constexpr uint32_t kIdescDh = idesc_bf16(128, kDhN, 0, 1);
+constexpr uint32_t kDhBBytes = (kDhN / 128) * 64 * 128; // this CTA's 2 column atoms x 64 rows
+constexpr uint32_t kIdescDh = idesc_bf16(256, kDhN, 0, 1);
 
 struct DhSmem {
   uint8_t a[kDhStages][kDhABytes];
@@ -104,9 +106,9 @@ struct DhSmem {
 };
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
-    dh_gemm_kernel(const __grid_constant__ CUtensorMap tmW, int d, int V, int rb0, int cap,
-                   const int32_t *counters, const int32_t *tok_idx, const uint8_t *gimg,
-                   float *dH, int32_t *dev_err) {
+    dh_gemm_kernel(const __grid_constant__ CUtensorMap tmG, const __grid_constant__ CUtensorMap tmW,
+                   int d, int V, int rb0, int cap, const int32_t *counters,
+                   const int32_t *tok_idx, float *dH, int32_t *dev_err) {
   const int Teff = counters[0];
   const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
   if (nrb == 0) return;  // no token in this chunk
@@ -122,25 +124,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kDhStages; ++s) {
-      mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], 2);  // both CTAs' MMAs done with the stage
+      mbar_init(&sm.full[s], 1);   // the even CTA's expect_tx (both CTAs' bytes)
+      mbar_init(&sm.empty[s], 1);  // the pair MMA's commit
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&sm.acc_full[s], 1);
-      mbar_init(&sm.acc_empty[s], 128);
+      mbar_init(&sm.acc_empty[s], 2 * 128);  // both CTAs' epilogue threads
     }
     mbar_init(&sm.mma_done, 1);
     sm.abort = 0;
     fence_mbar_init();
+    prefetch_tmap(&tmG);
     prefetch_tmap(&tmW);
   }
   if (warp == 1) {
-    tmem_alloc(&sm.tmem_base, 512);
-    tmem_relinquish();
+    tmem_alloc_pair(&sm.tmem_base, 512);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
-  cluster_sync();  // the peer's barriers exist before any multicast lands
+  cluster_sync();  // the pair's barriers exist before any copy or commit lands
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   volatile int *abort = &sm.abort;
@@ -155,59 +158,66 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int u = pid; u < n_units && ok; u += npairs) {
         const int tp = u / nq, q = u - tp * nq;
         const int b = min(2 * tp + r, nrb - 1);
-        const uint8_t *arow = gimg + (size_t)b * n_vt * kGImgTileBytes;
+        const int atom0 = b * nks;  // the block's first image atom
         for (int ks = 0; ks < nks; ++ks) {
           if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
           if (elect_one()) {
-            mbar_expect_tx(&sm.full[stage], kDhABytes + kDhBBytes);
-            bulk_load(sm.a[stage], arow + (size_t)ks * kAtom128, kAtom128, &sm.full[stage]);
-            tma_load_3d_mc(sm.b[stage] + r * (kDhBBytes / 2), &tmW, &sm.full[stage], 0, 64 * ks,
-                           q * (kDhN / 64) + r * (kDhN / 128), (uint16_t)3);
+            if (r == 0) mbar_expect_tx(&sm.full[stage], 2 * (kDhABytes + kDhBBytes));
+            const uint32_t fb = mapa(smem_u32(&sm.full[stage]), 0);
+            tma_load_3d_pair(sm.a[stage], &tmG, fb, 0, 0, atom0 + ks);
+            tma_load_3d_pair(sm.b[stage], &tmW, fb, 0, 64 * ks,
+                             q * (kDhN / 64) + r * (kDhN / 128));
           }
           __syncwarp();
           last_ph[stage] = (int)ph;
           if (++stage == kDhStages) { stage = 0; ph ^= 1; }
         }
       }
+      // The last copy of every stage: completed on the even CTA, consumed by
+      // the pair MMA on the odd one (both CTAs issue the same sequence).
       for (int s = 0; s < kDhStages; ++s)
         if (last_ph[s] >= 0) {
           volatile int never = 0;
-          wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+          if (r == 0)
+            wait_cluster(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+          else
+            wait_cluster(&sm.empty[s], (uint32_t)last_ph[s], &never, dev_err);
         }
     }
   } else if (warp == 1) {
-    {  // whole warp: uniform loop state; elected lane issues
+    if (r == 0) {  // whole warp: uniform loop state; elected lane issues
       // A: K-major atom, 16 tokens of K = 32 bytes along the swizzled row.
-      // B: 4 column atoms of 64 vocabulary rows (LBO 8 KB), row groups of 8
-      // (SBO 1 KB); 16 vocabulary rows = 2 KB.
+      // B: this CTA's 2 column atoms of 64 vocabulary rows (LBO 8 KB), row
+      // groups of 8 (SBO 1 KB); 16 vocabulary rows = 2 KB.
       const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
       const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 64 * 128, 1024);
       int stage = 0, acc = 0;
       uint32_t ph = 0, acc_ph = 0;
       bool ok = true;
       for (int u = pid; u < n_units && ok; u += npairs) {
-        if (!(ok = wait(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
+        if (!(ok = wait_cluster(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
         tc_fence_after();
         const uint32_t dt = tmem + acc * kDhN;
         for (int ks = 0; ks < nks; ++ks) {
-          if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+          if (!(ok = wait_cluster(&sm.full[stage], ph, abort, dev_err))) break;
+          tc_fence_after();
           const uint64_t da = da0 + (uint64_t)stage * (kDhABytes >> 4);
           const uint64_t db = db0 + (uint64_t)stage * (kDhBBytes >> 4);
           if (elect_one()) {
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              mma_bf16(dt, da + 2 * kk, db + kk * (2048 >> 4), kIdescDh, (ks | kk) != 0);
-            mma_commit_multicast(&sm.empty[stage], (uint16_t)3);
+              mma_bf16_pair(dt, da + 2 * kk, db + kk * (2048 >> 4), kIdescDh, (ks | kk) != 0);
+            mma_commit_pair(&sm.empty[stage], (uint16_t)3);
           }
           __syncwarp();
           if (++stage == kDhStages) { stage = 0; ph ^= 1; }
         }
         if (!ok) break;
-        if (elect_one()) mma_commit(&sm.acc_full[acc]);
+        if (elect_one()) mma_commit_pair(&sm.acc_full[acc], (uint16_t)3);
         __syncwarp();
         if (++acc == 2) { acc = 0; acc_ph ^= 1; }
       }
-      if (elect_one()) mma_commit(&sm.mma_done);
+      if (elect_one()) mma_commit_pair(&sm.mma_done, (uint16_t)1);
       __syncwarp();
       volatile int never = 0;
       wait(&sm.mma_done, 0, &never, dev_err);
@@ -225,7 +235,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const bool valid = 2 * tp + r < nrb && t < Teff;
       float4 *dst =
           valid ? reinterpret_cast<float4 *>(dH + (int64_t)tok_idx[t] * d + q * kDhN) : nullptr;
-      if (!(ok = wait_sleepy(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
+      if (!(ok = wait_sleepy_cluster(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
       tc_fence_after();
 #pragma unroll 1
       for (int c = 0; c < kDhN / 32; ++c) {
@@ -238,7 +248,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
       }
       tc_fence_before();
-      mbar_arrive(&sm.acc_empty[acc]);
+      mbar_arrive_cluster(mapa(smem_u32(&sm.acc_empty[acc]), 0));
       if (++acc == 2) { acc = 0; acc_ph ^= 1; }
     }
   }
@@ -248,7 +258,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   cluster_sync();  // no CTA leaves while its peer may still signal or fill it
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 512);
+    tmem_dealloc_pair(tmem, 512);
   }
 }
 
@@ -263,21 +273,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 //     dW[v, :] (+)= sum_t Gs[t, v] Hc[t, :]
 // with no logit recomputation.
 //
-// CTA pairs (2-CTA clusters) share one 512-column chunk of Hc: CTA r of the
-// pair fetches half of each Hc stage and multicasts it into both CTAs; each
-// CTA fetches the Gs^T stage of its own 128 vocabulary rows. Work unit =
-// (vocabulary block pair, 512-column chunk of d); CTA r accumulates
-// dW[block 2 p + r, chunk] (128 x 512 fp32 = all of TMEM) over the chunk's
-// tokens, 32 token rows per stage, and drains it with plain stores (first
-// chunk) or read-add-writes (later chunks; this CTA owns those rows).
-// An odd last block is computed twice (the pair's other CTA repeats the
-// last block) so both CTAs run the same stage sequence; only one stores it.
+// CTA pairs (2-CTA clusters) share one 512-column chunk of Hc as two M = 256
+// tiles of 256 columns each: the even CTA issues every MMA of the pair
+// (cta_group::2) over both CTAs' Gs^T stages (each CTA fetches the one of its
+// own 128 vocabulary rows) and each 256-column half's four Hc column atoms,
+// two in each CTA. Work unit = (vocabulary block pair, 512-column chunk of
+// d); CTA r accumulates dW[block 2 p + r, chunk] (128 x 512 fp32 = all of
+// TMEM) over the chunk's tokens, 32 token rows per stage, and drains it with
+// plain stores (first chunk) or read-add-writes (later chunks; this CTA owns
+// those rows). An odd last block is computed twice (the pair's other CTA
+// repeats the last block) so both CTAs run the same stage sequence; only one
+// stores it.
 constexpr int kDwKS = 32;                                 // token rows per stage
 constexpr int kDwStages = 5;
 constexpr int kDwN = 512;                                 // output columns per CTA
 constexpr uint32_t kDwGBytes = 2 * kDwKS * 128;           // 2 vocabulary atoms x 32 rows
-constexpr uint32_t kDwHBytes = (kDwN / 64) * kDwKS * 128; // 8 column atoms x 32 rows
-constexpr uint32_t kIdescDw = idesc_bf16(128, 256, 1, 1); // both operands MN-major
+constexpr uint32_t kDwHBytes = (kDwN / 128) * kDwKS * 128; // this CTA's 4 column atoms x 32 rows
+constexpr uint32_t kIdescDw = idesc_bf16(256, 256, 1, 1); // both operands MN-major
 
 struct DwSmem {
   uint8_t g[kDwStages][kDwGBytes];  // Gs^T: MN-major A, atoms 4 KB apart
@@ -309,11 +321,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kDwStages; ++s) {
-      mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], 2);  // both CTAs' MMAs done with the stage
+      mbar_init(&sm.full[s], 1);   // the even CTA's expect_tx (both CTAs' bytes)
+      mbar_init(&sm.empty[s], 1);  // the pair MMA's commit
     }
     mbar_init(&sm.acc_full, 1);
-    mbar_init(&sm.acc_empty, 128);
+    mbar_init(&sm.acc_empty, 2 * 128);  // both CTAs' epilogue threads
     mbar_init(&sm.mma_done, 1);
     sm.abort = 0;
     fence_mbar_init();
@@ -321,12 +333,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmH);
   }
   if (warp == 1) {
-    tmem_alloc(&sm.tmem_base, 512);
-    tmem_relinquish();
+    tmem_alloc_pair(&sm.tmem_base, 512);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
-  cluster_sync();  // the peer's barriers exist before any multicast lands
+  cluster_sync();  // the pair's barriers exist before any copy or commit lands
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   volatile int *abort = &sm.abort;
@@ -345,12 +357,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const int rbl = ks >> 2, j = ks & 3;
           if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
           if (elect_one()) {
-            mbar_expect_tx(&sm.full[stage], kDwGBytes + kDwHBytes);
-            tma_load_3d(sm.g[stage], &tmG, &sm.full[stage], 0, kDwKS * j,
-                        2 * (rbl * n_vb + vb));
-            tma_load_3d_mc(sm.h[stage] + r * (kDwHBytes / 2), &tmH, &sm.full[stage], 0,
-                           (rb0 + rbl) * 128 + kDwKS * j, q * (kDwN / 64) + r * (kDwN / 128),
-                           (uint16_t)3);
+            if (r == 0) mbar_expect_tx(&sm.full[stage], 2 * (kDwGBytes + kDwHBytes));
+            const uint32_t fb = mapa(smem_u32(&sm.full[stage]), 0);
+            const int t0 = (rb0 + rbl) * 128 + kDwKS * j;
+            tma_load_3d_pair(sm.g[stage], &tmG, fb, 0, kDwKS * j, 2 * (rbl * n_vb + vb));
+            // Column atoms 2r, 2r + 1 of each 256-column half of the chunk.
+            tma_load_3d_pair(sm.h[stage], &tmH, fb, 0, t0, q * (kDwN / 64) + 2 * r);
+            tma_load_3d_pair(sm.h[stage] + kDwHBytes / 2, &tmH, fb, 0, t0,
+                             q * (kDwN / 64) + 4 + 2 * r);
           }
           __syncwarp();
           last_ph[stage] = (int)ph;
@@ -358,29 +372,35 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
       }
       // Never leave a copy in flight: wait (bounded) for the last one issued
-      // on every stage.
+      // on every stage: completed on the even CTA, consumed by the pair MMA
+      // on the odd one (both CTAs issue the same sequence).
       for (int s = 0; s < kDwStages; ++s)
         if (last_ph[s] >= 0) {
           volatile int never = 0;
-          wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+          if (r == 0)
+            wait_cluster(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+          else
+            wait_cluster(&sm.empty[s], (uint32_t)last_ph[s], &never, dev_err);
         }
     }
   } else if (warp == 1) {
-    {  // whole warp: uniform loop state; elected lane issues
+    if (r == 0) {  // whole warp: uniform loop state; elected lane issues
       // A: 2 vocabulary atoms (LBO 4 KB), token groups of 8 rows (SBO 1 KB);
-      // B: 8 column atoms (LBO 4 KB), the same token groups. One K step of 16
-      // tokens advances both by 2 KB; B's second 256-column half is 16 KB on.
+      // B: this CTA's 2 column atoms of each half (LBO 4 KB), the same token
+      // groups. One K step of 16 tokens advances both by 2 KB; B's second
+      // 256-column half is 8 KB on.
       const uint64_t dg0 = sdesc_sw128(smem_u32(sm.g[0]), kDwKS * 128, 1024);
       const uint64_t dh0 = sdesc_sw128(smem_u32(sm.h[0]), kDwKS * 128, 1024);
       int stage = 0;
       uint32_t ph = 0, acc_ph = 0;
       bool ok = true;
       for (int u = pid; u < n_units && ok && nks > 0; u += npairs) {
-        if (!(ok = wait(&sm.acc_empty, acc_ph ^ 1, abort, dev_err))) break;
+        if (!(ok = wait_cluster(&sm.acc_empty, acc_ph ^ 1, abort, dev_err))) break;
         acc_ph ^= 1;
         tc_fence_after();
         for (int ks = 0; ks < nks; ++ks) {
-          if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+          if (!(ok = wait_cluster(&sm.full[stage], ph, abort, dev_err))) break;
+          tc_fence_after();
           const uint64_t dg = dg0 + (uint64_t)stage * (kDwGBytes >> 4);
           const uint64_t dh = dh0 + (uint64_t)stage * (kDwHBytes >> 4);
           if (elect_one()) {
@@ -388,19 +408,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             for (int kk = 0; kk < kDwKS / 16; ++kk)
 #pragma unroll
               for (int nh = 0; nh < 2; ++nh)
-                mma_bf16(tmem + nh * 256, dg + kk * (2048 >> 4),
-                         dh + nh * ((kDwHBytes / 2) >> 4) + kk * (2048 >> 4), kIdescDw,
-                         (ks | kk) != 0);
-            mma_commit_multicast(&sm.empty[stage], (uint16_t)3);
+                mma_bf16_pair(tmem + nh * 256, dg + kk * (2048 >> 4),
+                              dh + nh * ((kDwHBytes / 2) >> 4) + kk * (2048 >> 4), kIdescDw,
+                              (ks | kk) != 0);
+            mma_commit_pair(&sm.empty[stage], (uint16_t)3);
           }
           __syncwarp();
           if (++stage == kDwStages) { stage = 0; ph ^= 1; }
         }
         if (!ok) break;
-        if (elect_one()) mma_commit(&sm.acc_full);
+        if (elect_one()) mma_commit_pair(&sm.acc_full, (uint16_t)3);
         __syncwarp();
       }
-      if (elect_one()) mma_commit(&sm.mma_done);
+      if (elect_one()) mma_commit_pair(&sm.mma_done, (uint16_t)1);
       __syncwarp();
       volatile int never = 0;
       wait(&sm.mma_done, 0, &never, dev_err);
@@ -421,7 +441,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           for (int c = 0; c < kDwN / 4; ++c) dst[c] = make_float4(0.f, 0.f, 0.f, 0.f);
         continue;
       }
-      if (!(ok = wait_sleepy(&sm.acc_full, acc_ph, abort, dev_err))) break;
+      if (!(ok = wait_sleepy_cluster(&sm.acc_full, acc_ph, abort, dev_err))) break;
       acc_ph ^= 1;
       tc_fence_after();
 #pragma unroll 1
@@ -441,7 +461,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
       }
       tc_fence_before();
-      mbar_arrive(&sm.acc_empty);
+      mbar_arrive_cluster(mapa(smem_u32(&sm.acc_empty), 0));
     }
   }
 
@@ -450,7 +470,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   cluster_sync();  // no CTA leaves while its peer may still signal or fill it
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 512);
+    tmem_dealloc_pair(tmem, 512);
   }
 }
 
@@ -463,11 +483,13 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
   const int cap = w.gimg_rb;
   const int rb0 = (int)(c * cap);
   const int n_vt = (g.V + 127) / 128;
-  CUtensorMap mG, mH3, mW3;
+  CUtensorMap mG, mGA, mH3, mW3;
   if (!make_map3(&mG, w.gimg, {64, 128, (cuuint64_t)2 * cap * n_vt}, {128, 16384}, {64, 32, 2},
                  CU_TENSOR_MAP_SWIZZLE_NONE) ||
+      !make_map3(&mGA, w.gimg, {64, 128, (cuuint64_t)2 * cap * n_vt}, {128, 16384}, {64, 128, 1},
+                 CU_TENSOR_MAP_SWIZZLE_NONE) ||
       !make_map3(&mH3, w.Hc, {64, (cuuint64_t)w.Tpad, (cuuint64_t)g.d / 64},
-                 {(cuuint64_t)g.d * 2, 128}, {64, (cuuint32_t)kDwKS, 4},
+                 {(cuuint64_t)g.d * 2, 128}, {64, (cuuint32_t)kDwKS, 2},
                  CU_TENSOR_MAP_SWIZZLE_128B) ||
       !make_map3(&mW3, g.W, {64, (cuuint64_t)g.V, (cuuint64_t)g.d / 64},
                  {(cuuint64_t)g.d * 2, 128}, {64, 64, 2}, CU_TENSOR_MAP_SWIZZLE_128B))
@@ -485,7 +507,7 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("dh_gemm_tc", s);
   dh_gemm_kernel<<<pair_grid((const void *)dh_gemm_kernel, dh_smem, &dh_cache), kThreads,
-                   dh_smem, s>>>(mW3, g.d, g.V, rb0, cap, w.counters, w.tok_idx, gimg, g.dH,
+                   dh_smem, s>>>(mGA, mW3, g.d, g.V, rb0, cap, w.counters, w.tok_idx, g.dH,
                                  g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("dw_gemm_tc", s);

@@ -12,15 +12,17 @@ using namespace tc;
 using namespace tck;
 
 // ------------------------------------------------------------------ LSE
-constexpr int kLseBN = 256;
-constexpr int kLseStages = 4;
-constexpr uint32_t kLseStageTx = (128 + kLseBN) * 64 * 2;
-constexpr int kLsePair = 2;  // CTAs per cluster sharing each vocabulary tile
-constexpr uint32_t kIdescLse = idesc_bf16(128, kLseBN, 0, 0);
+constexpr int kLseBN = 256;     // vocabulary rows per tile (N of the pair MMA)
+constexpr int kLseStages = 6;
+constexpr int kLsePair = 2;     // CTAs per cluster: one M = 256 MMA per K step
+// Bytes that complete one stage, counted on the even CTA's barrier: each CTA
+// lands its token atom and its 128 vocabulary rows.
+constexpr uint32_t kLseStageTx = kLsePair * 2 * kAtom128;
+constexpr uint32_t kIdescLse = idesc_bf16(256, kLseBN, 0, 0);
 
 struct LseSmem {
-  uint8_t a[kLseStages][kAtom128];
-  uint8_t b[kLseStages][2 * kAtom128];
+  uint8_t a[kLseStages][kAtom128];  // this CTA's token block, one K-atom (128 x 64)
+  uint8_t b[kLseStages][kAtom128];  // this CTA's half of the vocabulary tile (128 x 64)
   uint8_t stg[2][128 * 128];  // kept-term staging: per warp 32 rows x 64 fp16, SWIZZLE_128B
   uint64_t full[kLseStages], empty[kLseStages];
   uint64_t acc_full[2], acc_empty[2];
@@ -45,12 +47,15 @@ __device__ __forceinline__ void lse_unit(int u, int n_pairs, int nsplit, int &pa
 }
 
 // CTA pairs (2-CTA clusters) work on two token blocks of the same vocabulary
-// split in lockstep: each CTA fetches its own token atom and one half (128
-// rows) of the shared 256-row vocabulary atom, multicast into both CTAs'
-// stage. A stage is refilled only after both CTAs' MMAs released it (each
-// MMA warp commits to the empty barrier of both CTAs). This halves the
-// vocabulary bytes each SM's copy engine requests, which is what limits the
-// loads here (the engine's outstanding requests wait on DRAM-latency tiles).
+// split in lockstep, as one M = 256 tile: the even CTA issues every MMA of
+// the pair (cta_group::2), over the 256 token rows of both CTAs' A stages and
+// the 256 vocabulary rows of their B stages (128 in each CTA), and each CTA's
+// TMEM receives the logits of its own token block. Each CTA fetches only its
+// own token atom and its own half of the vocabulary atom, so a stage is 32 KB
+// per CTA and six stages fit beside the staging buffers; the even CTA's full
+// barrier counts both CTAs' bytes, and the MMA's commits release the stage
+// and publish the accumulator in both CTAs. The odd CTA's epilogue returns
+// each accumulator buffer to the even CTA's acc_empty barrier.
 __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
     lse_kernel(const __grid_constant__ CUtensorMap tmH,
                const __grid_constant__ CUtensorMap tmW,
@@ -89,12 +94,12 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kLseStages; ++s) {
-      mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], kLsePair);  // both CTAs' MMAs done with the stage
+      mbar_init(&sm.full[s], 1);   // the even CTA's expect_tx (both CTAs' bytes)
+      mbar_init(&sm.empty[s], 1);  // the pair MMA's commit
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&sm.acc_full[s], 1);
-      mbar_init(&sm.acc_empty[s], 128);
+      mbar_init(&sm.acc_empty[s], kLsePair * 128);  // both CTAs' epilogue threads
     }
     mbar_init(&sm.mma_done, 1);
     sm.abort = 0;
@@ -103,12 +108,12 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmW);
   }
   if (warp == 1) {
-    tmem_alloc(&sm.tmem_base, 512);
-    tmem_relinquish();
+    tmem_alloc_pair(&sm.tmem_base, 512);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
-  cluster_sync();  // the peer's barriers exist before any multicast lands
+  cluster_sync();  // the pair's barriers exist before any copy or commit lands
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   volatile int *abort = &sm.abort;
@@ -130,10 +135,10 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
           for (int k = 0; k < nk; ++k) {
             if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
             if (elect_one()) {
-              mbar_expect_tx(&sm.full[stage], kLseStageTx);
-              tma_load_2d(sm.a[stage], &tmH, &sm.full[stage], k * 64, tb * 128);
-              tma_load_2d_mc(sm.b[stage] + r * (kLseBN / 2) * 128, &tmW, &sm.full[stage],
-                             k * 64, vt * kLseBN + r * (kLseBN / 2), (uint16_t)3);
+              if (r == 0) mbar_expect_tx(&sm.full[stage], kLseStageTx);
+              const uint32_t fb = mapa(smem_u32(&sm.full[stage]), 0);
+              tma_load_2d_pair(sm.a[stage], &tmH, fb, k * 64, tb * 128);
+              tma_load_2d_pair(sm.b[stage], &tmW, fb, k * 64, vt * kLseBN + r * (kLseBN / 2));
             }
             __syncwarp();
             last_ph[stage] = (int)ph;
@@ -142,15 +147,19 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
         }
       }
       // Never leave a copy in flight: wait (bounded) for the last one issued
-      // on every stage.
+      // on every stage: its completion on the even CTA, its consumption by
+      // the pair MMA on the odd one (both CTAs issue the same sequence).
       for (int s = 0; s < kLseStages; ++s)
         if (last_ph[s] >= 0) {
           volatile int never = 0;
-          wait(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+          if (r == 0)
+            wait_cluster(&sm.full[s], (uint32_t)last_ph[s], &never, dev_err);
+          else
+            wait_cluster(&sm.empty[s], (uint32_t)last_ph[s], &never, dev_err);
         }
     }
   } else if (warp == 1) {
-    {  // whole warp: uniform loop state; elected lane issues
+    if (r == 0) {  // whole warp: uniform loop state; elected lane issues
       int stage = 0, acc = 0;
       uint32_t ph = 0, acc_ph = 0;
       const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
@@ -162,29 +171,30 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
         const int vt0 = (int)((int64_t)sp * n_vt / nsplit);
         const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
         for (int vt = vt0; vt < vt1 && ok; ++vt) {
-          if (!(ok = wait(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
+          if (!(ok = wait_cluster(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
           tc_fence_after();
           const uint32_t dt = tmem + acc * kLseBN;
           for (int k = 0; k < nk; ++k) {
-            if (!(ok = wait(&sm.full[stage], ph, abort, dev_err))) break;
+            if (!(ok = wait_cluster(&sm.full[stage], ph, abort, dev_err))) break;
+            tc_fence_after();
             const uint64_t da = da0 + (uint64_t)stage * (kAtom128 >> 4);
-            const uint64_t db = db0 + (uint64_t)stage * ((2 * kAtom128) >> 4);
+            const uint64_t db = db0 + (uint64_t)stage * (kAtom128 >> 4);
             if (elect_one()) {
 #pragma unroll
               for (int kk = 0; kk < 4; ++kk)
-                mma_bf16(dt, da + 2 * kk, db + 2 * kk, kIdescLse, (k | kk) != 0);
-              mma_commit_multicast(&sm.empty[stage], (uint16_t)3);
+                mma_bf16_pair(dt, da + 2 * kk, db + 2 * kk, kIdescLse, (k | kk) != 0);
+              mma_commit_pair(&sm.empty[stage], (uint16_t)3);
             }
             __syncwarp();
             if (++stage == kLseStages) { stage = 0; ph ^= 1; }
           }
           if (!ok) break;
-          if (elect_one()) mma_commit(&sm.acc_full[acc]);
+          if (elect_one()) mma_commit_pair(&sm.acc_full[acc], (uint16_t)3);
           __syncwarp();
           if (++acc == 2) { acc = 0; acc_ph ^= 1; }
         }
       }
-      if (elect_one()) mma_commit(&sm.mma_done);
+      if (elect_one()) mma_commit_pair(&sm.mma_done, (uint16_t)1);
       __syncwarp();
       volatile int never = 0;
       wait(&sm.mma_done, 0, &never, dev_err);
@@ -211,7 +221,7 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
       float m2 = -INFINITY, l = 0.f, zt = 0.f;
       bool found = false;
       for (int vt = vt0; vt < vt1; ++vt) {
-        if (!(ok = wait_sleepy(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
+        if (!(ok = wait_sleepy_cluster(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
         tc_fence_after();
 #pragma unroll 1
         for (int c = 0; c < kLseBN / 32; ++c) {
@@ -289,7 +299,7 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
           }
         }
         tc_fence_before();
-        mbar_arrive(&sm.acc_empty[acc]);
+        mbar_arrive_cluster(mapa(smem_u32(&sm.acc_empty[acc]), 0));
         if (++acc == 2) { acc = 0; acc_ph ^= 1; }
       }
       if (!ok) break;
@@ -308,7 +318,7 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
   cluster_sync();  // no CTA leaves while its peer may still signal or fill it
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 512);
+    tmem_dealloc_pair(tmem, 512);
   }
 }
 

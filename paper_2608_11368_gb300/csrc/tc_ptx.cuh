@@ -371,6 +371,87 @@ __device__ __forceinline__ void mma_commit_multicast(uint64_t *bar, uint16_t mas
       : "memory");
 }
 
+// ------------------------------------------------------ CTA pairs (2-SM MMA)
+//
+// The cta_group::2 forms: one MMA instruction, issued by the even CTA of a
+// cluster pair, computes an M = 256 tile whose rows [0, 128) come from the
+// even CTA's A operand and land in its TMEM, rows [128, 256) from the odd
+// CTA's A at the same shared-memory offset into the odd CTA's TMEM; each
+// CTA holds half of the B operand's N rows (the even CTA the first half).
+// TMEM is allocated for both CTAs at once (one warp of each CTA takes part),
+// and a kernel uses these forms for all its tcgen05 allocation, MMA and
+// commit instructions.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t *dst, uint32_t ncols) {
+  asm volatile(
+      "tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+          smem_u32(dst)),
+      "r"(ncols)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr),
+               "r"(ncols)
+               : "memory");
+}
+// D[tmem] (+)= A * B^T over the pair (M = 256), kind::f16.
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                              uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive once on the mbarrier at the same shared offset in every cluster CTA
+// of `mask` when all pair MMAs this thread issued before have completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t *bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster."
+      "multicast::cluster.b64 [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(mask)
+      : "memory");
+}
+// Tile loads into this CTA's shared memory whose completed bytes count on an
+// mbarrier that may sit in the pair's other CTA (bar_caddr is a
+// shared::cluster address, e.g. from mapa).
+__device__ __forceinline__ void tma_load_2d_pair(void *dst, const CUtensorMap *map,
+                                                 uint32_t bar_caddr, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_"
+      "tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_caddr), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_3d_pair(void *dst, const CUtensorMap *map,
+                                                 uint32_t bar_caddr, int x, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_"
+      "tx::bytes [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_caddr), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+// wait_sleepy with cluster-scope acquire (phases completed by the pair's
+// other CTA).
+__device__ __forceinline__ bool wait_sleepy_cluster(uint64_t *bar, uint32_t parity,
+                                                    volatile int *abort, int32_t *dev_err) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    __nanosleep(128);
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *abort = 1;
+      flag_error(dev_err, PAIR_DEV_ERR_TIMEOUT);
+      return false;
+    }
+  }
+}
+
 // Bulk copy of `bytes` (multiple of 16) from this CTA's shared memory to a
 // cluster CTA's shared memory, completing `bytes` of transaction count on
 // that CTA's mbarrier (dst and mbar are shared::cluster addresses).
