@@ -13,7 +13,7 @@ using namespace tck;
 
 // ------------------------------------------------------------------ LSE
 constexpr int kLseBN = 256;     // vocabulary rows per tile (N of the pair MMA)
-constexpr int kLseStages = 6;
+constexpr int kLseStages = 5;
 constexpr int kLsePair = 2;     // CTAs per cluster: one M = 256 MMA per K step
 // Bytes that complete one stage, counted on the even CTA's barrier: each CTA
 // lands its token atom and its 128 vocabulary rows.
@@ -52,10 +52,13 @@ __device__ __forceinline__ void lse_unit(int u, int n_pairs, int nsplit, int &pa
 // the 256 vocabulary rows of their B stages (128 in each CTA), and each CTA's
 // TMEM receives the logits of its own token block. Each CTA fetches only its
 // own token atom and its own half of the vocabulary atom, so a stage is 32 KB
-// per CTA and six stages fit beside the staging buffers; the even CTA's full
-// barrier counts both CTAs' bytes, and the MMA's commits release the stage
-// and publish the accumulator in both CTAs. The odd CTA's epilogue returns
-// each accumulator buffer to the even CTA's acc_empty barrier.
+// per CTA; the even CTA's full barrier counts both CTAs' bytes, and the MMA's
+// commits release the stage and publish the accumulator in both CTAs. The
+// odd CTA's epilogue returns each accumulator buffer to the even CTA's
+// acc_empty barrier. Five stages: a sixth fits beside the staging buffers but
+// measured slower over the whole step (deeper pipelines let the pairs drift
+// apart in the vocabulary, so fewer of them share W rows in L2), four starve
+// the MMA.
 __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
     lse_kernel(const __grid_constant__ CUtensorMap tmH,
                const __grid_constant__ CUtensorMap tmW,
