@@ -96,6 +96,26 @@ constexpr uint32_t kDhABytes = kAtom128;               // 128 tokens x 64 vocabu
 constexpr uint32_t kDhBBytes = (kDhN / 128) * 64 * 128; // this CTA's 2 column atoms x 64 rows
 constexpr uint32_t kIdescDh = idesc_bf16(256, kDhN, 0, 1);
 
+// Work list of dh_gemm_kernel: the units that fill whole rounds of the
+// persistent grid (ncl clusters) run over all of V; the R < ncl units left
+// for the last round are cut into S vocabulary parts each (R S <= ncl, at
+// most `cap` partial tiles of scratch), so that round takes a part's time
+// instead of a unit's. Work item i < full_end is unit i; item full_end + j
+// is part j % S of unit full_end + j / S, over image atoms
+// [part nks / S, (part + 1) nks / S); its fp32 tile goes to scratch slot j
+// and dh_tail_combine_kernel adds the S parts in order (deterministic).
+struct DhTail {
+  int full_end, R, S;
+};
+__host__ __device__ __forceinline__ DhTail dh_tail(int n_units, int ncl, int cap, int nks) {
+  const int rem = n_units % ncl;
+  int S = rem ? ncl / rem : 1;
+  if (rem && S * rem > cap) S = cap / rem;
+  if (S > nks) S = nks;
+  if (S < 2) return DhTail{n_units, 0, 1};
+  return DhTail{n_units - rem, rem, S};
+}
+
 struct DhSmem {
   uint8_t a[kDhStages][kDhABytes];
   uint8_t b[kDhStages][kDhBBytes];
@@ -108,7 +128,8 @@ struct DhSmem {
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     dh_gemm_kernel(const __grid_constant__ CUtensorMap tmG, const __grid_constant__ CUtensorMap tmW,
                    int d, int V, int rb0, int cap, const int32_t *counters,
-                   const int32_t *tok_idx, float *dH, int32_t *dev_err) {
+                   const int32_t *tok_idx, float *dH, float *scratch, int scratch_cap,
+                   int32_t *dev_err) {
   const int Teff = counters[0];
   const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
   if (nrb == 0) return;  // no token in this chunk
@@ -121,6 +142,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int nks = 2 * n_vt;  // 64-wide vocabulary steps (image atoms)
   const int nq = d / kDhN;
   const int n_units = (nrb + 1) / 2 * nq;
+  const DhTail tl = dh_tail(n_units, npairs, scratch_cap, nks);
+  const int n_items = tl.full_end + tl.R * tl.S;
+  // Work item i -> unit, its image-atom range [k0, k1) and scratch slot (-1:
+  // a whole unit, stored to dH).
+  auto item = [&](int i, int &u, int &k0, int &k1, int &slot) {
+    if (i < tl.full_end) {
+      u = i; k0 = 0; k1 = nks; slot = -1;
+    } else {
+      const int j = i - tl.full_end, part = j % tl.S;
+      u = tl.full_end + j / tl.S;
+      k0 = (int)((int64_t)part * nks / tl.S);
+      k1 = (int)((int64_t)(part + 1) * nks / tl.S);
+      slot = j;
+    }
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kDhStages; ++s) {
@@ -155,11 +191,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int last_ph[kDhStages];
       for (int s = 0; s < kDhStages; ++s) last_ph[s] = -1;
       bool ok = true;
-      for (int u = pid; u < n_units && ok; u += npairs) {
+      for (int i = pid; i < n_items && ok; i += npairs) {
+        int u, k0, k1, slot;
+        item(i, u, k0, k1, slot);
         const int tp = u / nq, q = u - tp * nq;
         const int b = min(2 * tp + r, nrb - 1);
         const int atom0 = b * nks;  // the block's first image atom
-        for (int ks = 0; ks < nks; ++ks) {
+        for (int ks = k0; ks < k1; ++ks) {
           if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
           if (elect_one()) {
             if (r == 0) mbar_expect_tx(&sm.full[stage], 2 * (kDhABytes + kDhBBytes));
@@ -194,11 +232,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int stage = 0, acc = 0;
       uint32_t ph = 0, acc_ph = 0;
       bool ok = true;
-      for (int u = pid; u < n_units && ok; u += npairs) {
+      for (int i = pid; i < n_items && ok; i += npairs) {
+        int u, k0, k1, slot;
+        item(i, u, k0, k1, slot);
         if (!(ok = wait_cluster(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
         tc_fence_after();
         const uint32_t dt = tmem + acc * kDhN;
-        for (int ks = 0; ks < nks; ++ks) {
+        for (int ks = k0; ks < k1; ++ks) {
           if (!(ok = wait_cluster(&sm.full[stage], ph, abort, dev_err))) break;
           tc_fence_after();
           const uint64_t da = da0 + (uint64_t)stage * (kDhABytes >> 4);
@@ -206,7 +246,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (elect_one()) {
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              mma_bf16_pair(dt, da + 2 * kk, db + kk * (2048 >> 4), kIdescDh, (ks | kk) != 0);
+              mma_bf16_pair(dt, da + 2 * kk, db + kk * (2048 >> 4), kIdescDh,
+                            (ks != k0) | (kk != 0));
             mma_commit_pair(&sm.empty[stage], (uint16_t)3);
           }
           __syncwarp();
@@ -229,19 +270,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     int acc = 0;
     uint32_t acc_ph = 0;
     bool ok = true;
-    for (int u = pid; u < n_units && ok; u += npairs) {
+    for (int i = pid; i < n_items && ok; i += npairs) {
+      int u, k0, k1, slot;
+      item(i, u, k0, k1, slot);
       const int tp = u / nq, q = u - tp * nq;
       const int t = (rb0 + 2 * tp + r) * 128 + row;
       const bool valid = 2 * tp + r < nrb && t < Teff;
       float4 *dst =
-          valid ? reinterpret_cast<float4 *>(dH + (int64_t)tok_idx[t] * d + q * kDhN) : nullptr;
+          slot >= 0
+              ? reinterpret_cast<float4 *>(scratch + (((int64_t)slot * 2 + r) * 128 + row) * kDhN)
+          : valid ? reinterpret_cast<float4 *>(dH + (int64_t)tok_idx[t] * d + q * kDhN)
+                  : nullptr;
       if (!(ok = wait_sleepy_cluster(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
       tc_fence_after();
 #pragma unroll 1
       for (int c = 0; c < kDhN / 32; ++c) {
         float x[32];
         tmem_ld32(tmem + lane_off + acc * kDhN + c * 32, x);
-        if (valid) {
+        if (dst) {
 #pragma unroll
           for (int e = 0; e < 8; ++e)
             dst[c * 8 + e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
@@ -259,6 +305,40 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc_pair(tmem, 512);
+  }
+}
+
+// dH of the units dh_gemm_kernel split into vocabulary parts (see DhTail):
+// the sum of their S partial tiles in part order.
+__global__ void __launch_bounds__(256)
+    dh_tail_combine_kernel(int d, int V, int rb0, int cap, int ncl, int scratch_cap,
+                           const int32_t *counters, const int32_t *tok_idx,
+                           const float *__restrict__ scratch, float *dH) {
+  const int Teff = counters[0];
+  const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  if (nrb == 0) return;
+  const int nks = 2 * ((V + 127) / 128);
+  const int nq = d / kDhN;
+  const DhTail tl = dh_tail((nrb + 1) / 2 * nq, ncl, scratch_cap, nks);
+  constexpr int kQ = kDhN / 4;  // float4 per tile row
+  const int64_t n4 = (int64_t)tl.R * 2 * 128 * kQ;
+  const float4 *src = reinterpret_cast<const float4 *>(scratch);
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n4;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int c4 = (int)(e % kQ);
+    const int row = (int)((e / kQ) % 128);
+    const int r = (int)((e / (kQ * 128)) % 2);
+    const int uj = (int)(e / (kQ * 256));
+    const int u = tl.full_end + uj;
+    const int tp = u / nq, q = u - tp * nq;
+    const int t = (rb0 + 2 * tp + r) * 128 + row;
+    if (2 * tp + r >= nrb || t >= Teff) continue;
+    float4 acc = src[(((int64_t)uj * tl.S * 2 + r) * 128 + row) * kQ + c4];
+    for (int p = 1; p < tl.S; ++p) {
+      const float4 v = src[((((int64_t)uj * tl.S + p) * 2 + r) * 128 + row) * kQ + c4];
+      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    }
+    reinterpret_cast<float4 *>(dH + (int64_t)tok_idx[t] * d + q * kDhN)[c4] = acc;
   }
 }
 
@@ -505,11 +585,23 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
   g_image_kernel<<<num_sms() * 3, 256, 0, s>>>(g.V, rb0, cap, w.counters, w.tok_c, w.lse,
                                                static_cast<const __half *>(w.sbuf), w.mbuf, gimg);
   PAIR_LAUNCH_CHECK(s);
+  // Scratch for the split last round of dH: the cluster path's tail rows
+  // (unused by this path), in 2 x 128 x kDhN fp32 tiles.
+  const int dh_grid = pair_grid((const void *)dh_gemm_kernel, dh_smem, &dh_cache);
+  const int scratch_cap =
+      w.tailbuf ? (int)((int64_t)kMaxClusters * 2 * 128 * g.d / (2 * 128 * kDhN)) : 0;
   PAIR_BEGIN("dh_gemm_tc", s);
-  dh_gemm_kernel<<<pair_grid((const void *)dh_gemm_kernel, dh_smem, &dh_cache), kThreads,
-                   dh_smem, s>>>(mGA, mW3, g.d, g.V, rb0, cap, w.counters, w.tok_idx, g.dH,
-                                 g.dev_err);
+  dh_gemm_kernel<<<dh_grid, kThreads, dh_smem, s>>>(mGA, mW3, g.d, g.V, rb0, cap, w.counters,
+                                                    w.tok_idx, g.dH, w.tailbuf, scratch_cap,
+                                                    g.dev_err);
   PAIR_LAUNCH_CHECK(s);
+  if (scratch_cap > 0) {
+    PAIR_BEGIN("dh_tail", s);
+    dh_tail_combine_kernel<<<num_sms() * 2, 256, 0, s>>>(g.d, g.V, rb0, cap, dh_grid / 2,
+                                                         scratch_cap, w.counters, w.tok_idx,
+                                                         w.tailbuf, g.dH);
+    PAIR_LAUNCH_CHECK(s);
+  }
   PAIR_BEGIN("dw_gemm_tc", s);
   dw_gemm_kernel<<<pair_grid((const void *)dw_gemm_kernel, dw_smem, &dw_cache), kThreads,
                    dw_smem, s>>>(mG, mH3, g.d, g.V, rb0, cap, c > 0 ? 1 : 0, w.counters, g.dW,
