@@ -96,24 +96,39 @@ constexpr uint32_t kDhABytes = kAtom128;               // 128 tokens x 64 vocabu
 constexpr uint32_t kDhBBytes = (kDhN / 128) * 64 * 128; // this CTA's 2 column atoms x 64 rows
 constexpr uint32_t kIdescDh = idesc_bf16(256, kDhN, 0, 1);
 
-// Work list of dh_gemm_kernel: the units that fill whole rounds of the
-// persistent grid (ncl clusters) run over all of V; the R < ncl units left
-// for the last round are cut into S vocabulary parts each (R S <= ncl, at
-// most `cap` partial tiles of scratch), so that round takes a part's time
-// instead of a unit's. Work item i < full_end is unit i; item full_end + j
-// is part j % S of unit full_end + j / S, over image atoms
-// [part nks / S, (part + 1) nks / S); its fp32 tile goes to scratch slot j
-// and dh_tail_combine_kernel adds the S parts in order (deterministic).
-struct DhTail {
+// Work list of the persistent backward GEMMs (dh_gemm_kernel,
+// dw_gemm_kernel): the units that fill whole rounds of the grid (ncl
+// clusters) run over all of their K extent; the R < ncl units left for the
+// last round are cut into S parts of K each (R S <= ncl, at most `cap`
+// partial tiles of scratch), so that round takes a part's time instead of a
+// unit's. Work item i < full_end is unit i; item full_end + j is part j % S
+// of unit full_end + j / S, over K steps [part nks / S, (part + 1) nks / S);
+// its fp32 tile goes to scratch slot j and the kernel's tail-combine pass
+// adds the S parts in order (deterministic).
+struct TailSplit {
   int full_end, R, S;
 };
-__host__ __device__ __forceinline__ DhTail dh_tail(int n_units, int ncl, int cap, int nks) {
+__host__ __device__ __forceinline__ TailSplit tail_split(int n_units, int ncl, int cap, int nks) {
   const int rem = n_units % ncl;
   int S = rem ? ncl / rem : 1;
   if (rem && S * rem > cap) S = cap / rem;
   if (S > nks) S = nks;
-  if (S < 2) return DhTail{n_units, 0, 1};
-  return DhTail{n_units - rem, rem, S};
+  if (S < 2) return TailSplit{n_units, 0, 1};
+  return TailSplit{n_units - rem, rem, S};
+}
+// Work item i of a TailSplit -> unit u, its K steps [k0, k1) and scratch
+// slot (-1: a whole unit).
+__device__ __forceinline__ void tail_item(const TailSplit &tl, int nks, int i, int &u, int &k0,
+                                          int &k1, int &slot) {
+  if (i < tl.full_end) {
+    u = i; k0 = 0; k1 = nks; slot = -1;
+  } else {
+    const int j = i - tl.full_end, part = j % tl.S;
+    u = tl.full_end + j / tl.S;
+    k0 = (int)((int64_t)part * nks / tl.S);
+    k1 = (int)((int64_t)(part + 1) * nks / tl.S);
+    slot = j;
+  }
 }
 
 struct DhSmem {
@@ -142,21 +157,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int nks = 2 * n_vt;  // 64-wide vocabulary steps (image atoms)
   const int nq = d / kDhN;
   const int n_units = (nrb + 1) / 2 * nq;
-  const DhTail tl = dh_tail(n_units, npairs, scratch_cap, nks);
+  const TailSplit tl = tail_split(n_units, npairs, scratch_cap, nks);
   const int n_items = tl.full_end + tl.R * tl.S;
-  // Work item i -> unit, its image-atom range [k0, k1) and scratch slot (-1:
-  // a whole unit, stored to dH).
-  auto item = [&](int i, int &u, int &k0, int &k1, int &slot) {
-    if (i < tl.full_end) {
-      u = i; k0 = 0; k1 = nks; slot = -1;
-    } else {
-      const int j = i - tl.full_end, part = j % tl.S;
-      u = tl.full_end + j / tl.S;
-      k0 = (int)((int64_t)part * nks / tl.S);
-      k1 = (int)((int64_t)(part + 1) * nks / tl.S);
-      slot = j;
-    }
-  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kDhStages; ++s) {
@@ -193,7 +195,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int i = pid; i < n_items && ok; i += npairs) {
         int u, k0, k1, slot;
-        item(i, u, k0, k1, slot);
+        tail_item(tl, nks, i, u, k0, k1, slot);
         const int tp = u / nq, q = u - tp * nq;
         const int b = min(2 * tp + r, nrb - 1);
         const int atom0 = b * nks;  // the block's first image atom
@@ -234,7 +236,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int i = pid; i < n_items && ok; i += npairs) {
         int u, k0, k1, slot;
-        item(i, u, k0, k1, slot);
+        tail_item(tl, nks, i, u, k0, k1, slot);
         if (!(ok = wait_cluster(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
         tc_fence_after();
         const uint32_t dt = tmem + acc * kDhN;
@@ -272,7 +274,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (int i = pid; i < n_items && ok; i += npairs) {
       int u, k0, k1, slot;
-      item(i, u, k0, k1, slot);
+      tail_item(tl, nks, i, u, k0, k1, slot);
       const int tp = u / nq, q = u - tp * nq;
       const int t = (rb0 + 2 * tp + r) * 128 + row;
       const bool valid = 2 * tp + r < nrb && t < Teff;
@@ -308,7 +310,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   }
 }
 
-// dH of the units dh_gemm_kernel split into vocabulary parts (see DhTail):
+// dH of the units dh_gemm_kernel split into vocabulary parts (see TailSplit):
 // the sum of their S partial tiles in part order.
 __global__ void __launch_bounds__(256)
     dh_tail_combine_kernel(int d, int V, int rb0, int cap, int ncl, int scratch_cap,
@@ -319,7 +321,7 @@ __global__ void __launch_bounds__(256)
   if (nrb == 0) return;
   const int nks = 2 * ((V + 127) / 128);
   const int nq = d / kDhN;
-  const DhTail tl = dh_tail((nrb + 1) / 2 * nq, ncl, scratch_cap, nks);
+  const TailSplit tl = tail_split((nrb + 1) / 2 * nq, ncl, scratch_cap, nks);
   constexpr int kQ = kDhN / 4;  // float4 per tile row
   const int64_t n4 = (int64_t)tl.R * 2 * 128 * kQ;
   const float4 *src = reinterpret_cast<const float4 *>(scratch);
@@ -383,7 +385,8 @@ struct DwSmem {
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     dw_gemm_kernel(const __grid_constant__ CUtensorMap tmG,
                    const __grid_constant__ CUtensorMap tmH, int d, int V, int rb0, int cap,
-                   int accumulate, const int32_t *counters, float *dW, int32_t *dev_err) {
+                   int accumulate, const int32_t *counters, float *dW, float *scratch,
+                   int scratch_cap, int32_t *dev_err) {
   const int Teff = counters[0];
   const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
   // A chunk past the last token adds nothing (the first chunk always runs:
@@ -398,6 +401,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int nq = d / kDwN;
   const int n_units = (n_vb + 1) / 2 * nq;
   const int nks = nrb * (128 / kDwKS);
+  const TailSplit tl = tail_split(n_units, npairs, scratch_cap, nks);
+  const int n_items = tl.full_end + tl.R * tl.S;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kDwStages; ++s) {
@@ -430,10 +435,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int last_ph[kDwStages];
       for (int s = 0; s < kDwStages; ++s) last_ph[s] = -1;
       bool ok = true;
-      for (int u = pid; u < n_units && ok; u += npairs) {
+      for (int i = pid; i < n_items && ok; i += npairs) {
+        int u, k0, k1, slot;
+        tail_item(tl, nks, i, u, k0, k1, slot);
         const int vp = u / nq, q = u - vp * nq;
         const int vb = min(2 * vp + r, n_vb - 1);
-        for (int ks = 0; ks < nks; ++ks) {
+        for (int ks = k0; ks < k1; ++ks) {
           const int rbl = ks >> 2, j = ks & 3;
           if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
           if (elect_one()) {
@@ -474,11 +481,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t ph = 0, acc_ph = 0;
       bool ok = true;
-      for (int u = pid; u < n_units && ok && nks > 0; u += npairs) {
+      for (int i = pid; i < n_items && ok && nks > 0; i += npairs) {
+        int u, k0, k1, slot;
+        tail_item(tl, nks, i, u, k0, k1, slot);
         if (!(ok = wait_cluster(&sm.acc_empty, acc_ph ^ 1, abort, dev_err))) break;
         acc_ph ^= 1;
         tc_fence_after();
-        for (int ks = 0; ks < nks; ++ks) {
+        for (int ks = k0; ks < k1; ++ks) {
           if (!(ok = wait_cluster(&sm.full[stage], ph, abort, dev_err))) break;
           tc_fence_after();
           const uint64_t dg = dg0 + (uint64_t)stage * (kDwGBytes >> 4);
@@ -490,7 +499,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
               for (int nh = 0; nh < 2; ++nh)
                 mma_bf16_pair(tmem + nh * 256, dg + kk * (2048 >> 4),
                               dh + nh * ((kDwHBytes / 2) >> 4) + kk * (2048 >> 4), kIdescDw,
-                              (ks | kk) != 0);
+                              (ks != k0) | (kk != 0));
             mma_commit_pair(&sm.empty[stage], (uint16_t)3);
           }
           __syncwarp();
@@ -511,11 +520,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     uint32_t acc_ph = 0;
     bool ok = true;
-    for (int u = pid; u < n_units && ok; u += npairs) {
+    for (int i = pid; i < n_items && ok; i += npairs) {
+      int u, k0, k1, slot;
+      tail_item(tl, nks, i, u, k0, k1, slot);
       const int vp = u / nq, q = u - vp * nq;
       const int v = (2 * vp + r) * 128 + row;
       const bool valid = 2 * vp + r < n_vb && v < V;
       float4 *dst = valid ? reinterpret_cast<float4 *>(dW + (int64_t)v * d + q * kDwN) : nullptr;
+      float4 *part_dst =
+          slot >= 0
+              ? reinterpret_cast<float4 *>(scratch + (((int64_t)slot * 2 + r) * 128 + row) * kDwN)
+              : nullptr;
       if (nks == 0) {
         if (valid)
           for (int c = 0; c < kDwN / 4; ++c) dst[c] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -528,7 +543,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int c = 0; c < kDwN / 32; ++c) {
         float x[32];
         tmem_ld32(tmem + lane_off + c * 32, x);
-        if (valid) {
+        if (part_dst) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            part_dst[c * 8 + e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+        } else if (valid) {
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             float4 o = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
@@ -551,6 +570,45 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc_pair(tmem, 512);
+  }
+}
+
+// dW rows of the units dw_gemm_kernel split into token parts (see
+// TailSplit): the sum of their S partial tiles in part order, stored or
+// (later token chunks) added.
+__global__ void __launch_bounds__(256)
+    dw_tail_combine_kernel(int d, int V, int rb0, int cap, int accumulate, int ncl,
+                           int scratch_cap, const int32_t *counters,
+                           const float *__restrict__ scratch, float *dW) {
+  const int Teff = counters[0];
+  const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
+  const int n_vb = (V + 127) / 128;
+  const int nq = d / kDwN;
+  const TailSplit tl = tail_split((n_vb + 1) / 2 * nq, ncl, scratch_cap, nrb * (128 / kDwKS));
+  constexpr int kQ = kDwN / 4;  // float4 per tile row
+  const int64_t n4 = (int64_t)tl.R * 2 * 128 * kQ;
+  const float4 *src = reinterpret_cast<const float4 *>(scratch);
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n4;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int c4 = (int)(e % kQ);
+    const int row = (int)((e / kQ) % 128);
+    const int r = (int)((e / (kQ * 128)) % 2);
+    const int uj = (int)(e / (kQ * 256));
+    const int u = tl.full_end + uj;
+    const int vp = u / nq, q = u - vp * nq;
+    const int v = (2 * vp + r) * 128 + row;
+    if (2 * vp + r >= n_vb || v >= V) continue;
+    float4 acc = src[(((int64_t)uj * tl.S * 2 + r) * 128 + row) * kQ + c4];
+    for (int p = 1; p < tl.S; ++p) {
+      const float4 x = src[((((int64_t)uj * tl.S + p) * 2 + r) * 128 + row) * kQ + c4];
+      acc.x += x.x; acc.y += x.y; acc.z += x.z; acc.w += x.w;
+    }
+    float4 *dst = reinterpret_cast<float4 *>(dW + (int64_t)v * d + q * kDwN) + c4;
+    if (accumulate) {
+      const float4 o = *dst;
+      acc.x += o.x; acc.y += o.y; acc.z += o.z; acc.w += o.w;
+    }
+    *dst = acc;
   }
 }
 
@@ -602,11 +660,21 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
                                                          w.tailbuf, g.dH);
     PAIR_LAUNCH_CHECK(s);
   }
+  const int dw_grid = pair_grid((const void *)dw_gemm_kernel, dw_smem, &dw_cache);
+  const int dw_scratch_cap =
+      w.tailbuf ? (int)((int64_t)kMaxClusters * 2 * 128 * g.d / (2 * 128 * kDwN)) : 0;
   PAIR_BEGIN("dw_gemm_tc", s);
-  dw_gemm_kernel<<<pair_grid((const void *)dw_gemm_kernel, dw_smem, &dw_cache), kThreads,
-                   dw_smem, s>>>(mG, mH3, g.d, g.V, rb0, cap, c > 0 ? 1 : 0, w.counters, g.dW,
-                                 g.dev_err);
+  dw_gemm_kernel<<<dw_grid, kThreads, dw_smem, s>>>(mG, mH3, g.d, g.V, rb0, cap, c > 0 ? 1 : 0,
+                                                    w.counters, g.dW, w.tailbuf, dw_scratch_cap,
+                                                    g.dev_err);
   PAIR_LAUNCH_CHECK(s);
+  if (dw_scratch_cap > 0) {
+    PAIR_BEGIN("dw_tail", s);
+    dw_tail_combine_kernel<<<num_sms() * 2, 256, 0, s>>>(g.d, g.V, rb0, cap, c > 0 ? 1 : 0,
+                                                         dw_grid / 2, dw_scratch_cap, w.counters,
+                                                         w.tailbuf, g.dW);
+    PAIR_LAUNCH_CHECK(s);
+  }
   return PAIR_OK;
 }
 
