@@ -514,10 +514,9 @@ __device__ __forceinline__ bool wait_count(const int *ctr, int target, volatile 
   }
 }
 
-// z_t[y_t] = <Hc_p, W_{y_p}> for every compacted token p (fp32 sums of bf16
-// products, a fixed order per token: lane-strided 8-element pieces, then the
-// warp's butterfly) and its log2-unit reference R_p = z log2 e for the fused
-// pass; also zeroes the fused pass's counters and row-block flags.
+// z_t[y_t] = <Hc_p, W_{y_p}> for every compacted token p (target_logit_dot)
+// and its log2-unit reference R_p = z log2 e for the fused pass; also zeroes
+// the fused pass's counters and row-block flags.
 __global__ void target_logit_kernel(int d, const int32_t *counters, const int32_t *tok_y,
                                     const __nv_bfloat16 *Hc, const __nv_bfloat16 *W,
                                     float *zy, float *ref, int *ready, int n_ready, int *rbflag,
@@ -529,22 +528,8 @@ __global__ void target_logit_kernel(int d, const int32_t *counters, const int32_
   const int Teff = counters[0];
   const int lane = threadIdx.x & 31;
   for (int p = tid >> 5; p < Teff; p += nth >> 5) {
-    const __nv_bfloat16 *h = Hc + (int64_t)p * d;
-    const __nv_bfloat16 *w = W + (int64_t)tok_y[p] * d;
-    float acc = 0.f;
-    for (int k = lane * 8; k < d; k += 256) {
-      const uint4 hu = *reinterpret_cast<const uint4 *>(h + k);
-      const uint4 wu = *reinterpret_cast<const uint4 *>(w + k);
-      const __nv_bfloat162 *hb = reinterpret_cast<const __nv_bfloat162 *>(&hu);
-      const __nv_bfloat162 *wb = reinterpret_cast<const __nv_bfloat162 *>(&wu);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float2 hf = __bfloat1622float2(hb[i]), wf = __bfloat1622float2(wb[i]);
-        acc = fmaf(hf.x, wf.x, acc);
-        acc = fmaf(hf.y, wf.y, acc);
-      }
-    }
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    const float acc =
+        target_logit_dot(d, Hc + (int64_t)p * d, W + (int64_t)tok_y[p] * d, lane);
     if (lane == 0) {
       zy[p] = acc;
       ref[p] = acc * kLog2e;

@@ -1,7 +1,12 @@
-// Backward of the bf16 LM-head path through the logit-gradient image: the
-// bf16 tiles Gs = -c_t softmax(z_t) formed once from the kept logit terms,
-// then dH = Gs W and dW = Gs^T Hc as plain tcgen05 GEMMs (no logit
-// recomputation), one token chunk at a time.
+// Backward of the bf16 LM-head path through the image the log-sum-exp pass
+// keeps: bf16 tiles of the softmax terms P_tv = 2^(z_tv log2 e - R_t)
+// relative to each token's reference R_t, whose row sums lsum_t the pass
+// also returns. With s_t = -c_t / lsum_t the softmax part of the logit
+// gradient is Gs_tv = s_t P_tv, so
+//     dH[t, :] = s_t sum_v P_tv W[v, :]     (dh_gemm, s_t in the epilogue)
+//     dW[v, :] = sum_t P_tv (s_t Hc[t, :])   (dw_gemm on pre-scaled rows)
+// as plain tcgen05 GEMMs (no logit recomputation, no pass over the image
+// between them), one token chunk at a time.
 #include "tc_kernels.cuh"
 
 namespace pairk {
@@ -10,76 +15,57 @@ namespace {
 using namespace tc;
 using namespace tck;
 
-// ------------------------------------------ logit-gradient image from S
+// --------------------------------------------- scaled rows for dW
 //
-// Gs_tv = -c_t exp(z_tv - lse_t) in bf16 for every tile of a chunk of token
-// blocks, from the chunk-relative terms the LSE pass kept (fp16 P_v =
-// 2^(z_v log2 e - m) and the fp32 chunk maximum m, per 32 columns):
-// Gs = -c_t 2^(m - lse_t log2 e) P_v, one exponential per 8 columns. One
-// 32 KB image tile per 128 tokens x 128 vocabulary rows, two K-major
-// SWIZZLE_128B atoms of 64 vocabulary columns (the layout both backward
-// GEMMs read). Columns >= V, rows >= T_eff and tokens with c_t = 0 give
-// exact zeros. Streaming kernel: 34 KB read and 32 KB written per tile.
-__global__ void __launch_bounds__(256) g_image_kernel(int V, int rb0, int cap,
-                                                      const int32_t *counters,
-                                                      const float *__restrict__ tok_c,
-                                                      const float *__restrict__ lse,
-                                                      const __half *__restrict__ sbuf,
-                                                      const float4 *__restrict__ mbuf,
-                                                      uint8_t *__restrict__ gimg) {
+// Hs[i, :] = s_t Hc[t, :] in bf16 for the chunk's token rows t = 128 rb0 + i,
+// s_t = -c_t / lsum_t (0 for c_t = 0); rows past T_eff are exact zeros.
+// Streaming kernel, 8 columns per thread.
+__global__ void __launch_bounds__(256)
+    scale_rows_kernel(int d, int rb0, int cap, const int32_t *counters,
+                      const float *__restrict__ tok_c, const float *__restrict__ lsum,
+                      const __nv_bfloat16 *__restrict__ Hc, __nv_bfloat16 *__restrict__ Hs) {
   const int Teff = counters[0];
   const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
-  const int n_vt = (V + 127) / 128;
-  const int64_t n_tiles = (int64_t)nrb * n_vt;
-  // Thread t of the block handles 8-column chunk (t & 15) of rows
-  // (t >> 4) + 16 k, k < 8; all eight loads are issued before any use.
-  const int ch = threadIdx.x & 15, r0 = threadIdx.x >> 4;
-  for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-    const int b = (int)(tile / n_vt), vt = (int)(tile - (int64_t)b * n_vt);
-    const __half *src = sbuf + tile * (128 * 128);
-    const float4 *mt = mbuf + tile * 128;
-    uint8_t *dst = gimg + tile * kGImgTileBytes;
-    const int col0 = vt * 128 + ch * 8;
-    uint4 h[8];
-    float4 m4[8];
+  const int d8 = d / 8;
+  const int64_t n8 = (int64_t)nrb * 128 * d8;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n8;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i = e / d8;
+    const int k8 = (int)(e - i * d8);
+    const int64_t t = (int64_t)rb0 * 128 + i;
+    uint4 out = make_uint4(0u, 0u, 0u, 0u);
+    if (t < Teff) {
+      const float c = tok_c[t];
+      if (c != 0.f) {
+        const float sc = -c / lsum[t];
+        const uint4 h = reinterpret_cast<const uint4 *>(Hc + t * d)[k8];
+        const uint32_t hw[4] = {h.x, h.y, h.z, h.w};
+        uint32_t pk[4];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const int row = r0 + 16 * k;
-      h[k] = *reinterpret_cast<const uint4 *>(src + row * 128 + ch * 8);
-      m4[k] = mt[row];
-    }
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const int row = r0 + 16 * k;
-      const int p = (rb0 + b) * 128 + row;
-      float sc = 0.f;
-      if (p < Teff && col0 < V) {
-        const float cc = tok_c[p];
-        const int q = ch >> 2;
-        const float m = q == 0 ? m4[k].x : q == 1 ? m4[k].y : q == 2 ? m4[k].z : m4[k].w;
-        if (cc != 0.f) sc = -cc * ex2_approx(m - lse[p] * kLog2e);
+        for (int q = 0; q < 4; ++q) {
+          const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&hw[q]));
+          __nv_bfloat162 b2 = __floats2bfloat162_rn(sc * f.x, sc * f.y);
+          pk[q] = *reinterpret_cast<uint32_t *>(&b2);
+        }
+        out = make_uint4(pk[0], pk[1], pk[2], pk[3]);
       }
-      const uint32_t hw[4] = {h[k].x, h[k].y, h[k].z, h[k].w};
-      uint32_t pk[4];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&hw[e]));
-        const float g0 = col0 + 2 * e < V ? sc * f.x : 0.f;
-        const float g1 = col0 + 2 * e + 1 < V ? sc * f.y : 0.f;
-        __nv_bfloat162 b2 = __floats2bfloat162_rn(g0, g1);
-        pk[e] = *reinterpret_cast<uint32_t *>(&b2);
-      }
-      *reinterpret_cast<uint4 *>(dst + (ch >> 3) * kAtom128 + sw128_offset(row, (ch & 7) * 8)) =
-          make_uint4(pk[0], pk[1], pk[2], pk[3]);
     }
+    reinterpret_cast<uint4 *>(Hs + i * d)[k8] = out;
   }
+}
+
+// Row scale of the softmax part of dH: s_t = -c_t / lsum_t.
+__device__ __forceinline__ float row_scale(const float *tok_c, const float *lsum, int t) {
+  const float c = tok_c[t];
+  return c != 0.f ? -c / lsum[t] : 0.f;
 }
 
 // ---------------------------------------------- dH from the stored image
 //
-// Softmax part of dH as the plain GEMM dH[t, :] = sum_v Gs[t, v] W[v, :],
+// Softmax part of dH as the plain GEMM dH[t, :] = s_t sum_v P[t, v] W[v, :],
 // with the image tiles as the K-major A operand (64 vocabulary rows per
-// stage, one 16 KB atom, copied verbatim) and W as the MN-major B operand.
+// stage, one 16 KB atom, copied verbatim), W as the MN-major B operand and
+// the row scale s_t applied when the accumulator is drained.
 // CTA pairs (2-CTA clusters) take two token blocks of the same 256-column
 // chunk of d as one M = 256 tile: the even CTA issues every MMA of the pair
 // (cta_group::2) over both CTAs' image atoms and the chunk's four W column
@@ -143,8 +129,8 @@ struct DhSmem {
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     dh_gemm_kernel(const __grid_constant__ CUtensorMap tmG, const __grid_constant__ CUtensorMap tmW,
                    int d, int V, int rb0, int cap, const int32_t *counters,
-                   const int32_t *tok_idx, float *dH, float *scratch, int scratch_cap,
-                   int32_t *dev_err) {
+                   const int32_t *tok_idx, const float *tok_c, const float *lsum, float *dH,
+                   float *scratch, int scratch_cap, int32_t *dev_err) {
   const int Teff = counters[0];
   const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
   if (nrb == 0) return;  // no token in this chunk
@@ -283,6 +269,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
               ? reinterpret_cast<float4 *>(scratch + (((int64_t)slot * 2 + r) * 128 + row) * kDhN)
           : valid ? reinterpret_cast<float4 *>(dH + (int64_t)tok_idx[t] * d + q * kDhN)
                   : nullptr;
+      // Partial tiles stay unscaled (the combine pass scales their sum).
+      const float sc = (slot < 0 && valid) ? row_scale(tok_c, lsum, t) : 1.f;
       if (!(ok = wait_sleepy_cluster(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
       tc_fence_after();
 #pragma unroll 1
@@ -292,7 +280,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (dst) {
 #pragma unroll
           for (int e = 0; e < 8; ++e)
-            dst[c * 8 + e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+            dst[c * 8 + e] = make_float4(sc * x[4 * e], sc * x[4 * e + 1], sc * x[4 * e + 2],
+                                         sc * x[4 * e + 3]);
         }
       }
       tc_fence_before();
@@ -311,10 +300,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 }
 
 // dH of the units dh_gemm_kernel split into vocabulary parts (see TailSplit):
-// the sum of their S partial tiles in part order.
+// the sum of their S partial tiles in part order, times the row scale.
 __global__ void __launch_bounds__(256)
     dh_tail_combine_kernel(int d, int V, int rb0, int cap, int ncl, int scratch_cap,
                            const int32_t *counters, const int32_t *tok_idx,
+                           const float *__restrict__ tok_c, const float *__restrict__ lsum,
                            const float *__restrict__ scratch, float *dH) {
   const int Teff = counters[0];
   const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
@@ -340,25 +330,27 @@ __global__ void __launch_bounds__(256)
       const float4 v = src[((((int64_t)uj * tl.S + p) * 2 + r) * 128 + row) * kQ + c4];
       acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
     }
-    reinterpret_cast<float4 *>(dH + (int64_t)tok_idx[t] * d + q * kDhN)[c4] = acc;
+    const float sc = row_scale(tok_c, lsum, t);
+    reinterpret_cast<float4 *>(dH + (int64_t)tok_idx[t] * d + q * kDhN)[c4] =
+        make_float4(sc * acc.x, sc * acc.y, sc * acc.z, sc * acc.w);
   }
 }
 
-// ------------------------------------- dW from the stored logit gradient
+// ------------------------------------- dW from the stored softmax terms
 //
-// With 128-wide column tiles the dH pass keeps every bf16 tile Gs it forms
-// (128 tokens x 128 vocabulary rows, one 32 KB image per tile in the
-// K-major SWIZZLE_128B layout of its own MMA operand) for a chunk of token
-// blocks. Read with the token index as K, the same bytes are the MN-major
-// SWIZZLE_128B layout of Gs^T (64 vocabulary rows per 128-byte line, one
-// line per token), so the softmax part of dW is the plain GEMM
-//     dW[v, :] (+)= sum_t Gs[t, v] Hc[t, :]
+// The image keeps every bf16 tile P of a chunk of token blocks (128 tokens x
+// 128 vocabulary rows, 32 KB, in the K-major SWIZZLE_128B layout of the dH
+// GEMM's A operand). Read with the token index as K, the same bytes are the
+// MN-major SWIZZLE_128B layout of P^T (64 vocabulary rows per 128-byte line,
+// one line per token), so with the pre-scaled rows Hs = s_t Hc[t, :] of the
+// chunk the softmax part of dW is the plain GEMM
+//     dW[v, :] (+)= sum_t P[t, v] Hs[t, :]
 // with no logit recomputation.
 //
-// CTA pairs (2-CTA clusters) share one 512-column chunk of Hc as two M = 256
+// CTA pairs (2-CTA clusters) share one 512-column chunk of Hs as two M = 256
 // tiles of 256 columns each: the even CTA issues every MMA of the pair
-// (cta_group::2) over both CTAs' Gs^T stages (each CTA fetches the one of its
-// own 128 vocabulary rows) and each 256-column half's four Hc column atoms,
+// (cta_group::2) over both CTAs' P^T stages (each CTA fetches the one of its
+// own 128 vocabulary rows) and each 256-column half's four Hs column atoms,
 // two in each CTA. Work unit = (vocabulary block pair, 512-column chunk of
 // d); CTA r accumulates dW[block 2 p + r, chunk] (128 x 512 fp32 = all of
 // TMEM) over the chunk's tokens, 32 token rows per stage, and drains it with
@@ -374,8 +366,8 @@ constexpr uint32_t kDwHBytes = (kDwN / 128) * kDwKS * 128; // this CTA's 4 colum
 constexpr uint32_t kIdescDw = idesc_bf16(256, 256, 1, 1); // both operands MN-major
 
 struct DwSmem {
-  uint8_t g[kDwStages][kDwGBytes];  // Gs^T: MN-major A, atoms 4 KB apart
-  uint8_t h[kDwStages][kDwHBytes];  // Hc[t, chunk]: MN-major B, atoms 4 KB apart
+  uint8_t g[kDwStages][kDwGBytes];  // P^T: MN-major A, atoms 4 KB apart
+  uint8_t h[kDwStages][kDwHBytes];  // Hs[t, chunk]: MN-major B, atoms 4 KB apart
   uint64_t full[kDwStages], empty[kDwStages];
   uint64_t acc_full, acc_empty, mma_done;
   uint32_t tmem_base;
@@ -446,7 +438,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (elect_one()) {
             if (r == 0) mbar_expect_tx(&sm.full[stage], 2 * (kDwGBytes + kDwHBytes));
             const uint32_t fb = mapa(smem_u32(&sm.full[stage]), 0);
-            const int t0 = (rb0 + rbl) * 128 + kDwKS * j;
+            const int t0 = rbl * 128 + kDwKS * j;  // chunk row of Hs
             tma_load_3d_pair(sm.g[stage], &tmG, fb, 0, kDwKS * j, 2 * (rbl * n_vb + vb));
             // Column atoms 2r, 2r + 1 of each 256-column half of the chunk.
             tma_load_3d_pair(sm.h[stage], &tmH, fb, 0, t0, q * (kDwN / 64) + 2 * r);
@@ -626,7 +618,7 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
                  CU_TENSOR_MAP_SWIZZLE_NONE) ||
       !make_map3(&mGA, w.gimg, {64, 128, (cuuint64_t)2 * cap * n_vt}, {128, 16384}, {64, 128, 1},
                  CU_TENSOR_MAP_SWIZZLE_NONE) ||
-      !make_map3(&mH3, w.Hc, {64, (cuuint64_t)w.Tpad, (cuuint64_t)g.d / 64},
+      !make_map3(&mH3, w.hs, {64, (cuuint64_t)cap * 128, (cuuint64_t)g.d / 64},
                  {(cuuint64_t)g.d * 2, 128}, {64, (cuuint32_t)kDwKS, 2},
                  CU_TENSOR_MAP_SWIZZLE_128B) ||
       !make_map3(&mW3, g.W, {64, (cuuint64_t)g.V, (cuuint64_t)g.d / 64},
@@ -638,10 +630,10 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
   PAIR_CUDA_TRY(cudaFuncSetAttribute(dw_gemm_kernel,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dw_smem));
   static int dh_cache = 0, dw_cache = 0;
-  uint8_t *gimg = static_cast<uint8_t *>(w.gimg);
-  PAIR_BEGIN("g_image", s);
-  g_image_kernel<<<num_sms() * 3, 256, 0, s>>>(g.V, rb0, cap, w.counters, w.tok_c, w.lse,
-                                               static_cast<const __half *>(w.sbuf), w.mbuf, gimg);
+  PAIR_BEGIN("scale_rows", s);
+  scale_rows_kernel<<<num_sms() * 4, 256, 0, s>>>(
+      g.d, rb0, cap, w.counters, w.tok_c, w.lsum, static_cast<const __nv_bfloat16 *>(w.Hc),
+      static_cast<__nv_bfloat16 *>(w.hs));
   PAIR_LAUNCH_CHECK(s);
   // Scratch for the split last round of dH: the cluster path's tail rows
   // (unused by this path), in 2 x 128 x kDhN fp32 tiles.
@@ -650,14 +642,14 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
       w.tailbuf ? (int)((int64_t)kMaxClusters * 2 * 128 * g.d / (2 * 128 * kDhN)) : 0;
   PAIR_BEGIN("dh_gemm_tc", s);
   dh_gemm_kernel<<<dh_grid, kThreads, dh_smem, s>>>(mGA, mW3, g.d, g.V, rb0, cap, w.counters,
-                                                    w.tok_idx, g.dH, w.tailbuf, scratch_cap,
-                                                    g.dev_err);
+                                                    w.tok_idx, w.tok_c, w.lsum, g.dH, w.tailbuf,
+                                                    scratch_cap, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   if (scratch_cap > 0) {
     PAIR_BEGIN("dh_tail", s);
     dh_tail_combine_kernel<<<num_sms() * 2, 256, 0, s>>>(g.d, g.V, rb0, cap, dh_grid / 2,
                                                          scratch_cap, w.counters, w.tok_idx,
-                                                         w.tailbuf, g.dH);
+                                                         w.tok_c, w.lsum, w.tailbuf, g.dH);
     PAIR_LAUNCH_CHECK(s);
   }
   const int dw_grid = pair_grid((const void *)dw_gemm_kernel, dw_smem, &dw_cache);
@@ -681,23 +673,22 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
 
 }  // namespace tck
 
-// Memory the backward may use for kept logit terms (fp16 terms and fp32
-// chunk maxima) and bf16 logit-gradient tiles, 66 KB per 128 x 128 tile;
-// larger problems run in token chunks.
+// Memory the backward may use for the image of softmax terms (32 KB per
+// 128 x 128 tile) and the scaled hidden rows of a chunk (128 d bf16 per token
+// block); larger problems run in token chunks.
 constexpr int64_t kImageBudget = int64_t(24) << 30;
-constexpr size_t kImageTileBytes = kGImgTileBytes + 128 * 128 * 2 + 128 * 16;
 
 int grad_gimg_rows(int64_t T, int32_t d, int32_t V, pair_dtype dt) {
   if (dt != PAIR_BF16 || d < 512 || d % kDwN != 0) return 0;
   const int64_t n_rb = (T + 127) / 128;
-  const int64_t per_rb = (int64_t)((V + 127) / 128) * (int64_t)kImageTileBytes;
+  const int64_t per_rb = (int64_t)grad_image_block_bytes(d, V);
   int64_t cap = kImageBudget / per_rb;
   if (cap < 32) cap = 32;
   return (int)(n_rb < cap ? n_rb : cap);
 }
 
-size_t grad_image_block_bytes(int32_t V) {
-  return (size_t)((V + 127) / 128) * kImageTileBytes;
+size_t grad_image_block_bytes(int32_t d, int32_t V) {
+  return (size_t)((V + 127) / 128) * kGImgTileBytes + (size_t)128 * d * 2;
 }
 
 }  // namespace pairk

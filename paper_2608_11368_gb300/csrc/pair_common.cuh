@@ -82,15 +82,15 @@ struct GradWorkspace {
   // Fused log-sum-exp + dH pass (cluster path; null otherwise).
   float *ref;          // [Tpad] per-token reference of the softmax terms (log2 units)
   float *mrow;         // [Tpad] row maximum of the logits (log2 units)
+  float *lsum;         // [Tpad] image path: sum of 2^(z log2 e - ref) over the vocabulary
   int32_t *rbflag;     // [n_rbmax] row block needs the fix-up pass
   int32_t *rb_list;    // [n_rbmax] row blocks of the fix-up pass (count in counters[1])
   int32_t *ready;      // [n_slots] per-unit publication counters
   float *lpart;        // [n_slots][8][2][128] per-CTA row partials (l, maximum)
   float *tail_l;       // [kMaxClusters][2][2][128] tail units' row partials
   int n_rbmax, n_slots;
-  void *gimg;          // bf16 logit-gradient tiles of gimg_rb token blocks, or null
-  void *sbuf;          // fp16 chunk-relative logit terms of the same blocks (LSE pass)
-  float4 *mbuf;        // fp32 maxima of their 32-column chunks, one float4 per tile row
+  void *gimg;          // bf16 softmax-term tiles 2^(z log2 e - ref) of gimg_rb token blocks
+  void *hs;            // [gimg_rb * 128][d] bf16 rows s_t Hc_t of a chunk (s_t = -c_t / lsum_t)
   int gimg_rb;         // token blocks (128 rows) per backward chunk; 0 = no image
   int64_t Tpad;
   int nsplit;
@@ -99,12 +99,11 @@ struct GradWorkspace {
 // Whether the bf16 backward runs as 8-CTA clusters: d = 512 A, 1 <= A <= 6.
 inline bool grad_cluster_path(int d) { return d % 512 == 0 && d >= 512 && d <= 3072; }
 
-// Token blocks per backward chunk for which the bf16 path keeps the fp32
-// logits and the bf16 logit-gradient image (0 where that path does not
-// apply: fp32, or d not a multiple of 512), and the bytes one block of both
-// takes.
+// Token blocks per backward chunk for which the bf16 path keeps the image of
+// softmax terms and the scaled hidden rows (0 where that path does not apply:
+// fp32, or d not a multiple of 512), and the bytes one block of both takes.
 int grad_gimg_rows(int64_t T, int32_t d, int32_t V, pair_dtype dt);
-size_t grad_image_block_bytes(int32_t V);
+size_t grad_image_block_bytes(int32_t d, int32_t V);
 constexpr uint32_t kGImgTileBytes = 128 * 128 * 2;  // one 128 x 128 bf16 tile
 
 // Workspace layout with gimg_rb token blocks of logit-gradient image (0 =

@@ -410,11 +410,15 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   const size_t o_hc = take((size_t)Tpad * d * esz);
   const size_t o_ring = dt == PAIR_BF16 ? take((size_t)kMaxClusters * kRingBytesPerCluster) : off;
   const bool cl = dt == PAIR_BF16 && grad_cluster_path(d);
+  // Hidden sizes the image backward takes (grad_gimg_rows): per-token
+  // reference and softmax sum of its log-sum-exp pass.
+  const bool img = dt == PAIR_BF16 && d >= 512 && d % 512 == 0;
   const size_t o_tail = cl ? take((size_t)kMaxClusters * 2 * 128 * d * sizeof(float)) : off;
   const int n_rbmax = (int)(Tpad / 128);
   const int n_slots = n_rbmax + 2 * kMaxClusters;
-  const size_t o_ref = cl ? take((size_t)Tpad * 4) : off;
-  const size_t o_mrow = cl ? take((size_t)Tpad * 4) : off;
+  const size_t o_ref = (cl || img) ? take((size_t)Tpad * 4) : off;
+  const size_t o_mrow = (cl || img) ? take((size_t)Tpad * 4) : off;
+  const size_t o_lsum = img ? take((size_t)Tpad * 4) : off;
   const size_t o_rbflag = cl ? take((size_t)n_rbmax * 4) : off;
   const size_t o_rblist = cl ? take((size_t)n_rbmax * 4) : off;
   const size_t o_ready = cl ? take((size_t)n_slots * 4) : off;
@@ -423,8 +427,7 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   // The image comes last, so that a larger workspace only adds token blocks.
   const size_t n_vt = (size_t)((V + 127) / 128);
   const size_t o_gimg = gimg_rb ? take((size_t)gimg_rb * n_vt * kGImgTileBytes) : off;
-  const size_t o_sbuf = gimg_rb ? take((size_t)gimg_rb * n_vt * 128 * 128 * 2) : off;
-  const size_t o_mbuf = gimg_rb ? take((size_t)gimg_rb * n_vt * 128 * 16) : off;
+  const size_t o_hs = gimg_rb ? take((size_t)gimg_rb * 128 * d * 2) : off;
   if (out) {
     char *b = static_cast<char *>(base);
     out->counters = reinterpret_cast<int32_t *>(b + o_cnt);
@@ -442,8 +445,9 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->Hc = b + o_hc;
     out->gring = b + o_ring;
     out->tailbuf = cl ? reinterpret_cast<float *>(b + o_tail) : nullptr;
-    out->ref = cl ? reinterpret_cast<float *>(b + o_ref) : nullptr;
-    out->mrow = cl ? reinterpret_cast<float *>(b + o_mrow) : nullptr;
+    out->ref = (cl || img) ? reinterpret_cast<float *>(b + o_ref) : nullptr;
+    out->mrow = (cl || img) ? reinterpret_cast<float *>(b + o_mrow) : nullptr;
+    out->lsum = img ? reinterpret_cast<float *>(b + o_lsum) : nullptr;
     out->rbflag = cl ? reinterpret_cast<int32_t *>(b + o_rbflag) : nullptr;
     out->rb_list = cl ? reinterpret_cast<int32_t *>(b + o_rblist) : nullptr;
     out->ready = cl ? reinterpret_cast<int32_t *>(b + o_ready) : nullptr;
@@ -452,8 +456,7 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->n_rbmax = n_rbmax;
     out->n_slots = n_slots;
     out->gimg = gimg_rb ? b + o_gimg : nullptr;
-    out->sbuf = gimg_rb ? b + o_sbuf : nullptr;
-    out->mbuf = gimg_rb ? reinterpret_cast<float4 *>(b + o_mbuf) : nullptr;
+    out->hs = gimg_rb ? b + o_hs : nullptr;
     out->gimg_rb = gimg_rb;
     out->Tpad = Tpad;
     out->nsplit = kNSplit;
@@ -467,7 +470,7 @@ int grad_gimg_rows_fit(int64_t T, int32_t d, int32_t V, int32_t R, pair_dtype dt
   if (ws_bytes < base) return -1;
   const int pref = grad_gimg_rows(T, d, V, dt);
   if (pref == 0) return 0;
-  const size_t fit = (ws_bytes - base) / grad_image_block_bytes(V);
+  const size_t fit = (ws_bytes - base) / grad_image_block_bytes(d, V);
   return fit < (size_t)pref ? (int)fit : pref;
 }
 

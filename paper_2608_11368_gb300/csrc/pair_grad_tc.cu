@@ -65,21 +65,6 @@ bool make_map3(CUtensorMap *m, const void *ptr, const cuuint64_t (&dims)[3],
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// fp16 [rows][128] map with 64-column x 32-row SWIZZLE_128B boxes (the
-// kept chunk-relative terms, stored by the LSE pass one warp's rows at a
-// time).
-bool make_map_s(CUtensorMap *m, const void *ptr, int64_t rows) {
-  auto fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[2] = {128, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {128 * 2};
-  cuuint32_t box[2] = {64, 32};
-  cuuint32_t estr[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(ptr), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 int num_sms() {
   static int n = 0;
   if (!n) {
@@ -113,16 +98,20 @@ int pair_grid(const void *kernel, size_t smem, int *cache) {
 using namespace tck;
 
 // Forward half: per-token log-sum-exp and target logit over every active
-// token (with an image, the first chunk's logits are kept for the backward).
+// token (with an image, relative to each token's reference, and the first
+// chunk's softmax terms are kept for the backward).
 pair_status grad_lse_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
-  if (image_path(w)) return launch_lse(g, w, s, 0, kAllBlocks, true, w.gimg_rb);
+  if (image_path(w)) {
+    const pair_status st = launch_ref(g, w, s);
+    return st != PAIR_OK ? st : launch_lse(g, w, s, 0, kAllBlocks, true, w.gimg_rb);
+  }
   return launch_lse(g, w, s, 0, kAllBlocks, false, 0);
 }
 
 // Backward half: softmax parts of dH and dW from the token coefficients,
 // after grad_lse_tc. With an image, token blocks run in chunks of
-// w.gimg_rb: the first chunk uses the logit terms grad_lse_tc kept, later
-// chunks recompute theirs.
+// w.gimg_rb: the first chunk uses the softmax terms grad_lse_tc kept, later
+// chunks recompute theirs (with the references grad_lse_tc settled).
 pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
   if (image_path(w)) {
     const int64_t nc = image_chunks(g, w);
@@ -140,21 +129,25 @@ pair_status grad_bwd_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t 
   return grad_bwd_recompute(g, w, s);
 }
 
-// The backward through the logit-gradient image runs whenever the workspace
-// holds one: token blocks in chunks of w.gimg_rb, and for each chunk
-//   g_image   Gs (bf16 tiles) from the kept fp16 logit terms, lse and c_t,
-//   dh_gemm   dH rows of the chunk = Gs . W,
-//   dw_gemm   dW (+)= Gs^T . Hc (the first chunk stores, later ones add).
-// The number of chunks follows from T, so the launch sequence needs no
-// device-to-host read; chunks past the last active token exit at once.
+// The backward through the image runs whenever the workspace holds one:
+// token blocks in chunks of w.gimg_rb, and for each chunk
+//   scale_rows  Hs = s_t Hc[t, :] in bf16, s_t = -c_t / lsum_t,
+//   dh_gemm     dH rows of the chunk = s_t (P . W),
+//   dw_gemm     dW (+)= P^T . Hs (the first chunk stores, later ones add),
+// P being the bf16 softmax terms 2^(z log2 e - R_t) the chunk's log-sum-exp
+// pass kept. The number of chunks follows from T, so the launch sequence
+// needs no device-to-host read; chunks past the last active token exit at
+// once.
 //
-// Whole head: with an image, each chunk's log-sum-exp pass keeps its logits
-// for that chunk's backward (no recomputation); otherwise, where the cluster
-// kernels apply, the fused log-sum-exp + dH pass and the recomputing dW pass
-// (no logit-sized tensor in HBM), else forward, then the recomputing
-// backward.
+// Whole head: with an image, the references R_t, then each chunk's
+// log-sum-exp pass keeps its softmax terms for that chunk's backward (no
+// recomputation); otherwise, where the cluster kernels apply, the fused
+// log-sum-exp + dH pass and the recomputing dW pass (no logit-sized tensor in
+// HBM), else forward, then the recomputing backward.
 pair_status grad_head_tc(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
   if (image_path(w)) {
+    const pair_status st = launch_ref(g, w, s);
+    if (st != PAIR_OK) return st;
     const int64_t nc = image_chunks(g, w);
     for (int64_t c = 0; c < nc; ++c) {
       pair_status st = launch_lse(g, w, s, (int)(c * w.gimg_rb), w.gimg_rb, true, w.gimg_rb);

@@ -59,26 +59,29 @@ __device__ __forceinline__ void lse_unit(int u, int n_pairs, int nsplit, int &pa
 // measured slower over the whole step (deeper pipelines let the pairs drift
 // apart in the vocabulary, so fewer of them share W rows in L2), four starve
 // the MMA.
+template <bool kImage>
 __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
     lse_kernel(const __grid_constant__ CUtensorMap tmH,
-               const __grid_constant__ CUtensorMap tmW,
-               const __grid_constant__ CUtensorMap tmS, int d, int V,
+               const __grid_constant__ CUtensorMap tmW, int d, int V,
                int nsplit, int64_t Tpad, const int32_t *counters,
-               const int32_t *tok_y, float2 *part, float *zy, int rb0, int cap,
-               const void *sbuf, float4 *mbuf, int s_blocks, int32_t *dev_err) {
+               const int32_t *tok_y, const float *ref, float2 *part, float *zy, int rb0,
+               int cap, uint8_t *gimg, int s_blocks, int fix, int32_t *dev_err) {
+  // The fix-up launch redoes the pass only if the first one flagged a row
+  // (the same value for every CTA: uniform exit before any cluster step).
+  if (kImage && fix && counters[2] == 0) return;
   extern __shared__ uint8_t smem_raw[];
   LseSmem &sm = *reinterpret_cast<LseSmem *>(align1k(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int Teff = counters[0];
-  // Token blocks [rb0, rb0 + n_tb) of this launch. With sbuf, the logits of
-  // its first s_blocks blocks are also kept, per 32-column chunk c of a row
-  // as P_j = 2^(z_j log2 e - m_c) in fp16 (in [0, 1]) with the chunk maximum
-  // m_c = max_j z_j log2 e in fp32: 128 x 128 tiles, tile (b, vt) at
-  // ((b * n_vt128 + vt) * 128 + row) * 128 + col of sbuf (written through
-  // tmS, a [rows][128] fp16 view: each epilogue warp stages its 32 rows of
-  // two chunks in shared memory and writes them with one TMA store), and
-  // the row's four maxima as one float4 at mbuf[(b * n_vt128 + vt) * 128 +
-  // row]. The same per-chunk terms P_j make up the log-sum-exp sum.
+  // Token blocks [rb0, rb0 + n_tb) of this launch. Per split, part holds
+  // (maximum, sum of terms) of each token's logits z (log2 units). Without
+  // kImage the terms are relative to the running maximum. With kImage they
+  // are P_v = 2^(z_v log2 e - R_t) for the token's reference R_t (ref), and
+  // the bf16 P of the first s_blocks blocks form the image: 128 x 128 tiles,
+  // tile (b, vt) at (b * n_vt128 + vt) * 32 KB of gimg as two K-major
+  // SWIZZLE_128B atoms of 64 columns (each epilogue warp stages 32 rows x 64
+  // columns in that layout and writes the 4 KB with one bulk copy). Columns
+  // in [V, 128 n_vt128) and rows past T_eff are exact zeros.
   const int n_tb = min(max((Teff + 127) / 128 - rb0, 0), cap);
   const int n_vt128 = (V + 127) / 128;
   const int s_lim = min(n_tb, s_blocks);
@@ -206,6 +209,7 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
     const int quad = warp & 3;
     const int row = quad * 32 + lane;
     const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    const int img_cols = n_vt128 * 128;  // image columns: V rounded up to a tile
     int acc = 0, sbuf_i = 0;
     uint32_t acc_ph = 0;
     bool ok = true;
@@ -218,8 +222,8 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
       const int vt1 = (int)((int64_t)(sp + 1) * n_vt / nsplit);
       const int p = tb * 128 + row;
       const bool valid = p < Teff;
-      const bool keep = sbuf && tbl < s_lim;  // uniform over the CTA
-      float mrow[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      const bool keep = kImage && tbl < s_lim;  // uniform over the CTA
+      const float R = (kImage && valid) ? ref[p] : 0.f;
       const int yt = valid ? tok_y[p] : -1;
       float m2 = -INFINITY, l = 0.f, zt = 0.f;
       bool found = false;
@@ -228,9 +232,10 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
         tc_fence_after();
 #pragma unroll 1
         for (int c = 0; c < kLseBN / 32; ++c) {
+          const int col0 = vt * kLseBN + c * 32;
+          if (kImage ? col0 >= img_cols : col0 >= V) break;  // the rest lies past V
           float v[32];
           tmem_ld32(lane_addr + acc * kLseBN + c * 32, v);
-          const int col0 = vt * kLseBN + c * 32;
           const int off = yt - col0;
           if (off >= 0 && off < 32) {
             found = true;
@@ -245,26 +250,36 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
             v[j] = (j < nvalid) ? v[j] * kLog2e : -INFINITY;
             mc = fmaxf(mc, v[j]);
           }
-          if (mc == -INFINITY) continue;  // the whole chunk lies past V
-          // Chunk terms relative to the chunk maximum, then folded into the
-          // running (max, sum): v[j] becomes P_j.
-          float s = 0.f;
+          if (kImage) {
+            // Terms relative to the token's reference: v[j] becomes P_j.
+            m2 = fmaxf(m2, mc);
+            float sum = 0.f;
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            v[j] = ex2_approx(v[j] - mc);
-            s += v[j];
-          }
-          if (mc > m2) {
-            l = l * ex2_approx(m2 - mc) + s;
-            m2 = mc;
+            for (int j = 0; j < 32; ++j) {
+              v[j] = valid ? ex2_approx(v[j] - R) : 0.f;
+              sum += v[j];
+            }
+            l += sum;
           } else {
-            l += s * ex2_approx(mc - m2);
+            if (mc == -INFINITY) continue;
+            // Chunk terms relative to the chunk maximum, folded into the
+            // running (maximum, sum).
+            float sum = 0.f;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) sum += ex2_approx(v[j] - mc);
+            if (mc > m2) {
+              l = l * ex2_approx(m2 - mc) + sum;
+              m2 = mc;
+            } else {
+              l += sum * ex2_approx(mc - m2);
+            }
           }
           if (keep) {
-            // Per warp: its 32 rows x 64 columns (two chunks) in fp16, in its
-            // own 4 KB buffer, stored by its lane 0 once both halves (or the
-            // last chunk before V) are in. The store that last read this
-            // buffer is done before the first half is written.
+            // Per warp: its 32 rows x 64 columns (two chunks) as bf16 in the
+            // image atom's swizzled layout, in its own 4 KB buffer, stored by
+            // its lane 0 once both halves are in (the image width is a
+            // multiple of 64 columns). The store that last read this buffer
+            // is done before the first half is written.
             const int half = c & 1;
             if (half == 0) {
               if (lane == 0) bulk_wait_group_read<1>();
@@ -276,28 +291,25 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
               uint32_t pk[4];
 #pragma unroll
               for (int q = 0; q < 4; ++q) {
-                __half2 h2 = __floats2half2_rn(v[8 * e + 2 * q], v[8 * e + 2 * q + 1]);
-                pk[q] = *reinterpret_cast<uint32_t *>(&h2);
+                __nv_bfloat162 b2 = __floats2bfloat162_rn(v[8 * e + 2 * q], v[8 * e + 2 * q + 1]);
+                pk[q] = *reinterpret_cast<uint32_t *>(&b2);
               }
               *reinterpret_cast<uint4 *>(buf + lane * 128 + (((half * 4 + e) ^ (lane & 7)) << 4)) =
                   make_uint4(pk[0], pk[1], pk[2], pk[3]);
             }
-            mrow[c & 3] = mc;
-            const bool last = col0 + 32 >= V;
-            if (half == 1 || last) {
+            if (half == 1) {
               fence_async_smem();
               __syncwarp();
               if (lane == 0) {
-                tma_store_2d_evict_first(&tmS, buf, col0 & 64,
-                                         (tbl * n_vt128 + (col0 >> 7)) * 128 + quad * 32);
+                const int acol = col0 & ~63;  // the atom's first column
+                uint8_t *dst = gimg +
+                               (((size_t)tbl * n_vt128 + (acol >> 7)) * 2 + ((acol >> 6) & 1)) *
+                                   kAtom128 +
+                               quad * 4096;
+                bulk_store_evict_first(dst, buf, 4096);
                 bulk_commit_group();
               }
               sbuf_i ^= 1;
-            }
-            if ((c & 3) == 3 || last) {
-              mbuf[((int64_t)tbl * n_vt128 + (col0 >> 7)) * 128 + row] =
-                  make_float4(mrow[0], mrow[1], mrow[2], mrow[3]);
-              mrow[0] = mrow[1] = mrow[2] = mrow[3] = -INFINITY;
             }
           }
         }
@@ -311,7 +323,7 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
         if (found) zy[p] = zt;
       }
     }
-    // Every kept-logit store has completed before the CTA leaves.
+    // Every image store has completed before the CTA leaves.
     if (lane == 0) bulk_wait_group<0>();
     __syncwarp();
   }
@@ -325,11 +337,23 @@ __global__ void __cluster_dims__(kLsePair, 1, 1) __launch_bounds__(kThreads, 1)
   }
 }
 
-// lse_t = ln 2 * (M + log2 sum_s l_s 2^(m_s - M)) over the vocabulary splits.
-// Tokens [128 rb0, 128 (rb0 + cap)) of the active ones.
-__global__ void lse_combine_kernel(int nsplit, int64_t Tpad,
-                                   const int32_t *counters, const float2 *part,
-                                   float *lse, int rb0, int cap) {
+// Largest distance (log2 units) of a row's maximum logit above its reference
+// that the image pass keeps: the terms stay below 2^64, their sums far from
+// the fp32 range. Rows beyond it are redone with the maximum as reference.
+constexpr float kImgFixLog2 = 64.f;
+
+// lse of tokens [128 rb0, 128 (rb0 + cap)) of the active ones, over the
+// vocabulary splits. Without kImage: lse = ln 2 (M + log2 sum_s l_s 2^(m_s -
+// M)). With kImage (terms relative to R_t): lsum_t = sum_s l_s and lse =
+// ln 2 (R_t + log2 lsum_t); in the first pass (fix = 0), a row whose maximum
+// m exceeds R_t by more than kImgFixLog2 instead gets R_t = m and is counted
+// in counters[2] for the fix-up pass; the fix-up pass (fix = 1) runs only if
+// some row was counted.
+template <bool kImage>
+__global__ void lse_combine_kernel(int nsplit, int64_t Tpad, int32_t *counters,
+                                   const float2 *part, float *lse, float *ref, float *lsum,
+                                   int rb0, int cap, int fix) {
+  if (kImage && fix && counters[2] == 0) return;
   const int Teff = counters[0];
   const int64_t hi64 = (int64_t)(rb0 + (int64_t)cap) * 128;
   const int p1 = (int)(hi64 < Teff ? hi64 : Teff);
@@ -338,11 +362,36 @@ __global__ void lse_combine_kernel(int nsplit, int64_t Tpad,
     float M = -INFINITY;
     for (int s = 0; s < nsplit; ++s) M = fmaxf(M, part[(int64_t)s * Tpad + p].x);
     float L = 0.f;
-    for (int s = 0; s < nsplit; ++s) {
-      const float2 q = part[(int64_t)s * Tpad + p];
-      if (q.y > 0.f) L += q.y * exp2f(q.x - M);
+    if (kImage) {
+      for (int s = 0; s < nsplit; ++s) L += part[(int64_t)s * Tpad + p].y;
+      const float R = ref[p];
+      if (!fix && M - R > kImgFixLog2) {
+        ref[p] = M;
+        atomicAdd(&counters[2], 1);
+      } else {
+        lsum[p] = L;
+        lse[p] = (R + log2f(L)) * 0.6931471805599453f;
+      }
+    } else {
+      for (int s = 0; s < nsplit; ++s) {
+        const float2 q = part[(int64_t)s * Tpad + p];
+        if (q.y > 0.f) L += q.y * exp2f(q.x - M);
+      }
+      lse[p] = (M + log2f(L)) * 0.6931471805599453f;
     }
-    lse[p] = (M + log2f(L)) * 0.6931471805599453f;
+  }
+}
+
+// Reference of the image pass: R_p = z_p[y_p] log2 e for every compacted
+// active token p (target_logit_dot).
+__global__ void ref_logit_kernel(int d, const int32_t *counters, const int32_t *tok_y,
+                                 const __nv_bfloat16 *Hc, const __nv_bfloat16 *W, float *ref) {
+  const int Teff = counters[0];
+  const int lane = threadIdx.x & 31;
+  const int nw = (gridDim.x * blockDim.x) >> 5;
+  for (int p = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; p < Teff; p += nw) {
+    const float z = target_logit_dot(d, Hc + (int64_t)p * d, W + (int64_t)tok_y[p] * d, lane);
+    if (lane == 0) ref[p] = z * kLog2e;
   }
 }
 
@@ -355,7 +404,8 @@ int lse_grid(size_t smem) {
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, (const void *)lse_kernel, &cfg) != cudaSuccess || n <= 0) {
+  if (cudaOccupancyMaxActiveClusters(&n, (const void *)lse_kernel<true>, &cfg) != cudaSuccess ||
+      n <= 0) {
     cudaGetLastError();
     n = num_sms() / kLsePair;
   }
@@ -367,30 +417,56 @@ int lse_grid(size_t smem) {
 
 namespace tck {
 
+pair_status launch_ref(const GradArgs &g, const GradWorkspace &w, cudaStream_t s) {
+  PAIR_BEGIN("ref_logit", s);
+  ref_logit_kernel<<<num_sms() * 8, 256, 0, s>>>(
+      g.d, w.counters, w.tok_y, static_cast<const __nv_bfloat16 *>(w.Hc),
+      static_cast<const __nv_bfloat16 *>(g.W), w.ref);
+  PAIR_LAUNCH_CHECK(s);
+  return PAIR_OK;
+}
+
 // Log-sum-exp pass over token blocks [rb0, rb0 + cap) (clipped to the active
-// ones), then lse for those tokens. With keep, the chunk-relative logit terms
-// of the first s_blocks of those blocks are kept in w.sbuf / w.mbuf.
+// ones), then lse for those tokens. With image, the terms are relative to
+// w.ref, the bf16 terms of the first s_blocks of those blocks are kept in
+// w.gimg, and a fix-up pass redoes the blocks (only if some row was flagged).
 pair_status launch_lse(const GradArgs &g, const GradWorkspace &w, cudaStream_t s, int rb0,
-                       int cap, bool keep, int s_blocks) {
-  void *sbuf = keep ? w.sbuf : nullptr;
-  CUtensorMap mH, mW128, mS = {};
+                       int cap, bool image, int s_blocks) {
+  CUtensorMap mH, mW128;
   if (!make_map(&mH, w.Hc, w.Tpad, g.d, 128) || !make_map(&mW128, g.W, g.V, g.d, 128))
-    return PAIR_ERR_CUDA;
-  if (sbuf && !make_map_s(&mS, sbuf, (int64_t)w.gimg_rb * ((g.V + 127) / 128) * 128))
     return PAIR_ERR_CUDA;
   const int nsm = num_sms();
   const size_t lse_smem = sizeof(LseSmem) + 1024;
-  PAIR_CUDA_TRY(cudaFuncSetAttribute(lse_kernel,
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(lse_kernel<true>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)lse_smem));
-  PAIR_BEGIN("lse_tc", s);
-  lse_kernel<<<lse_grid(lse_smem), kThreads, lse_smem, s>>>(
-      mH, mW128, mS, g.d, g.V, w.nsplit, w.Tpad, w.counters, w.tok_y, w.part, w.zy, rb0, cap, sbuf,
-      keep ? w.mbuf : nullptr, s_blocks, g.dev_err);
-  PAIR_LAUNCH_CHECK(s);
-  PAIR_BEGIN("lse_combine", s);
-  lse_combine_kernel<<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters, w.part, w.lse, rb0,
-                                             cap);
-  PAIR_LAUNCH_CHECK(s);
+  PAIR_CUDA_TRY(cudaFuncSetAttribute(lse_kernel<false>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)lse_smem));
+  const int grid = lse_grid(lse_smem);
+  if (!image) {
+    PAIR_BEGIN("lse_tc", s);
+    lse_kernel<false><<<grid, kThreads, lse_smem, s>>>(
+        mH, mW128, g.d, g.V, w.nsplit, w.Tpad, w.counters, w.tok_y, nullptr, w.part, w.zy, rb0,
+        cap, nullptr, 0, 0, g.dev_err);
+    PAIR_LAUNCH_CHECK(s);
+    PAIR_BEGIN("lse_combine", s);
+    lse_combine_kernel<false><<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters, w.part,
+                                                      w.lse, nullptr, nullptr, rb0, cap, 0);
+    PAIR_LAUNCH_CHECK(s);
+    return PAIR_OK;
+  }
+  uint8_t *gimg = static_cast<uint8_t *>(w.gimg);
+  PAIR_CUDA_TRY(cudaMemsetAsync(w.counters + 2, 0, sizeof(int32_t), s));
+  for (int fix = 0; fix < 2; ++fix) {
+    PAIR_BEGIN(fix ? "lse_fix" : "lse_tc", s);
+    lse_kernel<true><<<grid, kThreads, lse_smem, s>>>(
+        mH, mW128, g.d, g.V, w.nsplit, w.Tpad, w.counters, w.tok_y, w.ref, w.part, w.zy, rb0,
+        cap, gimg, s_blocks, fix, g.dev_err);
+    PAIR_LAUNCH_CHECK(s);
+    PAIR_BEGIN("lse_combine", s);
+    lse_combine_kernel<true><<<nsm * 4, 256, 0, s>>>(w.nsplit, w.Tpad, w.counters, w.part,
+                                                     w.lse, w.ref, w.lsum, rb0, cap, fix);
+    PAIR_LAUNCH_CHECK(s);
+  }
   return PAIR_OK;
 }
 

@@ -45,6 +45,42 @@ __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t b
       : "memory");
 }
 
+// Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned) from
+// this CTA's shared memory to global memory, tracked by this thread's bulk
+// groups, with an L2 evict-first hint.
+__device__ __forceinline__ void bulk_store_evict_first(void *dst, const void *src,
+                                                       uint32_t bytes) {
+  asm volatile(
+      "{\n\t.reg .b64 pol;\n\t"
+      "createpolicy.fractional.L2::evict_first.b64 pol, 1.0;\n\t"
+      "cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, pol;\n\t}" ::"l"(
+          reinterpret_cast<uint64_t>(dst)),
+      "r"(smem_u32(src)), "r"(bytes)
+      : "memory");
+}
+
+// <h, w> over d bf16 elements by one warp (d a multiple of 8, rows 16-byte
+// aligned): fp32 sums of the products in a fixed order (lane-strided
+// 8-element pieces, then the warp's butterfly); every lane gets the sum.
+__device__ __forceinline__ float target_logit_dot(int d, const __nv_bfloat16 *h,
+                                                  const __nv_bfloat16 *w, int lane) {
+  float acc = 0.f;
+  for (int k = lane * 8; k < d; k += 256) {
+    const uint4 hu = *reinterpret_cast<const uint4 *>(h + k);
+    const uint4 wu = *reinterpret_cast<const uint4 *>(w + k);
+    const __nv_bfloat162 *hb = reinterpret_cast<const __nv_bfloat162 *>(&hu);
+    const __nv_bfloat162 *wb = reinterpret_cast<const __nv_bfloat162 *>(&wu);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 hf = __bfloat1622float2(hb[i]), wf = __bfloat1622float2(wb[i]);
+      acc = fmaf(hf.x, wf.x, acc);
+      acc = fmaf(hf.y, wf.y, acc);
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  return acc;
+}
+
 __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
@@ -57,20 +93,22 @@ bool make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t cols, int b
 bool make_map3(CUtensorMap *m, const void *ptr, const cuuint64_t (&dims)[3],
                const cuuint64_t (&strides)[2], const cuuint32_t (&box)[3],
                CUtensorMapSwizzle sw);
-// fp16 [rows][128] map with 64-column x 32-row SWIZZLE_128B boxes.
-bool make_map_s(CUtensorMap *m, const void *ptr, int64_t rows);
 int num_sms();
 // CTAs of a persistent grid of 2-CTA clusters (occupancy API; cached in *cache).
 int pair_grid(const void *kernel, size_t smem, int *cache);
 
 // ---- stages of the head
+// Per-token reference of the image path's log-sum-exp pass: R_t = z_t[y_t]
+// log2 e for every active token (pair_lse.cu).
+pair_status launch_ref(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
 // Log-sum-exp pass over token blocks [rb0, rb0 + cap), then lse of those
-// tokens; with keep, the logit terms of its first s_blocks blocks are kept
-// (pair_lse.cu).
+// tokens. With image, the softmax terms are taken relative to the reference
+// (launch_ref first), the bf16 terms of its first s_blocks blocks are kept as
+// the image, and rows too far above their reference are redone (pair_lse.cu).
 pair_status launch_lse(const GradArgs &g, const GradWorkspace &w, cudaStream_t s, int rb0,
-                       int cap, bool keep, int s_blocks);
-// One token chunk of the image backward: g_image, dh_gemm, dw_gemm
-// (pair_bwd_image.cu).
+                       int cap, bool image, int s_blocks);
+// One token chunk of the image backward: scaled hidden rows, dh_gemm,
+// dw_gemm (pair_bwd_image.cu).
 pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStream_t s,
                              int64_t c);
 // Backward without an image, recomputing the logits (pair_bwd_cluster.cu).
@@ -81,7 +119,7 @@ pair_status grad_bwd_recompute(const GradArgs &g, const GradWorkspace &w, cudaSt
 bool onchip_fused_applies(int d);
 pair_status grad_head_onchip(const GradArgs &g, const GradWorkspace &w, cudaStream_t s);
 
-inline bool image_path(const GradWorkspace &w) { return w.gimg && w.sbuf && w.gimg_rb > 0; }
+inline bool image_path(const GradWorkspace &w) { return w.gimg && w.hs && w.gimg_rb > 0; }
 inline int64_t image_chunks(const GradArgs &g, const GradWorkspace &w) {
   return ((g.T + 127) / 128 + w.gimg_rb - 1) / w.gimg_rb;
 }

@@ -129,60 +129,6 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map,
       : "memory");
 }
 
-// tma_load_2d delivered to the same shared-memory offset (and completing
-// the same-offset mbarrier) in every cluster CTA of `mask`.
-__device__ __forceinline__ void tma_load_2d_mc(void *dst, const CUtensorMap *map,
-                                               uint64_t *bar, int x, int y, uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      ".multicast::cluster [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(mask)
-      : "memory");
-}
-
-// 3-D tile load (coordinates innermost first).
-__device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, uint64_t *bar,
-                                            int x, int y, int z) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z)
-      : "memory");
-}
-
-// tma_load_3d delivered to the same shared-memory offset (and completing
-// the same-offset mbarrier) in every cluster CTA of `mask`.
-__device__ __forceinline__ void tma_load_3d_mc(void *dst, const CUtensorMap *map, uint64_t *bar,
-                                               int x, int y, int z, uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      ".multicast::cluster [%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z),
-      "h"(mask)
-      : "memory");
-}
-
-// 2-D tile store shared -> global, tracked by this thread's bulk groups.
-__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, const void *src, int x,
-                                             int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
-          reinterpret_cast<uint64_t>(map)),
-      "r"(smem_u32(src)), "r"(x), "r"(y)
-      : "memory");
-}
-// tma_store_2d with an L2 evict-first policy: for streams written once and
-// read back much later, so they do not displace reused lines.
-__device__ __forceinline__ void tma_store_2d_evict_first(const CUtensorMap *map, const void *src,
-                                                         int x, int y) {
-  asm volatile(
-      "{\n\t.reg .b64 pol;\n\t"
-      "createpolicy.fractional.L2::evict_first.b64 pol, 1.0;\n\t"
-      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group.L2::cache_hint"
-      " [%0, {%2, %3}], [%1], pol;\n\t}" ::"l"(reinterpret_cast<uint64_t>(map)),
-      "r"(smem_u32(src)), "r"(x), "r"(y)
-      : "memory");
-}
 __device__ __forceinline__ void bulk_commit_group() {
   asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }

@@ -43,23 +43,22 @@ def test_workspace_size_rules(L):
     wmin = L.pair_grad_workspace_min_size
     # The fp32 path stages 4-byte hidden rows; bf16 stages 2-byte rows plus a
     # fixed ring of logit-gradient tiles, the clusters' tail scratch
-    # (24 x 2 x 128 x d fp32) and the fused LSE pass's per-token arrays
-    # (reference and row maximum, 2 x 4 bytes per padded token; one 8 x 256
-    # fp32 partial block per 128-token slot, ceil(T/128) + 48 slots), so fp32
-    # needs more once T is large.
+    # (24 x 2 x 128 x d fp32) and the per-token arrays of the log-sum-exp
+    # passes (reference, row maximum and softmax sum, 3 x 4 bytes per padded
+    # token; one 8 x 256 fp32 partial block per 128-token slot, ceil(T/128) +
+    # 48 slots), so fp32 needs more once T is large.
     tpad = (100000 + 127) // 128 * 128
-    fused = 2 * 4 * tpad + (tpad // 128 + 48) * 8 * 256 * 4 + (1 << 20)
+    fused = 3 * 4 * tpad + (tpad // 128 + 48) * 8 * 256 * 4 + (1 << 20)
     fixed = (12 << 20) + 24 * 2 * 128 * 2048 * 4 + (1 << 20) + fused
     assert (wmin(100000, 2048, 151936, 64, L.PAIR_F32)
             - wmin(100000, 2048, 151936, 64, L.PAIR_BF16) > 100000 * 2048 * 2 - fixed)
-    # For d a multiple of 512, bf16 also keeps the logit terms (fp16 per
-    # element, an fp32 maximum per 32 columns) and the bf16 logit-gradient
-    # image of min(ceil(T/128), max(32, 24 GiB // per_block)) token blocks,
-    # per_block = ceil(V/128) tiles of 32 + 2 + 32 KB; other widths and fp32
-    # keep none.
+    # For d a multiple of 512, bf16 also keeps the bf16 image of softmax
+    # terms and the scaled hidden rows of min(ceil(T/128), max(32, 24 GiB //
+    # per_block)) token blocks, per_block = ceil(V/128) tiles of 32 KB plus
+    # 128 rows of d bf16; other widths and fp32 keep none.
     for T, d, V in [(100000, 2048, 151936), (1000, 512, 1000), (10 ** 6, 1024, 10 ** 6),
                     (5000, 1536, 300), (70000, 2560, 151936), (3000, 3072, 4099)]:
-        per_block = (V + 127) // 128 * (32768 + 2048 + 32768)
+        per_block = (V + 127) // 128 * 32768 + 128 * d * 2
         blocks = min((T + 127) // 128, max(32, (24 << 30) // per_block))
         assert ws(T, d, V, 64, L.PAIR_BF16) - wmin(T, d, V, 64, L.PAIR_BF16) == blocks * per_block
     for d, dt in [(640, L.PAIR_BF16), (256, L.PAIR_BF16), (2048, L.PAIR_F32)]:
