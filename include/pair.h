@@ -37,12 +37,12 @@
  *    PAIR_ERR_UNSUPPORTED.
  *  - Single-GPU library: every call runs on the current device only, and
  *    every array it is given must live on that device. The tensor-core head
- *    kernels (the log-sum-exp pass and the two backward GEMMs) load tiles
- *    with TMA multicast to the CTAs of one thread-block cluster; their tensor
- *    maps cover only the caller's buffers and the workspace on the current
- *    device, never another GPU's memory. A multi-GPU trainer runs one
- *    independent call per GPU (whole prompt groups per GPU) and does its own
- *    exchange of dW outside the library.
+ *    kernels (the log-sum-exp pass and the two backward GEMMs) run one MMA
+ *    per pair of CTAs of a 2-CTA cluster; their tensor maps cover only the
+ *    caller's buffers and the workspace on the current device, never another
+ *    GPU's memory, and no kernel issues TMA multicast loads. A multi-GPU
+ *    trainer runs one independent call per GPU (whole prompt groups per GPU)
+ *    and does its own exchange of dW outside the library.
  */
 #ifndef PAIR_H_
 #define PAIR_H_
@@ -323,24 +323,28 @@ PAIR_API pair_status pair_allocate(int32_t B, int32_t G, const float *p_hat, con
  * pair_grad_clipped) should be given for T packed tokens, hidden size d,
  * vocabulary V, R rollouts and dtype dt. Returns 0 for arguments pair_grad
  * would reject.
- * For PAIR_BF16 with d in {512, 1024, 1536, 2048} this includes the
- * logit-gradient image: the bf16 tiles Gs = -c_t softmax(z_t) the dH pass
- * forms are kept, 32 KB per 128 tokens x 128 vocabulary rows, so that the dW
- * pass reads them instead of recomputing the logits. It holds
- * min(ceil(T/128), max(32, 2^33 / (ceil(V/128) * 32768))) token blocks of
- * ceil(V/128) tiles (at most about 8 GiB); longer batches run the backward
- * in token chunks of that many blocks.
+ * For PAIR_BF16 with d a multiple of 512 this includes the image of the
+ * backward: the log-sum-exp pass keeps the bf16 softmax terms
+ * 2^(z_tv log2 e - R_t) relative to each token's target logit R_t, 32 KB per
+ * 128 tokens x 128 vocabulary rows, which the dH and dW GEMMs read instead of
+ * recomputing the logits, plus the chunk's hidden rows scaled by
+ * -c_t / sum_v 2^(z_tv log2 e - R_t) (128 d bf16 per token block). It holds
+ * min(ceil(T/128), max(32, 24 GiB / per_block)) token blocks, per_block =
+ * ceil(V/128) * 32768 + 256 d bytes (at most about 24 GiB); longer batches
+ * run the backward in token chunks of that many blocks.
  */
 PAIR_API size_t pair_grad_workspace_size(int64_t T, int32_t d, int32_t V, int32_t R,
                                 pair_dtype dt);
 
 /*
  * pair_grad_workspace_min_size -- the smallest workspace pair_grad accepts:
- * pair_grad_workspace_size without the logit-gradient image. Any size from
- * here up to pair_grad_workspace_size is valid; the image then holds the
- * token blocks that fit (more chunks), and with none the dW pass recomputes
- * the logits. Results agree to fp32 rounding across sizes (the dW sums run
- * in a different order), and are bit-identical for the same size.
+ * pair_grad_workspace_size without the image. Any size from here up to
+ * pair_grad_workspace_size is valid; the image then holds the token blocks
+ * that fit (more chunks), and with none no logit-sized tensor is kept at all
+ * (the on-chip form: the log-sum-exp pass is fused with dH, and dW
+ * recomputes the logits). Results agree to bf16/fp32 rounding across sizes
+ * (the sums run in a different order), and are bit-identical for the same
+ * size.
  */
 PAIR_API size_t pair_grad_workspace_min_size(int64_t T, int32_t d, int32_t V, int32_t R,
                                     pair_dtype dt);
@@ -356,10 +360,10 @@ PAIR_API size_t pair_grad_workspace_min_size(int64_t T, int32_t d, int32_t V, in
  * The sequence score of Sec. 3.1 is the per-rollout sum over tokens (no
  * length normalisation). Rollouts with a_i == 0 (+0 or -0) are skipped
  * entirely; their tokens' dH rows, like those of mask = 0 tokens, are
- * written as exact zeros. No logit-sized tensor is written in fp32: the
- * log-sum-exp pass keeps the logits as fp16 terms relative to each
- * 32-column chunk maximum, from which the bf16 logit gradient is formed
- * once and read by the dH and dW GEMMs (see pair_grad_workspace_size).
+ * written as exact zeros. No logit-sized tensor is written in fp32: with the
+ * default workspace the log-sum-exp pass keeps the bf16 softmax terms once
+ * for the dH and dW GEMMs (see pair_grad_workspace_size); with the minimum
+ * workspace nothing logit-sized is written.
  *
  * In:  T >= 1 packed tokens; d hidden size; V vocabulary size; dt dtype of
  *      H and W (PAIR_BF16: fp32 accumulation on the tensor cores, requires
@@ -461,8 +465,8 @@ PAIR_API pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dty
  * size grows with T * d (the compacted hidden rows) plus, for bf16, a fixed
  * exchange buffer and, for d a multiple of 512, per-cluster partial rows of
  * width d. In this build the accepted range is, roughly: PAIR_F32, T (4 d +
- * 148) <= 33 MB (T <= 32,000 at d = 256); PAIR_BF16 with d a multiple of 512,
- * only d = 512 with T <= 7,000 (larger d need more than the array for the
+ * 148) <= 33 MB (T <= 28,000 at d = 256); PAIR_BF16 with d a multiple of 512,
+ * only d = 512 with T <= 6,000 (larger d need more than the array for the
  * partial rows alone); other PAIR_BF16 d, T (2 d + 148) <= 20.9 MB. Larger
  * heads (the Qwen3 shapes) need pair_grad with a caller-provided workspace.
  * The call allocates nothing.
