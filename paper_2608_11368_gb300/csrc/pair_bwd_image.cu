@@ -66,21 +66,24 @@ __device__ __forceinline__ float row_scale(const float *tok_c, const float *lsum
 // with the image tiles as the K-major A operand (64 vocabulary rows per
 // stage, one 16 KB atom, copied verbatim), W as the MN-major B operand and
 // the row scale s_t applied when the accumulator is drained.
-// CTA pairs (2-CTA clusters) take two token blocks of the same 256-column
-// chunk of d as one M = 256 tile: the even CTA issues every MMA of the pair
-// (cta_group::2) over both CTAs' image atoms and the chunk's four W column
-// atoms, two in each CTA, and each CTA's TMEM receives its own token block's
-// rows. Work unit = (token block pair, 256-column chunk); the fp32
-// accumulator (128 x 256 per CTA) is double-buffered in TMEM so the drain of
-// one unit overlaps the next. Each (token, column) is owned by one CTA and
-// summed over all of V in one fixed order: deterministic, no atomics. An odd
-// last block is computed twice (the pair's other CTA repeats it) and stored
-// once.
-constexpr int kDhN = 256;                              // output columns per unit
+// CTA pairs (2-CTA clusters) take two token blocks of the same 512-column
+// chunk of d as two M = 256 tiles of 256 columns each: the even CTA issues
+// every MMA of the pair (cta_group::2) over both CTAs' image atoms and each
+// 256-column half's four W column atoms, two in each CTA, and each CTA's TMEM
+// receives its own token block's rows (128 x 512 fp32, all of TMEM; a unit
+// runs long enough that its drain, not overlapped with the next unit, costs
+// well under 1 %). Work unit = (token block pair, 512-column chunk): the
+// units of one token pair read its image rows, and with d = 2048 the 76
+// pairs of a GB300 hold 19 token pairs' four units at once, so no token
+// pair's units straddle two rounds. Each (token, column) is owned by one CTA
+// and summed over all of V in one fixed order: deterministic, no atomics. An
+// odd last block is computed twice (the pair's other CTA repeats it) and
+// stored once.
+constexpr int kDhN = 512;                              // output columns per unit
 constexpr int kDhStages = 4;
 constexpr uint32_t kDhABytes = kAtom128;               // 128 tokens x 64 vocabulary
-constexpr uint32_t kDhBBytes = (kDhN / 128) * 64 * 128; // this CTA's 2 column atoms x 64 rows
-constexpr uint32_t kIdescDh = idesc_bf16(256, kDhN, 0, 1);
+constexpr uint32_t kDhBBytes = (kDhN / 128) * 64 * 128; // this CTA's 4 column atoms x 64 rows
+constexpr uint32_t kIdescDh = idesc_bf16(256, 256, 0, 1);
 
 // Work list of the persistent backward GEMMs (dh_gemm_kernel,
 // dw_gemm_kernel): the units that fill whole rounds of the grid (ncl
@@ -121,7 +124,7 @@ struct DhSmem {
   uint8_t a[kDhStages][kDhABytes];
   uint8_t b[kDhStages][kDhBBytes];
   uint64_t full[kDhStages], empty[kDhStages];
-  uint64_t acc_full[2], acc_empty[2], mma_done;
+  uint64_t acc_full, acc_empty, mma_done;
   uint32_t tmem_base;
   int abort;
 };
@@ -151,10 +154,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(&sm.full[s], 1);   // the even CTA's expect_tx (both CTAs' bytes)
       mbar_init(&sm.empty[s], 1);  // the pair MMA's commit
     }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&sm.acc_full[s], 1);
-      mbar_init(&sm.acc_empty[s], 2 * 128);  // both CTAs' epilogue threads
-    }
+    mbar_init(&sm.acc_full, 1);
+    mbar_init(&sm.acc_empty, 2 * 128);  // both CTAs' epilogue threads
     mbar_init(&sm.mma_done, 1);
     sm.abort = 0;
     fence_mbar_init();
@@ -191,8 +192,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             if (r == 0) mbar_expect_tx(&sm.full[stage], 2 * (kDhABytes + kDhBBytes));
             const uint32_t fb = mapa(smem_u32(&sm.full[stage]), 0);
             tma_load_3d_pair(sm.a[stage], &tmG, fb, 0, 0, atom0 + ks);
-            tma_load_3d_pair(sm.b[stage], &tmW, fb, 0, 64 * ks,
-                             q * (kDhN / 64) + r * (kDhN / 128));
+            // Column atoms 2r, 2r + 1 of each 256-column half of the chunk.
+            tma_load_3d_pair(sm.b[stage], &tmW, fb, 0, 64 * ks, q * (kDhN / 64) + 2 * r);
+            tma_load_3d_pair(sm.b[stage] + kDhBBytes / 2, &tmW, fb, 0, 64 * ks,
+                             q * (kDhN / 64) + 4 + 2 * r);
           }
           __syncwarp();
           last_ph[stage] = (int)ph;
@@ -213,19 +216,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     if (r == 0) {  // whole warp: uniform loop state; elected lane issues
       // A: K-major atom, 16 tokens of K = 32 bytes along the swizzled row.
-      // B: this CTA's 2 column atoms of 64 vocabulary rows (LBO 8 KB), row
-      // groups of 8 (SBO 1 KB); 16 vocabulary rows = 2 KB.
+      // B: per 256-column half, this CTA's 2 column atoms of 64 vocabulary
+      // rows (LBO 8 KB), row groups of 8 (SBO 1 KB); 16 vocabulary rows =
+      // 2 KB; the second half is 16 KB on.
       const uint64_t da0 = sdesc_sw128(smem_u32(sm.a[0]), 16, 1024);
       const uint64_t db0 = sdesc_sw128(smem_u32(sm.b[0]), 64 * 128, 1024);
-      int stage = 0, acc = 0;
+      int stage = 0;
       uint32_t ph = 0, acc_ph = 0;
       bool ok = true;
       for (int i = pid; i < n_items && ok; i += npairs) {
         int u, k0, k1, slot;
         tail_item(tl, nks, i, u, k0, k1, slot);
-        if (!(ok = wait_cluster(&sm.acc_empty[acc], acc_ph ^ 1, abort, dev_err))) break;
+        if (!(ok = wait_cluster(&sm.acc_empty, acc_ph ^ 1, abort, dev_err))) break;
+        acc_ph ^= 1;
         tc_fence_after();
-        const uint32_t dt = tmem + acc * kDhN;
         for (int ks = k0; ks < k1; ++ks) {
           if (!(ok = wait_cluster(&sm.full[stage], ph, abort, dev_err))) break;
           tc_fence_after();
@@ -234,17 +238,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (elect_one()) {
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk)
-              mma_bf16_pair(dt, da + 2 * kk, db + kk * (2048 >> 4), kIdescDh,
-                            (ks != k0) | (kk != 0));
+#pragma unroll
+              for (int nh = 0; nh < 2; ++nh)
+                mma_bf16_pair(tmem + nh * 256, da + 2 * kk,
+                              db + nh * ((kDhBBytes / 2) >> 4) + kk * (2048 >> 4), kIdescDh,
+                              (ks != k0) | (kk != 0));
             mma_commit_pair(&sm.empty[stage], (uint16_t)3);
           }
           __syncwarp();
           if (++stage == kDhStages) { stage = 0; ph ^= 1; }
         }
         if (!ok) break;
-        if (elect_one()) mma_commit_pair(&sm.acc_full[acc], (uint16_t)3);
+        if (elect_one()) mma_commit_pair(&sm.acc_full, (uint16_t)3);
         __syncwarp();
-        if (++acc == 2) { acc = 0; acc_ph ^= 1; }
       }
       if (elect_one()) mma_commit_pair(&sm.mma_done, (uint16_t)1);
       __syncwarp();
@@ -255,7 +261,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int quad = warp & 3;
     const int row = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-    int acc = 0;
     uint32_t acc_ph = 0;
     bool ok = true;
     for (int i = pid; i < n_items && ok; i += npairs) {
@@ -271,12 +276,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                   : nullptr;
       // Partial tiles stay unscaled (the combine pass scales their sum).
       const float sc = (slot < 0 && valid) ? row_scale(tok_c, lsum, t) : 1.f;
-      if (!(ok = wait_sleepy_cluster(&sm.acc_full[acc], acc_ph, abort, dev_err))) break;
+      if (!(ok = wait_sleepy_cluster(&sm.acc_full, acc_ph, abort, dev_err))) break;
+      acc_ph ^= 1;
       tc_fence_after();
 #pragma unroll 1
       for (int c = 0; c < kDhN / 32; ++c) {
         float x[32];
-        tmem_ld32(tmem + lane_off + acc * kDhN + c * 32, x);
+        tmem_ld32(tmem + lane_off + c * 32, x);
         if (dst) {
 #pragma unroll
           for (int e = 0; e < 8; ++e)
@@ -285,8 +291,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
       }
       tc_fence_before();
-      mbar_arrive_cluster(mapa(smem_u32(&sm.acc_empty[acc]), 0));
-      if (++acc == 2) { acc = 0; acc_ph ^= 1; }
+      mbar_arrive_cluster(mapa(smem_u32(&sm.acc_empty), 0));
     }
   }
 
