@@ -120,6 +120,35 @@ __device__ __forceinline__ void tail_item(const TailSplit &tl, int nks, int i, i
   }
 }
 
+// Pacing of dh_gemm_kernel's whole units: the CTA pairs of a round read the
+// same W rows (all of them read all of W, in step order) and four at a time
+// the same image rows, so they share those rows in L2 only while they stay
+// close in the vocabulary. Every kPaceEvery K steps the even CTA's producer
+// publishes its position (round * nks + step) and, while it is more than
+// kPaceLead steps ahead of the slowest pair still on a whole unit, waits
+// (at most kPaceCycles per check, then it goes on: the pacing only affects
+// speed, never results). A pair that has left its whole units publishes
+// INT_MAX.
+constexpr int kPaceEvery = 16;
+constexpr int kPaceLead = 64;
+constexpr long long kPaceCycles = 40000;
+
+__device__ __forceinline__ void pace_publish(int32_t *prog, int pid, int pos) {
+  *reinterpret_cast<volatile int32_t *>(prog + pid) = pos;
+}
+// Whole warp: bounded wait until every pair's position is at least pos - kPaceLead.
+__device__ __forceinline__ void pace_wait(const int32_t *prog, int ncl, int pos, int lane) {
+  const long long t0 = clock64();
+  while (true) {
+    int mn = 0x7fffffff;
+    for (int c = lane; c < ncl; c += 32)
+      mn = min(mn, *reinterpret_cast<const volatile int32_t *>(prog + c));
+    for (int o = 16; o > 0; o >>= 1) mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    if (mn >= pos - kPaceLead || clock64() - t0 > kPaceCycles) break;
+    __nanosleep(256);
+  }
+}
+
 struct DhSmem {
   uint8_t a[kDhStages][kDhABytes];
   uint8_t b[kDhStages][kDhBBytes];
@@ -133,7 +162,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     dh_gemm_kernel(const __grid_constant__ CUtensorMap tmG, const __grid_constant__ CUtensorMap tmW,
                    int d, int V, int rb0, int cap, const int32_t *counters,
                    const int32_t *tok_idx, const float *tok_c, const float *lsum, float *dH,
-                   float *scratch, int scratch_cap, int32_t *dev_err) {
+                   float *scratch, int scratch_cap, int32_t *prog, int32_t *dev_err) {
   const int Teff = counters[0];
   const int nrb = min(max((Teff + 127) / 128 - rb0, 0), cap);
   if (nrb == 0) return;  // no token in this chunk
@@ -180,13 +209,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int last_ph[kDhStages];
       for (int s = 0; s < kDhStages; ++s) last_ph[s] = -1;
       bool ok = true;
+      const bool pacing = prog != nullptr && r == 0 && npairs <= kMaxPairs;
+      if (pacing && lane == 0) pace_publish(prog, pid, 0);
       for (int i = pid; i < n_items && ok; i += npairs) {
         int u, k0, k1, slot;
         tail_item(tl, nks, i, u, k0, k1, slot);
         const int tp = u / nq, q = u - tp * nq;
         const int b = min(2 * tp + r, nrb - 1);
         const int atom0 = b * nks;  // the block's first image atom
+        const bool whole = pacing && slot < 0;
+        if (pacing && !whole && lane == 0) pace_publish(prog, pid, 0x7fffffff);
         for (int ks = k0; ks < k1; ++ks) {
+          if (whole && (ks & (kPaceEvery - 1)) == 0) {
+            const int pos = (i / npairs) * nks + ks;
+            if (lane == 0) pace_publish(prog, pid, pos);
+            pace_wait(prog, npairs, pos, lane);
+          }
           if (!(ok = wait_cluster(&sm.empty[stage], ph ^ 1, abort, dev_err))) break;
           if (elect_one()) {
             if (r == 0) mbar_expect_tx(&sm.full[stage], 2 * (kDhABytes + kDhBBytes));
@@ -202,6 +240,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (++stage == kDhStages) { stage = 0; ph ^= 1; }
         }
       }
+      if (pacing && lane == 0) pace_publish(prog, pid, 0x7fffffff);
       // The last copy of every stage: completed on the even CTA, consumed by
       // the pair MMA on the odd one (both CTAs issue the same sequence).
       for (int s = 0; s < kDhStages; ++s)
@@ -648,7 +687,7 @@ pair_status launch_chunk_bwd(const GradArgs &g, const GradWorkspace &w, cudaStre
   PAIR_BEGIN("dh_gemm_tc", s);
   dh_gemm_kernel<<<dh_grid, kThreads, dh_smem, s>>>(mGA, mW3, g.d, g.V, rb0, cap, w.counters,
                                                     w.tok_idx, w.tok_c, w.lsum, g.dH, w.tailbuf,
-                                                    scratch_cap, g.dev_err);
+                                                    scratch_cap, w.prog, g.dev_err);
   PAIR_LAUNCH_CHECK(s);
   if (scratch_cap > 0) {
     PAIR_BEGIN("dh_tail", s);

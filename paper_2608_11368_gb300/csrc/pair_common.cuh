@@ -11,6 +11,7 @@ namespace pairk {
 // Clusters the cluster backward may run at once (ring buffers are sized for
 // this many); each ring holds 8 owners x 2 tiles x 32 KB.
 constexpr int kMaxClusters = 24;
+constexpr int kMaxPairs = 256;  // 2-CTA clusters of a persistent grid, at most
 constexpr size_t kRingBytesPerCluster = 8 * 2 * 32768;
 
 constexpr float kLog2e = 1.4426950408889634f;
@@ -83,6 +84,7 @@ struct GradWorkspace {
   float *ref;          // [Tpad] per-token reference of the softmax terms (log2 units)
   float *mrow;         // [Tpad] row maximum of the logits (log2 units)
   float *lsum;         // [Tpad] image path: sum of 2^(z log2 e - ref) over the vocabulary
+  int32_t *prog;       // [kMaxPairs] image path: per-CTA-pair progress of the dH GEMM
   int32_t *rbflag;     // [n_rbmax] row block needs the fix-up pass
   int32_t *rb_list;    // [n_rbmax] row blocks of the fix-up pass (count in counters[1])
   int32_t *ready;      // [n_slots] per-unit publication counters

@@ -419,6 +419,7 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   const size_t o_ref = (cl || img) ? take((size_t)Tpad * 4) : off;
   const size_t o_mrow = (cl || img) ? take((size_t)Tpad * 4) : off;
   const size_t o_lsum = img ? take((size_t)Tpad * 4) : off;
+  const size_t o_prog = img ? take((size_t)kMaxPairs * 4) : off;
   const size_t o_rbflag = cl ? take((size_t)n_rbmax * 4) : off;
   const size_t o_rblist = cl ? take((size_t)n_rbmax * 4) : off;
   const size_t o_ready = cl ? take((size_t)n_slots * 4) : off;
@@ -448,6 +449,7 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->ref = (cl || img) ? reinterpret_cast<float *>(b + o_ref) : nullptr;
     out->mrow = (cl || img) ? reinterpret_cast<float *>(b + o_mrow) : nullptr;
     out->lsum = img ? reinterpret_cast<float *>(b + o_lsum) : nullptr;
+    out->prog = img ? reinterpret_cast<int32_t *>(b + o_prog) : nullptr;
     out->rbflag = cl ? reinterpret_cast<int32_t *>(b + o_rbflag) : nullptr;
     out->rb_list = cl ? reinterpret_cast<int32_t *>(b + o_rblist) : nullptr;
     out->ready = cl ? reinterpret_cast<int32_t *>(b + o_ready) : nullptr;
