@@ -374,16 +374,18 @@ def test_token_logp_matches_oracle(case):
     np.testing.assert_allclose(lps.cpu().numpy(), sums, rtol=1e-5, atol=1e-4)
 
 
+@pytest.mark.parametrize("blocks", [0, None, 1], ids=["onchip", "image", "image_chunked"])
 @pytest.mark.parametrize("case", [(512, 1000, 0.3, 3), (1024, 3001, 0.2, 8),
                                   (2048, 2000, 0.15, 5)],
                          ids=["d512_V1000", "d1024_V3001", "d2048_V2000"])
-def test_grad_onchip_fixup_rows(case):
-    """The on-chip path (minimum workspace) takes each token's softmax terms
-    relative to its target logit; a row whose maximum logit exceeds the
-    target's by more than 2^64 (in log2 units) is redone relative to its
-    maximum. Peaky logits (std 24) with some targets set to the least likely
-    token of their row force such rows, in full and in tail row blocks; the
-    result must still match the oracle."""
+def test_grad_fixup_rows(case, blocks):
+    """Both bf16 head forms take each token's softmax terms relative to its
+    target logit (the on-chip form with the minimum workspace, the image form
+    with the default one or with one token block per chunk); a row whose
+    maximum logit exceeds the target's by more than 2^64 (in log2 units) is
+    redone relative to its maximum. Peaky logits (std 24) with some targets
+    set to the least likely token of their row force such rows, in full and
+    in tail row blocks; the result must still match the oracle."""
     d, V, ls, stride = case
     inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 7, B=3, G=8, d=d, V=V,
                                    len_scale=ls, w_std_mult=24.0)
@@ -397,9 +399,9 @@ def test_grad_onchip_fixup_rows(case):
     inp["y"][idx[::stride]] = np.argmin(Z, axis=1).astype(np.int32)
     gap = (Z.max(axis=1) - Z.min(axis=1)) * np.log2(np.e)
     assert (gap > 80).mean() > 0.9    # far beyond the 2^64 threshold
-    _full_check(inp, a, image_blocks=0)
+    _full_check(inp, a, image_blocks=blocks)
     # Reruns are bit-identical (the fix-up pass included).
-    r0 = _run(inp, a, 0)
-    r1 = _run(inp, a, 0)
+    r0 = _run(inp, a, blocks)
+    r1 = _run(inp, a, blocks)
     assert r0[0] == 0 and r0[1] == r1[1]
     assert torch.equal(r0[2], r1[2]) and torch.equal(r0[3], r1[3])
