@@ -71,8 +71,8 @@ def parse_args():
     p.add_argument("--vocab", type=int, default=0,
                    help="override the head's vocabulary size (0 = the workload's)")
     p.add_argument("--ws-exact", action="store_true",
-                   help="size the pair_grad workspace for the active tokens (kept logits "
-                        "and logit-gradient image for ceil(T_eff/128) token blocks) instead "
+                   help="size the pair_grad workspace for the active tokens (image of "
+                        "softmax terms and scaled rows for ceil(T_eff/128) token blocks) instead "
                         "of pair_grad_workspace_size, which sizes it for the packed length")
     return p.parse_args()
 
@@ -422,8 +422,8 @@ def main():
     lps = torch.empty(R, dtype=torch.float32, device="cuda")
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
     if args.ws_exact:
-        # The coefficients fix which rollouts are active; kept logit terms and
-        # image for exactly their token blocks (one block's bytes: the size
+        # The coefficients fix which rollouts are active; image and scaled
+        # rows for exactly their token blocks (one block's bytes: the size
         # difference at T = 128).
         B.pair_coeffs(devb["r"], devb["J"], devb["rho"], a=a, active=active, edges=edges,
                       contrast_edges=contrast, dev_err=err)
@@ -471,7 +471,7 @@ def main():
                                              args.workload)
 
     # ---- the on-chip form: the same step with pair_grad_workspace_min_size,
-    # so no logit-sized tensor (logit terms or logit-gradient image) is kept
+    # so no logit-sized tensor (no image of softmax terms) is kept
     # in HBM; the backward recomputes the logits in clusters.
     onchip = None
     if not args.no_onchip:

@@ -458,7 +458,7 @@ PAIR_API pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dty
  * Arguments, outputs and numerics are those of pair_grad, minus ws and
  * ws_bytes. The workspace is a file-scope device array of
  * PAIR_NOALLOC_MAX_WORKSPACE bytes that every GPU loading this library
- * holds until the process exits. It keeps no logit-gradient image (the
+ * holds until the process exits. It keeps no image of softmax terms (the
  * backward recomputes the logits); a problem is accepted iff
  * pair_grad_workspace_min_size(T, d, V, R, dt) <= PAIR_NOALLOC_MAX_WORKSPACE
  * and rejected with PAIR_ERR_WORKSPACE before any launch otherwise. That

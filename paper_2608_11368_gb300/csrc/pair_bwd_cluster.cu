@@ -1,4 +1,4 @@
-// Backward of the bf16 LM-head path without a logit-gradient image (the
+// Backward of the bf16 LM-head path without an image of softmax terms (the
 // no-alloc path and minimum workspaces): the logits are recomputed. For
 // d = 512 A (A <= 6), 8-CTA clusters share each Gs tile through an L2 ring
 // (bwd_cluster_kernel); otherwise one CTA per row block and 256-wide d-slice
@@ -1289,7 +1289,7 @@ pair_status grad_head_fused(const GradArgs &g, const GradWorkspace &w, cudaStrea
 
 namespace tck {
 
-// The bf16 head without a logit-gradient image: the fused log-sum-exp + dH
+// The bf16 head without an image of softmax terms: the fused log-sum-exp + dH
 // pass and the recomputing dW pass (cluster form), for the hidden sizes the
 // cluster kernels take; false elsewhere (the caller runs the three passes).
 bool onchip_fused_applies(int d) { return use_cluster_path(d); }

@@ -108,7 +108,7 @@ int grad_gimg_rows(int64_t T, int32_t d, int32_t V, pair_dtype dt);
 size_t grad_image_block_bytes(int32_t d, int32_t V);
 constexpr uint32_t kGImgTileBytes = 128 * 128 * 2;  // one 128 x 128 bf16 tile
 
-// Workspace layout with gimg_rb token blocks of logit-gradient image (0 =
+// Workspace layout with gimg_rb token blocks of image and scaled rows (0 =
 // none; at most grad_gimg_rows). Returns its size in bytes.
 size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
                             pair_dtype dt, GradWorkspace *out, void *base, int gimg_rb);

@@ -1,8 +1,8 @@
 // Log-sum-exp pass of the bf16 LM-head path (Sec. 4.5 forward): per active
 // token the log-sum-exp of its logits z = W h and its target logit, on the
-// 5th-generation tensor cores. With a workspace that keeps them, the logit
-// terms of a chunk of token blocks are stored for the backward (fp16 terms
-// relative to each 32-column chunk maximum, and the maxima).
+// 5th-generation tensor cores. With a workspace that keeps them, the softmax
+// terms of a chunk of token blocks, relative to each token's target logit,
+// are stored for the backward as the bf16 image the dH and dW GEMMs read.
 #include "tc_kernels.cuh"
 
 namespace pairk {

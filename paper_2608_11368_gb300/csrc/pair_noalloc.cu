@@ -80,7 +80,7 @@ extern "C" pair_status pair_grad_noalloc(
   reset_launches();
   if (!H || !W || !y || !mask || !cu_seqlens || !a || !dH || !dW || !Jobj)
     return PAIR_ERR_INVALID_ARG;
-  // This path keeps no logit-gradient image (its dW pass recomputes the
+  // This path keeps no image of softmax terms (its dW pass recomputes the
   // logits), so it needs the workspace without one.
   const size_t need = pair_grad_workspace_min_size(T, d, V, R, dt);
   if (need == 0)

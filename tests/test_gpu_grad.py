@@ -34,7 +34,7 @@ def _coeffs(inp, scale=1.0):
 
 def _run(inp, a, image_blocks=None, **kw):
     """image_blocks: size the workspace to hold that many token blocks of
-    kept logits and logit-gradient image (0 = none: the recomputing
+    the image of softmax terms and scaled rows (0 = none: the recomputing
     backward); None = the default pair_grad_workspace_size."""
     B = _binding()
     t = head_inputs(inp, a)

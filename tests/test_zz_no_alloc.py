@@ -34,8 +34,8 @@ def test_noalloc_matches_pair_grad_twice():
                                           B.PAIR_BF16)
     assert 0 < need <= B.NOALLOC_MAX_WORKSPACE
     err = dev_err_word()
-    # pair_grad with the default workspace (dW from the kept logit-gradient
-    # tiles) agrees to rounding; with the minimum workspace it runs the same
+    # pair_grad with the default workspace (dH and dW from the kept image of
+    # softmax terms) agrees to rounding; with the minimum workspace it runs the same
     # kernels as the fixed array and agrees bit for bit.
     Jr, dHr, dWr, lpr = B.pair_grad(t["H"], t["W"], t["y"], t["mask"],
                                     t["cu_seqlens"], t["a"], dev_err=err)
