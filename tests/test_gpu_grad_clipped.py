@@ -45,9 +45,9 @@ def _case(inp, deltas=DELTAS):
 
 
 def _check(inp, a, lo, image_blocks=None):
-    """image_blocks: size the workspace for that many token blocks of kept
-    logit terms and image (several backward chunks, later ones recomputing
-    their log-sum-exp); None = pair_grad_workspace_size."""
+    """image_blocks: size the workspace for that many token blocks of the
+    image of softmax terms (several backward chunks, later ones recomputing
+    their terms); None = pair_grad_workspace_size."""
     B = _binding()
     t = head_inputs(inp, a)
     err = dev_err_word()
@@ -97,9 +97,9 @@ def test_clipped_fp32_reference_workload():
 
 
 CASES = [
-    ("qwen3_1p7b_head", 2048, 151936, 2, 4, 0.05, 1.0),  # cluster path, full head
-    ("qwen3_1p7b_head", 512, 1000, 3, 8, 0.3, 4.0),      # cluster path, long rollouts
-    ("qwen3_1p7b_head", 192, 1000, 3, 5, 0.05, 8.0),     # per-slice fallback
+    ("qwen3_1p7b_head", 2048, 151936, 2, 4, 0.05, 1.0),  # image form, full head
+    ("qwen3_1p7b_head", 512, 1000, 3, 8, 0.3, 4.0),      # image form, long rollouts
+    ("qwen3_1p7b_head", 192, 1000, 3, 5, 0.05, 8.0),     # per-slice fallback (d % 512 != 0)
 ]
 
 
@@ -114,7 +114,7 @@ def test_clipped_bf16_parity(case):
 
 @pytest.mark.parametrize("blocks", [1, 2])
 def test_clipped_backward_chunks(blocks):
-    """Several backward chunks: the first uses the logit terms the full
+    """Several backward chunks: the first uses the softmax terms the full
     log-sum-exp pass kept, later chunks recompute theirs."""
     inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 7, B=3, G=8, d=512,
                                    V=1000, len_scale=0.3, w_std_mult=4.0)
@@ -130,3 +130,28 @@ def test_clipped_on_policy_equals_pair_grad():
     a, lo = _case(inp, deltas=[0.0])
     ref = _check(inp, a, lo)
     np.testing.assert_allclose(ref["coef"], a, rtol=1e-5)
+
+
+@pytest.mark.parametrize("blocks", [None, 1], ids=["image", "image_chunked"])
+def test_clipped_fixup_rows(blocks):
+    """pair_grad_clipped runs the whole log-sum-exp first and the backward
+    after it (in chunks of one token block for blocks = 1, each recomputing
+    its softmax terms). Rows whose maximum logit lies more than 2^64 (log2
+    units) above the target logit are redone in that first pass with the row
+    maximum as reference, and the later chunks must use the settled
+    references. Peaky logits (std 24) with every 16th active token's target
+    set to the least likely token of its row force such rows; the ratio
+    offsets stay far from the clip boundaries."""
+    inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 7, B=3, G=8, d=512,
+                                   V=1000, len_scale=0.2, w_std_mult=24.0)
+    a0 = oracle.coeffs(inp["r"], inp["J"], inp["rho"])["a"].reshape(-1)
+    assert (a0 != 0).any()
+    idx, _, _ = oracle.compact_tokens(inp["cu_seqlens"], inp["mask"], a0)
+    pick = idx[::16]
+    Hf = synth.as_float(inp["H"][pick], "bf16").astype(np.float64)
+    Wf = synth.as_float(inp["W"], "bf16").astype(np.float64)
+    Z = Hf @ Wf.T
+    inp["y"][pick] = np.argmin(Z, axis=1).astype(np.int32)
+    assert ((Z.max(axis=1) - Z.min(axis=1)) * np.log2(np.e) > 80).mean() > 0.9
+    a, lo = _case(inp, deltas=[-0.6, 0.0, 0.6])
+    _check(inp, a, lo, image_blocks=blocks)
