@@ -92,15 +92,18 @@ CASES = [
     ("qwen3_1p7b_head", 192, 1000, 3, 5, 0.05, 8.0),     # ragged V, N=192 slice
     ("qwen3_4b_head", 320, 777, 2, 6, 0.03, 8.0),        # two slices (256 + 64)
     ("longctx_skew", 64, 300, 4, 4, 0.02, 1.0),          # minimal d
-    # Cluster backward (d = 512 * A): slice widths 64, 128, 192, with
-    # ragged vocabulary tails and several row blocks per cluster.
+    # d = 512 A: the image form (default workspace), with one, two, three
+    # 512-column units per token pair, ragged vocabulary tails, and fewer
+    # units than clusters (every unit split into vocabulary parts).
     ("qwen3_1p7b_head", 512, 1000, 3, 8, 0.3, 4.0),
     ("longctx_skew", 1024, 5003, 2, 8, 0.15, 2.0),
     ("qwen3_4b_head", 1536, 777, 2, 6, 0.08, 8.0),
-    # Wider hidden sizes: 96-wide (d = 2560, slice 320) and 64-wide
-    # (d = 3072, slice 384) column tiles, ragged in both directions.
+    # Wider hidden sizes, ragged in both directions: d = 2560 and 3072
+    # (the widest the cluster form's scratch covers), and d = 4096, where the
+    # image form runs without that scratch (no split last rounds).
     ("qwen3_4b_head", 2560, 4099, 2, 3, 0.05, 3.0),
     ("longctx_skew", 3072, 2011, 2, 4, 0.04, 3.0),
+    ("qwen3_4b_head", 4096, 1500, 2, 8, 0.1, 2.0),
 ]
 
 
@@ -126,10 +129,14 @@ CHUNKED = [
     # for d = 2560, 64 wide for d = 3072).
     ("qwen3_4b_head", 2560, 4099, 2, 3, 0.05, 3.0, 0),
     ("longctx_skew", 3072, 2011, 2, 4, 0.04, 3.0, 0),
-    # No image at d = 2048: 6-CTA clusters with 320- and 352-column slices,
-    # a ragged vocabulary and tail row blocks split across clusters.
+    # No image at d = 2048: the 8-CTA cluster form with a ragged vocabulary
+    # and tail row blocks split across clusters.
     ("qwen3_1p7b_head", 2048, 20000, 2, 8, 0.15, 1.0, 0),
     ("longctx_skew", 2048, 5003, 4, 8, 0.12, 2.0, 0),
+    # d = 4096: beyond the cluster form, so no image means the per-slice
+    # backward; one-block chunks of the image form.
+    ("qwen3_4b_head", 4096, 1500, 2, 8, 0.1, 2.0, 0),
+    ("qwen3_4b_head", 4096, 1500, 2, 8, 0.1, 2.0, 1),
 ]
 
 
@@ -179,7 +186,7 @@ def test_grad_nan_padding_is_ignored_and_deterministic():
 @pytest.mark.parametrize("blocks,d", [(None, 512), (0, 512), (2, 512), (0, 2048)])
 def test_grad_cluster_path_deterministic(blocks, d):
     """Cluster backward with tail row blocks split across clusters (and, for
-    blocks = 2, several token chunks; at d = 2048 with 6-CTA clusters): reruns
+    blocks = 2, several token chunks; at d = 2048 in the cluster form): reruns
     are bit-identical."""
     inp = synth.make_head_workload(synth.WORKLOADS["qwen3_1p7b_head"], 5, B=3, G=8, d=d,
                                    V=1000, len_scale=0.3, w_std_mult=4.0)
