@@ -470,35 +470,8 @@ def main():
     roofline, pair_grad_info = kernel_report(kern, args.steps, T_eff, V, d, peaks, traffic,
                                              args.workload)
 
-    # ---- the on-chip form: the same step with pair_grad_workspace_min_size,
-    # so no logit-sized tensor (no image of softmax terms) is kept
-    # in HBM; the backward recomputes the logits in clusters.
-    onchip = None
-    if not args.no_onchip:
-        ws_min = torch.empty(B.pair_grad_workspace_min_size(T, d, V, R, B.PAIR_BF16),
-                             dtype=torch.uint8, device="cuda")
-        oc_step = lambda: step(wsp=ws_min)
-        for _ in range(args.warmup):
-            oc_step()
-        if B.pair_status_sync(err) != 0:
-            raise SystemExit("on-chip warm-up step failed")
-        oc_steps = max(3, min(args.steps, 20))
-        sampler_oc = ClockSampler(0)
-        sampler_oc.start()
-        oc_ms, oc_kern = timed_steps(B, torch, oc_step, oc_steps, flush)
-        oc_clocks = sampler_oc.stop()
-        if B.pair_status_sync(err) != 0:
-            raise SystemExit("on-chip steps reported a device error")
-        oc_roof, oc_info = kernel_report(oc_kern, oc_steps, T_eff, V, d, peaks, traffic,
-                                         args.workload + ":onchip")
-        onchip = {"ms_per_step": sum(oc_ms) / oc_steps, "steps": oc_steps,
-                  "warmup": args.warmup,
-                  "value": T * oc_steps / (sum(oc_ms) / 1e3), "unit": "tokens/s",
-                  "workspace_bytes": ws_min.numel(), "roofline": oc_roof, "pair_grad": oc_info,
-                  "clocks": oc_clocks}
-        del ws_min
-
-    # ---- end-to-end through the C-ABI with host buffers: every step copies
+    # ---- end-to-end through the C-ABI with host buffers, right after the
+    # device-resident steps (same GPU state as `value`): every step copies
     # all of its inputs from pinned host memory and reads J and logp back.
     # Inputs are double-buffered on a copy stream, so step k + 1's copy runs
     # while step k computes (the way a trainer feeds the stream-ordered API);
@@ -543,6 +516,34 @@ def main():
     e2e = {"value": T * args.steps / (e2e_ms / 1e3), "unit": "tokens/s",
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
     del sets
+
+    # ---- the on-chip form: the same step with pair_grad_workspace_min_size,
+    # so no logit-sized tensor (no image of softmax terms) is kept
+    # in HBM; the backward recomputes the logits in clusters.
+    onchip = None
+    if not args.no_onchip:
+        ws_min = torch.empty(B.pair_grad_workspace_min_size(T, d, V, R, B.PAIR_BF16),
+                             dtype=torch.uint8, device="cuda")
+        oc_step = lambda: step(wsp=ws_min)
+        for _ in range(args.warmup):
+            oc_step()
+        if B.pair_status_sync(err) != 0:
+            raise SystemExit("on-chip warm-up step failed")
+        oc_steps = max(3, min(args.steps, 20))
+        sampler_oc = ClockSampler(0)
+        sampler_oc.start()
+        oc_ms, oc_kern = timed_steps(B, torch, oc_step, oc_steps, flush)
+        oc_clocks = sampler_oc.stop()
+        if B.pair_status_sync(err) != 0:
+            raise SystemExit("on-chip steps reported a device error")
+        oc_roof, oc_info = kernel_report(oc_kern, oc_steps, T_eff, V, d, peaks, traffic,
+                                         args.workload + ":onchip")
+        onchip = {"ms_per_step": sum(oc_ms) / oc_steps, "steps": oc_steps,
+                  "warmup": args.warmup,
+                  "value": T * oc_steps / (sum(oc_ms) / 1e3), "unit": "tokens/s",
+                  "workspace_bytes": ws_min.numel(), "roofline": oc_roof, "pair_grad": oc_info,
+                  "clocks": oc_clocks}
+        del ws_min
 
     # ---- the other head workloads (Qwen3-4B head; heavy-tailed long context).
     extra = None
