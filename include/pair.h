@@ -465,9 +465,9 @@ PAIR_API pair_status pair_grad_clipped(int64_t T, int32_t d, int32_t V, pair_dty
  * size grows with T * d (the compacted hidden rows) plus, for bf16, a fixed
  * exchange buffer and, for d a multiple of 512, per-cluster partial rows of
  * width d. In this build the accepted range is, roughly: PAIR_F32, T (4 d +
- * 148) <= 33 MB (T <= 28,000 at d = 256); PAIR_BF16 with d a multiple of 512,
+ * 152) <= 33 MB (T <= 28,000 at d = 256); PAIR_BF16 with d a multiple of 512,
  * only d = 512 with T <= 6,000 (larger d need more than the array for the
- * partial rows alone); other PAIR_BF16 d, T (2 d + 148) <= 20.9 MB. Larger
+ * partial rows alone); other PAIR_BF16 d, T (2 d + 152) <= 20.9 MB. Larger
  * heads (the Qwen3 shapes) need pair_grad with a caller-provided workspace.
  * The call allocates nothing.
  * The first call on each device looks up the array's device address (with

@@ -12,6 +12,7 @@ namespace pairk {
 // this many); each ring holds 8 owners x 2 tiles x 32 KB.
 constexpr int kMaxClusters = 24;
 constexpr int kMaxPairs = 256;  // 2-CTA clusters of a persistent grid, at most
+constexpr int kOneHotBucket = 16;  // vocabulary rows per bucket of the one-hot dW part
 constexpr size_t kRingBytesPerCluster = 8 * 2 * 32768;
 
 constexpr float kLog2e = 1.4426950408889634f;
@@ -78,6 +79,9 @@ struct GradWorkspace {
   float *ppo_c;        // [R] clipped-surrogate coefficients (pair_grad_clipped)
   double *ppo_L;       // [R] clipped-surrogate terms (pair_grad_clipped)
   void *Hc;            // [Tpad][d] compacted hidden rows (dt), zero tail
+  int32_t *bkt;        // [3][nb + 1] one-hot part of dW: per target bucket of
+                       // kOneHotBucket rows, token counts, offsets, fill counters
+  int32_t *blist;      // [Tpad] active tokens grouped by target bucket
   void *gring;         // per-cluster ring of published Gs tiles
   float *tailbuf;      // [kMaxClusters][2][128][d] partial tail units (cluster path)
   // Fused log-sum-exp + dH pass (cluster path; null otherwise).

@@ -220,10 +220,14 @@ __global__ void onehot_dh_kernel(int d, const int32_t *counters,
 }
 
 // dW_v += sum_{t: y_t = v} c_t h_t (the one-hot part of dJ/dW_v), exact in
-// fp32, tokens added in their packed order. One warp owns a bucket of
-// vocabulary rows and scans the compacted targets for matches (four 32-token
-// chunks per round, so the target loads overlap); a matching row is updated
-// with 16-byte vector accesses when d allows it.
+// fp32, tokens added in their packed order. The compacted tokens are grouped
+// by target bucket (kOneHotBucket vocabulary rows): counts, offsets and a
+// fill (in any order); then one warp owns a bucket and puts its tokens in
+// packed order: up to 32 by a bitonic sort in registers, up to
+// kOneHotRankMax by ranking each against all others into shared memory; a
+// heavier bucket instead scans the compacted targets in order for its rows
+// (four 32-token chunks per round, so the target loads overlap). A row is
+// updated with 16-byte vector accesses when d allows it.
 __device__ __forceinline__ void load8(const __nv_bfloat16 *h, float (&x)[8]) {
   const uint4 u = *reinterpret_cast<const uint4 *>(h);
   const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&u);
@@ -279,22 +283,158 @@ __device__ __forceinline__ void axpy_row(int d, float c, const Tin *__restrict__
   }
 }
 
+__global__ void onehot_count_kernel(const int32_t *counters, const int32_t *tok_y,
+                                    int32_t *cnt) {
+  const int Teff = counters[0];
+  for (int p = blockIdx.x * blockDim.x + threadIdx.x; p < Teff; p += gridDim.x * blockDim.x)
+    atomicAdd(&cnt[tok_y[p] / kOneHotBucket], 1);
+}
+
+// off[b] = sum of cnt[< b] for b <= nb (one block of 1024 threads).
+__global__ void __launch_bounds__(1024) onehot_scan_kernel(int nb, const int32_t *cnt,
+                                                           int32_t *off) {
+  __shared__ int32_t wsum[32];
+  __shared__ int32_t carry;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int base = 0; base <= nb; base += 1024) {
+    const int b = base + threadIdx.x;
+    const int v = b < nb ? cnt[b] : 0;
+    int x = v;  // inclusive warp scan
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) wsum[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+      int w = wsum[lane];
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, w, o);
+        if (lane >= o) w += y;
+      }
+      wsum[lane] = w;
+    }
+    __syncthreads();
+    const int excl = carry + (warp ? wsum[warp - 1] : 0) + x - v;
+    if (b <= nb) off[b] = excl;
+    __syncthreads();
+    if (threadIdx.x == 1023) carry = excl + v;
+    __syncthreads();
+  }
+}
+
+__global__ void onehot_fill_kernel(const int32_t *counters, const int32_t *tok_y,
+                                   const int32_t *off, int32_t *fill, int32_t *blist) {
+  const int Teff = counters[0];
+  for (int p = blockIdx.x * blockDim.x + threadIdx.x; p < Teff; p += gridDim.x * blockDim.x) {
+    const int b = tok_y[p] / kOneHotBucket;
+    blist[off[b] + atomicAdd(&fill[b], 1)] = p;
+  }
+}
+
+// row += c h over d elements by 8 lanes (lane8 = lane index within them).
 template <typename Tin>
-__global__ void onehot_dw_kernel(int d, int V, int bucket,
-                                 const int32_t *counters, const int32_t *tok_y,
-                                 const float *tok_c, const Tin *Hc, float *dW) {
-  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+__device__ __forceinline__ void axpy_row8(int d, float c, const Tin *__restrict__ h,
+                                          float *__restrict__ row, int lane8) {
+  if ((d & 7) == 0) {
+    for (int k0 = lane8 * 8; k0 < d; k0 += 64) {
+      float x[8];
+      load8(h + k0, x);
+      float4 ra = reinterpret_cast<float4 *>(row + k0)[0];
+      float4 rb = reinterpret_cast<float4 *>(row + k0)[1];
+      ra = make_float4(fmaf(c, x[0], ra.x), fmaf(c, x[1], ra.y), fmaf(c, x[2], ra.z),
+                       fmaf(c, x[3], ra.w));
+      rb = make_float4(fmaf(c, x[4], rb.x), fmaf(c, x[5], rb.y), fmaf(c, x[6], rb.z),
+                       fmaf(c, x[7], rb.w));
+      reinterpret_cast<float4 *>(row + k0)[0] = ra;
+      reinterpret_cast<float4 *>(row + k0)[1] = rb;
+    }
+  } else {
+    for (int k = lane8; k < d; k += 8) row[k] = fmaf(c, (float)h[k], row[k]);
+  }
+}
+
+// Adds the one-hot terms of tokens q_0 < q_1 < ... (packed positions, given
+// by get(i), i < n) in that order per target row: four consecutive tokens at
+// a time, 8 lanes each, when their four rows differ; one at a time otherwise.
+template <typename Tin, typename Get>
+__device__ __forceinline__ void onehot_apply_sorted(int d, int n, Get get, const int32_t *tok_y,
+                                                    const float *tok_c, const Tin *Hc,
+                                                    float *dW, int lane) {
+  int i = 0;
+  while (i < n) {
+    if (i + 4 <= n) {
+      const int q0 = get(i), q1 = get(i + 1), q2 = get(i + 2), q3 = get(i + 3);
+      const int y0 = tok_y[q0], y1 = tok_y[q1], y2 = tok_y[q2], y3 = tok_y[q3];
+      if (y0 != y1 && y0 != y2 && y0 != y3 && y1 != y2 && y1 != y3 && y2 != y3) {
+        const int g = lane >> 3;
+        const int q = g == 0 ? q0 : g == 1 ? q1 : g == 2 ? q2 : q3;
+        const int y = g == 0 ? y0 : g == 1 ? y1 : g == 2 ? y2 : y3;
+        axpy_row8(d, tok_c[q], Hc + (int64_t)q * d, dW + (int64_t)y * d, lane & 7);
+        __syncwarp();
+        i += 4;
+        continue;
+      }
+    }
+    const int q = get(i);
+    axpy_row(d, tok_c[q], Hc + (int64_t)q * d, dW + (int64_t)tok_y[q] * d, lane);
+    __syncwarp();
+    ++i;
+  }
+}
+
+constexpr int kOneHotRankMax = 512;  // bucket tokens ranked in shared memory, at most
+
+template <typename Tin>
+__global__ void __launch_bounds__(256)
+    onehot_dw_kernel(int d, int V, int nb, const int32_t *counters, const int32_t *tok_y,
+                     const float *tok_c, const int32_t *off, const int32_t *blist,
+                     const Tin *Hc, float *dW) {
+  __shared__ int32_t sorted[8][kOneHotRankMax];  // per warp of the block
+  const int bk = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
-  const int v0 = warp * bucket;
-  if (v0 >= V) return;
-  const int v1 = min(V, v0 + bucket);
+  if (bk >= nb) return;
+  const int b0 = off[bk], n = off[bk + 1] - b0;
+  if (n == 0) return;
+  if (n > 32 && n <= kOneHotRankMax) {
+    // Rank each token against all others of the bucket (positions are
+    // distinct), then add them in rank order.
+    int32_t *srt = sorted[threadIdx.x >> 5];
+    for (int i = lane; i < n; i += 32) {
+      const int p = blist[b0 + i];
+      int rank = 0;
+      for (int j = 0; j < n; ++j) rank += blist[b0 + j] < p ? 1 : 0;
+      srt[rank] = p;
+    }
+    __syncwarp();
+    onehot_apply_sorted(d, n, [&](int i) { return srt[i]; }, tok_y, tok_c, Hc, dW, lane);
+    return;
+  }
+  if (n <= 32) {
+    // Bitonic sort of the bucket's packed positions across the warp.
+    int p = lane < n ? blist[b0 + lane] : 0x7fffffff;
+#pragma unroll
+    for (int k = 2; k <= 32; k <<= 1)
+#pragma unroll
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        const int q = __shfl_xor_sync(0xffffffffu, p, j);
+        p = (((lane & j) == 0) == ((lane & k) == 0)) ? min(p, q) : max(p, q);
+      }
+    onehot_apply_sorted(
+        d, n, [&](int i) { return __shfl_sync(0xffffffffu, p, i); }, tok_y, tok_c, Hc, dW, lane);
+    return;
+  }
+  const int v0 = bk * kOneHotBucket;
+  const int v1 = min(V, v0 + kOneHotBucket);
   const int Teff = counters[0];
   for (int base = 0; base < Teff; base += 128) {
     int yt[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      const int p = base + 32 * i + lane;
-      yt[i] = p < Teff ? tok_y[p] : -1;
+      const int pp = base + 32 * i + lane;
+      yt[i] = pp < Teff ? tok_y[pp] : -1;
     }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -408,6 +548,9 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
   const size_t o_ppoc = take((size_t)R * 4);
   const size_t o_ppol = take((size_t)R * 8);
   const size_t o_hc = take((size_t)Tpad * d * esz);
+  const size_t nb = (size_t)((V + kOneHotBucket - 1) / kOneHotBucket);
+  const size_t o_bkt = take(3 * (nb + 1) * 4);
+  const size_t o_blist = take((size_t)Tpad * 4);
   const size_t o_ring = dt == PAIR_BF16 ? take((size_t)kMaxClusters * kRingBytesPerCluster) : off;
   const bool cl = dt == PAIR_BF16 && grad_cluster_path(d);
   // Hidden sizes the image backward takes (grad_gimg_rows): per-token
@@ -444,6 +587,8 @@ size_t grad_workspace_bytes(int64_t T, int32_t d, int32_t V, int32_t R,
     out->ppo_c = reinterpret_cast<float *>(b + o_ppoc);
     out->ppo_L = reinterpret_cast<double *>(b + o_ppol);
     out->Hc = b + o_hc;
+    out->bkt = reinterpret_cast<int32_t *>(b + o_bkt);
+    out->blist = reinterpret_cast<int32_t *>(b + o_blist);
     out->gring = b + o_ring;
     out->tailbuf = cl ? reinterpret_cast<float *>(b + o_tail) : nullptr;
     out->ref = (cl || img) ? reinterpret_cast<float *>(b + o_ref) : nullptr;
@@ -555,8 +700,20 @@ pair_status grad_ppo_finalize(const GradArgs &g, const GradWorkspace &w, cudaStr
 
 pair_status grad_onehot(const GradArgs &g, const GradWorkspace &w,
                         cudaStream_t s) {
-  const int bucket = 128;
-  const int warps = (int)ceil_div(g.V, bucket);
+  const int nb = (g.V + kOneHotBucket - 1) / kOneHotBucket;
+  int32_t *cnt = w.bkt, *off = w.bkt + (nb + 1), *fill = w.bkt + 2 * (nb + 1);
+  PAIR_CUDA_TRY(cudaMemsetAsync(cnt, 0, (size_t)(nb + 1) * sizeof(int32_t), s));
+  PAIR_CUDA_TRY(cudaMemsetAsync(fill, 0, (size_t)(nb + 1) * sizeof(int32_t), s));
+  PAIR_BEGIN("onehot_count", s);
+  onehot_count_kernel<<<152 * 4, 256, 0, s>>>(w.counters, w.tok_y, cnt);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("onehot_scan", s);
+  onehot_scan_kernel<<<1, 1024, 0, s>>>(nb, cnt, off);
+  PAIR_LAUNCH_CHECK(s);
+  PAIR_BEGIN("onehot_fill", s);
+  onehot_fill_kernel<<<152 * 4, 256, 0, s>>>(w.counters, w.tok_y, off, fill, w.blist);
+  PAIR_LAUNCH_CHECK(s);
+  const int blocks = (int)ceil_div(nb, 8);  // 8 warps (buckets) per block
   if (g.dt == PAIR_BF16) {
     const __nv_bfloat16 *W = static_cast<const __nv_bfloat16 *>(g.W);
     PAIR_BEGIN("onehot_dh", s);
@@ -564,8 +721,8 @@ pair_status grad_onehot(const GradArgs &g, const GradWorkspace &w,
         g.d, w.counters, w.tok_idx, w.tok_y, w.tok_c, W, g.dH);
     PAIR_LAUNCH_CHECK(s);
     PAIR_BEGIN("onehot_dw", s);
-    onehot_dw_kernel<__nv_bfloat16><<<(int)ceil_div(warps, 8), 256, 0, s>>>(
-        g.d, g.V, bucket, w.counters, w.tok_y, w.tok_c,
+    onehot_dw_kernel<__nv_bfloat16><<<blocks, 256, 0, s>>>(
+        g.d, g.V, nb, w.counters, w.tok_y, w.tok_c, off, w.blist,
         static_cast<const __nv_bfloat16 *>(w.Hc), g.dW);
     PAIR_LAUNCH_CHECK(s);
   } else {
@@ -575,8 +732,8 @@ pair_status grad_onehot(const GradArgs &g, const GradWorkspace &w,
         static_cast<const float *>(g.W), g.dH);
     PAIR_LAUNCH_CHECK(s);
     PAIR_BEGIN("onehot_dw", s);
-    onehot_dw_kernel<float><<<(int)ceil_div(warps, 8), 256, 0, s>>>(
-        g.d, g.V, bucket, w.counters, w.tok_y, w.tok_c,
+    onehot_dw_kernel<float><<<blocks, 256, 0, s>>>(
+        g.d, g.V, nb, w.counters, w.tok_y, w.tok_c, off, w.blist,
         static_cast<const float *>(w.Hc), g.dW);
     PAIR_LAUNCH_CHECK(s);
   }
