@@ -204,30 +204,7 @@ __global__ void objective_kernel(int R, const float *a, const double *seg_logp,
   }
 }
 
-// dH_t += c_t W[y_t]  (the one-hot part of dJ/dh_t, exact in fp32).
-template <typename Tin>
-__global__ void onehot_dh_kernel(int d, const int32_t *counters,
-                                 const int32_t *tok_idx, const int32_t *tok_y,
-                                 const float *tok_c, const Tin *W, float *dH) {
-  const int Teff = counters[0];
-  for (int p = blockIdx.x; p < Teff; p += gridDim.x) {
-    const float c = tok_c[p];
-    const Tin *w = W + (int64_t)tok_y[p] * d;
-    float *row = dH + (int64_t)tok_idx[p] * d;
-    for (int k = threadIdx.x; k < d; k += blockDim.x)
-      row[k] = fmaf(c, (float)w[k], row[k]);
-  }
-}
-
-// dW_v += sum_{t: y_t = v} c_t h_t (the one-hot part of dJ/dW_v), exact in
-// fp32, tokens added in their packed order. The compacted tokens are grouped
-// by target bucket (kOneHotBucket vocabulary rows): counts, offsets and a
-// fill (in any order); then one warp owns a bucket and puts its tokens in
-// packed order: up to 32 by a bitonic sort in registers, up to
-// kOneHotRankMax by ranking each against all others into shared memory; a
-// heavier bucket instead scans the compacted targets in order for its rows
-// (four 32-token chunks per round, so the target loads overlap). A row is
-// updated with 16-byte vector accesses when d allows it.
+// Eight consecutive elements as fp32.
 __device__ __forceinline__ void load8(const __nv_bfloat16 *h, float (&x)[8]) {
   const uint4 u = *reinterpret_cast<const uint4 *>(h);
   const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&u);
@@ -245,6 +222,61 @@ __device__ __forceinline__ void load8(const float *h, float (&x)[8]) {
   x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
 }
 
+// dH_t += c_t W[y_t]  (the one-hot part of dJ/dh_t, exact in fp32): 8
+// columns per thread with vector accesses (d is a multiple of 8 on both
+// paths), two tokens in flight per block.
+template <typename Tin>
+__global__ void onehot_dh_kernel(int d, const int32_t *counters,
+                                 const int32_t *tok_idx, const int32_t *tok_y,
+                                 const float *tok_c, const Tin *W, float *dH) {
+  const int Teff = counters[0];
+  const int d8 = d / 8;
+  for (int p0 = 2 * blockIdx.x; p0 < Teff; p0 += 2 * gridDim.x) {
+    const bool two = p0 + 1 < Teff;
+    const float c0 = tok_c[p0], c1 = two ? tok_c[p0 + 1] : 0.f;
+    const Tin *w0 = W + (int64_t)tok_y[p0] * d;
+    const Tin *w1 = two ? W + (int64_t)tok_y[p0 + 1] * d : w0;
+    float *r0 = dH + (int64_t)tok_idx[p0] * d;
+    float *r1 = two ? dH + (int64_t)tok_idx[p0 + 1] * d : r0;
+    for (int k8 = threadIdx.x; k8 < d8; k8 += blockDim.x) {
+      const int k = 8 * k8;
+      float x0[8], x1[8];
+      load8(w0 + k, x0);
+      float4 a0 = reinterpret_cast<float4 *>(r0 + k)[0];
+      float4 b0 = reinterpret_cast<float4 *>(r0 + k)[1];
+      float4 a1 = a0, b1 = b0;
+      if (two) {
+        load8(w1 + k, x1);
+        a1 = reinterpret_cast<float4 *>(r1 + k)[0];
+        b1 = reinterpret_cast<float4 *>(r1 + k)[1];
+      }
+      reinterpret_cast<float4 *>(r0 + k)[0] =
+          make_float4(fmaf(c0, x0[0], a0.x), fmaf(c0, x0[1], a0.y), fmaf(c0, x0[2], a0.z),
+                      fmaf(c0, x0[3], a0.w));
+      reinterpret_cast<float4 *>(r0 + k)[1] =
+          make_float4(fmaf(c0, x0[4], b0.x), fmaf(c0, x0[5], b0.y), fmaf(c0, x0[6], b0.z),
+                      fmaf(c0, x0[7], b0.w));
+      if (two) {
+        reinterpret_cast<float4 *>(r1 + k)[0] =
+            make_float4(fmaf(c1, x1[0], a1.x), fmaf(c1, x1[1], a1.y), fmaf(c1, x1[2], a1.z),
+                        fmaf(c1, x1[3], a1.w));
+        reinterpret_cast<float4 *>(r1 + k)[1] =
+            make_float4(fmaf(c1, x1[4], b1.x), fmaf(c1, x1[5], b1.y), fmaf(c1, x1[6], b1.z),
+                        fmaf(c1, x1[7], b1.w));
+      }
+    }
+  }
+}
+
+// dW_v += sum_{t: y_t = v} c_t h_t (the one-hot part of dJ/dW_v), exact in
+// fp32, tokens added in their packed order. The compacted tokens are grouped
+// by target bucket (kOneHotBucket vocabulary rows): counts, offsets and a
+// fill (in any order); then one warp owns a bucket and puts its tokens in
+// packed order: up to 32 by a bitonic sort in registers, up to
+// kOneHotRankMax by ranking each against all others into shared memory; a
+// heavier bucket instead scans the compacted targets in order for its rows
+// (four 32-token chunks per round, so the target loads overlap). A row is
+// updated with 16-byte vector accesses when d allows it.
 template <typename Tin>
 __device__ __forceinline__ void axpy_row(int d, float c, const Tin *__restrict__ h,
                                          float *__restrict__ row, int lane) {
