@@ -140,18 +140,28 @@ __global__ void copy_rows_kernel(int64_t Tpad, int d, const int32_t *counters,
 }
 
 // Zero the dH rows of tokens outside the objective (mask = 0 or a = 0).
+constexpr int kZeroCuSmem = 8192;  // rollout offsets staged in shared memory, at most
+
 __global__ void zero_inactive_rows_kernel(int64_t T, int d, int R,
                                           const int32_t *cu,
                                           const uint8_t *mask, const float *a,
                                           float *dH) {
+  // The rollout offsets are searched once per row by every thread: from
+  // shared memory when they fit, so the search costs no global round trips.
+  extern __shared__ int32_t cu_s[];
+  const bool staged = R + 1 <= kZeroCuSmem;
+  if (staged)
+    for (int i = threadIdx.x; i <= R; i += blockDim.x) cu_s[i] = cu[i];
+  __syncthreads();
+  const int32_t *cs = staged ? cu_s : cu;
   for (int64_t t = blockIdx.x; t < T; t += gridDim.x) {
     // rollout of t: last i with cu[i] <= t
     int lo = 0, hi = R - 1;
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (cu[mid] <= t) lo = mid; else hi = mid - 1;
+      if (cs[mid] <= t) lo = mid; else hi = mid - 1;
     }
-    const bool live = mask[t] && coef_nonzero(a[lo]) && cu[lo] <= t && t < cu[lo + 1];
+    const bool live = mask[t] && coef_nonzero(a[lo]) && cs[lo] <= t && t < cs[lo + 1];
     if (live) continue;
     float4 *row = reinterpret_cast<float4 *>(dH + t * d);
     if ((d & 3) == 0) {
@@ -678,8 +688,9 @@ pair_status grad_prepare(const GradArgs &g, const GradWorkspace &w,
         static_cast<float *>(w.Hc));
   PAIR_LAUNCH_CHECK(s);
   PAIR_BEGIN("zero_inactive", s);
-  zero_inactive_rows_kernel<<<rows_grid, 128, 0, s>>>(g.T, g.d, g.R, g.cu,
-                                                      g.mask, g.a, g.dH);
+  const size_t cu_smem = g.R + 1 <= kZeroCuSmem ? (size_t)(g.R + 1) * sizeof(int32_t) : 0;
+  zero_inactive_rows_kernel<<<rows_grid, 128, cu_smem, s>>>(g.T, g.d, g.R, g.cu,
+                                                            g.mask, g.a, g.dH);
   PAIR_LAUNCH_CHECK(s);
   return PAIR_OK;
 }
