@@ -12,9 +12,9 @@ line also carries pair_coeffs / pair_estimate_dense GB/s on the
 4096 x 64 coefficient stress workload.
 
 Usage: python bench.py [--steps K] [--warmup W] [--impl gb300|reference]
-The library is single-GPU: its tensor-core kernels multicast TMA tiles within
-a thread-block cluster of this GPU, and every call runs on the current device
-alone. --gpus N with N > 1 (or a torchrun launch with WORLD_SIZE > 1) exits
+The library is single-GPU: every call runs on the current device alone, its
+tensor-core kernels pairing CTAs within thread-block clusters of that GPU.
+--gpus N with N > 1 (or a torchrun launch with WORLD_SIZE > 1) exits
 with an error for the GPU arm; the reference arm (the fp64 CPU oracle) runs
 on rank 0 only.
 """
@@ -384,8 +384,8 @@ def main():
     if args.impl == "reference":
         return run_reference(args, rank)
     if args.gpus != 1 or world != 1:
-        print("bench.py: single-GPU library (the head kernels multicast TMA tiles within a "
-              "cluster of one GPU); run it with --gpus 1", file=sys.stderr)
+        print("bench.py: single-GPU library (every call runs on the current device); "
+              "run it with --gpus 1", file=sys.stderr)
         return 2
 
     import torch
